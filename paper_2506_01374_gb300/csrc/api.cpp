@@ -1,0 +1,613 @@
+// Host-side C ABI: operators (programs P0), schedules (transformed
+// programs) and their legality. The problem statement (Sec. 2, Eq. 1)
+// defines a program transformed by a sequence of semantics-preserving
+// transformations; here a schedule is the canonical knob vector that such a
+// sequence produces, one vector per stage (kernel) of the op.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+
+#include "rc_internal.h"
+
+namespace {
+thread_local std::string g_err;
+
+constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
+
+// Tensor-core GEMM shared-memory footprint: a ring of `stages` A (128 x 64)
+// and B (bn x 64) bf16 tiles plus 1 KB alignment slack and barriers.
+int64_t tc_smem_bytes(int bn_mma, int stages) {
+  return (int64_t)stages * (128 * 64 * 2 + (int64_t)bn_mma * 64 * 2) + 1024 + 256;
+}
+
+bool tc_gemm_ok(int bn_mma, int stages, std::string* why) {
+  if (bn_mma % 16 != 0 || bn_mma < 16 || bn_mma > 256) {
+    if (why) *why = "UMMA N must be a multiple of 16 in [16, 256]";
+    return false;
+  }
+  if (tc_smem_bytes(bn_mma, stages) > kSmemLimit) {
+    if (why) *why = "operand ring exceeds 227 KB of shared memory";
+    return false;
+  }
+  return true;
+}
+
+const char* kind_name(int k) {
+  switch (k) {
+    case RC_OP_GEMM_F32: return "gemm_f32";
+    case RC_OP_LINEAR: return "linear";
+    case RC_OP_SWIGLU: return "swiglu";
+    case RC_OP_MLP: return "mlp";
+    case RC_OP_ATTENTION: return "attention";
+    case RC_OP_CONV2D: return "conv2d";
+    case RC_OP_MOE_ROUTE: return "moe_route";
+    case RC_OP_MOE: return "moe";
+  }
+  return "?";
+}
+
+int n_stages_of(int kind) {
+  switch (kind) {
+    case RC_OP_MLP: return 2;
+    case RC_OP_MOE: return 3;
+    default: return 1;
+  }
+}
+
+bool pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+}  // namespace
+
+rc_status rc_fail(rc_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return st;
+}
+
+void rc_clear_error() { g_err.clear(); }
+
+extern "C" const char* rc_last_error(void) { return g_err.c_str(); }
+extern "C" const char* rc_version(void) { return "rc 0.1 (sm_103a)"; }
+
+// ------------------------------------------------------------ knob spaces --
+// The transformation vocabulary of the paper's prompt (App. A: TileSize,
+// Parallel, ComputeLocation, Unroll) extended with loop order, fusion,
+// layout, vectorisation, pipeline stages and split-K. Every value listed
+// selects a distinct compiled kernel variant or launch configuration.
+std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
+  std::vector<KnobSpec> v;
+  const int kind = op->d.kind;
+  auto gemm_common = [&](std::vector<int32_t> tn) {
+    v.push_back({RC_T_TILE_SIZE, 1, tn, {}});
+    v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 6}, {}});
+    v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1, 8}});
+  };
+  switch (kind) {
+    case RC_OP_GEMM_F32:
+      v.push_back({RC_T_TILE_SIZE, 0, {16, 32, 64}, {}});
+      v.push_back({RC_T_TILE_SIZE, 1, {16, 32, 64}, {}});
+      v.push_back({RC_T_TILE_SIZE, 2, {16, 32, 64}, {}});
+      v.push_back({RC_T_UNROLL, 0, {1, 4}, {}});
+      break;
+    case RC_OP_LINEAR:
+      gemm_common({64, 128, 256});
+      v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
+      break;
+    case RC_OP_SWIGLU:
+      gemm_common({32, 64, 128});
+      v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      break;
+    case RC_OP_MLP:
+      if (stage == 0) {
+        gemm_common({32, 64, 128});
+        v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      } else {
+        gemm_common({64, 128, 256});
+        v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
+      }
+      break;
+    case RC_OP_CONV2D:
+      gemm_common({64, 80, 160});
+      v.push_back({RC_T_SPLIT_K, 0, {1, 3, 5}, {}});
+      v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      break;
+    case RC_OP_ATTENTION:
+      v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});
+      v.push_back({RC_T_PIPELINE_STAGES, 0, {2, 3}, {}});
+      v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1}});
+      break;
+    case RC_OP_MOE_ROUTE:
+      v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
+      break;
+    case RC_OP_MOE:
+      if (stage == 0) {
+        v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
+      } else if (stage == 1) {
+        gemm_common({32, 64, 128});
+      } else {
+        gemm_common({64, 128, 256});
+        v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      }
+      break;
+  }
+  return v;
+}
+
+rc_knobs rc_default_knobs(const rc_op_s* op, int stage) {
+  rc_knobs k;
+  memset(&k, 0, sizeof k);
+  k.tile_m = 128;
+  k.tile_k = 64;
+  k.unroll = 1;
+  k.stages = 1;
+  k.split_k = 1;
+  k.raster = 0;
+  k.group = 1;
+  k.persistent = 0;
+  k.fuse = 0;
+  k.layout = 0;
+  k.vec = 16;
+  k.location = 0;
+  switch (op->d.kind) {
+    case RC_OP_GEMM_F32:
+      k.tile_m = k.tile_n = k.tile_k = 16;
+      k.vec = 4;
+      k.fuse = 1;
+      break;
+    case RC_OP_LINEAR: k.tile_n = 64; break;
+    case RC_OP_SWIGLU: k.tile_n = 32; break;
+    case RC_OP_MLP: k.tile_n = stage == 0 ? 32 : 64; break;
+    case RC_OP_CONV2D: k.tile_n = 64; break;
+    case RC_OP_ATTENTION:
+      k.tile_n = 64;
+      k.stages = 2;
+      break;
+    case RC_OP_MOE_ROUTE: k.tile_m = 4; break;
+    case RC_OP_MOE:
+      if (stage == 0) k.tile_m = 4;
+      else k.tile_n = stage == 1 ? 32 : 64;
+      break;
+  }
+  return k;
+}
+
+static bool in(const std::vector<int32_t>& v, int32_t x) {
+  for (int32_t y : v)
+    if (y == x) return true;
+  return false;
+}
+
+bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string* why) {
+  // 1) every tunable knob holds one of its listed values; untunable knobs keep P0's value
+  const rc_knobs d = rc_default_knobs(op, stage);
+  const auto space = rc_knob_space(op, stage);
+  auto spec_of = [&](int tk, int axis) -> const KnobSpec* {
+    for (auto& s : space)
+      if (s.tkind == tk && s.axis == axis) return &s;
+    return nullptr;
+  };
+  struct F { int tk, axis; int32_t v, dv; } fields[] = {
+      {RC_T_TILE_SIZE, 0, k.tile_m, d.tile_m},       {RC_T_TILE_SIZE, 1, k.tile_n, d.tile_n},
+      {RC_T_TILE_SIZE, 2, k.tile_k, d.tile_k},       {RC_T_UNROLL, 0, k.unroll, d.unroll},
+      {RC_T_PIPELINE_STAGES, 0, k.stages, d.stages}, {RC_T_SPLIT_K, 0, k.split_k, d.split_k},
+      {RC_T_LOOP_ORDER, 0, k.raster, d.raster},      {RC_T_PARALLEL, 0, k.persistent, d.persistent},
+      {RC_T_FUSE, 0, k.fuse, d.fuse},                {RC_T_LAYOUT, 0, k.layout, d.layout},
+      {RC_T_VECTORIZE, 0, k.vec, d.vec},             {RC_T_COMPUTE_LOCATION, 0, k.location, d.location},
+  };
+  for (auto& f : fields) {
+    const KnobSpec* s = spec_of(f.tk, f.axis);
+    if (s ? !in(s->values, f.v) : f.v != f.dv) {
+      if (why) *why = "knob value outside this op's transformation space";
+      return false;
+    }
+  }
+  const KnobSpec* lo = spec_of(RC_T_LOOP_ORDER, 0);
+  if (lo ? !in(lo->values1, k.group) : k.group != d.group) {
+    if (why) *why = "raster group outside this op's transformation space";
+    return false;
+  }
+  // 2) resource and shape rules of the kernel the knobs select
+  const rc_op_desc& o = op->d;
+  switch (o.kind) {
+    case RC_OP_LINEAR:
+      return tc_gemm_ok(k.tile_n, k.stages, why);
+    case RC_OP_SWIGLU:
+      return tc_gemm_ok(2 * k.tile_n, k.stages, why);
+    case RC_OP_MLP:
+      return tc_gemm_ok(stage == 0 ? 2 * k.tile_n : k.tile_n, k.stages, why);
+    case RC_OP_CONV2D:
+      if (o.c_out % k.tile_n != 0) {
+        if (why) *why = "conv N tile must divide Cout";
+        return false;
+      }
+      return tc_gemm_ok(k.tile_n, k.stages, why);
+    case RC_OP_MOE:
+      if (stage == 0) return true;
+      return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, why);
+    default:
+      return true;
+  }
+}
+
+// -------------------------------------------------------------- op slots --
+std::vector<SlotInfo> rc_slots(const rc_op_s* op) {
+  const rc_op_desc& d = op->d;
+  std::vector<SlotInfo> s;
+  const size_t b2 = 2, b4 = 4;
+  switch (d.kind) {
+    case RC_OP_GEMM_F32:
+      s = {{b4 * d.m * d.k, true, false, false},
+           {b4 * d.k * d.n, true, false, false},
+           {b4 * d.n, true, false, true},
+           {b4 * d.m * d.n, false, true, false}};
+      break;
+    case RC_OP_LINEAR:
+      s = {{b2 * d.m * d.k, true, false, false},
+           {b2 * d.n * d.k, true, false, false},
+           {b2 * d.m * d.n, false, true, false}};
+      break;
+    case RC_OP_SWIGLU:
+      s = {{b2 * d.m * d.k, true, false, false},
+           {b2 * 2 * d.n * d.k, true, false, false},
+           {b2 * d.m * d.n, false, true, false}};
+      break;
+    case RC_OP_MLP:
+      s = {{b2 * d.m * d.k, true, false, false},
+           {b2 * 2 * d.n * d.k, true, false, false},
+           {b2 * d.k * d.n, true, false, false},
+           {b2 * d.m * d.k, false, true, false}};
+      break;
+    case RC_OP_ATTENTION: {
+      const size_t q = b2 * d.batch * d.seq * d.heads_q * d.head_dim;
+      const size_t kv = b2 * d.batch * d.seq * d.heads_kv * d.head_dim;
+      s = {{q, true, false, false},
+           {kv, true, false, false},
+           {kv, true, false, false},
+           {q, false, true, false},
+           {b4 * d.batch * d.heads_q * d.seq, false, true, true}};
+      break;
+    }
+    case RC_OP_CONV2D:
+      s = {{b2 * d.img_n * d.img_h * d.img_w * d.c_in, true, false, false},
+           {b2 * d.c_out * d.kr * d.ks * d.c_in, true, false, false},
+           {b2 * d.c_out, true, false, true},
+           {b2 * d.img_n * d.img_h * d.img_w * d.c_out, false, true, false}};
+      break;
+    case RC_OP_MOE_ROUTE: {
+      const size_t lg = (d.logits_fp32 ? b4 : b2) * d.tokens * d.experts;
+      const size_t tk = (size_t)d.tokens * d.top_k;
+      s = {{lg, true, false, false},
+           {b4 * tk, false, true, false},
+           {b4 * tk, false, true, false},
+           {b4 * (d.experts + 1), false, true, false},
+           {b4 * tk, false, true, false}};
+      break;
+    }
+    case RC_OP_MOE: {
+      const size_t lg = (d.logits_fp32 ? b4 : b2) * d.tokens * d.experts;
+      const size_t tk = (size_t)d.tokens * d.top_k;
+      s = {{lg, true, false, false},
+           {b2 * d.tokens * d.hidden, true, false, false},
+           {b2 * d.experts * 2 * d.inter * d.hidden, true, false, false},
+           {b2 * d.experts * d.hidden * d.inter, true, false, false},
+           {b2 * d.tokens * d.hidden, false, true, false},
+           {b4 * tk, false, true, true},
+           {b4 * tk, false, true, true},
+           {b4 * (d.experts + 1), false, true, true},
+           {b4 * tk, false, true, true}};
+      break;
+    }
+  }
+  return s;
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+size_t rc_workspace_bytes(const rc_op_s* op, const rc_schedule_s* s) {
+  const rc_op_desc& d = op->d;
+  const rc_knobs* k = s ? s->k : nullptr;
+  switch (d.kind) {
+    case RC_OP_LINEAR:
+      return (k && k[0].split_k > 1) ? align256(4ull * k[0].split_k * d.m * d.n) : 0;
+    case RC_OP_SWIGLU:
+      return (k && !k[0].fuse) ? align256(2ull * d.m * 2 * d.n) : 0;
+    case RC_OP_MLP: {
+      size_t b = align256(2ull * d.m * d.n);                          // h
+      if (k && !k[0].fuse) b += align256(2ull * d.m * 2 * d.n);       // gate|up before SwiGLU
+      if (k && k[1].split_k > 1) b += align256(4ull * k[1].split_k * d.m * d.k);
+      return b;
+    }
+    case RC_OP_CONV2D: {
+      const size_t rows = (size_t)d.img_n * d.img_h * d.img_w;
+      size_t b = 0;
+      if (k && k[0].split_k > 1) b += align256(4ull * k[0].split_k * rows * d.c_out);
+      if (k && (!k[0].fuse || k[0].split_k > 1)) b += align256(2ull * rows * d.c_out);
+      return b;
+    }
+    case RC_OP_MOE: {
+      const size_t slots = (size_t)d.tokens * d.top_k;
+      size_t b = 0;
+      b += align256(4 * slots) * 4 + align256(4 * (d.experts + 1));  // ids, w, perm, inv_perm, offsets
+      b += align256(2 * slots * d.hidden);                            // gathered X
+      b += align256(2 * slots * d.inter);                             // H
+      b += align256(2 * slots * d.hidden);                            // Y (bf16) for gather-reduce
+      b += align256(4ull * d.tokens * d.hidden);                      // fp32 out for atomic combine
+      return b;
+    }
+    default:
+      return 0;
+  }
+}
+
+// -------------------------------------------------------------- describe --
+extern "C" rc_status rc_op_describe(const rc_op_desc* desc, rc_op** out) {
+  if (!desc || !out) return rc_fail(RC_ERR_INVALID_ARG, "rc_op_describe: NULL argument");
+  *out = nullptr;
+  rc_op_desc d = *desc;
+  rc_op_info_t info;
+  memset(&info, 0, sizeof info);
+  auto bad = [&](const char* what) {
+    return rc_fail(RC_ERR_INVALID_ARG, "rc_op_describe(%s): %s", kind_name(d.kind), what);
+  };
+  auto unsup = [&](const char* what) {
+    return rc_fail(RC_ERR_UNSUPPORTED_OP, "rc_op_describe(%s): %s", kind_name(d.kind), what);
+  };
+  const double ridge = 283.0;  // bf16 tensor FLOP per HBM byte on GB300 (measured peaks ratio)
+  switch (d.kind) {
+    case RC_OP_GEMM_F32:
+      if (d.m <= 0 || d.n <= 0 || d.k <= 0) return bad("m, n, k must be positive");
+      info.flops = 2.0 * d.m * d.n * d.k;
+      info.bytes = 4.0 * (d.m * d.k + d.k * d.n + d.n + d.m * d.n);
+      info.bound = RC_BOUND_FP32_SIMT;
+      info.n_tensors = 4;
+      break;
+    case RC_OP_LINEAR:
+    case RC_OP_SWIGLU:
+    case RC_OP_MLP: {
+      if (d.m <= 0 || d.n <= 0 || d.k <= 0) return bad("m, n, k must be positive");
+      if (d.k % 8 || d.n % 8) return unsup("k and n must be multiples of 8 (16-byte rows)");
+      const double ncols = d.kind == RC_OP_SWIGLU ? 2.0 * d.n : (double)d.n;
+      if (d.kind == RC_OP_MLP) {
+        info.flops = 6.0 * d.m * d.n * d.k;
+        info.bytes = 2.0 * (2.0 * d.m * d.k + 3.0 * d.n * d.k);
+        info.n_tensors = 4;
+      } else {
+        info.flops = 2.0 * d.m * ncols * d.k;
+        info.bytes = 2.0 * (d.m * d.k + ncols * d.k + (double)d.m * d.n);
+        info.n_tensors = 3;
+      }
+      info.bound = info.flops / info.bytes >= ridge ? RC_BOUND_TENSOR : RC_BOUND_HBM;
+      break;
+    }
+    case RC_OP_ATTENTION: {
+      if (d.batch <= 0 || d.seq <= 0 || d.heads_q <= 0 || d.heads_kv <= 0 || d.head_dim <= 0)
+        return bad("sizes must be positive");
+      if (d.heads_q % d.heads_kv) return bad("heads_q must be a multiple of heads_kv");
+      if (d.head_dim != 128) return unsup("head_dim must be 128");
+      if (d.scale == 0.0) d.scale = 1.0 / std::sqrt((double)d.head_dim);
+      const double pairs = d.causal ? 0.5 * (double)d.seq * (d.seq + 1) : (double)d.seq * d.seq;
+      info.flops = 4.0 * d.head_dim * d.heads_q * d.batch * pairs;
+      info.bytes = 2.0 * d.batch * d.seq * d.head_dim * (2.0 * d.heads_q + 2.0 * d.heads_kv) +
+                   4.0 * d.batch * d.heads_q * d.seq;
+      info.bound = RC_BOUND_TENSOR;
+      info.n_tensors = 5;
+      break;
+    }
+    case RC_OP_CONV2D: {
+      if (d.img_n <= 0 || d.img_h <= 0 || d.img_w <= 0 || d.c_in <= 0 || d.c_out <= 0 || d.kr <= 0 ||
+          d.ks <= 0)
+        return bad("sizes must be positive");
+      if (d.stride == 0) d.stride = 1;
+      if (d.stride != 1 || d.kr != d.ks || d.kr % 2 == 0 || d.pad != (d.kr - 1) / 2)
+        return unsup("only stride-1 'same' convolutions with an odd square kernel");
+      if (d.c_in % 64) return unsup("c_in must be a multiple of 64");
+      if (d.c_out % 16) return unsup("c_out must be a multiple of 16");
+      if (!pow2(d.img_w) || d.img_w < 8 || d.img_w > 128 || d.img_h % (128 / d.img_w))
+        return unsup("img_w must be a power of two in [8, 128] and img_h a multiple of 128/img_w");
+      const double pix = (double)d.img_n * d.img_h * d.img_w;
+      info.flops = 2.0 * pix * d.c_out * d.kr * d.ks * d.c_in;
+      info.bytes = 2.0 * (pix * d.c_in + (double)d.c_out * d.kr * d.ks * d.c_in + d.c_out + pix * d.c_out);
+      info.bound = info.flops / info.bytes >= ridge ? RC_BOUND_TENSOR : RC_BOUND_HBM;
+      info.n_tensors = 4;
+      break;
+    }
+    case RC_OP_MOE_ROUTE:
+    case RC_OP_MOE: {
+      if (d.tokens <= 0 || d.experts <= 0 || d.top_k <= 0) return bad("sizes must be positive");
+      if (d.top_k > d.experts) return bad("top_k must not exceed experts");
+      if (d.experts > 256 || d.top_k > 16) return unsup("experts <= 256 and top_k <= 16");
+      const double slots = (double)d.tokens * d.top_k;
+      const double lg = (d.logits_fp32 ? 4.0 : 2.0) * d.tokens * d.experts;
+      if (d.kind == RC_OP_MOE_ROUTE) {
+        info.flops = 0.0;
+        info.bytes = lg + 12.0 * slots + 4.0 * (d.experts + 1);
+        info.bound = RC_BOUND_HBM;
+        info.n_tensors = 5;
+      } else {
+        if (d.hidden <= 0 || d.inter <= 0) return bad("hidden and inter must be positive");
+        if (d.hidden % 64 || d.inter % 64) return unsup("hidden and inter must be multiples of 64");
+        info.flops = 6.0 * slots * d.hidden * d.inter;
+        info.bytes = lg + 2.0 * (2.0 * d.tokens * d.hidden + 3.0 * d.experts * d.hidden * d.inter);
+        info.bound = info.flops / info.bytes >= ridge ? RC_BOUND_TENSOR : RC_BOUND_HBM;
+        info.n_tensors = 9;
+      }
+      break;
+    }
+    default:
+      return rc_fail(RC_ERR_UNSUPPORTED_OP, "rc_op_describe: unknown op kind %d", d.kind);
+  }
+  rc_op_s* op = new (std::nothrow) rc_op_s;
+  if (!op) return rc_fail(RC_ERR_OOM, "rc_op_describe: out of host memory");
+  op->d = d;
+  op->n_stages = n_stages_of(d.kind);
+  rc_schedule_s p0;
+  p0.op_kind = d.kind;
+  p0.n_stages = op->n_stages;
+  for (int i = 0; i < op->n_stages; ++i) p0.k[i] = rc_default_knobs(op, i);
+  info.workspace_bytes = (int64_t)rc_workspace_bytes(op, &p0);
+  op->info = info;
+  *out = op;
+  return RC_OK;
+}
+
+extern "C" rc_status rc_op_info(const rc_op* op, rc_op_info_t* info) {
+  if (!op || !info) return rc_fail(RC_ERR_INVALID_ARG, "rc_op_info: NULL argument");
+  *info = op->info;
+  return RC_OK;
+}
+
+// rc_op_destroy lives in run.cu (it frees device memory).
+
+// -------------------------------------------------------------- schedules --
+static rc_status apply_one(const rc_op_s* op, rc_schedule_s* s, const rc_transform& t) {
+  if (t.stage < 0 || t.stage >= s->n_stages)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "transform stage %d out of range", t.stage);
+  if (t.reserved != 0) return rc_fail(RC_ERR_INVALID_ARG, "rc_transform.reserved must be 0");
+  rc_knobs& k = s->k[t.stage];
+  const int32_t v = (int32_t)t.value[0];
+  if ((int64_t)v != t.value[0]) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "transform value out of range");
+  switch (t.kind) {
+    case RC_T_TILE_SIZE:
+      if (t.axis == 0) k.tile_m = v;
+      else if (t.axis == 1) k.tile_n = v;
+      else if (t.axis == 2) k.tile_k = v;
+      else return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "TileSize axis %d", t.axis);
+      break;
+    case RC_T_PARALLEL: k.persistent = v; break;
+    case RC_T_COMPUTE_LOCATION: k.location = v; break;
+    case RC_T_UNROLL: k.unroll = v; break;
+    case RC_T_LOOP_ORDER:
+      k.raster = v;
+      k.group = t.value[1] > 0 ? (int32_t)t.value[1] : 1;
+      break;
+    case RC_T_FUSE: k.fuse = v; break;
+    case RC_T_LAYOUT: k.layout = v; break;
+    case RC_T_VECTORIZE: k.vec = v; break;
+    case RC_T_PIPELINE_STAGES: k.stages = v; break;
+    case RC_T_SPLIT_K: k.split_k = v; break;
+    default: return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "unknown transform kind %d", t.kind);
+  }
+  (void)op;
+  return RC_OK;
+}
+
+extern "C" rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base, const rc_transform* seq,
+                                       size_t n, rc_schedule** out) {
+  if (!op || !out || (n && !seq)) return rc_fail(RC_ERR_INVALID_ARG, "rc_schedule_apply: NULL argument");
+  *out = nullptr;
+  rc_schedule_s s;
+  memset(&s, 0, sizeof s);
+  if (base) {
+    if (base->op_kind != op->d.kind || base->n_stages != op->n_stages)
+      return rc_fail(RC_ERR_INVALID_ARG, "rc_schedule_apply: base schedule belongs to another op kind");
+    s = *base;
+  } else {
+    s.op_kind = op->d.kind;
+    s.n_stages = op->n_stages;
+    for (int i = 0; i < op->n_stages; ++i) s.k[i] = rc_default_knobs(op, i);
+  }
+  for (size_t i = 0; i < n; ++i) RC_TRY(apply_one(op, &s, seq[i]));
+  for (int i = 0; i < s.n_stages; ++i) {
+    std::string why;
+    if (!rc_knobs_legal(op, i, s.k[i], &why))
+      return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "stage %d: %s", i, why.c_str());
+  }
+  rc_schedule_s* r = new (std::nothrow) rc_schedule_s(s);
+  if (!r) return rc_fail(RC_ERR_OOM, "rc_schedule_apply: out of host memory");
+  *out = r;
+  return RC_OK;
+}
+
+extern "C" rc_status rc_schedule_knobs(const rc_schedule* s, int32_t stage, rc_knobs* out) {
+  if (!s || !out) return rc_fail(RC_ERR_INVALID_ARG, "rc_schedule_knobs: NULL argument");
+  if (stage < 0 || stage >= s->n_stages) return rc_fail(RC_ERR_INVALID_ARG, "stage out of range");
+  *out = s->k[stage];
+  return RC_OK;
+}
+
+extern "C" int32_t rc_schedule_num_stages(const rc_schedule* s) { return s ? s->n_stages : 0; }
+
+extern "C" uint64_t rc_schedule_hash(const rc_schedule* s) {
+  if (!s) return 0;
+  // FNV-1a over the op kind and the canonical knob vectors
+  uint64_t h = 1469598103934665603ull;
+  auto mixin = [&](int32_t v) {
+    for (int b = 0; b < 4; ++b) {
+      h ^= (uint64_t)((v >> (8 * b)) & 0xFF);
+      h *= 1099511628211ull;
+    }
+  };
+  mixin(s->op_kind);
+  mixin(s->n_stages);
+  for (int i = 0; i < s->n_stages; ++i) {
+    const rc_knobs& k = s->k[i];
+    for (int32_t v : {k.tile_m, k.tile_n, k.tile_k, k.unroll, k.stages, k.split_k, k.raster, k.group,
+                      k.persistent, k.fuse, k.layout, k.vec, k.location})
+      mixin(v);
+  }
+  return h;
+}
+
+extern "C" rc_status rc_schedule_to_string(const rc_schedule* s, char* buf, size_t cap, size_t* needed) {
+  if (!s) return rc_fail(RC_ERR_INVALID_ARG, "rc_schedule_to_string: NULL schedule");
+  std::string out = std::string("op=") + kind_name(s->op_kind);
+  char tmp[256];
+  for (int i = 0; i < s->n_stages; ++i) {
+    const rc_knobs& k = s->k[i];
+    snprintf(tmp, sizeof tmp,
+             ";s%d:tile=%dx%dx%d,unroll=%d,stages=%d,split_k=%d,raster=%d/%d,persistent=%d,fuse=%d,"
+             "layout=%d,vec=%d,loc=%d",
+             i, k.tile_m, k.tile_n, k.tile_k, k.unroll, k.stages, k.split_k, k.raster, k.group,
+             k.persistent, k.fuse, k.layout, k.vec, k.location);
+    out += tmp;
+  }
+  if (needed) *needed = out.size() + 1;
+  if (buf && cap) {
+    size_t n = out.size() < cap - 1 ? out.size() : cap - 1;
+    memcpy(buf, out.data(), n);
+    buf[n] = 0;
+  }
+  return RC_OK;
+}
+
+extern "C" rc_status rc_schedule_clone(const rc_schedule* s, rc_schedule** out) {
+  if (!s || !out) return rc_fail(RC_ERR_INVALID_ARG, "rc_schedule_clone: NULL argument");
+  *out = new (std::nothrow) rc_schedule_s(*s);
+  return *out ? RC_OK : rc_fail(RC_ERR_OOM, "rc_schedule_clone: out of host memory");
+}
+
+extern "C" void rc_schedule_destroy(rc_schedule* s) { delete s; }
+
+extern "C" rc_status rc_transform_space(const rc_op* op, rc_transform* buf, size_t cap, size_t* n) {
+  if (!op || !n) return rc_fail(RC_ERR_INVALID_ARG, "rc_transform_space: NULL argument");
+  size_t cnt = 0;
+  for (int st = 0; st < op->n_stages; ++st) {
+    for (const KnobSpec& ks : rc_knob_space(op, st)) {
+      const size_t n1 = ks.values1.empty() ? 1 : ks.values1.size();
+      if (ks.values.size() * n1 < 2) continue;  // nothing to choose
+      for (int32_t v : ks.values) {
+        for (size_t j = 0; j < n1; ++j) {
+          if (buf && cnt < cap) {
+            rc_transform t;
+            memset(&t, 0, sizeof t);
+            t.kind = ks.tkind;
+            t.axis = ks.axis;
+            t.stage = st;
+            t.value[0] = v;
+            if (!ks.values1.empty()) t.value[1] = ks.values1[j];
+            buf[cnt] = t;
+          }
+          ++cnt;
+        }
+      }
+    }
+  }
+  *n = cnt;
+  if (buf && cnt > cap) return rc_fail(RC_ERR_INVALID_ARG, "rc_transform_space: buffer too small");
+  return RC_OK;
+}

@@ -1,0 +1,22 @@
+// Launchers of kernels that this build does not provide yet: they report
+// RC_ERR_UNSUPPORTED_OP so callers see a clear error instead of a fallback.
+#include "rc_internal.h"
+
+rc_status rc_launch_tc_gemm(const rc_knobs&, const TcGemmArgs&, const LaunchCtx&) {
+  return rc_fail(RC_ERR_UNSUPPORTED_OP, "tensor-core GEMM not built");
+}
+rc_status rc_launch_attention(const rc_knobs&, const rc_op_desc&, const void*, const void*, const void*, void*,
+                              float*, const LaunchCtx&) {
+  return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention not built");
+}
+rc_status rc_launch_moe_route(const rc_knobs&, const rc_op_desc&, const void*, int*, float*, int*, int*, int*,
+                              const LaunchCtx&) {
+  return rc_fail(RC_ERR_UNSUPPORTED_OP, "MoE routing not built");
+}
+rc_status rc_launch_moe_gather(const void*, const int*, int64_t, int64_t, int, void*, int, const LaunchCtx&) {
+  return rc_fail(RC_ERR_UNSUPPORTED_OP, "MoE gather not built");
+}
+rc_status rc_launch_moe_combine(const void*, const float*, const int*, int64_t, int64_t, int, void*, int,
+                                const LaunchCtx&) {
+  return rc_fail(RC_ERR_UNSUPPORTED_OP, "MoE combine not built");
+}

@@ -1,0 +1,123 @@
+"""C-ABI checks that need no GPU: the library loads, exports every symbol that
+include/rc.h declares, validates ops, and canonicalises schedules."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2506_01374_gb300 import rc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_functions():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if not h.endswith(".h"):
+            continue
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        for m in re.finditer(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b(rc_\w+)\s*\(", src, flags=re.M):
+            names.add(m.group(1))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    names = _declared_functions()
+    assert {"rc_op_describe", "rc_schedule_apply", "rc_candidate_measure", "rc_search_step"} <= names
+    L = ctypes.CDLL(rc.LIB_PATH)
+    missing = [n for n in sorted(names) if not hasattr(L, n)]
+    assert not missing, missing
+
+
+def test_op_validation_errors():
+    with pytest.raises(rc.RcError) as e:
+        rc.Op(rc.OP_GEMM_F32, m=0, n=4, k=4)
+    assert e.value.status == rc.ERR_INVALID_ARG
+    with pytest.raises(rc.RcError) as e:
+        rc.Op(rc.OP_ATTENTION, batch=1, seq=16, heads_q=4, heads_kv=2, head_dim=64)
+    assert e.value.status == rc.ERR_UNSUPPORTED_OP
+    with pytest.raises(rc.RcError) as e:
+        rc.Op(rc.OP_ATTENTION, batch=1, seq=16, heads_q=3, heads_kv=2, head_dim=128)
+    assert e.value.status == rc.ERR_INVALID_ARG
+    with pytest.raises(rc.RcError) as e:
+        rc.Op(99)
+    assert e.value.status == rc.ERR_UNSUPPORTED_OP
+
+
+def test_algorithmic_work_of_the_workloads():
+    # Flop counts of the five workloads (2 flops per multiply-add).
+    assert rc.Op(rc.OP_GEMM_F32, m=256, n=256, k=256).info["flops"] == 2 * 256 ** 3
+    mlp = rc.Op(rc.OP_MLP, m=2048, n=14336, k=4096).info
+    assert mlp["flops"] == 6 * 2048 * 14336 * 4096 and mlp["bound"] == "tensor"
+    att = rc.Op(rc.OP_ATTENTION, batch=1, seq=2048, heads_q=32, heads_kv=8, head_dim=128, causal=1).info
+    assert att["flops"] == 4 * 128 * 32 * 2048 * 2049 // 2
+    conv = rc.Op(rc.OP_CONV2D, img_n=2, img_h=64, img_w=64, c_in=320, c_out=320, kr=3, ks=3, stride=1, pad=1,
+                 flags=rc.EPI_BIAS | rc.EPI_SILU).info
+    assert conv["flops"] == 2 * 8192 * 320 * 2880
+    moe = rc.Op(rc.OP_MOE, tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8).info
+    assert moe["flops"] == 6 * 4096 * 8 * 7168 * 2048
+
+
+def test_schedule_canonical_form_last_writer_wins():
+    op = rc.Op(rc.OP_GEMM_F32, m=256, n=256, k=256, flags=rc.EPI_BIAS | rc.EPI_RELU)
+    a = op.schedule(rc.T(rc.T_TILE_SIZE, 32, axis=0), rc.T(rc.T_TILE_SIZE, 64, axis=0), rc.T(rc.T_UNROLL, 4))
+    b = op.schedule(rc.T(rc.T_UNROLL, 4), rc.T(rc.T_TILE_SIZE, 64, axis=0))
+    assert a.hash == b.hash and str(a) == str(b)
+    assert a.knobs()["tile_m"] == 64 and a.knobs()["unroll"] == 4
+    c = op.schedule(rc.T(rc.T_TILE_SIZE, 32, axis=1), base=a)
+    assert c.knobs()["tile_n"] == 32 and c.knobs()["tile_m"] == 64 and c.hash != a.hash
+    p0 = op.schedule()
+    assert (p0.knobs()["tile_m"], p0.knobs()["tile_n"], p0.knobs()["tile_k"], p0.knobs()["unroll"]) == (16, 16, 16, 1)
+
+
+def test_gemm_f32_space_is_the_54_point_grid():
+    op = rc.Op(rc.OP_GEMM_F32, m=256, n=256, k=256)
+    space = op.transform_space()
+    got = [(t.kind, t.axis, t.value[0]) for t in space]
+    want = [(rc.T_TILE_SIZE, ax, v) for ax in range(3) for v in (16, 32, 64)] + [(rc.T_UNROLL, 0, 1),
+                                                                                (rc.T_UNROLL, 0, 4)]
+    assert got == want
+    hashes = set()
+    for bm in (16, 32, 64):
+        for bn in (16, 32, 64):
+            for bk in (16, 32, 64):
+                for u in (1, 4):
+                    s = op.schedule(rc.T(rc.T_TILE_SIZE, bm, axis=0), rc.T(rc.T_TILE_SIZE, bn, axis=1),
+                                    rc.T(rc.T_TILE_SIZE, bk, axis=2), rc.T(rc.T_UNROLL, u))
+                    hashes.add(s.hash)
+    assert len(hashes) == 54
+
+
+def test_illegal_schedules_are_rejected():
+    op = rc.Op(rc.OP_LINEAR, m=512, n=1024, k=1024)
+    for t in [rc.T(rc.T_TILE_SIZE, 96, axis=1), rc.T(rc.T_SPLIT_K, 3), rc.T(rc.T_UNROLL, 2),
+              rc.T(rc.T_TILE_SIZE, 64, axis=5), rc.T(rc.T_PIPELINE_STAGES, 2, stage=1)]:
+        with pytest.raises(rc.RcError) as e:
+            op.schedule(t)
+        assert e.value.status == rc.ERR_ILLEGAL_SCHEDULE
+    # 256-wide tiles with 6 stages overflow 227 KB of shared memory
+    with pytest.raises(rc.RcError) as e:
+        op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=1), rc.T(rc.T_PIPELINE_STAGES, 6))
+    assert e.value.status == rc.ERR_ILLEGAL_SCHEDULE
+    ok = op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=1), rc.T(rc.T_PIPELINE_STAGES, 4))
+    assert ok.knobs()["tile_n"] == 256
+
+
+def test_composite_op_stages_are_independent():
+    op = rc.Op(rc.OP_MLP, m=256, n=512, k=256)
+    s = op.schedule(rc.T(rc.T_TILE_SIZE, 128, axis=1, stage=0), rc.T(rc.T_TILE_SIZE, 256, axis=1, stage=1),
+                    rc.T(rc.T_SPLIT_K, 2, stage=1), rc.T(rc.T_FUSE, 1, stage=0))
+    assert s.num_stages == 2
+    assert s.knobs(0)["tile_n"] == 128 and s.knobs(0)["fuse"] == 1
+    assert s.knobs(1)["tile_n"] == 256 and s.knobs(1)["split_k"] == 2
+    with pytest.raises(rc.RcError):
+        op.schedule(rc.T(rc.T_SPLIT_K, 2, stage=0))  # split-K belongs to the down GEMM
+
+
+def test_schedule_string_round_trip_size():
+    op = rc.Op(rc.OP_MOE, tokens=64, hidden=128, experts=8, inter=64, top_k=2)
+    s = op.schedule()
+    txt = str(s)
+    assert txt.startswith("op=moe;s0:") and ";s2:" in txt
