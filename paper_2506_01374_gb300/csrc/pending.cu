@@ -2,9 +2,6 @@
 // RC_ERR_UNSUPPORTED_OP so callers see a clear error instead of a fallback.
 #include "rc_internal.h"
 
-rc_status rc_launch_tc_gemm(const rc_knobs&, const TcGemmArgs&, const LaunchCtx&) {
-  return rc_fail(RC_ERR_UNSUPPORTED_OP, "tensor-core GEMM not built");
-}
 rc_status rc_launch_attention(const rc_knobs&, const rc_op_desc&, const void*, const void*, const void*, void*,
                               float*, const LaunchCtx&) {
   return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention not built");

@@ -124,7 +124,8 @@ struct TcGemmArgs {
   int64_t b_group_rows;
   int64_t max_tiles_m;     // upper bound on m-tiles over all groups
   const float* row_scale;  // TC_EPI_SCALE_ATOMIC
-  const int* row_map;      // TC_EPI_SCALE_ATOMIC
+  const int* row_map;      // TC_EPI_SCALE_ATOMIC: A row -> slot; output row = slot / row_div
+  int row_div;
 };
 rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 // Split-K reduction: out_bf16[M][N] = sum_z part[z][M][N].

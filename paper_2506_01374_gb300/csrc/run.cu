@@ -123,7 +123,10 @@ rc_status run_linear(const rc_knobs& k, int64_t M, int64_t N, int64_t K, const v
 rc_status run_swiglu(const rc_knobs& k, int64_t M, int64_t I, int64_t K, const void* X, const void* W1, void* h,
                      void* gu, const LaunchCtx& c) {
   if (k.fuse) return rc_launch_tc_gemm(k, gemm_args(M, 2 * I, K, X, W1, h, I, TC_EPI_SWIGLU), c);
-  RC_TRY(rc_launch_tc_gemm(k, gemm_args(M, 2 * I, K, X, W1, gu, 2 * I, TC_EPI_STORE_BF16), c));
+  // unfused: the same UMMA shape (N = 2 x the output tile) writes gate|up, then a pass
+  rc_knobs kg = k;
+  kg.tile_n = 2 * k.tile_n;
+  RC_TRY(rc_launch_tc_gemm(kg, gemm_args(M, 2 * I, K, X, W1, gu, 2 * I, TC_EPI_STORE_BF16), c));
   return rc_launch_swiglu_pass(gu, M, I, h, k.vec, c);
 }
 
@@ -218,6 +221,7 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
         g2.epilogue = TC_EPI_SCALE_ATOMIC;
         g2.row_scale = w;
         g2.row_map = perm;
+        g2.row_div = (int)d.top_k;
         g2.ldd = d.hidden;
         RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
         return rc_launch_f32_to_bf16(acc, d.tokens * d.hidden, p[4], c);

@@ -1,0 +1,386 @@
+// Tensor-core GEMM family for sm_103a: D = A B^T, A[M][K] and B[N][K] bf16
+// K-major, fp32 accumulation in tensor memory (TMEM).
+//
+// One CTA computes one 128 x BN output tile (cta_group::1, UMMA M = 128):
+//   warp 0     : TMA producer. One elected thread streams 128 x 64 A tiles and
+//                BN x 64 B tiles (128-byte swizzle) into a ring of `stages`
+//                shared-memory buffers, signalling a "full" mbarrier per stage.
+//   warp 1     : allocates TMEM, and one elected thread issues 4 UMMAs
+//                (K = 16 each) per stage, releasing the stage through
+//                tcgen05.commit onto its "empty" mbarrier; a final commit
+//                signals the accumulator.
+//   warps 2..5 : epilogue. Warp w reads TMEM lanes 32*(w%4) .. +31 with
+//                tcgen05.ld (one output row per thread), applies the fused
+//                epilogue and stores 16-byte vectors.
+//
+// Schedule knobs that select variants here: the N tile (template BN), the
+// ring depth (runtime `stages`), split-K (grid z), tile raster order and
+// group (runtime), and the fused epilogue (template EPI). The A operand is a
+// plain matrix or, for convolutions, an implicit im2col view loaded with a
+// 4-D TMA box whose out-of-range coordinates are zero-filled (the padding).
+// Grouped mode (MoE) partitions A's rows into segments with their own B.
+#pragma once
+
+#include <cstring>
+
+#include "rc_internal.h"
+#include "tc_common.cuh"
+
+namespace tcg {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int kThreads = 192;
+
+struct Params {
+  int M, N, K;          // N: UMMA columns of the whole problem (2I for SwiGLU)
+  int tiles_m, tiles_n;
+  int kb_total, kb_per;
+  int raster, group;
+  void* D;
+  long long ldd;
+  const __nv_bfloat16* bias;
+  int silu;
+  int swiglu_I;         // SwiGLU: output width I (also the offset of the up rows)
+  int out_cols;         // columns of D that exist (store bound)
+  // implicit-GEMM convolution
+  int img_hw, img_w, cblocks, ks, pad;
+  // grouped rows (MoE)
+  const int* offsets;
+  int groups;
+  int b_group_rows;
+  const float* row_scale;
+  const int* row_map;
+  int row_div;
+  int* status;
+};
+
+// Linear CTA index -> (m tile, n tile) under the raster order knob.
+__device__ __forceinline__ void map_tile(const Params& p, int t, int& mt, int& nt) {
+  const int G = p.group;
+  if (p.raster == 0) {  // M fastest within bands of G n-tiles
+    const int band = t / (p.tiles_m * G), in = t - band * p.tiles_m * G;
+    const int gw = min(G, p.tiles_n - band * G);
+    mt = in / gw;
+    nt = band * G + (in - (in / gw) * gw);
+  } else {  // N fastest within bands of G m-tiles
+    const int band = t / (p.tiles_n * G), in = t - band * p.tiles_n * G;
+    const int gh = min(G, p.tiles_m - band * G);
+    nt = in / gh;
+    mt = band * G + (in - (in / gh) * gh);
+  }
+}
+
+union Pack8 {
+  uint4 u;
+  __nv_bfloat162 h2[4];
+};
+
+__device__ __forceinline__ uint4 pack8(const float* v) {
+  Pack8 p;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) p.h2[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+  return p.u;
+}
+
+template <int BN, int EPI>
+__device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r, int row_end, int nt, int split,
+                                         bool have_acc) {
+  const bool row_ok = r < row_end;
+  if constexpr (EPI == TC_EPI_SWIGLU) {
+    constexpr int HALF = BN / 2;
+    __nv_bfloat16* out = (__nv_bfloat16*)p.D + (long long)r * p.ldd;
+    const int n0 = nt * HALF;
+#pragma unroll 1
+    for (int c = 0; c < HALF; c += 16) {
+      uint32_t g[16], u[16];
+      tc::tmem_ld16(taddr + c, g);
+      tc::tmem_ld16(taddr + HALF + c, u);
+      tc::tmem_ld_wait();
+      float v[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float gv = have_acc ? __uint_as_float(g[j]) : 0.f;
+        const float uv = have_acc ? __uint_as_float(u[j]) : 0.f;
+        v[j] = tc::silu(gv) * uv;
+      }
+      const int col = n0 + c;
+      if (row_ok) {
+        if (col < p.out_cols) *reinterpret_cast<uint4*>(out + col) = pack8(v);
+        if (col + 8 < p.out_cols) *reinterpret_cast<uint4*>(out + col + 8) = pack8(v + 8);
+      }
+    }
+  } else {
+    const int n0 = nt * BN;
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 16) {
+      uint32_t a[16];
+      tc::tmem_ld16(taddr + c, a);
+      tc::tmem_ld_wait();
+      float v[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = have_acc ? __uint_as_float(a[j]) : 0.f;
+      const int col = n0 + c;
+      if (!row_ok) continue;
+      if constexpr (EPI == TC_EPI_STORE_BF16 || EPI == TC_EPI_BIAS_SILU) {
+        if constexpr (EPI == TC_EPI_BIAS_SILU) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            float x = v[j];
+            if (p.bias && col + j < p.out_cols) x += __bfloat162float(p.bias[col + j]);
+            v[j] = p.silu ? tc::silu(x) : x;
+          }
+        }
+        __nv_bfloat16* out = (__nv_bfloat16*)p.D + (long long)r * p.ldd;
+        if (col < p.out_cols) *reinterpret_cast<uint4*>(out + col) = pack8(v);
+        if (col + 8 < p.out_cols) *reinterpret_cast<uint4*>(out + col + 8) = pack8(v + 8);
+      } else if constexpr (EPI == TC_EPI_PARTIAL_F32) {
+        float* out = (float*)p.D + (long long)split * p.M * p.ldd + (long long)r * p.ldd;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (col + 4 * q < p.out_cols)
+            *reinterpret_cast<float4*>(out + col + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      } else if constexpr (EPI == TC_EPI_SCALE_ATOMIC) {
+        const int slot = p.row_map[r];
+        const float s = p.row_scale[slot];
+        float* out = (float*)p.D + (long long)(slot / p.row_div) * p.ldd;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (col + 4 * q < p.out_cols)
+            atomicAdd(reinterpret_cast<float4*>(out + col + 4 * q),
+                      make_float4(s * v[4 * q], s * v[4 * q + 1], s * v[4 * q + 2], s * v[4 * q + 3]));
+      }
+    }
+  }
+}
+
+template <int BN, int EPI, int AMODE, bool GROUPED>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const Params p,
+                const int stages) {
+  constexpr int A_BYTES = BM * BK * 2;
+  constexpr int B_BYTES = BN * BK * 2;
+  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static_assert(B_BYTES % 1024 == 0, "B tile must keep stage buffers 1024-byte aligned");
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = (uint64_t*)(smem + (size_t)stages * STAGE_BYTES);
+  uint64_t* empty = full + stages;
+  uint64_t* accum = empty + stages;
+  uint64_t* drain = accum + 1;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+
+  int mt, nt;
+  map_tile(p, blockIdx.x, mt, nt);
+  int row0, row_end, brow0 = 0;
+  if constexpr (GROUPED) {
+    int acc = 0, g = 0;
+    row0 = -1;
+    row_end = 0;
+    for (; g < p.groups; ++g) {
+      const int lo = p.offsets[g], hi = p.offsets[g + 1];
+      const int n_g = (hi - lo + BM - 1) / BM;
+      if (mt < acc + n_g) {
+        row0 = lo + (mt - acc) * BM;
+        row_end = hi;
+        break;
+      }
+      acc += n_g;
+    }
+    if (row0 < 0) return;  // more m-tiles were launched than the groups need
+    brow0 = g * p.b_group_rows;
+  } else {
+    row0 = mt * BM;
+    row_end = p.M;
+  }
+  const int split = blockIdx.z;
+  const int kb0 = split * p.kb_per;
+  const int nkb = max(0, min(p.kb_total, kb0 + p.kb_per) - kb0);
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&full[s], 1);
+      tc::mbar_init(&empty[s], 1);
+    }
+    tc::mbar_init(accum, 1);
+    tc::mbar_init(drain, 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmA);
+      tc::prefetch_tmap(&tmB);
+      int i = 0;
+      for (; i < nkb; ++i) {
+        const int s = i % stages;
+        const uint32_t ph = (uint32_t)(i / stages) & 1u;
+        if (!tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          break;
+        }
+        uint8_t* sa = smem + (size_t)s * STAGE_BYTES;
+        uint8_t* sb = sa + A_BYTES;
+        tc::mbar_expect_tx(&full[s], STAGE_BYTES);
+        const int kb = kb0 + i;
+        if constexpr (AMODE == TC_A_CONV) {
+          const int rs = kb / p.cblocks, cb = kb - rs * p.cblocks;
+          const int rr = rs / p.ks, ss = rs - rr * p.ks;
+          const int img = row0 / p.img_hw;
+          const int prow = (row0 - img * p.img_hw) / p.img_w;
+          tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
+        } else {
+          tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, row0);
+        }
+        if constexpr (EPI == TC_EPI_SWIGLU) {
+          const int nh = nt * (BN / 2);
+          tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, brow0 + nh);
+          tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], kb * BK, brow0 + p.swiglu_I + nh);
+        } else {
+          tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, brow0 + nt * BN);
+        }
+      }
+      // let the copies issued in the last `stages` iterations land before exit
+      for (int j = max(0, i - stages); j < i; ++j)
+        if (!tc::mbar_wait_drain(&full[j % stages], (uint32_t)(j / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+      bool ok = true;
+      for (int i = 0; i < nkb; ++i) {
+        const int s = i % stages;
+        const uint32_t ph = (uint32_t)(i / stages) & 1u;
+        if (!tc::mbar_wait(&full[s], ph, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_FULL);
+          ok = false;
+          break;
+        }
+        tc::tc_fence_after();
+        const uint32_t sa = tc::smem_u32(smem + (size_t)s * STAGE_BYTES);
+        const uint64_t da = tc::sw128_desc(sa), db = tc::sw128_desc(sa + A_BYTES);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k)
+          tc::umma_bf16(tmem, da + 2 * k, db + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        tc::umma_commit(&empty[s]);
+      }
+      if (ok) {
+        tc::umma_commit(accum);
+      } else {
+        tc::umma_commit(drain);  // wait for the MMAs already issued before TMEM is freed
+        if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    const int r = row0 + 32 * q + lane;
+    if (tc::mbar_wait(accum, 0, abort_flag, status)) {
+      tc::tc_fence_after();
+      epilogue<BN, EPI>(p, tmem + ((uint32_t)(32 * q) << 16), r, row_end, nt, split, nkb > 0);
+    } else if (!*abort_flag) {
+      fail(RC_DEV_TIMEOUT_ACCUM);
+    }
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------ host --
+rc_status encode_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows);
+rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uint64_t h, uint64_t n);
+
+template <typename Kern>
+rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tmB, const Params& p, int stages,
+                        int splits, size_t smem, const LaunchCtx& c) {
+  const long long tiles = (long long)p.tiles_m * p.tiles_n;
+  if (tiles <= 0 || tiles > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: %lld tiles", tiles);
+  dim3 grid((unsigned)tiles, 1, (unsigned)splits);
+  kern<<<grid, kThreads, smem, (cudaStream_t)c.stream>>>(tmA, tmB, p, stages);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
+  return RC_OK;
+}
+
+inline size_t smem_bytes(int bn, int stages) {
+  return (size_t)stages * (BM * BK * 2 + (size_t)bn * BK * 2) + 1024 + 256;
+}
+
+template <int BN, int EPI, int AMODE, bool GROUPED>
+rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
+  auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED>;
+  const size_t smem = smem_bytes(BN, k.stages);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+    if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "tc_gemm: smem attribute: %s", cudaGetErrorString(e));
+    attr_set = true;
+  }
+  CUtensorMap tmA, tmB;
+  if constexpr (AMODE == TC_A_CONV) {
+    RC_TRY(encode_conv(&tmA, a.A, a.c_in, a.img_w, a.img_h, a.img_n));
+  } else {
+    RC_TRY(encode_2d(&tmA, a.A, a.K, a.M, BM));
+  }
+  const int64_t b_rows = GROUPED ? (int64_t)a.groups * a.b_group_rows : a.N;
+  RC_TRY(encode_2d(&tmB, a.B, a.K, b_rows, EPI == TC_EPI_SWIGLU ? BN / 2 : BN));
+  Params p;
+  memset(&p, 0, sizeof p);
+  p.M = (int)a.M;
+  p.N = (int)a.N;
+  p.K = (int)a.K;
+  const int out_w = EPI == TC_EPI_SWIGLU ? (int)(a.N / 2) : (int)a.N;
+  const int tile_out = EPI == TC_EPI_SWIGLU ? BN / 2 : BN;
+  p.tiles_n = (out_w + tile_out - 1) / tile_out;
+  p.tiles_m = GROUPED ? (int)a.max_tiles_m : (int)((a.M + BM - 1) / BM);
+  p.kb_total = (int)((a.K + BK - 1) / BK);
+  const int splits = EPI == TC_EPI_PARTIAL_F32 ? k.split_k : 1;
+  p.kb_per = (p.kb_total + splits - 1) / splits;
+  p.raster = k.raster;
+  p.group = k.group > 0 ? k.group : 1;
+  p.D = a.D;
+  p.ldd = a.ldd;
+  p.bias = (const __nv_bfloat16*)a.bias;
+  p.silu = a.silu;
+  p.swiglu_I = (int)(a.N / 2);
+  p.out_cols = out_w;
+  if constexpr (AMODE == TC_A_CONV) {
+    p.img_hw = (int)(a.img_h * a.img_w);
+    p.img_w = (int)a.img_w;
+    p.cblocks = (int)(a.c_in / 64);
+    p.ks = (int)a.ks;
+    p.pad = (int)a.pad;
+  }
+  p.offsets = a.offsets;
+  p.groups = a.groups;
+  p.b_group_rows = (int)a.b_group_rows;
+  p.row_scale = a.row_scale;
+  p.row_map = a.row_map;
+  p.row_div = a.row_div > 0 ? a.row_div : 1;
+  p.status = c.status;
+  return launch_kernel(kern, tmA, tmB, p, k.stages, splits, smem, c);
+}
+
+}  // namespace tcg
