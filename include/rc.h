@@ -220,6 +220,13 @@ typedef struct {
  * allocated on first use and cached in the op (not thread safe per op). */
 rc_status rc_run(const rc_op* op, const rc_schedule* s, const rc_tensors* io, void* stream);
 
+/* rc_run with CUDA events recorded between the op's stages (MLP: gate/up,
+ * down; MOE: routing+gather, grouped gate/up, grouped down+combine; other
+ * ops: one stage). Synchronises the stream; stage_ms[i] = device time of
+ * stage i in milliseconds; *n_stages = stages written (<= cap). */
+rc_status rc_run_profiled(const rc_op* op, const rc_schedule* s, const rc_tensors* io, void* stream,
+                          double* stage_ms, size_t cap, size_t* n_stages);
+
 /* End-to-end form of rc_run: io holds HOST pointers. Inputs are copied to
  * device staging buffers owned by the op, the op runs, outputs are copied
  * back, and the stream is synchronised before returning. Host buffers

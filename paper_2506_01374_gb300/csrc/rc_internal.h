@@ -85,7 +85,13 @@ struct LaunchCtx {
   void* stream;
   int* status;
   int num_sms;
+  // optional stage markers (rc_run_profiled): event i is recorded after stage i
+  void** stage_events = nullptr;
+  int n_stage_events = 0;
+  mutable int next_event = 0;
 };
+// Record the next stage marker on the stream, if markers were requested.
+rc_status rc_mark_stage(const LaunchCtx& c);
 
 rc_status rc_launch_gemm_f32(const rc_knobs& k, int64_t M, int64_t N, int64_t K, const float* A,
                              const float* B, const float* bias, float* C, bool relu,

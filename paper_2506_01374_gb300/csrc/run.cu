@@ -147,7 +147,9 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       void* gu = s->k[0].fuse ? nullptr : ws.take(2ull * d.m * 2 * d.n);
       void* part = s->k[1].split_k > 1 ? ws.take(4ull * s->k[1].split_k * d.m * d.k) : nullptr;
       RC_TRY(run_swiglu(s->k[0], d.m, d.n, d.k, p[0], p[1], h, gu, c));
-      return run_linear(s->k[1], d.m, d.k, d.n, h, p[2], p[3], part, c);
+      RC_TRY(rc_mark_stage(c));
+      RC_TRY(run_linear(s->k[1], d.m, d.k, d.n, h, p[2], p[3], part, c));
+      return rc_mark_stage(c);
     }
     case RC_OP_CONV2D: {
       const rc_knobs& k = s->k[0];
@@ -202,6 +204,7 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       float* acc = (float*)ws.take(4ull * d.tokens * d.hidden);
       RC_TRY(rc_launch_moe_route(s->k[0], d, p[0], ids, w, offsets, perm, inv, c));
       RC_TRY(rc_launch_moe_gather(p[1], perm, slots, d.hidden, (int)d.top_k, Xp, 16, c));
+      RC_TRY(rc_mark_stage(c));
       const int64_t max_tiles = slots / 128 + d.experts;
       TcGemmArgs g1 = gemm_args(slots, 2 * d.inter, d.hidden, Xp, p[2], Hb, d.inter, TC_EPI_SWIGLU);
       g1.groups = (int)d.experts;
@@ -209,6 +212,7 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       g1.b_group_rows = 2 * d.inter;
       g1.max_tiles_m = max_tiles;
       RC_TRY(rc_launch_tc_gemm(s->k[1], g1, c));
+      RC_TRY(rc_mark_stage(c));
       TcGemmArgs g2 = gemm_args(slots, d.hidden, d.inter, Hb, p[3], Yb, d.hidden, TC_EPI_STORE_BF16);
       g2.groups = (int)d.experts;
       g2.offsets = offsets;
@@ -224,10 +228,12 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
         g2.row_div = (int)d.top_k;
         g2.ldd = d.hidden;
         RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
-        return rc_launch_f32_to_bf16(acc, d.tokens * d.hidden, p[4], c);
+        RC_TRY(rc_launch_f32_to_bf16(acc, d.tokens * d.hidden, p[4], c));
+        return rc_mark_stage(c);
       }
       RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
-      return rc_launch_moe_combine(Yb, w, inv, d.tokens, d.hidden, (int)d.top_k, p[4], 16, c);
+      RC_TRY(rc_launch_moe_combine(Yb, w, inv, d.tokens, d.hidden, (int)d.top_k, p[4], 16, c));
+      return rc_mark_stage(c);
     }
   }
   return rc_fail(RC_ERR_UNSUPPORTED_OP, "rc_run: op kind %d", d.kind);
@@ -279,6 +285,46 @@ extern "C" rc_status rc_run(const rc_op* op, const rc_schedule* s, const rc_tens
   RC_TRY(prepare(op, s, &c, stream));
   RC_TRY(check_io(op, io));
   return run_impl(op, s, io, c);
+}
+
+rc_status rc_mark_stage(const LaunchCtx& c) {
+  if (!c.stage_events || c.next_event >= c.n_stage_events) return RC_OK;
+  return cuda_err(cudaEventRecord((cudaEvent_t)c.stage_events[c.next_event++], (cudaStream_t)c.stream),
+                  "cudaEventRecord(stage)");
+}
+
+extern "C" rc_status rc_run_profiled(const rc_op* op, const rc_schedule* s, const rc_tensors* io, void* stream,
+                                     double* stage_ms, size_t cap, size_t* n_stages) {
+  if (!stage_ms || !n_stages) return rc_fail(RC_ERR_INVALID_ARG, "rc_run_profiled: NULL output");
+  LaunchCtx c;
+  RC_TRY(prepare(op, s, &c, stream));
+  RC_TRY(check_io(op, io));
+  void* ev[RC_MAX_STAGES + 1] = {};
+  for (int i = 0; i <= RC_MAX_STAGES; ++i) {
+    rc_status st = cuda_err(cudaEventCreate((cudaEvent_t*)&ev[i]), "cudaEventCreate");
+    if (st != RC_OK) {
+      for (int j = 0; j < i; ++j) cudaEventDestroy((cudaEvent_t)ev[j]);
+      return st;
+    }
+  }
+  c.stage_events = ev + 1;
+  c.n_stage_events = RC_MAX_STAGES;
+  rc_status st = cuda_err(cudaEventRecord((cudaEvent_t)ev[0], (cudaStream_t)stream), "cudaEventRecord");
+  if (st == RC_OK) st = run_impl(op, s, io, c);
+  if (st == RC_OK && c.next_event == 0) st = rc_mark_stage(c);  // single-stage ops: mark the end
+  if (st == RC_OK) st = cuda_err(cudaStreamSynchronize((cudaStream_t)stream), "cudaStreamSynchronize");
+  if (st == RC_OK) st = read_status(op);
+  size_t n = 0;
+  if (st == RC_OK) {
+    for (int i = 0; i < c.next_event && n < cap; ++i, ++n) {
+      float ms = 0.f;
+      cudaEventElapsedTime(&ms, (cudaEvent_t)ev[i], (cudaEvent_t)ev[i + 1]);
+      stage_ms[n] = ms;
+    }
+  }
+  *n_stages = n;
+  for (int i = 0; i <= RC_MAX_STAGES; ++i) cudaEventDestroy((cudaEvent_t)ev[i]);
+  return st;
 }
 
 // Synchronise the stream and report device-side failures of earlier runs.

@@ -120,6 +120,8 @@ _PROTOS = {
     "rc_transform_space": (C.c_int, [_P, C.POINTER(Transform), C.c_size_t, C.POINTER(C.c_size_t)]),
     "rc_run": (C.c_int, [_P, _P, C.POINTER(Tensors), _P]),
     "rc_run_host": (C.c_int, [_P, _P, C.POINTER(Tensors), _P]),
+    "rc_run_profiled": (C.c_int, [_P, _P, C.POINTER(Tensors), _P, C.POINTER(C.c_double), C.c_size_t,
+                                  C.POINTER(C.c_size_t)]),
     "rc_op_check": (C.c_int, [_P, _P]),
     "rc_candidate_measure": (C.c_int, [_P, C.POINTER(_P), C.c_size_t, C.POINTER(Tensors), _P,
                                        C.POINTER(MeasureOpts), C.POINTER(Measurement)]),
@@ -279,6 +281,15 @@ class Op:
     def run(self, sched: Schedule, tensors: Sequence, stream=None):
         t = _tensors(tensors)
         _check(lib().rc_run(self.h, sched.h, C.byref(t), _stream(stream)), "rc_run")
+
+    def run_profiled(self, sched: Schedule, tensors: Sequence, stream=None) -> list:
+        """Run once with events between stages; returns per-stage device ms (synchronises)."""
+        t = _tensors(tensors)
+        out = (C.c_double * MAX_STAGES)()
+        n = C.c_size_t(0)
+        _check(lib().rc_run_profiled(self.h, sched.h, C.byref(t), _stream(stream), out, MAX_STAGES, C.byref(n)),
+               "rc_run_profiled")
+        return [out[i] for i in range(n.value)]
 
     def run_host(self, sched: Schedule, arrays: Sequence, stream=None):
         t = _tensors(arrays)
