@@ -45,7 +45,11 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--samples", type=int, default=120, help="schedules the search measures")
-    ap.add_argument("--cpu-rows", type=int, default=48, help="token rows of the CPU-oracle sample")
+    ap.add_argument("--cpu-rows", type=int, default=1024,
+                    help="token rows of the CPU-oracle sample (0 = skip)")
+    ap.add_argument("--schedule", default="",
+                    help="fixed schedule instead of a search, e.g. 's0:tile_n=128,stages=4,fuse=1;s1:tile_n=256'")
+    ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
 
@@ -107,6 +111,25 @@ class Clocks:
         reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": num(rows[0][2]),
                 "reasons": reasons, "samples": len(rows)}
+
+
+def parse_schedule(op, text, rc):
+    """'s0:tile_n=128,stages=4;s1:split_k=2' -> schedule (raster=R/G sets loop order and group)."""
+    KNOB_T = {"tile_n": (rc.T_TILE_SIZE, 1), "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0),
+              "fuse": (rc.T_FUSE, 0), "raster": (rc.T_LOOP_ORDER, 0), "persistent": (rc.T_PARALLEL, 0)}
+    ts = []
+    for part in filter(None, text.split(";")):
+        stage_s, kvs = part.split(":")
+        stage = int(stage_s.strip()[1:])
+        for kv in filter(None, kvs.split(",")):
+            k, v = kv.split("=")
+            kind, axis = KNOB_T[k.strip()]
+            if k.strip() == "raster":
+                r, g = (v.split("/") + ["1"])[:2]
+                ts.append(rc.T(kind, int(r), stage=stage, group=int(g)))
+            else:
+                ts.append(rc.T(kind, int(v), axis=axis, stage=stage))
+    return op.schedule(*ts)
 
 
 def dist_setup(args):
@@ -179,17 +202,21 @@ def run_ours(args):
     # 1) schedule search, every candidate measured on the device
     search = rc.Search(op, seed=args.seed)
     res, n_meas, t_search = [], 0, 0.0
-    while n_meas < args.samples:
-        nxt = search.step(res)
-        if not nxt:
-            break
-        t0 = time.perf_counter()
-        res = op.measure(nxt, io, warmup=2, repeats=5)
-        t_search += time.perf_counter() - t0
-        n_meas += len(nxt)
-    if res:
-        search.step(res)
-    best, best_m = search.best()
+    if args.schedule:
+        best = parse_schedule(op, args.schedule, rc)
+        best_m = None
+    else:
+        while n_meas < args.samples:
+            nxt = search.step(res)
+            if not nxt:
+                break
+            t0 = time.perf_counter()
+            res = op.measure(nxt, io, warmup=2, repeats=5)
+            t_search += time.perf_counter() - t0
+            n_meas += len(nxt)
+        if res:
+            search.step(res)
+        best, best_m = search.best()
 
     # 2) timed steps of the best schedule
     flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
@@ -225,18 +252,20 @@ def run_ours(args):
     h2 = torch.from_numpy(W2.view(np.int16)).pin_memory().numpy()
     hY = torch.empty(T_TOK, HID, dtype=torch.int16).pin_memory().numpy()
     host_io = [hX, h1, h2, hY]
-    for _ in range(max(1, args.warmup)):
-        op.run_host(best, host_io)
-    e2e_t = []
-    for _ in range(args.steps):
-        t0 = time.perf_counter()
-        op.run_host(best, host_io)
-        e2e_t.append(time.perf_counter() - t0)
-    e2e_s = statistics.fmean(e2e_t)
-    if world > 1:
-        t = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = t.item()
+    e2e_s = None
+    if not args.skip_e2e:
+        for _ in range(max(1, args.warmup)):
+            op.run_host(best, host_io)
+        e2e_t = []
+        for _ in range(args.steps):
+            t0 = time.perf_counter()
+            op.run_host(best, host_io)
+            e2e_t.append(time.perf_counter() - t0)
+        e2e_s = statistics.fmean(e2e_t)
+        if world > 1:
+            t = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e2e_s = t.item()
     h2d = X.nbytes + W1.nbytes + W2.nbytes
     d2h = T_TOK * HID * 2
 
@@ -246,6 +275,7 @@ def run_ours(args):
         achieved = gate_up_flops / (ms_stage0 * 1e-3) / 1e12
         k0, k1 = best.knobs(0), best.knobs(1)
         launches_per_step = (1 if k0["fuse"] else 2) + (1 if k1["split_k"] == 1 else 2)
+        kname = "gate/up GEMM" + (" + fused SwiGLU epilogue" if k0["fuse"] else " + SwiGLU pass") + " (stage 0)"
         out = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -254,20 +284,23 @@ def run_ours(args):
                        "parallelism": "replicas" if world > 1 else "single",
                        "l2": "flushed between steps (flush outside the timed events)",
                        "schedule": str(best)},
-            "roofline": {"bound": "tensor", "kernel": "gate/up GEMM + fused SwiGLU (stage 0)",
+            "roofline": {"bound": "tensor", "kernel": kname,
                          "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
                          "frac": achieved / pk["bf16_tflops"], "peak_source": pk["source"] + " bf16 burst",
                          "traffic": None},
             "step_frac_of_peak": value / world / pk["bf16_tflops"],
             "search": {"samples": n_meas, "candidates_per_s": n_meas / t_search if t_search else None,
-                       "best_search_tflops": best_m.tflops, "stats": search.stats()},
-            "e2e": {"value": world * info["flops"] / e2e_s / 1e12, "unit": "TFLOP/s",
-                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                       "best_search_tflops": best_m.tflops if best_m else None, "stats": search.stats()},
+            "e2e": None if e2e_s is None else {"value": world * info["flops"] / e2e_s / 1e12, "unit": "TFLOP/s",
+                                               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": args.steps * launches_per_step,
             "clocks": clk,
         }
-        out["cpu_baseline"] = cpu_oracle_sample(X, W1, W2, args.cpu_rows)
-        out["cpu_baseline"].pop("seconds", None)
+        if args.cpu_rows > 0:
+            out["cpu_baseline"] = cpu_oracle_sample(X, W1, W2, args.cpu_rows)
+            out["cpu_baseline"].pop("seconds", None)
+        else:
+            out["cpu_baseline"] = None
         print(json.dumps(out))
     if world > 1:
         torch.distributed.destroy_process_group()
