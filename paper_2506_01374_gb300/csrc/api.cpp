@@ -329,10 +329,13 @@ size_t rc_workspace_bytes(const rc_op_s* op, const rc_schedule_s* s) {
       if (k && (!k[0].fuse || k[0].split_k > 1)) b += align256(2ull * rows * d.c_out);
       return b;
     }
+    case RC_OP_MOE_ROUTE:
+      return align256(4ull * d.experts);  // per-expert counts
     case RC_OP_MOE: {
       const size_t slots = (size_t)d.tokens * d.top_k;
       size_t b = 0;
       b += align256(4 * slots) * 4 + align256(4 * (d.experts + 1));  // ids, w, perm, inv_perm, offsets
+      b += align256(4ull * d.experts);                                // per-expert counts
       b += align256(2 * slots * d.hidden);                            // gathered X
       b += align256(2 * slots * d.inter);                             // H
       b += align256(2 * slots * d.hidden);                            // Y (bf16) for gather-reduce

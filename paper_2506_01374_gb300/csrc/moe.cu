@@ -1,0 +1,276 @@
+// MoE routing, gather and combine kernels.
+//
+// Routing (bit-exact ids / offsets / permutation):
+//   1) route_topk: one warp per token. The E logits are widened exactly to
+//      fp32, the softmax normaliser z = sum_e exp(l_e - max) is reduced over
+//      the warp, and k arg-max rounds pick the experts in the order
+//      (logit descending, expert id ascending) by comparing the widened
+//      logits only. Weights w_j = exp(l_j - max) / z, renormalised over the k
+//      picks when requested.
+//   2) route_count: one CTA per expert counts the tokens routed to it.
+//   3) route_permute: one CTA per expert takes the exclusive prefix of the
+//      counts as its offset and ranks its tokens in token order with a
+//      block-wide ballot scan, so slot s = t*k + j lands at
+//      perm[offset[e] + rank] - the (expert, token, j) order - with no
+//      dependence on thread timing.
+// Gather: Xp[pos] = X[perm[pos] / k], 16-byte vectors, one warp per row.
+// Combine: out[t] = sum_{j<k} w[t,j] * Y[inv_perm[t*k+j]] in fp32, in j order,
+//   rounded once to bf16.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "rc_internal.h"
+
+namespace {
+
+constexpr int kMaxE = 256;
+constexpr int kMaxPerLane = kMaxE / 32;
+constexpr int kMaxK = 16;
+
+// (value, id) order of the selection: a beats b if larger, or equal and lower id.
+__device__ __forceinline__ bool beats(float va, int ia, float vb, int ib) {
+  return va > vb || (va == vb && ia < ib);
+}
+
+template <bool FP32>
+__global__ void route_topk_kernel(const void* __restrict__ logits, int T, int E, int K, int renorm,
+                                  int* __restrict__ ids, float* __restrict__ w) {
+  const int warps = blockDim.x / 32;
+  const int t = blockIdx.x * warps + threadIdx.x / 32;
+  const int lane = threadIdx.x % 32;
+  if (t >= T) return;
+  float v[kMaxPerLane];
+  bool taken[kMaxPerLane];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kMaxPerLane; ++i) {
+    const int e = lane + 32 * i;
+    taken[i] = false;
+    if (e < E) {
+      v[i] = FP32 ? ((const float*)logits)[(size_t)t * E + e]
+                  : __bfloat162float(((const __nv_bfloat16*)logits)[(size_t)t * E + e]);
+      mx = fmaxf(mx, v[i]);
+    } else {
+      v[i] = -INFINITY;
+      taken[i] = true;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float z = 0.f;
+#pragma unroll
+  for (int i = 0; i < kMaxPerLane; ++i)
+    if (lane + 32 * i < E) z += expf(v[i] - mx);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+
+  float pk[kMaxK];
+  int ik[kMaxK];
+  float sel = 0.f;
+  for (int j = 0; j < K; ++j) {
+    // best untaken candidate of this lane
+    float bv = -INFINITY;
+    int bi = 0x7fffffff;
+#pragma unroll
+    for (int i = 0; i < kMaxPerLane; ++i) {
+      const int e = lane + 32 * i;
+      if (!taken[i] && beats(v[i], e, bv, bi)) {
+        bv = v[i];
+        bi = e;
+      }
+    }
+    // warp arg-max under the same order
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (beats(ov, oi, bv, bi)) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    if ((bi & 31) == lane) taken[bi >> 5] = true;
+    const float p = expf(bv - mx) / z;
+    pk[j] = p;
+    ik[j] = bi;
+    sel += p;
+  }
+  if (lane < K) {
+    float p = 0.f;
+    int id = 0;
+    for (int j = 0; j < K; ++j)
+      if (j == lane) {
+        p = pk[j];
+        id = ik[j];
+      }
+    ids[(size_t)t * K + lane] = id;
+    w[(size_t)t * K + lane] = renorm ? p / sel : p;
+  }
+}
+
+__device__ __forceinline__ bool routes_to(const int* __restrict__ ids, int t, int K, int e, int* jpos) {
+  for (int j = 0; j < K; ++j)
+    if (ids[(size_t)t * K + j] == e) {
+      *jpos = j;
+      return true;
+    }
+  return false;
+}
+
+__global__ void route_count_kernel(const int* __restrict__ ids, int T, int K, int* __restrict__ counts) {
+  const int e = blockIdx.x;
+  int c = 0;
+  for (int t = threadIdx.x; t < T; t += blockDim.x) {
+    int j;
+    c += routes_to(ids, t, K, e, &j) ? 1 : 0;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  __shared__ int part[32];
+  if (threadIdx.x % 32 == 0) part[threadIdx.x / 32] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int s = 0;
+    for (int i = 0; i < (int)(blockDim.x / 32); ++i) s += part[i];
+    counts[e] = s;
+  }
+}
+
+__global__ void route_permute_kernel(const int* __restrict__ ids, int T, int K, int E,
+                                     const int* __restrict__ counts, int* __restrict__ offsets,
+                                     int* __restrict__ perm, int* __restrict__ inv_perm) {
+  const int e = blockIdx.x;
+  __shared__ int base_s;
+  __shared__ int warp_tot[32];
+  if (threadIdx.x == 0) {
+    int off = 0;
+    for (int i = 0; i < e; ++i) off += counts[i];
+    base_s = off;
+    offsets[e] = off;
+    if (e == E - 1) offsets[E] = off + counts[e];
+  }
+  __syncthreads();
+  int running = base_s;
+  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32, nw = blockDim.x / 32;
+  for (int t0 = 0; t0 < T; t0 += blockDim.x) {
+    const int t = t0 + threadIdx.x;
+    int j = 0;
+    const bool in = t < T && routes_to(ids, t, K, e, &j);
+    const unsigned bal = __ballot_sync(0xffffffffu, in);
+    if (lane == 0) warp_tot[warp] = __popc(bal);
+    __syncthreads();
+    int before = 0, total = 0;
+    for (int i = 0; i < nw; ++i) {
+      const int c = warp_tot[i];
+      before += i < warp ? c : 0;
+      total += c;
+    }
+    if (in) {
+      const int pos = running + before + __popc(bal & ((1u << lane) - 1u));
+      const int slot = t * K + j;
+      perm[pos] = slot;
+      if (inv_perm) inv_perm[slot] = pos;
+    }
+    running += total;
+    __syncthreads();
+  }
+}
+
+__global__ void gather_rows_kernel(const uint4* __restrict__ X, const int* __restrict__ perm, int rows, int H16,
+                                   int K, uint4* __restrict__ Xp) {
+  const int warps = blockDim.x / 32;
+  const int lane = threadIdx.x % 32;
+  for (int r = blockIdx.x * warps + threadIdx.x / 32; r < rows; r += gridDim.x * warps) {
+    const int t = perm[r] / K;
+    const uint4* src = X + (size_t)t * H16;
+    uint4* dst = Xp + (size_t)r * H16;
+    for (int i = lane; i < H16; i += 32) dst[i] = src[i];
+  }
+}
+
+union V8 {
+  uint4 u;
+  __nv_bfloat162 h[4];
+};
+
+__global__ void combine_kernel(const uint4* __restrict__ Y, const float* __restrict__ w,
+                               const int* __restrict__ inv_perm, int T, int H8, int K, uint4* __restrict__ out) {
+  const int warps = blockDim.x / 32;
+  const int lane = threadIdx.x % 32;
+  for (int t = blockIdx.x * warps + threadIdx.x / 32; t < T; t += gridDim.x * warps) {
+    int rows[kMaxK];
+    float ws[kMaxK];
+    for (int j = 0; j < K; ++j) {
+      rows[j] = inv_perm[(size_t)t * K + j];
+      ws[j] = w[(size_t)t * K + j];
+    }
+    for (int i = lane; i < H8; i += 32) {
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      for (int j = 0; j < K; ++j) {
+        V8 y;
+        y.u = Y[(size_t)rows[j] * H8 + i];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __bfloat1622float2(y.h[q]);
+          acc[2 * q] = fmaf(ws[j], f.x, acc[2 * q]);
+          acc[2 * q + 1] = fmaf(ws[j], f.y, acc[2 * q + 1]);
+        }
+      }
+      V8 o;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) o.h[q] = __floats2bfloat162_rn(acc[2 * q], acc[2 * q + 1]);
+      out[(size_t)t * H8 + i] = o.u;
+    }
+  }
+}
+
+rc_status launched(const char* what) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "%s launch: %s", what, cudaGetErrorString(e));
+  return RC_OK;
+}
+
+}  // namespace
+
+rc_status rc_launch_moe_route(const rc_knobs& k, const rc_op_desc& d, const void* logits, int* ids, float* w,
+                              int* offsets, int* perm, int* inv_perm, int* counts, const LaunchCtx& c) {
+  const int T = (int)d.tokens, E = (int)d.experts, K = (int)d.top_k;
+  if (E > kMaxE || K > kMaxK || K > E) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: E <= 256, k <= 16");
+  if ((int64_t)T * K > 0x7fffffff) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: too many slots");
+  cudaStream_t st = (cudaStream_t)c.stream;
+  const int warps = k.tile_m > 0 ? k.tile_m : 4;
+  const int blocks = (T + warps - 1) / warps;
+  if (d.logits_fp32)
+    route_topk_kernel<true><<<blocks, 32 * warps, 0, st>>>(logits, T, E, K, d.renorm, ids, w);
+  else
+    route_topk_kernel<false><<<blocks, 32 * warps, 0, st>>>(logits, T, E, K, d.renorm, ids, w);
+  RC_TRY(launched("route_topk"));
+  route_count_kernel<<<E, 256, 0, st>>>(ids, T, K, counts);
+  RC_TRY(launched("route_count"));
+  route_permute_kernel<<<E, 256, 0, st>>>(ids, T, K, E, counts, offsets, perm, inv_perm);
+  return launched("route_permute");
+}
+
+rc_status rc_launch_moe_gather(const void* X, const int* perm, int64_t rows, int64_t H, int topk, void* Xp, int vec,
+                               const LaunchCtx& c) {
+  (void)vec;
+  if (H % 8) return rc_fail(RC_ERR_UNSUPPORTED_OP, "gather: H %% 8 != 0");
+  const int warps = 8;
+  int64_t blocks = (rows + warps - 1) / warps;
+  if (blocks > (int64_t)c.num_sms * 16) blocks = (int64_t)c.num_sms * 16;
+  gather_rows_kernel<<<(unsigned)blocks, 32 * warps, 0, (cudaStream_t)c.stream>>>(
+      (const uint4*)X, perm, (int)rows, (int)(H / 8), topk, (uint4*)Xp);
+  return launched("gather");
+}
+
+rc_status rc_launch_moe_combine(const void* Y, const float* w, const int* inv_perm, int64_t T, int64_t H, int topk,
+                                void* out, int vec, const LaunchCtx& c) {
+  (void)vec;
+  if (H % 8 || topk > kMaxK) return rc_fail(RC_ERR_UNSUPPORTED_OP, "combine: H %% 8 != 0 or k > 16");
+  const int warps = 8;
+  int64_t blocks = (T + warps - 1) / warps;
+  if (blocks > (int64_t)c.num_sms * 16) blocks = (int64_t)c.num_sms * 16;
+  combine_kernel<<<(unsigned)blocks, 32 * warps, 0, (cudaStream_t)c.stream>>>(
+      (const uint4*)Y, w, inv_perm, (int)T, (int)(H / 8), topk, (uint4*)out);
+  return launched("combine");
+}

@@ -6,14 +6,3 @@ rc_status rc_launch_attention(const rc_knobs&, const rc_op_desc&, const void*, c
                               float*, const LaunchCtx&) {
   return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention not built");
 }
-rc_status rc_launch_moe_route(const rc_knobs&, const rc_op_desc&, const void*, int*, float*, int*, int*, int*,
-                              const LaunchCtx&) {
-  return rc_fail(RC_ERR_UNSUPPORTED_OP, "MoE routing not built");
-}
-rc_status rc_launch_moe_gather(const void*, const int*, int64_t, int64_t, int, void*, int, const LaunchCtx&) {
-  return rc_fail(RC_ERR_UNSUPPORTED_OP, "MoE gather not built");
-}
-rc_status rc_launch_moe_combine(const void*, const float*, const int*, int64_t, int64_t, int, void*, int,
-                                const LaunchCtx&) {
-  return rc_fail(RC_ERR_UNSUPPORTED_OP, "MoE combine not built");
-}

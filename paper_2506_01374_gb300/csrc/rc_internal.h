@@ -149,8 +149,10 @@ rc_status rc_launch_l2_flush(void* buf, size_t bytes, void* stream);
 // Attention and MoE launchers.
 rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K,
                               const void* V, void* O, float* lse, const LaunchCtx& c);
+// Routing: counts is device scratch of E ints; inv_perm may be NULL.
 rc_status rc_launch_moe_route(const rc_knobs& k, const rc_op_desc& d, const void* logits, int* ids,
-                              float* w, int* offsets, int* perm, int* inv_perm, const LaunchCtx& c);
+                              float* w, int* offsets, int* perm, int* inv_perm, int* counts,
+                              const LaunchCtx& c);
 rc_status rc_launch_moe_gather(const void* X, const int* perm, int64_t rows, int64_t H, int topk,
                                void* Xp, int vec, const LaunchCtx& c);
 rc_status rc_launch_moe_combine(const void* Y, const float* w, const int* inv_perm, int64_t T,

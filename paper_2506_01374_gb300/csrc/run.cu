@@ -189,7 +189,9 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
     case RC_OP_ATTENTION:
       return rc_launch_attention(s->k[0], d, p[0], p[1], p[2], p[3], (float*)p[4], c);
     case RC_OP_MOE_ROUTE: {
-      return rc_launch_moe_route(s->k[0], d, p[0], (int*)p[1], (float*)p[2], (int*)p[3], (int*)p[4], nullptr, c);
+      int* counts = (int*)ws.take(4 * d.experts);
+      return rc_launch_moe_route(s->k[0], d, p[0], (int*)p[1], (float*)p[2], (int*)p[3], (int*)p[4], nullptr,
+                                 counts, c);
     }
     case RC_OP_MOE: {
       const int64_t slots = d.tokens * d.top_k;
@@ -198,11 +200,12 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       int* offsets = p[7] ? (int*)p[7] : (int*)ws.take(4 * (d.experts + 1));
       int* perm = p[8] ? (int*)p[8] : (int*)ws.take(4 * slots);
       int* inv = (int*)ws.take(4 * slots);
+      int* counts = (int*)ws.take(4 * d.experts);
       void* Xp = ws.take(2ull * slots * d.hidden);
       void* Hb = ws.take(2ull * slots * d.inter);
       void* Yb = ws.take(2ull * slots * d.hidden);
       float* acc = (float*)ws.take(4ull * d.tokens * d.hidden);
-      RC_TRY(rc_launch_moe_route(s->k[0], d, p[0], ids, w, offsets, perm, inv, c));
+      RC_TRY(rc_launch_moe_route(s->k[0], d, p[0], ids, w, offsets, perm, inv, counts, c));
       RC_TRY(rc_launch_moe_gather(p[1], perm, slots, d.hidden, (int)d.top_k, Xp, 16, c));
       RC_TRY(rc_mark_stage(c));
       const int64_t max_tiles = slots / 128 + d.experts;

@@ -26,7 +26,10 @@ layer (router logits N(0, 1), activations N(0, 1), weights N(0, 0.02)).
 from __future__ import annotations
 
 import concurrent.futures as _cf
+import ctypes
 import os
+import subprocess
+import threading
 
 import numpy as np
 
@@ -87,13 +90,7 @@ def uniform(k: int, n: int, lo: float = 0.0, hi: float = 1.0) -> np.ndarray:
 def normal(k: int, n: int, mean: float = 0.0, std: float = 1.0) -> np.ndarray:
     """n doubles ~ N(mean, std^2) from stream k (element i uses draws 2i, 2i+1)."""
 
-    def fn(s, m):
-        d = _draws(k, 2 * s, 2 * m)
-        u1 = _unit(d[0::2])
-        u2 = _unit(d[1::2])
-        return mean + std * np.sqrt(-2.0 * np.log1p(-u1)) * np.cos(2.0 * np.pi * u2)
-
-    return _parallel(n, fn)
+    return _parallel(n, lambda s, m: _normal_chunk(k, s, m, mean, std))
 
 
 def to_bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -114,9 +111,54 @@ def bf16_bits_to_f64(b: np.ndarray) -> np.ndarray:
     return u.view(np.float32).astype(np.float64)
 
 
+def _normal_chunk(k: int, s: int, m: int, mean: float, std: float) -> np.ndarray:
+    d = _draws(k, 2 * s, 2 * m)
+    u1 = _unit(d[0::2])
+    u2 = _unit(d[1::2])
+    return mean + std * np.sqrt(-2.0 * np.log1p(-u1)) * np.cos(2.0 * np.pi * u2)
+
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SYNTH_SRC = os.path.join(_HERE, "synth.c")
+_SYNTH_LIB = os.path.join(_HERE, "libsynth.so")
+_synth = None
+_synth_lock = threading.Lock()
+
+
+def build_synth(force: bool = False) -> str:
+    """Compile synth.c (the generator's C fast path) into libsynth.so."""
+    if not force and os.path.exists(_SYNTH_LIB) and os.path.getmtime(_SYNTH_LIB) >= os.path.getmtime(_SYNTH_SRC):
+        return _SYNTH_LIB
+    tmp = _SYNTH_LIB + f".tmp{os.getpid()}"
+    base = ["gcc", "-O2", "-std=c11", "-shared", "-fPIC", _SYNTH_SRC, "-o", tmp, "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True, capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    os.replace(tmp, _SYNTH_LIB)
+    return _SYNTH_LIB
+
+
+def _synth_lib():
+    global _synth
+    with _synth_lock:
+        if _synth is None:
+            L = ctypes.CDLL(build_synth())
+            L.synth_bf16_normal.restype = None
+            L.synth_bf16_normal.argtypes = [ctypes.c_uint64, ctypes.c_int64, ctypes.c_int64, ctypes.c_double,
+                                            ctypes.c_double, ctypes.c_void_p]
+            _synth = L
+    return _synth
+
+
 def _bf16_normal(seed, tid, shape, std):
+    """N(0, std^2) bf16 bits of stream (seed, tid), drawn by the C fast path
+    (the same definition as to_bf16_bits(normal(...)), without a float64 copy)."""
     n = int(np.prod(shape))
-    return to_bf16_bits(normal(key(seed, tid), n, 0.0, std)).reshape(shape)
+    out = np.empty(n, dtype=np.uint16)
+    if n:
+        _synth_lib().synth_bf16_normal(key(seed, tid), 0, n, 0.0, float(std), out.ctypes.data)
+    return out.reshape(shape)
 
 
 # ---------------------------------------------------------------- workloads --

@@ -1,0 +1,125 @@
+"""MoE routing (bit-exact) and the routed SwiGLU FFN layer on the GPU against
+the fp64 oracle. Routing ids, offsets and the permutation must be identical;
+weights agree to fp32 rounding; layer outputs to 2e-2 normwise (bf16)."""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2506_01374_gb300 import inputs, rc
+
+from .gpu_util import empty_bf16, from_dev_bf16, rel_err, to_dev, torch
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+
+
+def run_route(logits, E, K, tile_m=4, renorm=True):
+    T = logits.shape[0]
+    fp32 = logits.dtype == np.float32
+    op = rc.Op(rc.OP_MOE_ROUTE, tokens=T, experts=E, top_k=K, logits_fp32=int(fp32), renorm=int(renorm))
+    ids = torch.empty(T, K, dtype=torch.int32, device="cuda")
+    w = torch.empty(T, K, dtype=torch.float32, device="cuda")
+    off = torch.empty(E + 1, dtype=torch.int32, device="cuda")
+    perm = torch.empty(T * K, dtype=torch.int32, device="cuda")
+    op.run(op.schedule(rc.T(rc.T_TILE_SIZE, tile_m, axis=0)), [to_dev(logits), ids, w, off, perm])
+    op.check()
+    return ids.cpu().numpy(), w.cpu().numpy(), off.cpu().numpy(), perm.cpu().numpy()
+
+
+@pytest.mark.parametrize("T,E,K,fp32", [(4096, 64, 8, False), (1000, 16, 4, False), (333, 256, 16, False),
+                                        (517, 33, 3, True), (64, 16, 16, False), (1, 8, 1, False)])
+def test_routing_bit_exact(T, E, K, fp32):
+    logits, _, _, _ = inputs.moe(T, 8, E, 8, seed=41, logits_fp32=fp32)
+    r_ids, r_w, r_off, r_perm = oracle.moe_route(logits, K)
+    for tm in (4, 8, 16):
+        ids, w, off, perm = run_route(logits, E, K, tm)
+        np.testing.assert_array_equal(ids, r_ids)
+        np.testing.assert_array_equal(off, r_off)
+        np.testing.assert_array_equal(perm, r_perm)
+        np.testing.assert_allclose(w, r_w, rtol=2e-6, atol=1e-7)
+    _, w_raw, _, _ = run_route(logits, E, K, renorm=False)
+    np.testing.assert_allclose(w_raw, oracle.moe_route(logits, K, renorm=False)[1], rtol=2e-6, atol=1e-7)
+
+
+def test_routing_ties_and_imbalance():
+    T, E, K = 300, 64, 8
+    L = np.zeros((T, E))
+    L[100:, :] = np.random.default_rng(0).standard_normal((T - 100, E)).round(1)  # coarse values: many ties
+    L[200:, :8] += 5.0  # 100 tokens all pick experts 0..7
+    logits = inputs.to_bf16_bits(L)
+    r = oracle.moe_route(logits, K)
+    g = run_route(logits, E, K)
+    for a, b in zip(g[:1] + g[2:], r[:1] + r[2:]):
+        np.testing.assert_array_equal(a, b)
+    assert list(g[0][0]) == list(range(8))  # all-equal row: lowest ids first
+
+
+def moe_op(T, H, E, I, K):
+    return rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
+
+
+def moe_sched(op, tm, tn1, st1, tn2, st2, fuse):
+    return op.schedule(rc.T(rc.T_TILE_SIZE, tm, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
+                       rc.T(rc.T_PIPELINE_STAGES, st1, stage=1), rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2),
+                       rc.T(rc.T_PIPELINE_STAGES, st2, stage=2), rc.T(rc.T_FUSE, fuse, stage=2))
+
+
+def test_moe_layer_schedule_sweep():
+    T, H, E, I, K = 200, 128, 8, 64, 2
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=42)
+    ids, w, off, perm = oracle.moe_route(logits, K)
+    ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
+    op = moe_op(T, H, E, I, K)
+    dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
+    for tn1, tn2, fuse, st in itertools.product((32, 64, 128), (64, 128, 256), (0, 1), (1, 3)):
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
+        gp = torch.empty(T * K, dtype=torch.int32, device="cuda")
+        op.run(moe_sched(op, 8, tn1, st, tn2, st, fuse), [dl, dX, d1, d2, out, gi, None, None, gp])
+        op.check()
+        np.testing.assert_array_equal(gi.cpu().numpy(), ids)
+        np.testing.assert_array_equal(gp.cpu().numpy(), perm)
+        err = rel_err(from_dev_bf16(out), ref)
+        assert err <= TOL, (tn1, tn2, fuse, st, err)
+
+
+def test_moe_layer_imbalanced_and_empty_experts():
+    T, H, E, I, K = 300, 128, 16, 128, 4
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=43)
+    L = inputs.bf16_bits_to_f64(logits)
+    L[:, :4] += 8.0  # every token routes to experts 0..3: 300 rows each, 12 experts empty
+    logits = inputs.to_bf16_bits(L)
+    ids, w, off, _ = oracle.moe_route(logits, K)
+    assert (np.diff(off)[4:] == 0).all() and (np.diff(off)[:4] == T).all()
+    ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
+    op = moe_op(T, H, E, I, K)
+    for fuse in (0, 1):
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.check()
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, fuse
+
+
+def test_moe_full_size_sampled_tokens():
+    # T=4096 tokens, H=7168, 64 experts with I=2048, top-8 softmax routing.
+    T, H, E, I, K = 4096, 7168, 64, 2048, 8
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=6)
+    ids, w, off, perm = oracle.moe_route(logits, K)
+    tok = np.array([0, 1, 2047, 4095], dtype=np.int64)
+    ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w, tok=tok)
+    op = moe_op(T, H, E, I, K)
+    dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
+    del W1, W2
+    for s in [op.schedule(), moe_sched(op, 8, 128, 2, 256, 2, 0), moe_sched(op, 16, 64, 4, 128, 3, 1)]:
+        out = empty_bf16(T, H)
+        gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
+        go = torch.empty(E + 1, dtype=torch.int32, device="cuda")
+        gp = torch.empty(T * K, dtype=torch.int32, device="cuda")
+        op.run(s, [dl, dX, d1, d2, out, gi, None, go, gp])
+        op.check()
+        np.testing.assert_array_equal(gi.cpu().numpy(), ids)
+        np.testing.assert_array_equal(go.cpu().numpy(), off)
+        np.testing.assert_array_equal(gp.cpu().numpy(), perm)
+        assert rel_err(from_dev_bf16(out)[tok], ref) <= TOL, str(s)

@@ -31,6 +31,12 @@ def test_splitmix64_published_sequence():
     assert [int(x) for x in d] == [0xE220A8397B1DCDAF, 0x6E789E6AA1B965F4, 0x06C45D188009454F]
 
 
+def test_bf16_fast_path_matches_numpy_definition():
+    a = inputs._bf16_normal(3, 2, (300, 700), 0.02)
+    b = inputs.to_bf16_bits(inputs.normal(inputs.key(3, 2), 300 * 700, 0.0, 0.02)).reshape(300, 700)
+    np.testing.assert_array_equal(a, b)
+
+
 def test_bf16_rne():
     x = np.array([1.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -2.5, 0.0])
     # 1 + 2^-8 is a tie between 1 and 1 + 2^-7: even mantissa wins (1.0)
