@@ -307,6 +307,41 @@ rc_status rc_search_node(const rc_search* s, int64_t i, int64_t* parent, double*
                          uint64_t* sched_hash);
 void rc_search_destroy(rc_search* s);
 
+/* ------------------------------------------------- no-allocation routing -- */
+
+/* The paper has no counterpart to this entry point; it exists for callers
+ * that cannot allocate device memory. Examples: a process whose GPU memory
+ * has been reserved by another allocator (a framework's caching pool), or a
+ * latency-critical path where cudaMalloc is off limits because it can
+ * synchronise the device and has no time bound.
+ *
+ * It computes exactly what rc_run does for an RC_OP_MOE_ROUTE op with
+ * renorm/logits_fp32 as given (same kernels, same bit-exact ids, offsets and
+ * permutation), but allocates nothing: the per-expert counts it needs live
+ * in a fixed device array of RC_NOALLOC_MAX_EXPERTS ints inside the library,
+ * which every GPU that loads the library keeps until the process exits.
+ *
+ *   logits  : device bf16 (logits_fp32 = 0) or f32 [tokens][experts]
+ *   ids     : device i32 [tokens][top_k]      (output)
+ *   weights : device f32 [tokens][top_k]      (output)
+ *   offsets : device i32 [experts + 1]        (output)
+ *   perm    : device i32 [tokens * top_k]     (output, slot s = t*top_k + j)
+ * All tensors are caller-owned and 16-byte aligned. experts above
+ * RC_NOALLOC_MAX_EXPERTS gives RC_ERR_INVALID_ARG; top_k above 16 gives
+ * RC_ERR_UNSUPPORTED_OP. Kernels are queued on `stream` (no synchronisation).
+ *
+ * The first call on each device looks up the array's device address with
+ * that device current (cudaGetSymbolAddress); make that first call before
+ * any stream capture. Every call on a device shares the one array, so calls
+ * whose kernels overlap on the GPU (different streams, no ordering) race;
+ * order them on one stream or with events. The array keeps the last call's
+ * counts; each call overwrites the entries it uses, so nothing needs
+ * clearing. */
+#define RC_NOALLOC_MAX_EXPERTS 256
+rc_status rc_moe_route_noalloc(const void* logits, int32_t logits_fp32, int64_t tokens, int64_t experts,
+                               int64_t top_k, int32_t renorm, int32_t* ids, float* weights, int32_t* offsets,
+                               int32_t* perm, void* stream);
+
 /* Thread-local message of the last failing call on this thread. */
 const char* rc_last_error(void);
 /* Library version string. */

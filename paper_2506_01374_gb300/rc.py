@@ -133,6 +133,8 @@ _PROTOS = {
     "rc_search_node": (C.c_int, [_P, C.c_int64, C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                  C.POINTER(C.c_int64), C.POINTER(C.c_uint64)]),
     "rc_search_destroy": (None, [_P]),
+    "rc_moe_route_noalloc": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int64, C.c_int64, C.c_int32, _P, _P, _P, _P,
+                                       _P]),
     "rc_last_error": (C.c_char_p, []),
     "rc_version": (C.c_char_p, []),
 }
@@ -354,6 +356,14 @@ class Search:
         p, q, n, h = C.c_int64(), C.c_double(), C.c_int64(), C.c_uint64()
         _check(lib().rc_search_node(self.h, i, C.byref(p), C.byref(q), C.byref(n), C.byref(h)))
         return {"parent": p.value, "Q": q.value, "N": n.value, "hash": h.value}
+
+
+def moe_route_noalloc(logits, tokens: int, experts: int, top_k: int, ids, weights, offsets, perm,
+                      renorm: bool = True, logits_fp32: bool = False, stream=None):
+    """rc_moe_route_noalloc: routing without any device allocation (fixed library scratch)."""
+    _check(lib().rc_moe_route_noalloc(_ptr(logits), int(logits_fp32), tokens, experts, top_k, int(renorm), _ptr(ids),
+                                      _ptr(weights), _ptr(offsets), _ptr(perm), _stream(stream)),
+           "rc_moe_route_noalloc")
 
 
 def version() -> str:
