@@ -120,6 +120,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});
       v.push_back({RC_T_PIPELINE_STAGES, 0, {2, 3}, {}});
       v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1}});
+      v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // V as [keys][d] or transposed to [d][keys]
       break;
     case RC_OP_MOE_ROUTE:
       v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
@@ -166,6 +167,7 @@ rc_knobs rc_default_knobs(const rc_op_s* op, int stage) {
     case RC_OP_ATTENTION:
       k.tile_n = 64;
       k.stages = 2;
+      k.layout = 1;
       break;
     case RC_OP_MOE_ROUTE: k.tile_m = 4; break;
     case RC_OP_MOE:
@@ -229,6 +231,20 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
     case RC_OP_MOE:
       if (stage == 0) return true;
       return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, why);
+    case RC_OP_ATTENTION: {
+      // Q tile + ring of K and V tiles + P tile + slack, all bf16
+      const int64_t smem = 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 + 128 * (int64_t)k.tile_n * 2 +
+                           1024 + 256;
+      if (smem > kSmemLimit) {
+        if (why) *why = "attention ring exceeds 227 KB of shared memory";
+        return false;
+      }
+      if (k.layout == 1 && o.seq % 8) {
+        if (why) *why = "transposed V needs seq % 8 == 0 (16-byte TMA rows)";
+        return false;
+      }
+      return true;
+    }
     default:
       return true;
   }
@@ -329,6 +345,8 @@ size_t rc_workspace_bytes(const rc_op_s* op, const rc_schedule_s* s) {
       if (k && (!k[0].fuse || k[0].split_k > 1)) b += align256(2ull * rows * d.c_out);
       return b;
     }
+    case RC_OP_ATTENTION:
+      return (k && k[0].layout == 1) ? align256(2ull * d.batch * d.heads_kv * d.head_dim * d.seq) : 0;
     case RC_OP_MOE_ROUTE:
       return align256(4ull * d.experts);  // per-expert counts
     case RC_OP_MOE: {

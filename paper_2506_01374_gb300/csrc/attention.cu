@@ -1,0 +1,423 @@
+// Fused attention core O = softmax(scale * Q K^T + mask) V with grouped-query
+// heads, on the sm_103a tensor cores (tcgen05, TMEM accumulators, TMA).
+//
+// One CTA owns one (batch, query head h, block of 128 queries); the KV head is
+// g = h / (Hq / Hkv). Per key block j of BN keys:
+//   warp 0     : TMA producer - Q once, then K_j (2 x [BN][64] swizzled
+//                halves of the head dimension) and V_j into a ring of stages.
+//   warp 1     : one thread issues S = Q K_j^T into TMEM columns [0, BN)
+//                (8 UMMAs of K = 16 over the 128-wide head dimension), then,
+//                once P_j is in shared memory, O += P_j V_j into TMEM columns
+//                [BN, BN + 128).
+//   warps 2..5 : softmax, one query row per thread (TMEM lane = row). Pass 1
+//                reads S and takes the masked row maximum; the running maximum
+//                m and sum l follow the online softmax in the log2 domain
+//                (p = 2^(s * scale * log2 e - m)); O is rescaled in TMEM by
+//                2^(m_old - m_new) when the maximum moved; pass 2 writes P as
+//                bf16 in the 128-byte-swizzled K-major layout the UMMA reads.
+// The epilogue divides O by l, stores bf16 O and LSE = ln 2 * (m + log2 l).
+//
+// Schedule knobs: BN (template), ring depth (runtime), query-block order
+// (natural or longest-first for the causal triangle), and the layout of V:
+// as given ([keys][d], an MN-major UMMA B operand) or pre-transposed by a pass
+// into [d][keys] (K-major). Masking: key j is visible to query i when j < S and
+// (not causal or j <= i). Every wait is bounded as in the GEMM kernels.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstring>
+
+#include "rc_internal.h"
+#include "tc_common.cuh"
+
+namespace tcg {
+rc_status encode_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows);
+}
+
+namespace attn {
+
+constexpr int BM = 128;
+constexpr int D = 128;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 256;
+
+struct Params {
+  int B, S, Hq, Hkv, group;
+  int q_blocks;
+  int causal;
+  float scale_log2;  // softmax scale * log2(e)
+  int raster;
+  __nv_bfloat16* O;
+  float* lse;
+  int* status;
+};
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+template <int BN, bool VT>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  static_assert(BN == 64 || BN == 128, "key block");
+  constexpr int Q_BYTES = BM * D * 2;   // two [128][64] halves
+  constexpr int KV_TILE = BN * D * 2;   // one K or V tile
+  constexpr int P_BYTES = BM * BN * 2;  // BN/64 atoms of [128][64]
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;
+  uint8_t* ring = smem + Q_BYTES;
+  uint8_t* sP = ring + (size_t)stages * 2 * KV_TILE;
+  uint64_t* q_full = (uint64_t*)(sP + P_BYTES);
+  uint64_t* kv_full = q_full + 1;
+  uint64_t* kv_empty = kv_full + stages;
+  uint64_t* s_full = kv_empty + stages;
+  uint64_t* s_free = s_full + 1;
+  uint64_t* p_full = s_free + 1;
+  uint64_t* pv_full = p_full + 1;
+  uint64_t* drain = pv_full + 1;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int BH = p.B * p.Hq;
+  int qb, bh;
+  if (p.raster == 0) {
+    qb = blockIdx.x % p.q_blocks;
+    bh = blockIdx.x / p.q_blocks;
+  } else {  // longest causal rows first
+    qb = p.q_blocks - 1 - (int)(blockIdx.x / BH);
+    bh = blockIdx.x % BH;
+  }
+  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
+  const int q0 = qb * BM;
+  const int kv_end = p.causal ? min(q0 + BM, p.S) : p.S;
+  const int nkb = (kv_end + BN - 1) / BN;
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&kv_full[s], 1);
+      tc::mbar_init(&kv_empty[s], 1);
+    }
+    tc::mbar_init(s_full, 1);
+    tc::mbar_init(s_free, 128);
+    tc::mbar_init(p_full, 128);
+    tc::mbar_init(pv_full, 1);
+    tc::mbar_init(drain, 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(tmem_slot, kTmemCols);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::prefetch_tmap(&tmV);
+      tc::mbar_expect_tx(q_full, Q_BYTES);
+      const int qrow = b * p.S + q0;
+      tc::tma_load_2d(sQ, &tmQ, q_full, h * D, qrow);
+      tc::tma_load_2d(sQ + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
+      int j = 0;
+      for (; j < nkb; ++j) {
+        const int s = j % stages;
+        const uint32_t ph = (uint32_t)(j / stages) & 1u;
+        if (!tc::mbar_wait(&kv_empty[s], ph ^ 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          break;
+        }
+        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
+        uint8_t* sv = sk + KV_TILE;
+        tc::mbar_expect_tx(&kv_full[s], 2 * KV_TILE);
+        const int krow = b * p.S + j * BN;
+        tc::tma_load_2d(sk, &tmK, &kv_full[s], g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, &kv_full[s], g * D + 64, krow);
+        if constexpr (VT) {
+#pragma unroll
+          for (int a = 0; a < BN / 64; ++a)
+            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &kv_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
+        } else {
+          tc::tma_load_2d(sv, &tmV, &kv_full[s], g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, &kv_full[s], g * D + 64, krow);
+        }
+      }
+      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      for (int i = max(0, j - stages); i < j; ++i)
+        if (!tc::mbar_wait_drain(&kv_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+      const uint32_t tS = tmem, tO = tmem + BN;
+      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
+      if (!ok) fail(RC_DEV_TIMEOUT_FULL);
+      const uint32_t sq = tc::smem_u32(sQ);
+      for (int j = 0; ok && j < nkb; ++j) {
+        const int s = j % stages;
+        const uint32_t ph = (uint32_t)(j / stages) & 1u;
+        if (!tc::mbar_wait(&kv_full[s], ph, abort_flag, status) ||
+            (j > 0 && !tc::mbar_wait(s_free, (uint32_t)(j - 1) & 1u, abort_flag, status))) {
+          fail(RC_DEV_TIMEOUT_FULL);
+          ok = false;
+          break;
+        }
+        tc::tc_fence_after();
+        const uint32_t sk = tc::smem_u32(ring + (size_t)s * 2 * KV_TILE);
+        const uint32_t sv = sk + KV_TILE;
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
+                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(s_full);
+        if (!tc::mbar_wait(p_full, (uint32_t)j & 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_FULL);
+          ok = false;
+          break;
+        }
+        tc::tc_fence_after();
+        const uint32_t sp = tc::smem_u32(sP);
+#pragma unroll
+        for (int ks = 0; ks < BN / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          const uint64_t da = tc::sw128_desc(sp + (ks / 4) * (BM * 128) + off);
+          uint64_t db;
+          if constexpr (VT)
+            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
+          else
+            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
+          tc::umma_bf16(tO, da, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        tc::umma_commit(pv_full);
+        tc::umma_commit(&kv_empty[s]);
+      }
+      if (!ok) {
+        tc::umma_commit(drain);
+        if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int q = warp & 3;
+    const int row = 32 * q + lane;
+    const int qi = q0 + row;
+    const uint32_t lane_base = (uint32_t)(32 * q) << 16;
+    const uint32_t tS = tmem + lane_base, tO = tmem + lane_base + BN;
+    float m = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkb; ++j) {
+      if (!tc::mbar_wait(s_full, (uint32_t)j & 1u, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        ok = false;
+        break;
+      }
+      tc::tc_fence_after();
+      const int k0 = j * BN;
+      // pass 1: masked row maximum
+      float mx = -INFINITY;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t r[16];
+        tc::tmem_ld16(tS + c, r);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int key = k0 + c + i;
+          const bool vis = key < p.S && (!p.causal || key <= qi);
+          mx = fmaxf(mx, vis ? __uint_as_float(r[i]) : -INFINITY);
+        }
+      }
+      const float m_new = fmaxf(m, mx * p.scale_log2);
+      const float alpha = (m == -INFINITY) ? 0.f : exp2f(m - m_new);
+      const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+      if (j > 0) {
+        // O holds P_{j-1} V_{j-1}; P's buffer is free again; rescale O
+        if (!tc::mbar_wait(pv_full, (uint32_t)(j - 1) & 1u, abort_flag, status)) {
+          if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+          ok = false;
+          break;
+        }
+        tc::tc_fence_after();
+        if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll 1
+          for (int c = 0; c < D; c += 16) {
+            uint32_t r[16];
+            tc::tmem_ld16(tO + c, r);
+            tc::tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+            tc::tmem_st16(tO + c, r);
+          }
+          tc::tmem_st_wait();
+        }
+      }
+      // pass 2: probabilities -> P (bf16, swizzled K-major rows), row sum
+      float lsum = 0.f;
+      uint8_t* rowp0 = sP + (row / 8) * 1024 + (row % 8) * 128;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 16) {
+        uint32_t r[16];
+        tc::tmem_ld16(tS + c, r);
+        tc::tmem_ld_wait();
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 16; i += 2) {
+          const int key = k0 + c + i;
+          const bool v0 = key < p.S && (!p.causal || key <= qi);
+          const bool v1 = key + 1 < p.S && (!p.causal || key + 1 <= qi);
+          const float p0 = v0 ? exp2f(__uint_as_float(r[i]) * p.scale_log2 - m_use) : 0.f;
+          const float p1 = v1 ? exp2f(__uint_as_float(r[i + 1]) * p.scale_log2 - m_use) : 0.f;
+          lsum += p0 + p1;
+          pk[i / 2] = pack2(p0, p1);
+        }
+        uint8_t* rowp = rowp0 + (c / 64) * (BM * 128);
+        const int ch = (c % 64) / 8;
+        *reinterpret_cast<uint4*>(rowp + ((ch ^ (row % 8)) * 16)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        *reinterpret_cast<uint4*>(rowp + (((ch + 1) ^ (row % 8)) * 16)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      }
+      l = l * alpha + lsum;
+      m = m_new;
+      tc::tc_fence_before();
+      tc::fence_proxy_async_smem();
+      tc::mbar_arrive(s_free);
+      tc::mbar_arrive(p_full);
+    }
+    if (ok) {
+      if (tc::mbar_wait(pv_full, (uint32_t)(nkb - 1) & 1u, abort_flag, status)) {
+        tc::tc_fence_after();
+        const float inv_l = l > 0.f ? 1.f / l : 0.f;
+        __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + qi) * p.Hq + h) * D;
+        const bool row_ok = qi < p.S;
+#pragma unroll 1
+        for (int c = 0; c < D; c += 16) {
+          uint32_t r[16];
+          tc::tmem_ld16(tO + c, r);
+          tc::tmem_ld_wait();
+          uint32_t pk[8];
+#pragma unroll
+          for (int i = 0; i < 16; i += 2)
+            pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
+          if (row_ok) {
+            *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
+        }
+        if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m + log2f(l));
+      } else if (!*abort_flag) {
+        fail(RC_DEV_TIMEOUT_ACCUM);
+      }
+    }
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// Vt[(b*Hkv + g)*D + d][s] = V[b][s][g][d] (64 x 64 tiles through shared memory).
+__global__ void transpose_v_kernel(const __nv_bfloat16* __restrict__ V, int S, int Hkv, __nv_bfloat16* __restrict__ Vt) {
+  __shared__ __nv_bfloat16 tile[64][66];
+  const int bg = blockIdx.z;  // b * Hkv + g
+  const int b = bg / Hkv, g = bg - b * Hkv;
+  const int s0 = blockIdx.x * 64, d0 = blockIdx.y * 64;
+  for (int i = threadIdx.y; i < 64; i += blockDim.y) {
+    const int s = s0 + i;
+    for (int k = threadIdx.x; k < 64; k += blockDim.x)
+      tile[i][k] = s < S ? V[(((size_t)b * S + s) * Hkv + g) * D + d0 + k] : __float2bfloat16_rn(0.f);
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 64; i += blockDim.y) {
+    const int d = d0 + i;
+    for (int k = threadIdx.x; k < 64; k += blockDim.x) {
+      const int s = s0 + k;
+      if (s < S) Vt[((size_t)bg * D + d) * S + s] = tile[k][i];
+    }
+  }
+}
+
+size_t smem_bytes(int bn, int stages) {
+  return (size_t)BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)BM * bn * 2 + 1024 + 256;
+}
+
+template <int BN, bool VT>
+rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
+                 float* lse, const LaunchCtx& c) {
+  auto kern = attn_kernel<BN, VT>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+    if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention: smem attribute: %s", cudaGetErrorString(e));
+    attr = true;
+  }
+  const uint64_t BS = (uint64_t)d.batch * d.seq;
+  CUtensorMap tq, tk, tv;
+  RC_TRY(tcg::encode_2d(&tq, Q, (uint64_t)d.heads_q * D, BS, BM));
+  RC_TRY(tcg::encode_2d(&tk, K, (uint64_t)d.heads_kv * D, BS, BN));
+  if (VT)
+    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.seq, (uint64_t)d.batch * d.heads_kv * D, BM));
+  else
+    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.heads_kv * D, BS, BN));
+  Params p;
+  memset(&p, 0, sizeof p);
+  p.B = (int)d.batch;
+  p.S = (int)d.seq;
+  p.Hq = (int)d.heads_q;
+  p.Hkv = (int)d.heads_kv;
+  p.group = (int)(d.heads_q / d.heads_kv);
+  p.q_blocks = (int)((d.seq + BM - 1) / BM);
+  p.causal = d.causal ? 1 : 0;
+  p.scale_log2 = (float)(d.scale * 1.4426950408889634);
+  p.raster = k.raster;
+  p.O = (__nv_bfloat16*)O;
+  p.lse = lse;
+  p.status = c.status;
+  const long long ctas = (long long)p.B * p.Hq * p.q_blocks;
+  if (ctas > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
+  kern<<<(unsigned)ctas, kThreads, smem_bytes(BN, k.stages), (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention launch: %s", cudaGetErrorString(e));
+  return RC_OK;
+}
+
+}  // namespace attn
+
+rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V,
+                              void* O, float* lse, void* workspace, const LaunchCtx& c) {
+  if (d.head_dim != attn::D) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: head_dim must be 128");
+  if (d.batch * d.seq > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: B*S too large");
+  const void* Vuse = V;
+  if (k.layout == 1) {
+    if (d.seq % 8) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: transposed V needs seq %% 8 == 0");
+    dim3 grid((unsigned)((d.seq + 63) / 64), attn::D / 64, (unsigned)(d.batch * d.heads_kv));
+    attn::transpose_v_kernel<<<grid, dim3(64, 8), 0, (cudaStream_t)c.stream>>>(
+        (const __nv_bfloat16*)V, (int)d.seq, (int)d.heads_kv, (__nv_bfloat16*)workspace);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "V transpose launch: %s", cudaGetErrorString(e));
+    Vuse = workspace;
+  }
+  const bool vt = k.layout == 1;
+  if (k.tile_n == 64) return vt ? attn::launch<64, true>(k, d, Q, K, Vuse, O, lse, c)
+                                : attn::launch<64, false>(k, d, Q, K, Vuse, O, lse, c);
+  if (k.tile_n == 128) return vt ? attn::launch<128, true>(k, d, Q, K, Vuse, O, lse, c)
+                                 : attn::launch<128, false>(k, d, Q, K, Vuse, O, lse, c);
+  return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: key block %d", k.tile_n);
+}

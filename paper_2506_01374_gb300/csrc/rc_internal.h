@@ -147,8 +147,9 @@ rc_status rc_launch_bias_silu_pass(const void* y, const void* bias, int64_t rows
 rc_status rc_launch_l2_flush(void* buf, size_t bytes, void* stream);
 
 // Attention and MoE launchers.
+// Attention: workspace holds the transposed V when k.layout == 1.
 rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K,
-                              const void* V, void* O, float* lse, const LaunchCtx& c);
+                              const void* V, void* O, float* lse, void* workspace, const LaunchCtx& c);
 // Routing: counts is device scratch of E ints; inv_perm may be NULL.
 rc_status rc_launch_moe_route(const rc_knobs& k, const rc_op_desc& d, const void* logits, int* ids,
                               float* w, int* offsets, int* perm, int* inv_perm, int* counts,

@@ -187,7 +187,7 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       return rc_launch_bias_silu_pass(y, p[2], rows, d.c_out, silu, p[3], k.vec, c);
     }
     case RC_OP_ATTENTION:
-      return rc_launch_attention(s->k[0], d, p[0], p[1], p[2], p[3], (float*)p[4], c);
+      return rc_launch_attention(s->k[0], d, p[0], p[1], p[2], p[3], (float*)p[4], op->ws, c);
     case RC_OP_MOE_ROUTE: {
       int* counts = (int*)ws.take(4 * d.experts);
       return rc_launch_moe_route(s->k[0], d, p[0], (int*)p[1], (float*)p[2], (int*)p[3], (int*)p[4], nullptr,

@@ -1,0 +1,80 @@
+"""Fused causal GQA attention on the GPU against the fp64 oracle.
+
+Every legal schedule (key block, ring depth, query-block order, V layout) must
+match the oracle (Sec. 2: transformations preserve semantics). O is bf16
+(2e-2 normwise); LSE is fp32 (1e-3 normwise).
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2506_01374_gb300 import inputs, rc
+
+from .gpu_util import empty_bf16, from_dev_bf16, rel_err, to_dev, torch
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+TOL_LSE = 1e-3
+
+
+def att_op(B, S, Hq, Hkv, causal=True):
+    return rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=128, causal=int(causal))
+
+
+def sched(op, bn, stages, raster, layout):
+    return op.schedule(rc.T(rc.T_TILE_SIZE, bn, axis=1), rc.T(rc.T_PIPELINE_STAGES, stages),
+                       rc.T(rc.T_LOOP_ORDER, raster, group=1), rc.T(rc.T_LAYOUT, layout))
+
+
+def run(op, s, Q, K, V):
+    B, S, Hq, D = Q.shape
+    dO = empty_bf16(B, S, Hq, D).fill_(0x7FC0)
+    lse = torch.full((B, Hq, S), float("nan"), dtype=torch.float32, device="cuda")
+    op.run(s, [to_dev(Q), to_dev(K), to_dev(V), dO, lse])
+    op.check()
+    return from_dev_bf16(dO), lse.cpu().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("causal", [True, False])
+@pytest.mark.parametrize("B,S,Hq,Hkv", [(2, 296, 4, 2), (1, 128, 2, 2), (1, 200, 8, 1)])
+def test_attention_schedule_sweep(B, S, Hq, Hkv, causal):
+    Q, K, V = inputs.attention(B, S, Hq, Hkv, 128, seed=61)
+    O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=causal)
+    op = att_op(B, S, Hq, Hkv, causal)
+    n = 0
+    for bn, st, ra, lay in itertools.product((64, 128), (2, 3), (0, 1), (0, 1)):
+        try:
+            s = sched(op, bn, st, ra, lay)
+        except rc.RcError:
+            continue  # illegal here (shared memory, or S % 8 for the transposed V)
+        O, L = run(op, s, Q, K, V)
+        assert rel_err(O, O_ref) <= TOL, (bn, st, ra, lay, rel_err(O, O_ref))
+        assert rel_err(L, L_ref) <= TOL_LSE, (bn, st, ra, lay)
+        n += 1
+    assert n >= 6
+
+
+def test_attention_single_token_and_no_lse():
+    Q, K, V = inputs.attention(1, 1, 4, 2, 128, seed=62)
+    op = att_op(1, 1, 4, 2)
+    O, L = run(op, op.schedule(rc.T(rc.T_LAYOUT, 0)), Q, K, V)
+    for h in range(4):  # a single visible key returns its value row
+        np.testing.assert_allclose(O[0, 0, h], inputs.bf16_bits_to_f64(V)[0, 0, h // 2], rtol=1e-2, atol=1e-2)
+    dO = empty_bf16(1, 1, 4, 128)
+    op.run(op.schedule(rc.T(rc.T_LAYOUT, 0)), [to_dev(Q), to_dev(K), to_dev(V), dO, None])
+    op.check()
+
+
+def test_attention_full_size_sampled_queries():
+    # Llama-3-8B-shaped layer: batch 1, seq 2048, 32 query heads, 8 KV heads, d = 128, causal.
+    B, S, Hq, Hkv = 1, 2048, 32, 8
+    Q, K, V = inputs.attention(B, S, Hq, Hkv, 128, seed=4)
+    qpos = np.array([0, 1, 63, 64, 127, 128, 129, 1000, 1023, 1024, 2000, 2046, 2047], dtype=np.int64)
+    O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=True, qpos=qpos)
+    op = att_op(B, S, Hq, Hkv)
+    for s in [op.schedule(), sched(op, 128, 2, 1, 0), sched(op, 64, 3, 0, 1)]:
+        O, L = run(op, s, Q, K, V)
+        assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
+        assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
