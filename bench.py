@@ -44,12 +44,15 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--samples", type=int, default=120, help="schedules the search measures")
-    ap.add_argument("--cpu-rows", type=int, default=1024,
+    ap.add_argument("--samples", type=int, default=400, help="schedules the search measures")
+    ap.add_argument("--cpu-rows", type=int, default=2048,
                     help="token rows of the CPU-oracle sample (0 = skip)")
     ap.add_argument("--schedule", default="",
                     help="fixed schedule instead of a search, e.g. 's0:tile_n=128,stages=4,fuse=1;s1:tile_n=256'")
     ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--ops", default="gemm_f32,conv2d,attention,moe",
+                    help="other workloads to search and report per op ('' = none)")
+    ap.add_argument("--op-samples", type=int, default=48, help="schedules measured per extra op")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
 
@@ -132,6 +135,79 @@ def parse_schedule(op, text, rc):
     return op.schedule(*ts)
 
 
+# FP32 SIMT peak of one GB300: 152 SMs x 128 FP32 lanes x 2 flops x 2.07 GHz.
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def search_best(op, io, samples, seed=0):
+    """MCTS over op's schedule space with device-timed candidates; returns (best, m, n, cand/s)."""
+    from paper_2506_01374_gb300 import rc
+    search = rc.Search(op, seed=seed)
+    res, n, t, pending = [], 0, 0.0, False
+    while n < samples:
+        nxt = search.step(res)
+        pending = False
+        if not nxt:
+            break
+        t0 = time.perf_counter()
+        res = op.measure(nxt, io, warmup=2, repeats=5)
+        t += time.perf_counter() - t0
+        n += len(nxt)
+        pending = True
+    if pending:  # hand the last batch's measurements to the search
+        search.step(res)
+    best, m = search.best()
+    return search, best, m, n, (n / t if t else None)
+
+
+def extra_ops(args, peak_tf):
+    """Search each other workload of the hot path and report its best schedule."""
+    import numpy as np
+    import torch
+
+    from paper_2506_01374_gb300 import inputs, rc
+
+    def dev(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16) if a.dtype == np.uint16 else a).cuda()
+
+    out = {}
+    for name in [x for x in args.ops.split(",") if x]:
+        if name == "gemm_f32":
+            A, B, bias = inputs.gemm_f32(256, 256, 256, seed=0)
+            op = rc.Op(rc.OP_GEMM_F32, m=256, n=256, k=256, flags=rc.EPI_BIAS | rc.EPI_RELU)
+            io = [dev(A), dev(B), dev(bias), torch.empty(256, 256, dtype=torch.float32, device="cuda")]
+            wl, bound, peak = "gemm_bias_relu_f32_256^3", "alu", FP32_ALU_TFLOPS
+        elif name == "conv2d":
+            x, w, b = inputs.conv2d(2, 64, 64, 320, 320, seed=5)
+            op = rc.Op(rc.OP_CONV2D, img_n=2, img_h=64, img_w=64, c_in=320, c_out=320, kr=3, ks=3, stride=1, pad=1,
+                       flags=rc.EPI_BIAS | rc.EPI_SILU)
+            io = [dev(x), dev(w), dev(b), torch.empty(2, 64, 64, 320, dtype=torch.int16, device="cuda")]
+            wl, bound, peak = "conv2d_nhwc_3x3_N2_64x64_C320_bias_silu_bf16", "tensor", peak_tf
+        elif name == "attention":
+            Q, K, V = inputs.attention(1, 2048, 32, 8, 128, seed=4)
+            op = rc.Op(rc.OP_ATTENTION, batch=1, seq=2048, heads_q=32, heads_kv=8, head_dim=128, causal=1)
+            io = [dev(Q), dev(K), dev(V), torch.empty(1, 2048, 32, 128, dtype=torch.int16, device="cuda"),
+                  torch.empty(1, 32, 2048, dtype=torch.float32, device="cuda")]
+            wl, bound, peak = "causal_gqa_attention_S2048_Hq32_Hkv8_d128_bf16", "tensor", peak_tf
+        elif name == "moe":
+            logits, X, W1, W2 = inputs.moe(4096, 7168, 64, 2048, seed=6)
+            op = rc.Op(rc.OP_MOE, tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
+            io = [dev(logits), dev(X), dev(W1), dev(W2), torch.empty(4096, 7168, dtype=torch.int16, device="cuda")]
+            del W1, W2
+            wl, bound, peak = "moe_T4096_H7168_E64_I2048_top8_bf16", "tensor", peak_tf
+        else:
+            continue
+        search, best, m, n, cps = search_best(op, io, args.op_samples)
+        # time the best schedule again with more repeats
+        m2 = op.measure([best], io, warmup=3, repeats=20)[0]
+        tf = op.info["flops"] / (m2.ms_median * 1e-3) / 1e12
+        out[name] = {"workload": wl, "tflops": tf, "ms": m2.ms_median, "bound": bound, "peak": peak,
+                     "frac": tf / peak, "samples": n, "candidates_per_s": cps, "schedule": str(best)}
+        del io
+        torch.cuda.empty_cache()
+    return out
+
+
 def dist_setup(args):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -206,17 +282,8 @@ def run_ours(args):
         best = parse_schedule(op, args.schedule, rc)
         best_m = None
     else:
-        while n_meas < args.samples:
-            nxt = search.step(res)
-            if not nxt:
-                break
-            t0 = time.perf_counter()
-            res = op.measure(nxt, io, warmup=2, repeats=5)
-            t_search += time.perf_counter() - t0
-            n_meas += len(nxt)
-        if res:
-            search.step(res)
-        best, best_m = search.best()
+        search, best, best_m, n_meas, cps = search_best(op, io, args.samples, seed=args.seed)
+        t_search = n_meas / cps if cps else 0.0
 
     # 2) timed steps of the best schedule
     flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
@@ -296,6 +363,8 @@ def run_ours(args):
             "gpu_launches": args.steps * launches_per_step,
             "clocks": clk,
         }
+        if args.ops:
+            out["ops"] = extra_ops(args, pk["bf16_tflops"])
         if args.cpu_rows > 0:
             out["cpu_baseline"] = cpu_oracle_sample(X, W1, W2, args.cpu_rows)
             out["cpu_baseline"].pop("seconds", None)
