@@ -86,6 +86,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
     v.push_back({RC_T_TILE_SIZE, 1, tn, {}});
     v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 6}, {}});
     v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1, 8}});
+    v.push_back({RC_T_PARALLEL, 0, {0, 1}, {}});  // one CTA per tile, or persistent CTAs
   };
   switch (kind) {
     case RC_OP_GEMM_F32:
@@ -95,7 +96,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       v.push_back({RC_T_UNROLL, 0, {1, 4}, {}});
       break;
     case RC_OP_LINEAR:
-      gemm_common({64, 128, 256});
+      gemm_common({64, 128, 224, 256});
       v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       break;
     case RC_OP_SWIGLU:
@@ -107,7 +108,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         gemm_common({32, 64, 128});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
       } else {
-        gemm_common({64, 128, 256});
+        gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       }
       break;
@@ -131,7 +132,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       } else if (stage == 1) {
         gemm_common({32, 64, 128});
       } else {
-        gemm_common({64, 128, 256});
+        gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
       }
       break;

@@ -53,6 +53,8 @@ struct Params {
   const int* row_map;
   int row_div;
   int* status;
+  int persistent;       // 1: grid-stride loop over tiles with two TMEM accumulators
+  int splits;           // split-K factor (work items = tiles x splits)
 };
 
 // Linear CTA index -> (m tile, n tile) under the raster order knob.
@@ -154,6 +156,47 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
   }
 }
 
+// Work item -> (A rows, B rows, n tile, split, k-block range). Grouped mode
+// maps the m tile onto the segment that owns it; `valid` is false for the
+// spare m tiles launched beyond what the segments need.
+struct Item {
+  bool valid;
+  int row0, row_end, brow0, nt, split, kb0, nkb;
+};
+
+template <bool GROUPED>
+__device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
+  Item it;
+  const long long tiles = (long long)p.tiles_m * p.tiles_n;
+  it.split = (int)(w / tiles);
+  int mt;
+  map_tile(p, (int)(w - (long long)it.split * tiles), mt, it.nt);
+  it.valid = true;
+  it.brow0 = 0;
+  if constexpr (GROUPED) {
+    int acc = 0, g = 0;
+    it.valid = false;
+    for (; g < p.groups; ++g) {
+      const int lo = p.offsets[g], hi = p.offsets[g + 1];
+      const int n_g = (hi - lo + BM - 1) / BM;
+      if (mt < acc + n_g) {
+        it.row0 = lo + (mt - acc) * BM;
+        it.row_end = hi;
+        it.valid = true;
+        break;
+      }
+      acc += n_g;
+    }
+    it.brow0 = g * p.b_group_rows;
+  } else {
+    it.row0 = mt * BM;
+    it.row_end = p.M;
+  }
+  it.kb0 = it.split * p.kb_per;
+  it.nkb = max(0, min(p.kb_total, it.kb0 + p.kb_per) - it.kb0);
+  return it;
+}
+
 template <int BN, int EPI, int AMODE, bool GROUPED>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const Params p,
@@ -161,47 +204,24 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int A_BYTES = BM * BK * 2;
   constexpr int B_BYTES = BN * BK * 2;
   constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   static_assert(B_BYTES % 1024 == 0, "B tile must keep stage buffers 1024-byte aligned");
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* full = (uint64_t*)(smem + (size_t)stages * STAGE_BYTES);
   uint64_t* empty = full + stages;
-  uint64_t* accum = empty + stages;
-  uint64_t* drain = accum + 1;
+  uint64_t* acc_full = empty + stages;  // [2]
+  uint64_t* acc_empty = acc_full + 2;   // [2]
+  uint64_t* drain = acc_empty + 2;
   uint32_t* tmem_slot = (uint32_t*)(drain + 1);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
   volatile int* status = p.status;
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-
-  int mt, nt;
-  map_tile(p, blockIdx.x, mt, nt);
-  int row0, row_end, brow0 = 0;
-  if constexpr (GROUPED) {
-    int acc = 0, g = 0;
-    row0 = -1;
-    row_end = 0;
-    for (; g < p.groups; ++g) {
-      const int lo = p.offsets[g], hi = p.offsets[g + 1];
-      const int n_g = (hi - lo + BM - 1) / BM;
-      if (mt < acc + n_g) {
-        row0 = lo + (mt - acc) * BM;
-        row_end = hi;
-        break;
-      }
-      acc += n_g;
-    }
-    if (row0 < 0) return;  // more m-tiles were launched than the groups need
-    brow0 = g * p.b_group_rows;
-  } else {
-    row0 = mt * BM;
-    row_end = p.M;
-  }
-  const int split = blockIdx.z;
-  const int kb0 = split * p.kb_per;
-  const int nkb = max(0, min(p.kb_total, kb0 + p.kb_per) - kb0);
+  const int n_acc = p.persistent ? 2 : 1;  // accumulator buffers in TMEM
+  const uint32_t tmem_cols = ACC_COLS * (uint32_t)n_acc;
+  const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;
 
   auto fail = [&](int code) {
     *abort_flag = 1;
@@ -213,12 +233,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&full[s], 1);
       tc::mbar_init(&empty[s], 1);
     }
-    tc::mbar_init(accum, 1);
+    for (int b = 0; b < 2; ++b) {
+      tc::mbar_init(&acc_full[b], 1);
+      tc::mbar_init(&acc_empty[b], 128);
+    }
     tc::mbar_init(drain, 1);
     *abort_flag = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
+  if (warp == 1) tc::tmem_alloc(tmem_slot, tmem_cols);
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
@@ -228,62 +251,85 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       tc::prefetch_tmap(&tmA);
       tc::prefetch_tmap(&tmB);
-      int i = 0;
-      for (; i < nkb; ++i) {
-        const int s = i % stages;
-        const uint32_t ph = (uint32_t)(i / stages) & 1u;
-        if (!tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status)) {
-          fail(RC_DEV_TIMEOUT_EMPTY);
-          break;
-        }
-        uint8_t* sa = smem + (size_t)s * STAGE_BYTES;
-        uint8_t* sb = sa + A_BYTES;
-        tc::mbar_expect_tx(&full[s], STAGE_BYTES);
-        const int kb = kb0 + i;
-        if constexpr (AMODE == TC_A_CONV) {
-          const int rs = kb / p.cblocks, cb = kb - rs * p.cblocks;
-          const int rr = rs / p.ks, ss = rs - rr * p.ks;
-          const int img = row0 / p.img_hw;
-          const int prow = (row0 - img * p.img_hw) / p.img_w;
-          tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
-        } else {
-          tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, row0);
-        }
-        if constexpr (EPI == TC_EPI_SWIGLU) {
-          const int nh = nt * (BN / 2);
-          tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, brow0 + nh);
-          tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], kb * BK, brow0 + p.swiglu_I + nh);
-        } else {
-          tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, brow0 + nt * BN);
+      uint32_t g = 0;  // k-blocks issued so far (ring position)
+      bool ok = true;
+      for (long long w = blockIdx.x; ok && w < items; w += gridDim.x) {
+        const Item it = resolve_item<GROUPED>(p, w);
+        if (!it.valid) continue;
+        for (int i = 0; i < it.nkb; ++i, ++g) {
+          const int s = (int)(g % (uint32_t)stages);
+          const uint32_t ph = (g / (uint32_t)stages) & 1u;
+          if (!tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status)) {
+            fail(RC_DEV_TIMEOUT_EMPTY);
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + (size_t)s * STAGE_BYTES;
+          uint8_t* sb = sa + A_BYTES;
+          tc::mbar_expect_tx(&full[s], STAGE_BYTES);
+          const int kb = it.kb0 + i;
+          if constexpr (AMODE == TC_A_CONV) {
+            const int rs = kb / p.cblocks, cb = kb - rs * p.cblocks;
+            const int rr = rs / p.ks, ss = rs - rr * p.ks;
+            const int img = it.row0 / p.img_hw;
+            const int prow = (it.row0 - img * p.img_hw) / p.img_w;
+            tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
+          } else {
+            tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, it.row0);
+          }
+          if constexpr (EPI == TC_EPI_SWIGLU) {
+            const int nh = it.nt * (BN / 2);
+            tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + nh);
+            tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], kb * BK, it.brow0 + p.swiglu_I + nh);
+          } else {
+            tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + it.nt * BN);
+          }
         }
       }
-      // let the copies issued in the last `stages` iterations land before exit
-      for (int j = max(0, i - stages); j < i; ++j)
-        if (!tc::mbar_wait_drain(&full[j % stages], (uint32_t)(j / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+      // let the copies issued in the last `stages` ring slots land before exit
+      const uint32_t first = g > (uint32_t)stages ? g - (uint32_t)stages : 0u;
+      for (uint32_t j = first; j < g; ++j)
+        if (!tc::mbar_wait_drain(&full[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u))
+          fail(RC_DEV_TIMEOUT_DRAIN);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+      uint32_t g = 0, li = 0;
       bool ok = true;
-      for (int i = 0; i < nkb; ++i) {
-        const int s = i % stages;
-        const uint32_t ph = (uint32_t)(i / stages) & 1u;
-        if (!tc::mbar_wait(&full[s], ph, abort_flag, status)) {
-          fail(RC_DEV_TIMEOUT_FULL);
+      for (long long w = blockIdx.x; ok && w < items; w += gridDim.x) {
+        const Item it = resolve_item<GROUPED>(p, w);
+        if (!it.valid) continue;
+        const uint32_t buf = li % (uint32_t)n_acc;
+        const uint32_t aph = (li / (uint32_t)n_acc) & 1u;
+        if (!tc::mbar_wait(&acc_empty[buf], aph ^ 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_ACCUM);
           ok = false;
           break;
         }
         tc::tc_fence_after();
-        const uint32_t sa = tc::smem_u32(smem + (size_t)s * STAGE_BYTES);
-        const uint64_t da = tc::sw128_desc(sa), db = tc::sw128_desc(sa + A_BYTES);
+        const uint32_t dacc = tmem + buf * ACC_COLS;
+        for (int i = 0; i < it.nkb; ++i, ++g) {
+          const int s = (int)(g % (uint32_t)stages);
+          const uint32_t ph = (g / (uint32_t)stages) & 1u;
+          if (!tc::mbar_wait(&full[s], ph, abort_flag, status)) {
+            fail(RC_DEV_TIMEOUT_FULL);
+            ok = false;
+            break;
+          }
+          tc::tc_fence_after();
+          const uint32_t sa = tc::smem_u32(smem + (size_t)s * STAGE_BYTES);
+          const uint64_t da = tc::sw128_desc(sa), db = tc::sw128_desc(sa + A_BYTES);
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k)
-          tc::umma_bf16(tmem, da + 2 * k, db + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
-        tc::umma_commit(&empty[s]);
+          for (int k = 0; k < BK / 16; ++k)
+            tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          tc::umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        tc::umma_commit(&acc_full[buf]);  // accumulator ready (also when nkb == 0)
+        ++li;
       }
-      if (ok) {
-        tc::umma_commit(accum);
-      } else {
+      if (!ok) {
         tc::umma_commit(drain);  // wait for the MMAs already issued before TMEM is freed
         if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
       }
@@ -291,12 +337,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     const int q = warp & 3;
-    const int r = row0 + 32 * q + lane;
-    if (tc::mbar_wait(accum, 0, abort_flag, status)) {
+    uint32_t li = 0;
+    for (long long w = blockIdx.x; w < items; w += gridDim.x) {
+      const Item it = resolve_item<GROUPED>(p, w);
+      if (!it.valid) continue;
+      const uint32_t buf = li % (uint32_t)n_acc;
+      const uint32_t aph = (li / (uint32_t)n_acc) & 1u;
+      if (!tc::mbar_wait(&acc_full[buf], aph, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        break;
+      }
       tc::tc_fence_after();
-      epilogue<BN, EPI>(p, tmem + ((uint32_t)(32 * q) << 16), r, row_end, nt, split, nkb > 0);
-    } else if (!*abort_flag) {
-      fail(RC_DEV_TIMEOUT_ACCUM);
+      epilogue<BN, EPI>(p, tmem + buf * ACC_COLS + ((uint32_t)(32 * q) << 16), it.row0 + 32 * q + lane,
+                        it.row_end, it.nt, it.split, it.nkb > 0);
+      tc::tc_fence_before();
+      tc::mbar_arrive(&acc_empty[buf]);
+      ++li;
     }
   }
   tc::tc_fence_before();
@@ -304,7 +360,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     __syncwarp();
     tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, TMEM_COLS);
+    tc::tmem_dealloc(tmem, tmem_cols);
   }
 }
 
@@ -314,10 +370,20 @@ rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uin
 
 template <typename Kern>
 rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tmB, const Params& p, int stages,
-                        int splits, size_t smem, const LaunchCtx& c) {
-  const long long tiles = (long long)p.tiles_m * p.tiles_n;
-  if (tiles <= 0 || tiles > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: %lld tiles", tiles);
-  dim3 grid((unsigned)tiles, 1, (unsigned)splits);
+                        int acc_cols, size_t smem, const LaunchCtx& c) {
+  const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;
+  if (items <= 0 || items > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: %lld work items", items);
+  long long ctas = items;
+  if (p.persistent) {
+    // as many CTAs as fit on the SMs at once (shared memory and 512 TMEM columns)
+    long long per_sm = 233472 / (long long)(smem + 1024);
+    const long long by_tmem = 512 / (2LL * acc_cols);
+    if (by_tmem < per_sm) per_sm = by_tmem;
+    if (per_sm < 1) per_sm = 1;
+    const long long resident = per_sm * (c.num_sms > 0 ? c.num_sms : 1);
+    if (resident < ctas) ctas = resident;
+  }
+  dim3 grid((unsigned)ctas, 1, 1);
   kern<<<grid, kThreads, smem, (cudaStream_t)c.stream>>>(tmA, tmB, p, stages);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
@@ -358,6 +424,8 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.kb_total = (int)((a.K + BK - 1) / BK);
   const int splits = EPI == TC_EPI_PARTIAL_F32 ? k.split_k : 1;
   p.kb_per = (p.kb_total + splits - 1) / splits;
+  p.splits = splits;
+  p.persistent = k.persistent ? 1 : 0;
   p.raster = k.raster;
   p.group = k.group > 0 ? k.group : 1;
   p.D = a.D;
@@ -380,7 +448,8 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.row_map = a.row_map;
   p.row_div = a.row_div > 0 ? a.row_div : 1;
   p.status = c.status;
-  return launch_kernel(kern, tmA, tmB, p, k.stages, splits, smem, c);
+  constexpr int acc_cols = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  return launch_kernel(kern, tmA, tmB, p, k.stages, acc_cols, smem, c);
 }
 
 }  // namespace tcg

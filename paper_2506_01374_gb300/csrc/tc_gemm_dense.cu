@@ -1,4 +1,4 @@
-// Dense 2-D instantiations of the tensor-core GEMM: N tile {64, 128, 256}
+// Dense 2-D instantiations of the tensor-core GEMM: N tile {64, 128, 224, 256}
 // (SwiGLU: 2 x {32, 64, 128}) x epilogue {bf16 store, SwiGLU, fp32 split-K}.
 #include "tc_gemm.cuh"
 
@@ -17,6 +17,10 @@ rc_status tc_dispatch_dense(const rc_knobs& k, const TcGemmArgs& a, const Launch
     RC_CASE(64)
     RC_CASE(128)
     RC_CASE(256)
+    case 224:  // 16 x 19 tiles of a 2048 x 4096 output = 2 full waves on 152 SMs
+      if (a.epilogue == TC_EPI_STORE_BF16) return launch<224, TC_EPI_STORE_BF16, TC_A_2D, false>(k, a, c);
+      if (a.epilogue == TC_EPI_PARTIAL_F32) return launch<224, TC_EPI_PARTIAL_F32, TC_A_2D, false>(k, a, c);
+      break;
   }
 #undef RC_CASE
   return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm dense: no variant for N tile %d epilogue %d", bn, a.epilogue);

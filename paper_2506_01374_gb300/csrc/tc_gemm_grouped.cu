@@ -1,4 +1,4 @@
-// Grouped (MoE) instantiations of the tensor-core GEMM: N tile {64, 128, 256}
+// Grouped (MoE) instantiations of the tensor-core GEMM: N tile {64, 128, 224, 256}
 // (SwiGLU: 2 x {32, 64, 128}) x epilogue {SwiGLU, bf16 store, scaled fp32
 // atomic combine}.
 #include "tc_gemm.cuh"
@@ -18,6 +18,10 @@ rc_status tc_dispatch_grouped(const rc_knobs& k, const TcGemmArgs& a, const Laun
     RC_CASE(64)
     RC_CASE(128)
     RC_CASE(256)
+    case 224:
+      if (a.epilogue == TC_EPI_STORE_BF16) return launch<224, TC_EPI_STORE_BF16, TC_A_2D, true>(k, a, c);
+      if (a.epilogue == TC_EPI_SCALE_ATOMIC) return launch<224, TC_EPI_SCALE_ATOMIC, TC_A_2D, true>(k, a, c);
+      break;
   }
 #undef RC_CASE
   return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm grouped: no variant for N tile %d epilogue %d", bn, a.epilogue);

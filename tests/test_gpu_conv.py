@@ -24,9 +24,9 @@ def conv_op(N, H, W, Cin, Cout, flags=rc.EPI_BIAS | rc.EPI_SILU):
                  flags=flags)
 
 
-def sched(op, tile_n, stages, split_k=1, fuse=1):
+def sched(op, tile_n, stages, split_k=1, fuse=1, persistent=0):
     return op.schedule(rc.T(rc.T_TILE_SIZE, tile_n, axis=1), rc.T(rc.T_PIPELINE_STAGES, stages),
-                       rc.T(rc.T_SPLIT_K, split_k), rc.T(rc.T_FUSE, fuse))
+                       rc.T(rc.T_SPLIT_K, split_k), rc.T(rc.T_FUSE, fuse), rc.T(rc.T_PARALLEL, persistent))
 
 
 @pytest.mark.parametrize("N,H,W,Cin", [(2, 16, 16, 128), (1, 16, 8, 64), (1, 4, 32, 64), (1, 2, 64, 192),
@@ -51,12 +51,12 @@ def test_conv_split_k_and_unfused_epilogue():
     ref = oracle.conv2d_nhwc_bf16(x, w, b)
     op = conv_op(N, H, W, Cin, Cout)
     dx, dw, db = to_dev(x), to_dev(w), to_dev(b)
-    for sk, fuse, tn in itertools.product((1, 3, 5), (0, 1), (80, 160)):
+    for sk, fuse, tn, pe in itertools.product((1, 3, 5), (0, 1), (80, 160), (0, 1)):
         dy = empty_bf16(N, H, W, Cout).fill_(0x7FC0)
-        op.run(sched(op, tn, 3, sk, fuse), [dx, dw, db, dy])
+        op.run(sched(op, tn, 3, sk, fuse, pe), [dx, dw, db, dy])
         op.check()
         err = rel_err(from_dev_bf16(dy).reshape(-1, Cout), ref)
-        assert err <= TOL, (sk, fuse, tn, err)
+        assert err <= TOL, (sk, fuse, tn, pe, err)
 
 
 def test_conv_without_bias_or_silu():
@@ -83,7 +83,8 @@ def test_conv_full_size_sampled_pixels():
     corners = [0, W - 1, (H - 1) * W, H * W - 1, H * W, 2 * H * W - 1, 63 * 64 + 5, 64 * 5]
     pix = np.unique(np.concatenate([corners, rng.integers(0, N * H * W, 120)])).astype(np.int64)
     ref = oracle.conv2d_nhwc_bf16(x, w, b, pix=pix)
-    for s in [op.schedule(), sched(op, 160, 4), sched(op, 80, 3, 5, 1), sched(op, 64, 6, 3, 0)]:
+    for s in [op.schedule(), sched(op, 160, 4), sched(op, 80, 3, 5, 1), sched(op, 64, 6, 3, 0),
+              sched(op, 160, 3, 1, 1, 1), sched(op, 80, 4, 3, 1, 1)]:
         op.run(s, [dx, dw, db, dy])
         op.check()
         got = from_dev_bf16(dy).reshape(-1, C)[pix]

@@ -22,7 +22,7 @@ TOL = 2e-2
 def sched(op, stage=0, base=None, **kv):
     ts = []
     names = {"tile_n": (rc.T_TILE_SIZE, 1), "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0),
-             "fuse": (rc.T_FUSE, 0)}
+             "fuse": (rc.T_FUSE, 0), "persistent": (rc.T_PARALLEL, 0)}
     for k, v in kv.items():
         if k == "raster":
             ts.append(rc.T(rc.T_LOOP_ORDER, v[0], stage=stage, group=v[1]))
@@ -38,13 +38,13 @@ def test_linear_schedule_sweep(M, N, K):
     ref = oracle.linear_bf16(X, W)
     op = rc.Op(rc.OP_LINEAR, m=M, n=N, k=K)
     dX, dW = to_dev(X), to_dev(W)
-    for tn, st, sk in itertools.product((64, 128, 256), (1, 2, 4), (1, 2, 4)):
-        s = sched(op, tile_n=tn, stages=st, split_k=sk)
+    for tn, st, sk, pe in itertools.product((64, 128, 224, 256), (1, 2, 4), (1, 2, 4), (0, 1)):
+        s = sched(op, tile_n=tn, stages=st, split_k=sk, persistent=pe)
         dY = empty_bf16(M, N).fill_(0x7FC0)  # NaN canary
         op.run(s, [dX, dW, dY])
         op.check()
         err = rel_err(from_dev_bf16(dY), ref)
-        assert err <= TOL, (tn, st, sk, err)
+        assert err <= TOL, (tn, st, sk, pe, err)
 
 
 def test_linear_raster_orders():
@@ -53,9 +53,9 @@ def test_linear_raster_orders():
     ref = oracle.linear_bf16(X, W)
     op = rc.Op(rc.OP_LINEAR, m=M, n=N, k=K)
     dX, dW = to_dev(X), to_dev(W)
-    for raster in [(0, 1), (1, 1), (0, 8), (1, 8)]:
+    for raster, pe in itertools.product([(0, 1), (1, 1), (0, 8), (1, 8)], (0, 1)):
         dY = empty_bf16(M, N).fill_(0x7FC0)
-        op.run(sched(op, tile_n=128, stages=3, raster=raster), [dX, dW, dY])
+        op.run(sched(op, tile_n=128, stages=3, raster=raster, persistent=pe), [dX, dW, dY])
         op.check()
         assert rel_err(from_dev_bf16(dY), ref) <= TOL, raster
 
@@ -66,12 +66,12 @@ def test_swiglu_fused_and_unfused(M, I, K):
     ref = oracle.swiglu_bf16(X, W1)
     op = rc.Op(rc.OP_SWIGLU, m=M, n=I, k=K)
     dX, dW = to_dev(X), to_dev(W1)
-    for tn, st, fuse in itertools.product((32, 64, 128), (1, 3), (0, 1)):
+    for tn, st, fuse, pe in itertools.product((32, 64, 128), (1, 3), (0, 1), (0, 1)):
         dh = empty_bf16(M, I).fill_(0x7FC0)
-        op.run(sched(op, tile_n=tn, stages=st, fuse=fuse), [dX, dW, dh])
+        op.run(sched(op, tile_n=tn, stages=st, fuse=fuse, persistent=pe), [dX, dW, dh])
         op.check()
         err = rel_err(from_dev_bf16(dh), ref)
-        assert err <= TOL, (tn, st, fuse, err)
+        assert err <= TOL, (tn, st, fuse, pe, err)
 
 
 def test_mlp_block_small():
@@ -81,7 +81,9 @@ def test_mlp_block_small():
     op = rc.Op(rc.OP_MLP, m=T, n=I, k=H)
     dX, d1, d2 = to_dev(X), to_dev(W1), to_dev(W2)
     cases = [dict(), dict(s0=dict(tile_n=128, stages=4, fuse=1), s1=dict(tile_n=256, stages=3, split_k=2)),
-             dict(s0=dict(tile_n=64, stages=2, fuse=0), s1=dict(tile_n=64, stages=6, split_k=4))]
+             dict(s0=dict(tile_n=64, stages=2, fuse=0), s1=dict(tile_n=64, stages=6, split_k=4)),
+             dict(s0=dict(tile_n=128, stages=4, fuse=1, persistent=1),
+                  s1=dict(tile_n=256, stages=4, split_k=2, persistent=1))]
     for c in cases:
         s = op.schedule()
         if c:
