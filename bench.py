@@ -1,21 +1,26 @@
 #!/usr/bin/env python
 """Benchmark of the schedule-search hot path on GB300.
 
-Workload (one GPU): the Llama-3-8B-shaped SwiGLU MLP block, bf16, tokens
-T=2048, hidden H=4096, intermediate I=14336, weights N(0, 0.02), activations
-N(0, 1), synthetic seeded inputs. A run
-  1. searches the block's schedule space with the LLM-free MCTS
+Default workload (one GPU): the Llama-3-8B-shaped SwiGLU MLP block, bf16,
+tokens T=2048, hidden H=4096, intermediate I=14336, weights N(0, 0.02),
+activations N(0, 1), synthetic seeded inputs. ``--workload`` selects one of
+the other hot-path workloads instead (attention, conv2d, moe, gemm_f32).
+
+A run
+  1. searches the workload's schedule space with the LLM-free MCTS
      (rc_search_step), every candidate timed on the device
      (rc_candidate_measure) -> candidates measured per second;
   2. times K steps of the best schedule found (rc_run_profiled: per-stage
      CUDA events on the launching stream; L2 flushed between steps, outside
-     the timed events) -> best-schedule TFLOP/s and the roofline fraction of
-     the dominant kernel (the gate/up GEMM with the fused SwiGLU epilogue);
+     the timed events) -> best-schedule TFLOP/s, and the roofline fraction of
+     the dominant kernel measured live;
   3. times K end-to-end steps through rc_run_host (pinned host buffers,
-     host->device inputs and device->host output inside the timed region);
-  4. times the fp64 CPU oracle on a bounded sample of token rows.
-Under torchrun (N > 1) every rank runs an independent replica (the path
-has no exchange step); value = all ranks' work / the slowest rank's time.
+     host->device inputs and device->host outputs inside the timed region);
+  4. searches the other workloads briefly and reports each one's best
+     schedule and roofline fraction (``ops``);
+  5. times the fp64 CPU oracle on a bounded sample of the workload.
+Under torchrun (N > 1) every rank runs an independent replica (the path has
+no exchange step); value = all ranks' work / the slowest rank's time.
 
 ``--impl reference`` times the CPU oracle alone as the reference arm.
 """
@@ -33,9 +38,8 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-T_TOK, HID, INTER = 2048, 4096, 14336
-WORKLOAD = "llama3_8b_mlp_swiglu_bf16_T2048_H4096_I14336"
-METRIC = "best-schedule TFLOP/s (Llama-3-8B MLP block, bf16)"
+# FP32 SIMT peak of one GB300: 152 SMs x 128 FP32 lanes x 2 flops x 2.07 GHz.
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
 def parse():
@@ -44,14 +48,16 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="mlp", choices=["mlp", "attention", "conv2d", "moe", "gemm_f32"])
     ap.add_argument("--samples", type=int, default=400, help="schedules the search measures")
-    ap.add_argument("--cpu-rows", type=int, default=2048,
-                    help="token rows of the CPU-oracle sample (0 = skip)")
+    ap.add_argument("--cpu-sample", type=int, default=0,
+                    help="size of the CPU-oracle sample (rows/queries/pixels/tokens; 0 = workload default, "
+                         "-1 = skip)")
     ap.add_argument("--schedule", default="",
                     help="fixed schedule instead of a search, e.g. 's0:tile_n=128,stages=4,fuse=1;s1:tile_n=256'")
     ap.add_argument("--skip-e2e", action="store_true")
-    ap.add_argument("--ops", default="gemm_f32,conv2d,attention,moe",
-                    help="other workloads to search and report per op ('' = none)")
+    ap.add_argument("--ops", default=None,
+                    help="other workloads to search and report ('' = none; default: all others for mlp)")
     ap.add_argument("--op-samples", type=int, default=48, help="schedules measured per extra op")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
@@ -116,10 +122,185 @@ class Clocks:
                 "reasons": reasons, "samples": len(rows)}
 
 
+# ------------------------------------------------------------------ workloads --
+
+class Workload:
+    """One hot-path workload: op, seeded host inputs, output slots, dominant kernel."""
+
+    def __init__(self, name):
+        import numpy as np
+
+        from paper_2506_01374_gb300 import inputs, rc
+        self.name = name
+        if name == "mlp":
+            T, H, I = 2048, 4096, 14336
+            X, W1, W2 = inputs.mlp(T, H, I, seed=1)
+            self.op = rc.Op(rc.OP_MLP, m=T, n=I, k=H)
+            self.host = [X, W1, W2, None]
+            self.outs = {3: ((T, H), np.uint16)}
+            self.label = "llama3_8b_mlp_swiglu_bf16_T2048_H4096_I14336"
+            self.config = {"tokens": T, "hidden": H, "inter": I}
+            self.metric = "best-schedule TFLOP/s (Llama-3-8B MLP block, bf16)"
+            self.dom_stage, self.dom_flops = 0, 2.0 * T * (2 * I) * H
+            self.dom_name = "gate/up GEMM{} (stage 0)"
+            self.bound = "tensor"
+            self.dtype = "bf16"
+        elif name == "attention":
+            B, S, Hq, Hkv, D = 1, 2048, 32, 8, 128
+            Q, K, V = inputs.attention(B, S, Hq, Hkv, D, seed=4)
+            self.op = rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=1)
+            self.host = [Q, K, V, None, None]
+            self.outs = {3: ((B, S, Hq, D), np.uint16), 4: ((B, Hq, S), np.float32)}
+            self.label = "causal_gqa_attention_B1_S2048_Hq32_Hkv8_d128_bf16"
+            self.config = {"batch": B, "seq": S, "heads_q": Hq, "heads_kv": Hkv, "head_dim": D, "causal": True}
+            self.metric = "best-schedule TFLOP/s (causal GQA attention, bf16)"
+            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_name = "fused attention kernel"
+            self.bound = "tensor"
+            self.dtype = "bf16"
+        elif name == "conv2d":
+            N, H, W, C = 2, 64, 64, 320
+            x, w, b = inputs.conv2d(N, H, W, C, C, seed=5)
+            self.op = rc.Op(rc.OP_CONV2D, img_n=N, img_h=H, img_w=W, c_in=C, c_out=C, kr=3, ks=3, stride=1, pad=1,
+                            flags=rc.EPI_BIAS | rc.EPI_SILU)
+            self.host = [x, w, b, None]
+            self.outs = {3: ((N, H, W, C), np.uint16)}
+            self.label = "conv2d_nhwc_3x3_N2_64x64_C320_bias_silu_bf16"
+            self.config = {"n": N, "h": H, "w": W, "c_in": C, "c_out": C, "kernel": 3}
+            self.metric = "best-schedule TFLOP/s (UNet conv2d 3x3 + bias + SiLU, bf16)"
+            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_name = "implicit-GEMM conv kernel"
+            self.bound = "tensor"
+            self.dtype = "bf16"
+        elif name == "moe":
+            T, H, E, I, K = 4096, 7168, 64, 2048, 8
+            logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=6)
+            self.op = rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
+            self.host = [logits, X, W1, W2, None]
+            self.outs = {4: ((T, H), np.uint16)}
+            self.label = "moe_T4096_H7168_E64_I2048_top8_bf16"
+            self.config = {"tokens": T, "hidden": H, "experts": E, "inter": I, "top_k": K}
+            self.metric = "best-schedule TFLOP/s (MoE layer, 64 experts, top-8, bf16)"
+            self.dom_stage, self.dom_flops = 1, 2.0 * T * K * (2 * I) * H
+            self.dom_name = "grouped gate/up GEMM + SwiGLU (stage 1)"
+            self.bound = "tensor"
+            self.dtype = "bf16"
+        elif name == "gemm_f32":
+            M = N = K = 256
+            A, B, bias = inputs.gemm_f32(M, N, K, seed=0)
+            self.op = rc.Op(rc.OP_GEMM_F32, m=M, n=N, k=K, flags=rc.EPI_BIAS | rc.EPI_RELU)
+            self.host = [A, B, bias, None]
+            self.outs = {3: ((M, N), np.float32)}
+            self.label = "gemm_bias_relu_f32_256^3"
+            self.config = {"m": M, "n": N, "k": K}
+            self.metric = "best-schedule TFLOP/s (fp32 GEMM + bias + ReLU, 256^3)"
+            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_name = "fp32 SIMT GEMM"
+            self.bound = "alu"
+            self.dtype = "f32"
+        else:
+            raise ValueError(name)
+
+    def device_io(self):
+        import numpy as np
+        import torch
+        io = []
+        for i, a in enumerate(self.host):
+            if a is not None:
+                io.append(torch.from_numpy(a.view(np.int16) if a.dtype == np.uint16 else a).cuda())
+            elif i in self.outs:
+                shape, dt = self.outs[i]
+                io.append(torch.empty(shape, dtype=torch.int16 if dt == np.uint16 else torch.float32, device="cuda"))
+            else:
+                io.append(None)
+        return io
+
+    def host_io(self):
+        import numpy as np
+        import torch
+        io = []
+        for i, a in enumerate(self.host):
+            if a is not None:
+                io.append(torch.from_numpy(a.view(np.int16) if a.dtype == np.uint16 else a).pin_memory().numpy())
+            elif i in self.outs:
+                shape, dt = self.outs[i]
+                io.append(torch.empty(shape, dtype=torch.int16 if dt == np.uint16 else torch.float32)
+                          .pin_memory().numpy())
+            else:
+                io.append(None)
+        return io
+
+    def io_bytes(self):
+        import numpy as np
+        h2d = sum(a.nbytes for a in self.host if a is not None)
+        d2h = sum(int(np.prod(s)) * np.dtype(dt).itemsize for s, dt in self.outs.values())
+        return h2d, d2h
+
+    def cpu_sample(self, n):
+        """Time the fp64 oracle on a bounded sample; returns the cpu_baseline dict."""
+        import numpy as np
+
+        import oracle
+        oracle.build()
+        cores = os.cpu_count() or 1
+        if self.name == "mlp":
+            X, W1, W2 = self.host[:3]
+            n = n or 2048
+            sel = np.arange(n, dtype=np.int64) * (X.shape[0] // n)
+            t0 = time.perf_counter()
+            oracle.mlp_bf16(X, W1, W2, rows=sel)
+            dt = time.perf_counter() - t0
+            flops = 6.0 * n * X.shape[1] * (W1.shape[0] // 2)
+            what, used = f"{n} of {X.shape[0]} token rows of the MLP block", min(cores, n)
+        elif self.name == "attention":
+            Q, K, V = self.host[:3]
+            S = Q.shape[1]
+            n = n or 256
+            qpos = np.linspace(0, S - 1, n).astype(np.int64)
+            t0 = time.perf_counter()
+            oracle.attention_bf16(Q, K, V, causal=True, qpos=qpos)
+            dt = time.perf_counter() - t0
+            flops = float(sum(4.0 * Q.shape[3] * Q.shape[2] * (int(i) + 1) for i in qpos))
+            what, used = f"{n} of {S} query positions (all heads)", min(cores, n)
+        elif self.name == "conv2d":
+            x, w, b = self.host[:3]
+            total = x.shape[0] * x.shape[1] * x.shape[2]
+            n = n or 4096
+            pix = np.linspace(0, total - 1, n).astype(np.int64)
+            t0 = time.perf_counter()
+            oracle.conv2d_nhwc_bf16(x, w, b, pix=pix)
+            dt = time.perf_counter() - t0
+            flops = 2.0 * n * w.shape[0] * w.shape[1] * w.shape[2] * w.shape[3]
+            what, used = f"{n} of {total} output pixels", min(cores, n)
+        elif self.name == "moe":
+            logits, X, W1, W2 = self.host[:4]
+            n = n or 32
+            tok = np.linspace(0, X.shape[0] - 1, n).astype(np.int64)
+            t0 = time.perf_counter()
+            ids, w, _, _ = oracle.moe_route(logits, 8)
+            oracle.moe_ffn_bf16(X, W1, W2, ids, w, tok=tok)
+            dt = time.perf_counter() - t0
+            flops = 6.0 * n * 8 * X.shape[1] * (W1.shape[1] // 2)
+            what, used = f"routing of all tokens + expert FFN of {n} of {X.shape[0]} tokens", min(cores, n)
+        else:
+            A, B, bias = self.host[:3]
+            n = n or 40
+            t0 = time.perf_counter()
+            for _ in range(n):
+                oracle.gemm_bias_relu_f32(A, B, bias)
+            dt = time.perf_counter() - t0
+            flops = n * 2.0 * A.shape[0] * A.shape[1] * B.shape[1]
+            what, used = f"{n} full 256^3 GEMMs", min(cores, A.shape[0])
+        return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": used, "kind": "oracle",
+                "sample": what + ", fp64 loop nests", "seconds": dt}
+
+
 def parse_schedule(op, text, rc):
     """'s0:tile_n=128,stages=4;s1:split_k=2' -> schedule (raster=R/G sets loop order and group)."""
-    KNOB_T = {"tile_n": (rc.T_TILE_SIZE, 1), "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0),
-              "fuse": (rc.T_FUSE, 0), "raster": (rc.T_LOOP_ORDER, 0), "persistent": (rc.T_PARALLEL, 0)}
+    KNOB_T = {"tile_m": (rc.T_TILE_SIZE, 0), "tile_n": (rc.T_TILE_SIZE, 1), "tile_k": (rc.T_TILE_SIZE, 2),
+              "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0), "fuse": (rc.T_FUSE, 0),
+              "raster": (rc.T_LOOP_ORDER, 0), "persistent": (rc.T_PARALLEL, 0), "layout": (rc.T_LAYOUT, 0),
+              "unroll": (rc.T_UNROLL, 0)}
     ts = []
     for part in filter(None, text.split(";")):
         stage_s, kvs = part.split(":")
@@ -135,12 +316,8 @@ def parse_schedule(op, text, rc):
     return op.schedule(*ts)
 
 
-# FP32 SIMT peak of one GB300: 152 SMs x 128 FP32 lanes x 2 flops x 2.07 GHz.
-FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
-
-
 def search_best(op, io, samples, seed=0):
-    """MCTS over op's schedule space with device-timed candidates; returns (best, m, n, cand/s)."""
+    """MCTS over op's schedule space with device-timed candidates; returns (search, best, m, n, cand/s)."""
     from paper_2506_01374_gb300 import rc
     search = rc.Search(op, seed=seed)
     res, n, t, pending = [], 0, 0.0, False
@@ -160,130 +337,91 @@ def search_best(op, io, samples, seed=0):
     return search, best, m, n, (n / t if t else None)
 
 
-def extra_ops(args, peak_tf):
-    """Search each other workload of the hot path and report its best schedule."""
-    import numpy as np
+def extra_ops(names, samples, peak_tf):
+    """Search each other workload briefly and report its best schedule."""
     import torch
-
-    from paper_2506_01374_gb300 import inputs, rc
-
-    def dev(a):
-        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16) if a.dtype == np.uint16 else a).cuda()
-
     out = {}
-    for name in [x for x in args.ops.split(",") if x]:
-        if name == "gemm_f32":
-            A, B, bias = inputs.gemm_f32(256, 256, 256, seed=0)
-            op = rc.Op(rc.OP_GEMM_F32, m=256, n=256, k=256, flags=rc.EPI_BIAS | rc.EPI_RELU)
-            io = [dev(A), dev(B), dev(bias), torch.empty(256, 256, dtype=torch.float32, device="cuda")]
-            wl, bound, peak = "gemm_bias_relu_f32_256^3", "alu", FP32_ALU_TFLOPS
-        elif name == "conv2d":
-            x, w, b = inputs.conv2d(2, 64, 64, 320, 320, seed=5)
-            op = rc.Op(rc.OP_CONV2D, img_n=2, img_h=64, img_w=64, c_in=320, c_out=320, kr=3, ks=3, stride=1, pad=1,
-                       flags=rc.EPI_BIAS | rc.EPI_SILU)
-            io = [dev(x), dev(w), dev(b), torch.empty(2, 64, 64, 320, dtype=torch.int16, device="cuda")]
-            wl, bound, peak = "conv2d_nhwc_3x3_N2_64x64_C320_bias_silu_bf16", "tensor", peak_tf
-        elif name == "attention":
-            Q, K, V = inputs.attention(1, 2048, 32, 8, 128, seed=4)
-            op = rc.Op(rc.OP_ATTENTION, batch=1, seq=2048, heads_q=32, heads_kv=8, head_dim=128, causal=1)
-            io = [dev(Q), dev(K), dev(V), torch.empty(1, 2048, 32, 128, dtype=torch.int16, device="cuda"),
-                  torch.empty(1, 32, 2048, dtype=torch.float32, device="cuda")]
-            wl, bound, peak = "causal_gqa_attention_S2048_Hq32_Hkv8_d128_bf16", "tensor", peak_tf
-        elif name == "moe":
-            logits, X, W1, W2 = inputs.moe(4096, 7168, 64, 2048, seed=6)
-            op = rc.Op(rc.OP_MOE, tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
-            io = [dev(logits), dev(X), dev(W1), dev(W2), torch.empty(4096, 7168, dtype=torch.int16, device="cuda")]
-            del W1, W2
-            wl, bound, peak = "moe_T4096_H7168_E64_I2048_top8_bf16", "tensor", peak_tf
-        else:
-            continue
-        search, best, m, n, cps = search_best(op, io, args.op_samples)
-        # time the best schedule again with more repeats
-        m2 = op.measure([best], io, warmup=3, repeats=20)[0]
-        tf = op.info["flops"] / (m2.ms_median * 1e-3) / 1e12
-        out[name] = {"workload": wl, "tflops": tf, "ms": m2.ms_median, "bound": bound, "peak": peak,
+    for name in names:
+        wl = Workload(name)
+        io = wl.device_io()
+        _, best, _, n, cps = search_best(wl.op, io, samples)
+        m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
+        tf = wl.op.info["flops"] / (m.ms_median * 1e-3) / 1e12
+        peak = FP32_ALU_TFLOPS if wl.bound == "alu" else peak_tf
+        out[name] = {"workload": wl.label, "tflops": tf, "ms": m.ms_median, "bound": wl.bound, "peak": peak,
                      "frac": tf / peak, "samples": n, "candidates_per_s": cps, "schedule": str(best)}
-        del io
+        del io, wl
         torch.cuda.empty_cache()
     return out
 
 
-def dist_setup(args):
+def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return world, rank, local
 
 
-def cpu_oracle_sample(X, W1, W2, rows: int):
-    """Time the fp64 oracle on `rows` token rows of the MLP block."""
-    import numpy as np
-
-    import oracle
-    sel = np.arange(rows, dtype=np.int64) * (X.shape[0] // max(rows, 1))
-    oracle.build()
-    t0 = time.perf_counter()
-    oracle.mlp_bf16(X, W1, W2, rows=sel)
-    dt = time.perf_counter() - t0
-    flops = 6.0 * rows * HID * INTER
-    return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": min(os.cpu_count() or 1, rows),
-            "kind": "oracle", "sample": f"{rows} of {T_TOK} token rows of the MLP block, fp64 loop nests",
-            "seconds": dt}
-
-
 def run_reference(args):
-    world, rank, _ = dist_setup(args)
+    world, rank, _ = dist_setup()
     if rank != 0:
         return
-    from paper_2506_01374_gb300 import inputs
-    X, W1, W2 = inputs.mlp(T_TOK, HID, INTER, seed=1)
-    rows = max(1, min(args.cpu_rows, 16))
+    wl = Workload(args.workload)
+    n = args.cpu_sample if args.cpu_sample > 0 else {"mlp": 16, "attention": 32, "conv2d": 512, "moe": 4,
+                                                     "gemm_f32": 4}[args.workload]
     for _ in range(args.warmup):
-        cpu_oracle_sample(X, W1, W2, rows)
-    ts = [cpu_oracle_sample(X, W1, W2, rows)["seconds"] for _ in range(args.steps)]
-    ms = 1e3 * sum(ts) / len(ts)
-    val = 6.0 * rows * HID * INTER / (ms * 1e-3) / 1e12
-    cb = {"value": val, "unit": "TFLOP/s", "cores": min(os.cpu_count() or 1, rows), "kind": "oracle",
-          "sample": f"{rows} of {T_TOK} token rows per step, fp64 loop nests"}
-    print(json.dumps({"impl": "reference", "metric": METRIC, "value": val, "unit": "TFLOP/s", "n_gpus": world,
-                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-                      "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                      "config": {"workload": WORKLOAD, "tokens": T_TOK, "hidden": HID, "inter": INTER},
-                      "cpu_baseline": cb,
+        wl.cpu_sample(n)
+    samples = [wl.cpu_sample(n) for _ in range(args.steps)]
+    secs = statistics.fmean(s["seconds"] for s in samples)
+    val = statistics.fmean(s["value"] for s in samples)
+    cb = {k: v for k, v in samples[0].items() if k != "seconds"}
+    cb["value"] = val
+    print(json.dumps({"impl": "reference", "metric": wl.metric, "value": val, "unit": "TFLOP/s", "n_gpus": world,
+                      "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs,
+                      "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                      "data": "synthetic", "config": dict(workload=wl.label, **wl.config), "cpu_baseline": cb,
                       "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
 
 
+def launches_per_step(workload, s):
+    """Kernels of this library one step of the schedule launches (the L2 flush is a torch fill)."""
+    k = [s.knobs(i) for i in range(s.num_stages)]
+    if workload == "mlp":
+        return (1 if k[0]["fuse"] else 2) + (1 if k[1]["split_k"] == 1 else 2)
+    if workload == "attention":
+        return 1 + (1 if k[0]["layout"] == 1 else 0)
+    if workload == "conv2d":
+        return 1 + (1 if k[0]["split_k"] > 1 else 0) + (1 if (k[0]["split_k"] > 1 or not k[0]["fuse"]) else 0)
+    if workload == "moe":
+        # routing (3 kernels), gather, grouped gate/up, grouped down, combine (or memset + convert)
+        return 3 + 1 + 1 + 1 + 1
+    return 1
+
+
 def run_ours(args):
-    import numpy as np
     import torch
 
-    from paper_2506_01374_gb300 import inputs, rc
+    from paper_2506_01374_gb300 import rc
 
-    world, rank, local = dist_setup(args)
+    world, rank, local = dist_setup()
     torch.cuda.set_device(local)
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     stream = torch.cuda.current_stream()
 
-    X, W1, W2 = inputs.mlp(T_TOK, HID, INTER, seed=1)
-    dX = torch.from_numpy(X.view(np.int16)).cuda()
-    d1 = torch.from_numpy(W1.view(np.int16)).cuda()
-    d2 = torch.from_numpy(W2.view(np.int16)).cuda()
-    dY = torch.empty(T_TOK, HID, dtype=torch.int16, device="cuda")
-    io = [dX, d1, d2, dY]
-    op = rc.Op(rc.OP_MLP, m=T_TOK, n=INTER, k=HID)
+    wl = Workload(args.workload)
+    op = wl.op
     info = op.info
+    io = wl.device_io()
 
     # 1) schedule search, every candidate measured on the device
-    search = rc.Search(op, seed=args.seed)
-    res, n_meas, t_search = [], 0, 0.0
+    n_meas, cps, best_m = 0, None, None
+    search = None
     if args.schedule:
         best = parse_schedule(op, args.schedule, rc)
-        best_m = None
     else:
         search, best, best_m, n_meas, cps = search_best(op, io, args.samples, seed=args.seed)
-        t_search = n_meas / cps if cps else 0.0
 
     # 2) timed steps of the best schedule
     flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
@@ -295,32 +433,28 @@ def run_ours(args):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    step_ms, stage0_ms = [], []
+    step_ms, dom_ms = [], []
     for _ in range(args.steps):
         flush.fill_(1.0)
         st = op.run_profiled(best, io, stream)
         step_ms.append(sum(st))
-        stage0_ms.append(st[0])
+        dom_ms.append(st[wl.dom_stage])
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     clk = clocks.stop()
     ms = statistics.fmean(step_ms)
-    ms_stage0 = statistics.fmean(stage0_ms)
+    ms_dom = statistics.fmean(dom_ms)
     if world > 1:
-        t = torch.tensor([ms, ms_stage0], device="cuda", dtype=torch.float64)
+        t = torch.tensor([ms, ms_dom], device="cuda", dtype=torch.float64)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, ms_stage0 = t.tolist()
+        ms, ms_dom = t.tolist()
     value = world * info["flops"] / (ms * 1e-3) / 1e12
 
     # 3) end to end through the host-buffer entry point
-    hX = torch.from_numpy(X.view(np.int16)).pin_memory().numpy()
-    h1 = torch.from_numpy(W1.view(np.int16)).pin_memory().numpy()
-    h2 = torch.from_numpy(W2.view(np.int16)).pin_memory().numpy()
-    hY = torch.empty(T_TOK, HID, dtype=torch.int16).pin_memory().numpy()
-    host_io = [hX, h1, h2, hY]
     e2e_s = None
     if not args.skip_e2e:
+        host_io = wl.host_io()
         for _ in range(max(1, args.warmup)):
             op.run_host(best, host_io)
         e2e_t = []
@@ -333,41 +467,46 @@ def run_ours(args):
             t = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
             torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
             e2e_s = t.item()
-    h2d = X.nbytes + W1.nbytes + W2.nbytes
-    d2h = T_TOK * HID * 2
+    h2d, d2h = wl.io_bytes()
 
     if rank == 0:
         pk = peaks()
-        gate_up_flops = 2.0 * T_TOK * (2 * INTER) * HID
-        achieved = gate_up_flops / (ms_stage0 * 1e-3) / 1e12
-        k0, k1 = best.knobs(0), best.knobs(1)
-        launches_per_step = (1 if k0["fuse"] else 2) + (1 if k1["split_k"] == 1 else 2)
-        kname = "gate/up GEMM" + (" + fused SwiGLU epilogue" if k0["fuse"] else " + SwiGLU pass") + " (stage 0)"
+        peak = FP32_ALU_TFLOPS if wl.bound == "alu" else pk["bf16_tflops"]
+        peak_src = ("derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz" if wl.bound == "alu"
+                    else pk["source"] + " bf16 burst")
+        achieved = wl.dom_flops / (ms_dom * 1e-3) / 1e12
+        kname = wl.dom_name
+        if args.workload == "mlp":
+            kname = kname.format(" + fused SwiGLU epilogue" if best.knobs(0)["fuse"] else " + SwiGLU pass")
         out = {
-            "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "metric": wl.metric, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "tokens": T_TOK, "hidden": HID, "inter": INTER,
-                       "parallelism": "replicas" if world > 1 else "single",
-                       "l2": "flushed between steps (flush outside the timed events)",
-                       "schedule": str(best)},
-            "roofline": {"bound": "tensor", "kernel": kname,
-                         "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
-                         "frac": achieved / pk["bf16_tflops"], "peak_source": pk["source"] + " bf16 burst",
-                         "traffic": None},
-            "step_frac_of_peak": value / world / pk["bf16_tflops"],
-            "search": {"samples": n_meas, "candidates_per_s": n_meas / t_search if t_search else None,
-                       "best_search_tflops": best_m.tflops if best_m else None, "stats": search.stats()},
+            "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+            "config": dict(workload=wl.label, **wl.config,
+                           parallelism="replicas" if world > 1 else "single",
+                           l2="flushed between steps (flush outside the timed events)", schedule=str(best)),
+            "roofline": {"bound": wl.bound, "kernel": kname, "achieved": achieved, "peak": peak,
+                         "unit": "TFLOP/s", "frac": achieved / peak, "peak_source": peak_src, "traffic": None},
+            "step_frac_of_peak": value / world / peak,
+            "search": {"samples": n_meas, "candidates_per_s": cps,
+                       "best_search_tflops": best_m.tflops if best_m else None,
+                       "stats": search.stats() if search else None},
             "e2e": None if e2e_s is None else {"value": world * info["flops"] / e2e_s / 1e12, "unit": "TFLOP/s",
                                                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": args.steps * launches_per_step,
+            "gpu_launches": args.steps * launches_per_step(args.workload, best),
             "clocks": clk,
         }
-        if args.ops:
-            out["ops"] = extra_ops(args, pk["bf16_tflops"])
-        if args.cpu_rows > 0:
-            out["cpu_baseline"] = cpu_oracle_sample(X, W1, W2, args.cpu_rows)
-            out["cpu_baseline"].pop("seconds", None)
+        others = args.ops if args.ops is not None else (
+            "gemm_f32,conv2d,attention,moe" if args.workload == "mlp" else "")
+        names = [x for x in others.split(",") if x and x != args.workload]
+        if names:
+            del io
+            torch.cuda.empty_cache()
+            out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"])
+        if args.cpu_sample >= 0:
+            cb = wl.cpu_sample(args.cpu_sample)
+            cb.pop("seconds", None)
+            out["cpu_baseline"] = cb
         else:
             out["cpu_baseline"] = None
         print(json.dumps(out))

@@ -118,10 +118,13 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
       break;
     case RC_OP_ATTENTION:
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256 = two query tiles, ping-pong softmax
       v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});
-      v.push_back({RC_T_PIPELINE_STAGES, 0, {2, 3}, {}});
+      v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 5}, {}});
       v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1}});
       v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // V as [keys][d] or transposed to [d][keys]
+      v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});  // P stored in shared or tensor memory
+      v.push_back({RC_T_UNROLL, 0, {1, 2}, {}});  // key blocks in flight per query tile
       break;
     case RC_OP_MOE_ROUTE:
       v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
@@ -233,11 +236,26 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
       if (stage == 0) return true;
       return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, why);
     case RC_OP_ATTENTION: {
-      // Q tile + ring of K and V tiles + P tile + slack, all bf16
-      const int64_t smem = 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 + 128 * (int64_t)k.tile_n * 2 +
-                           1024 + 256;
+      // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
+      const int64_t qt = k.tile_m / 128;
+      const int64_t smem = qt * 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 +
+                           (k.location ? 0 : qt * 128 * (int64_t)k.tile_n * 2) + 1024 + 256;
+      if (k.location == 1 && k.tile_m != 256) {
+        if (why) *why = "P in tensor memory is a variant of the two-tile kernel";
+        return false;
+      }
+      if (k.unroll == 2 && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
+        // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
+        if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
+        return false;
+      }
       if (smem > kSmemLimit) {
         if (why) *why = "attention ring exceeds 227 KB of shared memory";
+        return false;
+      }
+      if (k.tile_m == 256 && k.stages < 2) {
+        // the ping-pong kernel issues S for key block j+1 before releasing block j
+        if (why) *why = "two query tiles per CTA need at least two K/V stages";
         return false;
       }
       if (k.layout == 1 && o.seq % 8) {

@@ -333,6 +333,380 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Two query tiles per CTA (TileSize M = 256), ping-pong between two softmax
+// warpgroups: the MMA warp issues S_0 = Q_0 K^T, S_1 = Q_1 K^T, then
+// O_0 += P_0 V as soon as P_0 is ready and the next S_0 right after it, so
+// one tile's softmax overlaps the other tile's tensor-core work. TMEM holds
+// S_0, S_1 (BN columns each) and O_0, O_1 (128 each). Each softmax thread
+// loads its whole S row with one wait. O is rescaled only when the running
+// maximum grows by more than 2^8 (kRescaleLog2); the exponents use that same
+// reference maximum, and so does the row sum l, so the result is exact.
+// S for key block j+1 is issued before block j's ring slot is released, so
+// this kernel needs a ring of at least two stages.
+constexpr int kThreads2 = 320;
+constexpr float kRescaleLog2 = 8.0f;
+
+
+template <int BN, bool VT, bool PT, bool SDB>
+__global__ void __launch_bounds__(kThreads2, 1)
+    attn2_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  static_assert(BN == 64 || BN == 128, "key block");
+  constexpr int Q_BYTES = BM * D * 2;   // one query tile: two [128][64] halves
+  constexpr int KV_TILE = BN * D * 2;
+  // P tiles live in shared memory (BN/64 atoms of [128][64]) or, when PT, in
+  // the first BN/2 TMEM columns of their S tile (two bf16 per column).
+  constexpr int P_BYTES = PT ? 0 : BM * BN * 2;
+  // SDB: two S buffers per query tile, so S for key block j+1 is computed
+  // while the softmax works on block j (two key blocks in flight per tile).
+  static_assert(!SDB || (PT && BN == 64), "double-buffered S needs P in TMEM and BN = 64");
+  // (SDB also needs >= 4 ring stages: S of block j+2 is issued while V of
+  // block j is still in use, and the next block should already be loading.)
+  constexpr int NSB = SDB ? 2 : 1;                     // S buffers per tile
+  constexpr uint32_t O_BASE = (uint32_t)(2 * NSB * BN);  // TMEM column of O_0
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;                                   // [2] tiles
+  uint8_t* ring = smem + 2 * Q_BYTES;
+  uint8_t* sP = ring + (size_t)stages * 2 * KV_TILE;    // [2] tiles
+  uint64_t* q_full = (uint64_t*)(sP + 2 * P_BYTES);
+  uint64_t* kv_full = q_full + 1;
+  uint64_t* kv_empty = kv_full + stages;
+  uint64_t* s_full = kv_empty + stages;  // [2 tiles][NSB buffers]
+  uint64_t* p_full = s_full + 2 * NSB;   // [2]
+  uint64_t* pv_full = p_full + 2;        // [2]
+  uint64_t* drain = pv_full + 2;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int pairs = (p.q_blocks + 1) / 2;
+  const int BH = p.B * p.Hq;
+  int pb, bh;
+  if (p.raster == 0) {
+    pb = blockIdx.x % pairs;
+    bh = blockIdx.x / pairs;
+  } else {
+    pb = pairs - 1 - (int)(blockIdx.x / BH);
+    bh = blockIdx.x % BH;
+  }
+  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
+  int q0[2], nkb[2];
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    q0[t] = (2 * pb + t) * BM;
+    const int end = p.causal ? min(q0[t] + BM, p.S) : p.S;
+    nkb[t] = q0[t] < p.S ? (end + BN - 1) / BN : 0;
+  }
+  const int nblk = max(nkb[0], nkb[1]);
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&kv_full[s], 1);
+      tc::mbar_init(&kv_empty[s], 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      for (int b2 = 0; b2 < NSB; ++b2) tc::mbar_init(&s_full[t * NSB + b2], 1);
+      tc::mbar_init(&p_full[t], 128);
+      tc::mbar_init(&pv_full[t], 1);
+    }
+    tc::mbar_init(drain, 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(tmem_slot, 512);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::prefetch_tmap(&tmV);
+      tc::mbar_expect_tx(q_full, 2 * Q_BYTES);
+#pragma unroll
+      for (int t = 0; t < 2; ++t) {
+        const int qrow = b * p.S + q0[t];
+        tc::tma_load_2d(sQ + t * Q_BYTES, &tmQ, q_full, h * D, qrow);
+        tc::tma_load_2d(sQ + t * Q_BYTES + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
+      }
+      int j = 0;
+      for (; j < nblk; ++j) {
+        const int s = j % stages;
+        const uint32_t ph = (uint32_t)(j / stages) & 1u;
+        if (!tc::mbar_wait(&kv_empty[s], ph ^ 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          break;
+        }
+        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
+        uint8_t* sv = sk + KV_TILE;
+        tc::mbar_expect_tx(&kv_full[s], 2 * KV_TILE);
+        const int krow = b * p.S + j * BN;
+        tc::tma_load_2d(sk, &tmK, &kv_full[s], g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, &kv_full[s], g * D + 64, krow);
+        if constexpr (VT) {
+#pragma unroll
+          for (int a = 0; a < BN / 64; ++a)
+            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &kv_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
+        } else {
+          tc::tma_load_2d(sv, &tmV, &kv_full[s], g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, &kv_full[s], g * D + 64, krow);
+        }
+      }
+      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      for (int i = max(0, j - stages); i < j; ++i)
+        if (!tc::mbar_wait_drain(&kv_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
+      if (!ok) fail(RC_DEV_TIMEOUT_FULL);
+      int loaded = -1;  // highest key block whose K/V arrival was awaited
+      auto await_block = [&](int j) -> bool {
+        if (j <= loaded) return true;
+        if (!tc::mbar_wait(&kv_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status)) return false;
+        loaded = j;
+        tc::tc_fence_after();
+        return true;
+      };
+      auto issue_s = [&](int t, int j) {
+        const uint32_t sq = tc::smem_u32(sQ + t * Q_BYTES);
+        const uint32_t sk = tc::smem_u32(ring + (size_t)(j % stages) * 2 * KV_TILE);
+        const int sb = t * NSB + (j % NSB);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          tc::umma_bf16(tmem + (uint32_t)sb * BN, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
+                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&s_full[sb]);
+      };
+      auto issue_pv = [&](int t, int j) {
+        const uint32_t sp = tc::smem_u32(sP + t * P_BYTES);
+        const uint32_t sv = tc::smem_u32(ring + (size_t)(j % stages) * 2 * KV_TILE) + KV_TILE;
+        const uint32_t tO = tmem + O_BASE + t * D;
+        const uint32_t tP = tmem + (uint32_t)(t * NSB + (j % NSB)) * BN;  // P aliases its S buffer
+#pragma unroll
+        for (int ks = 0; ks < BN / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          uint64_t db;
+          if constexpr (VT)
+            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
+          else
+            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
+          if constexpr (PT)
+            tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+          else
+            tc::umma_bf16(tO, tc::sw128_desc(sp + (ks / 4) * (BM * 128) + off), db, idO,
+                          (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        tc::umma_commit(&pv_full[t]);
+      };
+      // prologue: S for the first NSB key blocks of both tiles
+      for (int j0 = 0; ok && j0 < NSB && j0 < nblk; ++j0) {
+        ok = await_block(j0);
+        if (ok)
+          for (int t = 0; t < 2; ++t)
+            if (j0 < nkb[t]) issue_s(t, j0);
+      }
+      for (int j = 0; ok && j < nblk; ++j) {
+        for (int t = 0; t < 2; ++t) {
+          if (j >= nkb[t]) continue;
+          if (!tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          tc::tc_fence_after();
+          issue_pv(t, j);
+          if (j + NSB < nkb[t]) {
+            if (!await_block(j + NSB)) {
+              ok = false;
+              break;
+            }
+            issue_s(t, j + NSB);
+          }
+        }
+        if (!ok) break;
+        tc::umma_commit(&kv_empty[j % stages]);
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(drain);
+        if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else if (warp >= 2) {
+    const int t = (warp - 2) / 4;  // query tile of this warpgroup
+    const int qd = warp & 3;
+    const int row = 32 * qd + lane;
+    const int qi = q0[t] + row;
+    const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+    const uint32_t tO = tmem + lane_base + O_BASE + t * D;
+    uint8_t* rowp0 = sP + t * P_BYTES + (row / 8) * 1024 + (row % 8) * 128;
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int j = 0; j < nkb[t]; ++j) {
+      const uint32_t tS = tmem + lane_base + (uint32_t)(t * NSB + (j % NSB)) * BN;
+      if (!tc::mbar_wait(&s_full[t * NSB + (j % NSB)], (uint32_t)(j / NSB) & 1u, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        ok = false;
+        break;
+      }
+      tc::tc_fence_after();
+      const int k0 = j * BN;
+      // keys [k0, k0 + nvis) of this block are visible to query qi
+      int nvis = min(BN, p.S - k0);
+      if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
+      // the whole S row in registers: one TMEM round trip
+      uint32_t r[BN];
+#pragma unroll
+      for (int q = 0; q < BN; q += 16) tc::tmem_ld16(tS + q, *reinterpret_cast<uint32_t(*)[16]>(&r[q]));
+      tc::tmem_ld_wait();
+      if (nvis < BN) {
+#pragma unroll
+        for (int i = 0; i < BN; ++i)
+          if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
+      }
+      // row maximum: 8 independent partial maxima, then combine
+      float pm[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(r[u]);
+#pragma unroll
+      for (int i = 8; i < BN; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(r[i]));
+      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      const float mxs = mx * p.scale_log2;
+      float factor = 1.f;
+      if (m_ref == -INFINITY) {
+        m_ref = mxs;  // first visible scores: O and l are still zero
+      } else if (mxs > m_ref + kRescaleLog2) {
+        factor = exp2f(m_ref - mxs);
+        m_ref = mxs;
+      }
+      const bool rescale = __any_sync(0xffffffffu, factor != 1.f);
+      // pv_full completes once per key block (P_t V of that block). It is
+      // observed phase by phase, so a parity wait never meets a barrier more
+      // than one phase ahead: phase j-1 is awaited in iteration j, before the
+      // O rescale when there is one (O must hold P_t V of block j-1), before
+      // overwriting P's shared-memory buffer, or else after the probabilities
+      // are written. P V of block j is only issued after this thread's p_full.
+      bool pv_seen = j == 0;
+      auto await_pv = [&]() -> bool {
+        if (pv_seen) return true;
+        pv_seen = true;
+        if (!tc::mbar_wait(&pv_full[t], (uint32_t)(j - 1) & 1u, abort_flag, status)) {
+          if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+          return false;
+        }
+        tc::tc_fence_after();
+        return true;
+      };
+      if (rescale || !PT) {
+        if (!await_pv()) {
+          ok = false;
+          break;
+        }
+      }
+      if (rescale) {
+#pragma unroll 1
+        for (int c = 0; c < D; c += 16) {
+          uint32_t r[16];
+          tc::tmem_ld16(tO + c, r);
+          tc::tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
+          tc::tmem_st16(tO + c, r);
+        }
+        tc::tmem_st_wait();
+      }
+      // pass 2: probabilities -> P (bf16) and the row sum
+      const float mref = m_ref == -INFINITY ? 0.f : m_ref;
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < BN; c += 32) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          // masked scores are -inf: 2^-inf = +0
+          const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i]), p.scale_log2, -mref));
+          const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i + 1]), p.scale_log2, -mref));
+          ls[(i / 2) % 4] += p0 + p1;
+          pk[i / 2] = pack2(p0, p1);
+        }
+        if constexpr (PT) {
+          // P for keys [c, c + 32) goes to columns [c/2, c/2 + 16) of the S row (already in registers)
+          tc::tmem_st16(tS + c / 2, pk);
+        } else {
+#pragma unroll
+          for (int h2 = 0; h2 < 2; ++h2) {
+            const int cc = c + 16 * h2;
+            uint8_t* rowp = rowp0 + (cc / 64) * (BM * 128);
+            const int ch = (cc % 64) / 8;
+            *reinterpret_cast<uint4*>(rowp + ((ch ^ (row % 8)) * 16)) =
+                make_uint4(pk[8 * h2], pk[8 * h2 + 1], pk[8 * h2 + 2], pk[8 * h2 + 3]);
+            *reinterpret_cast<uint4*>(rowp + (((ch + 1) ^ (row % 8)) * 16)) =
+                make_uint4(pk[8 * h2 + 4], pk[8 * h2 + 5], pk[8 * h2 + 6], pk[8 * h2 + 7]);
+          }
+        }
+      }
+      l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+      if constexpr (PT) tc::tmem_st_wait();
+      if (!await_pv()) {
+        ok = false;
+        break;
+      }
+      tc::tc_fence_before();
+      if constexpr (!PT) tc::fence_proxy_async_smem();
+      tc::mbar_arrive(&p_full[t]);
+    }
+    if (ok && nkb[t] > 0) {
+      if (tc::mbar_wait(&pv_full[t], (uint32_t)(nkb[t] - 1) & 1u, abort_flag, status)) {
+        tc::tc_fence_after();
+        const float inv_l = l > 0.f ? 1.f / l : 0.f;
+        const bool row_ok = qi < p.S;
+        __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
+#pragma unroll 1
+        for (int c = 0; c < D; c += 16) {
+          uint32_t r[16];
+          tc::tmem_ld16(tO + c, r);
+          tc::tmem_ld_wait();
+          uint32_t pk[8];
+#pragma unroll
+          for (int i = 0; i < 16; i += 2)
+            pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
+          if (row_ok) {
+            *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
+        }
+        if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
+      } else if (!*abort_flag) {
+        fail(RC_DEV_TIMEOUT_ACCUM);
+      }
+    }
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
 // Vt[(b*Hkv + g)*D + d][s] = V[b][s][g][d] (64 x 64 tiles through shared memory).
 __global__ void transpose_v_kernel(const __nv_bfloat16* __restrict__ V, int S, int Hkv, __nv_bfloat16* __restrict__ Vt) {
   __shared__ __nv_bfloat16 tile[64][66];
@@ -354,14 +728,14 @@ __global__ void transpose_v_kernel(const __nv_bfloat16* __restrict__ V, int S, i
   }
 }
 
-size_t smem_bytes(int bn, int stages) {
-  return (size_t)BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)BM * bn * 2 + 1024 + 256;
+size_t smem_bytes(int bn, int stages, int qtiles) {
+  return (size_t)qtiles * BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)qtiles * BM * bn * 2 + 1024 + 256;
 }
 
-template <int BN, bool VT>
+template <int BN, bool VT, bool PINGPONG, bool PT = false, bool SDB = false>
 rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
                  float* lse, const LaunchCtx& c) {
-  auto kern = attn_kernel<BN, VT>;
+  auto kern = PINGPONG ? attn2_kernel<BN, VT, PT, SDB> : attn_kernel<BN, VT>;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
@@ -390,9 +764,10 @@ rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const vo
   p.O = (__nv_bfloat16*)O;
   p.lse = lse;
   p.status = c.status;
-  const long long ctas = (long long)p.B * p.Hq * p.q_blocks;
+  const long long ctas = (long long)p.B * p.Hq * (PINGPONG ? (p.q_blocks + 1) / 2 : p.q_blocks);
   if (ctas > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
-  kern<<<(unsigned)ctas, kThreads, smem_bytes(BN, k.stages), (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  const size_t smem = smem_bytes(BN, k.stages, PINGPONG ? 2 : 1) - (PT ? (size_t)2 * BM * BN * 2 : 0);
+  kern<<<(unsigned)ctas, PINGPONG ? kThreads2 : kThreads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention launch: %s", cudaGetErrorString(e));
   return RC_OK;
@@ -415,9 +790,27 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
     Vuse = workspace;
   }
   const bool vt = k.layout == 1;
-  if (k.tile_n == 64) return vt ? attn::launch<64, true>(k, d, Q, K, Vuse, O, lse, c)
-                                : attn::launch<64, false>(k, d, Q, K, Vuse, O, lse, c);
-  if (k.tile_n == 128) return vt ? attn::launch<128, true>(k, d, Q, K, Vuse, O, lse, c)
-                                 : attn::launch<128, false>(k, d, Q, K, Vuse, O, lse, c);
+  const bool pp = k.tile_m == 256;  // two query tiles per CTA, ping-pong softmax
+  if (pp && k.stages < 2) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: ping-pong needs >= 2 stages");
+  const bool pt = k.location == 1;  // P kept in tensor memory
+  if (pt && !pp) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: P in TMEM needs the ping-pong kernel");
+  if (k.unroll == 2) {  // two key blocks in flight per query tile
+    if (!(pp && pt && k.tile_n == 64 && k.stages >= 4))
+      return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: unroll 2 needs 2 query tiles, P in TMEM, BN 64, 4 stages");
+    return vt ? attn::launch<64, true, true, true, true>(k, d, Q, K, Vuse, O, lse, c)
+              : attn::launch<64, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c);
+  }
+#define RC_ATT(BN)                                                                                  \
+  if (k.tile_n == BN) {                                                                             \
+    if (pp && pt) return vt ? attn::launch<BN, true, true, true>(k, d, Q, K, Vuse, O, lse, c)       \
+                            : attn::launch<BN, false, true, true>(k, d, Q, K, Vuse, O, lse, c);     \
+    if (pp) return vt ? attn::launch<BN, true, true>(k, d, Q, K, Vuse, O, lse, c)                   \
+                      : attn::launch<BN, false, true>(k, d, Q, K, Vuse, O, lse, c);                 \
+    return vt ? attn::launch<BN, true, false>(k, d, Q, K, Vuse, O, lse, c)                          \
+              : attn::launch<BN, false, false>(k, d, Q, K, Vuse, O, lse, c);                        \
+  }
+  RC_ATT(64)
+  RC_ATT(128)
+#undef RC_ATT
   return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: key block %d", k.tile_n);
 }

@@ -23,9 +23,10 @@ def att_op(B, S, Hq, Hkv, causal=True):
     return rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=128, causal=int(causal))
 
 
-def sched(op, bn, stages, raster, layout):
-    return op.schedule(rc.T(rc.T_TILE_SIZE, bn, axis=1), rc.T(rc.T_PIPELINE_STAGES, stages),
-                       rc.T(rc.T_LOOP_ORDER, raster, group=1), rc.T(rc.T_LAYOUT, layout))
+def sched(op, bn, stages, raster, layout, bm=128, p_tmem=0, unroll=1):
+    return op.schedule(rc.T(rc.T_TILE_SIZE, bm, axis=0), rc.T(rc.T_TILE_SIZE, bn, axis=1),
+                       rc.T(rc.T_PIPELINE_STAGES, stages), rc.T(rc.T_LOOP_ORDER, raster, group=1),
+                       rc.T(rc.T_LAYOUT, layout), rc.T(rc.T_COMPUTE_LOCATION, p_tmem), rc.T(rc.T_UNROLL, unroll))
 
 
 def run(op, s, Q, K, V):
@@ -44,16 +45,19 @@ def test_attention_schedule_sweep(B, S, Hq, Hkv, causal):
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=causal)
     op = att_op(B, S, Hq, Hkv, causal)
     n = 0
-    for bn, st, ra, lay in itertools.product((64, 128), (2, 3), (0, 1), (0, 1)):
+    for bm, bn, st, ra, lay, pt, un in itertools.product((128, 256), (64, 128), (1, 2, 3, 4), (0, 1), (0, 1), (0, 1),
+                                                         (1, 2)):
         try:
-            s = sched(op, bn, st, ra, lay)
+            s = sched(op, bn, st, ra, lay, bm, pt, un)
         except rc.RcError:
-            continue  # illegal here (shared memory, or S % 8 for the transposed V)
+            continue  # illegal here (shared memory, S % 8 for the transposed V, variant combinations)
         O, L = run(op, s, Q, K, V)
-        assert rel_err(O, O_ref) <= TOL, (bn, st, ra, lay, rel_err(O, O_ref))
-        assert rel_err(L, L_ref) <= TOL_LSE, (bn, st, ra, lay)
+        assert rel_err(O, O_ref) <= TOL, (bm, bn, st, ra, lay, pt, un, rel_err(O, O_ref))
+        assert rel_err(L, L_ref) <= TOL_LSE, (bm, bn, st, ra, lay, pt, un)
         n += 1
-    assert n >= 6
+    assert n >= 16
+    with pytest.raises(rc.RcError):  # one K/V stage cannot feed the ping-pong kernel
+        sched(op, 64, 1, 0, 0, 256)
 
 
 def test_attention_single_token_and_no_lse():
@@ -74,7 +78,9 @@ def test_attention_full_size_sampled_queries():
     qpos = np.array([0, 1, 63, 64, 127, 128, 129, 1000, 1023, 1024, 2000, 2046, 2047], dtype=np.int64)
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=True, qpos=qpos)
     op = att_op(B, S, Hq, Hkv)
-    for s in [op.schedule(), sched(op, 128, 2, 1, 0), sched(op, 64, 3, 0, 1)]:
+    for s in [op.schedule(), sched(op, 128, 2, 1, 0), sched(op, 64, 3, 0, 1), sched(op, 64, 3, 1, 0, 256),
+              sched(op, 64, 2, 1, 1, 256), sched(op, 128, 2, 1, 0, 256, 1), sched(op, 64, 3, 1, 1, 256, 1),
+              sched(op, 64, 4, 1, 0, 256, 1, 2), sched(op, 64, 5, 0, 1, 256, 1, 2)]:
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
