@@ -49,7 +49,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mlp", choices=["mlp", "attention", "conv2d", "moe", "gemm_f32"])
-    ap.add_argument("--samples", type=int, default=400, help="schedules the search measures")
+    ap.add_argument("--samples", type=int, default=1200, help="schedules the search measures")
     ap.add_argument("--cpu-sample", type=int, default=0,
                     help="size of the CPU-oracle sample (rows/queries/pixels/tokens; 0 = workload default, "
                          "-1 = skip)")
@@ -58,7 +58,7 @@ def parse():
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--ops", default=None,
                     help="other workloads to search and report ('' = none; default: all others for mlp)")
-    ap.add_argument("--op-samples", type=int, default=48, help="schedules measured per extra op")
+    ap.add_argument("--op-samples", type=int, default=160, help="schedules measured per extra op")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
 
@@ -340,12 +340,17 @@ def search_best(op, io, samples, seed=0):
 def extra_ops(names, samples, peak_tf):
     """Search each other workload briefly and report its best schedule."""
     import torch
+
+    from paper_2506_01374_gb300 import rc
     out = {}
     for name in names:
         wl = Workload(name)
         io = wl.device_io()
         _, best, _, n, cps = search_best(wl.op, io, samples)
         m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
+        if m.status != rc.OK:
+            out[name] = {"workload": wl.label, "error": rc.STATUS_NAMES.get(m.status, m.status)}
+            continue
         tf = wl.op.info["flops"] / (m.ms_median * 1e-3) / 1e12
         peak = FP32_ALU_TFLOPS if wl.bound == "alu" else peak_tf
         out[name] = {"workload": wl.label, "tflops": tf, "ms": m.ms_median, "bound": wl.bound, "peak": peak,

@@ -342,10 +342,13 @@ class Search:
         return [Schedule(nxt[i], owned=False) for i in range(n.value)]
 
     def best(self):
+        """Best measured schedule (an owned copy, valid after the search is gone) and its measurement."""
         h = _P()
         m = Measurement()
         _check(lib().rc_search_best(self.h, C.byref(h), C.byref(m)), "rc_search_best")
-        return Schedule(h.value, owned=False), m
+        c = _P()
+        _check(lib().rc_schedule_clone(h.value, C.byref(c)), "rc_schedule_clone")
+        return Schedule(c.value), m
 
     def stats(self) -> dict:
         s = SearchStats()

@@ -152,3 +152,18 @@ def test_result_count_mismatch_is_an_error():
     s.step([])
     with pytest.raises(rc.RcError):
         s.step([])
+
+
+def test_best_schedule_outlives_the_search():
+    op = make_op()
+    s = rc.Search(op, seed=4)
+    res = []
+    for _ in range(5):
+        nxt = s.step(res)
+        res = [meas(lib_program(x)) for x in nxt]
+    best, m = s.best()
+    knobs = best.knobs()
+    del s
+    import gc
+    gc.collect()
+    assert best.knobs() == knobs and best.hash == m.sched_hash
