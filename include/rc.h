@@ -239,6 +239,14 @@ rc_status rc_run_host(const rc_op* op, const rc_schedule* s, const rc_tensors* h
  * word is cleared). */
 rc_status rc_op_check(const rc_op* op, void* stream);
 
+/* Self-test of the bounded device waits (no paper counterpart): one CTA
+ * waits on an mbarrier phase that nothing completes, with a wait limit of
+ * wait_ms (0 < wait_ms <= 2000). The wait gives up, records a timeout in a
+ * device status word and the call returns RC_ERR_DEVICE_TIMEOUT after
+ * synchronising `stream`; RC_OK would mean the wait did not give up. The
+ * CUDA context stays usable. Allocates and frees a 4-byte status word. */
+rc_status rc_selftest_bounded_wait(double wait_ms, void* stream);
+
 /* ---------------------------------------------------------- measurement -- */
 
 typedef struct {

@@ -284,9 +284,10 @@ extern "C" void rc_op_destroy(rc_op* op) {
 }
 
 extern "C" rc_status rc_run(const rc_op* op, const rc_schedule* s, const rc_tensors* io, void* stream) {
+  if (!op || !s) return rc_fail(RC_ERR_INVALID_ARG, "rc_run: NULL op or schedule");
+  RC_TRY(check_io(op, io));  // host-side argument checks come before any CUDA call
   LaunchCtx c;
   RC_TRY(prepare(op, s, &c, stream));
-  RC_TRY(check_io(op, io));
   return run_impl(op, s, io, c);
 }
 
@@ -299,9 +300,10 @@ rc_status rc_mark_stage(const LaunchCtx& c) {
 extern "C" rc_status rc_run_profiled(const rc_op* op, const rc_schedule* s, const rc_tensors* io, void* stream,
                                      double* stage_ms, size_t cap, size_t* n_stages) {
   if (!stage_ms || !n_stages) return rc_fail(RC_ERR_INVALID_ARG, "rc_run_profiled: NULL output");
+  if (!op || !s) return rc_fail(RC_ERR_INVALID_ARG, "rc_run_profiled: NULL op or schedule");
+  RC_TRY(check_io(op, io));
   LaunchCtx c;
   RC_TRY(prepare(op, s, &c, stream));
-  RC_TRY(check_io(op, io));
   void* ev[RC_MAX_STAGES + 1] = {};
   for (int i = 0; i <= RC_MAX_STAGES; ++i) {
     rc_status st = cuda_err(cudaEventCreate((cudaEvent_t*)&ev[i]), "cudaEventCreate");

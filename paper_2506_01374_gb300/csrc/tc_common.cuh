@@ -58,8 +58,8 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 
 // Wait for the phase with the given parity to complete. Returns false when
 // the wait gave up (timeout, CTA abort flag, or launch status already set).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          volatile int* status) {
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                              volatile int* status, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   for (uint32_t it = 1;; ++it) {
@@ -67,9 +67,14 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     if ((it & 63) == 0) {
       if (*abort_flag) return false;
       if (*status) return false;
-      if (globaltimer() - t0 > kWaitNs) return false;
+      if (globaltimer() - t0 > limit_ns) return false;
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          volatile int* status) {
+  return mbar_wait_for(bar, parity, abort_flag, status, kWaitNs);
 }
 
 // Wait without abort checks, bounded by time only (teardown draining).

@@ -135,6 +135,7 @@ _PROTOS = {
     "rc_search_destroy": (None, [_P]),
     "rc_moe_route_noalloc": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int64, C.c_int64, C.c_int32, _P, _P, _P, _P,
                                        _P]),
+    "rc_selftest_bounded_wait": (C.c_int, [C.c_double, _P]),
     "rc_last_error": (C.c_char_p, []),
     "rc_version": (C.c_char_p, []),
 }
@@ -367,6 +368,11 @@ def moe_route_noalloc(logits, tokens: int, experts: int, top_k: int, ids, weight
     _check(lib().rc_moe_route_noalloc(_ptr(logits), int(logits_fp32), tokens, experts, top_k, int(renorm), _ptr(ids),
                                       _ptr(weights), _ptr(offsets), _ptr(perm), _stream(stream)),
            "rc_moe_route_noalloc")
+
+
+def selftest_bounded_wait(wait_ms: float = 50.0, stream=None) -> int:
+    """Run the bounded-wait self-test; returns its status (ERR_DEVICE_TIMEOUT means it worked)."""
+    return lib().rc_selftest_bounded_wait(wait_ms, _stream(stream))
 
 
 def version() -> str:
