@@ -116,6 +116,8 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       gemm_common({64, 80, 160});
       v.push_back({RC_T_SPLIT_K, 0, {1, 3, 5}, {}});
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      // implicit zero padding (one 4-D box), or a padded copy read as one 4-D box or as row boxes
+      v.push_back({RC_T_LAYOUT, 0, {0, 1, 2}, {}});
       break;
     case RC_OP_ATTENTION:
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256 = two query tiles, ping-pong softmax
@@ -360,6 +362,7 @@ size_t rc_workspace_bytes(const rc_op_s* op, const rc_schedule_s* s) {
     case RC_OP_CONV2D: {
       const size_t rows = (size_t)d.img_n * d.img_h * d.img_w;
       size_t b = 0;
+      if (k && k[0].layout >= 1) b += align256(2ull * d.img_n * (d.img_h + 2 * d.pad) * (d.img_w + 2 * d.pad) * d.c_in);
       if (k && k[0].split_k > 1) b += align256(4ull * k[0].split_k * rows * d.c_out);
       if (k && (!k[0].fuse || k[0].split_k > 1)) b += align256(2ull * rows * d.c_out);
       return b;

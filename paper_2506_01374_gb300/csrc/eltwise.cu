@@ -83,6 +83,20 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits,
   }
 }
 
+// xp[n][p + pad][q + pad][c] = x[n][p][q][c], zero border of width `pad`.
+__global__ void pad_nhwc_kernel(const uint4* __restrict__ x, int64_t N, int64_t H, int64_t W, int64_t C16,
+                                int64_t pad, uint4* __restrict__ xp) {
+  const int64_t Hp = H + 2 * pad, Wp = W + 2 * pad;
+  const int64_t total = N * Hp * Wp * C16;
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < total; v += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t c = v % C16;
+    const int64_t pix = v / C16;
+    const int64_t q = pix % Wp, p = (pix / Wp) % Hp, n = pix / (Wp * Hp);
+    const int64_t ih = p - pad, iw = q - pad;
+    xp[v] = (ih >= 0 && ih < H && iw >= 0 && iw < W) ? x[((n * H + ih) * W + iw) * C16 + c] : make_uint4(0, 0, 0, 0);
+  }
+}
+
 __global__ void f32_to_bf16_kernel(const float* __restrict__ in, int64_t n4, __nv_bfloat16* __restrict__ out) {
   for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n4; v += (int64_t)gridDim.x * blockDim.x) {
     const float4 s = reinterpret_cast<const float4*>(in)[v];
@@ -138,6 +152,15 @@ rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, const Lau
   if (n % 4) return rc_fail(RC_ERR_UNSUPPORTED_OP, "f32->bf16: n %% 4 != 0");
   f32_to_bf16_kernel<<<grid_for(n / 4, c), 256, 0, (cudaStream_t)c.stream>>>(in, n / 4, (__nv_bfloat16*)out);
   return launched("f32->bf16");
+}
+
+rc_status rc_launch_pad_nhwc(const void* x, int64_t N, int64_t H, int64_t W, int64_t C, int64_t pad, void* xp,
+                              const LaunchCtx& c) {
+  if (C % 8) return rc_fail(RC_ERR_UNSUPPORTED_OP, "pad: C %% 8 != 0");
+  const int64_t total = N * (H + 2 * pad) * (W + 2 * pad) * (C / 8);
+  pad_nhwc_kernel<<<grid_for(total, c), 256, 0, (cudaStream_t)c.stream>>>((const uint4*)x, N, H, W, C / 8, pad,
+                                                                          (uint4*)xp);
+  return launched("pad");
 }
 
 rc_status rc_launch_l2_flush(void* buf, size_t bytes, void* stream) {

@@ -107,8 +107,9 @@ enum TcEpilogue {
   TC_EPI_SCALE_ATOMIC = 4  // row_scale[row] * D atomically added to fp32 out[row_map[row]]
 };
 enum TcAMode {
-  TC_A_2D = 0,    // A is a row-major [M][K] matrix
-  TC_A_CONV = 1   // A rows are output pixels of an NHWC 'same' conv; K = (r, s, c)
+  TC_A_2D = 0,         // A is a row-major [M][K] matrix
+  TC_A_CONV = 1,       // A rows are output pixels of an NHWC 'same' conv; K = (r, s, c); one 4-D box
+  TC_A_CONV_ROWS = 2   // as TC_A_CONV over an explicitly padded input, one 2-D box per image row
 };
 struct TcGemmArgs {
   int64_t M, N, K;         // N = UMMA columns of the whole problem (2I for SwiGLU)
@@ -120,8 +121,10 @@ struct TcGemmArgs {
   int a_mode;              // TcAMode
   const void* bias;        // TC_EPI_BIAS_SILU: bf16[N] (NULL = no bias)
   int silu;                // TC_EPI_BIAS_SILU: 1 = apply SiLU after the bias
-  // conv geometry (TC_A_CONV)
+  // conv geometry (TC_A_CONV); padded = 1: A is an explicitly padded copy
+  // [N][H+2pad][W+2pad][C] read without out-of-range coordinates
   int64_t img_n, img_h, img_w, c_in, kr, ks, pad;
+  int padded;
   // grouped (MoE) mode: groups > 0 means rows of A are partitioned into
   // `groups` segments by offsets[g] (device int32[groups+1]); segment g uses
   // B rows [g*b_group_rows, (g+1)*b_group_rows).
@@ -159,3 +162,6 @@ rc_status rc_launch_moe_gather(const void* X, const int* perm, int64_t rows, int
 rc_status rc_launch_moe_combine(const void* Y, const float* w, const int* inv_perm, int64_t T,
                                 int64_t H, int topk, void* out, int vec, const LaunchCtx& c);
 rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, const LaunchCtx& c);
+// Explicitly zero-padded copy of an NHWC tensor ([N][H+2p][W+2p][C]).
+rc_status rc_launch_pad_nhwc(const void* x, int64_t N, int64_t H, int64_t W, int64_t C, int64_t pad, void* xp,
+                             const LaunchCtx& c);

@@ -165,6 +165,15 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       a.ks = d.ks;
       a.pad = d.pad;
       a.bias = p[2];
+      if (k.layout >= 1) {
+        // layouts 1 and 2: explicitly zero-padded copy of x, read without out-of-range
+        // TMA coordinates, as one 4-D box (1) or one 2-D box per image row (2)
+        void* xp = ws.take(2ull * d.img_n * (d.img_h + 2 * d.pad) * (d.img_w + 2 * d.pad) * d.c_in);
+        RC_TRY(rc_launch_pad_nhwc(p[0], d.img_n, d.img_h, d.img_w, d.c_in, d.pad, xp, c));
+        a.A = xp;
+        a.padded = 1;
+        if (k.layout == 2) a.a_mode = TC_A_CONV_ROWS;
+      }
       const bool silu = (d.flags & RC_EPI_SILU) != 0;
       if (k.split_k > 1) {
         void* part = ws.take(4ull * k.split_k * rows * d.c_out);

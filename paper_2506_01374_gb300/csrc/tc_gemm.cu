@@ -52,15 +52,17 @@ rc_status encode_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t r
 }
 
 // NHWC activation x[n][h][w][c] seen as a 4-D tensor {c, w, h, n}; one box is
-// 64 channels x the full row width x (128 / w) rows of one image = the 128
-// output pixels of an M tile, shifted by the filter tap (r, s).
-rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uint64_t h, uint64_t n) {
+// 64 channels x box_w columns x box_h rows of one image = the 128 output
+// pixels of an M tile, shifted by the filter tap (r, s). For an explicitly
+// padded input the tensor is (w + 2 pad) wide and (h + 2 pad) high.
+rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uint64_t h, uint64_t n,
+                      uint64_t box_w, uint64_t box_h) {
   EncodeTiledFn fn;
   RC_TRY(get_encode(&fn));
   if ((uintptr_t)x % 16 || (c * 2) % 16) return rc_fail(RC_ERR_INVALID_ARG, "TMA: 16-byte alignment");
   cuuint64_t dims[4] = {c, w, h, n};
   cuuint64_t strides[3] = {c * 2, w * c * 2, h * w * c * 2};
-  cuuint32_t box[4] = {64, (cuuint32_t)w, (cuuint32_t)(128 / w), 1};
+  cuuint32_t box[4] = {64, (cuuint32_t)box_w, (cuuint32_t)box_h, 1};
   cuuint32_t estr[4] = {1, 1, 1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -75,7 +77,7 @@ rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const Launch
   if (a.M > 0x7fffffff || a.N > 0x7fffffff || a.K > 0x7fffffff)
     return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: dimension exceeds 2^31");
   if (k.stages < 1) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: stages < 1");
-  if (a.a_mode == TC_A_CONV) return tc_dispatch_conv(k, a, c);
+  if (a.a_mode == TC_A_CONV || a.a_mode == TC_A_CONV_ROWS) return tc_dispatch_conv(k, a, c);
   if (a.groups > 0) return tc_dispatch_grouped(k, a, c);
   return tc_dispatch_dense(k, a, c);
 }

@@ -43,8 +43,9 @@ struct Params {
   int silu;
   int swiglu_I;         // SwiGLU: output width I (also the offset of the up rows)
   int out_cols;         // columns of D that exist (store bound)
-  // implicit-GEMM convolution
-  int img_hw, img_w, cblocks, ks, pad;
+  // implicit-GEMM convolution (pad = coordinate shift of the filter taps;
+  // pad_rows = border width of an explicitly padded input)
+  int img_hw, img_w, cblocks, ks, pad, pad_rows;
   // grouped rows (MoE)
   const int* offsets;
   int groups;
@@ -274,6 +275,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int img = it.row0 / p.img_hw;
             const int prow = (it.row0 - img * p.img_hw) / p.img_w;
             tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
+          } else if constexpr (AMODE == TC_A_CONV_ROWS) {
+            // padded input [N][Hp][Wp][C] as rows of pixels: image row i of the tile, shifted by (r, s)
+            const int rs = kb / p.cblocks, cb = kb - rs * p.cblocks;
+            const int rr = rs / p.ks, ss = rs - rr * p.ks;
+            const int img = it.row0 / p.img_hw;
+            const int prow = (it.row0 - img * p.img_hw) / p.img_w;
+            const int wp = p.img_w + 2 * p.pad_rows, hp = p.img_hw / p.img_w + 2 * p.pad_rows;
+            for (int i = 0; i < BM / p.img_w; ++i)
+              tc::tma_load_2d(sa + i * p.img_w * 128, &tmA, &full[s], cb * 64,
+                              (img * hp + prow + i + rr) * wp + ss);
           } else {
             tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, it.row0);
           }
@@ -366,7 +377,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ------------------------------------------------------------------ host --
 rc_status encode_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows);
-rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uint64_t h, uint64_t n);
+rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uint64_t h, uint64_t n,
+                      uint64_t box_w, uint64_t box_h);
 
 template <typename Kern>
 rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tmB, const Params& p, int stages,
@@ -406,7 +418,11 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   }
   CUtensorMap tmA, tmB;
   if constexpr (AMODE == TC_A_CONV) {
-    RC_TRY(encode_conv(&tmA, a.A, a.c_in, a.img_w, a.img_h, a.img_n));
+    const uint64_t extra = a.padded ? 2 * (uint64_t)a.pad : 0;  // padded copy: no out-of-range coordinates
+    RC_TRY(encode_conv(&tmA, a.A, a.c_in, a.img_w + extra, a.img_h + extra, a.img_n, a.img_w, 128 / a.img_w));
+  } else if constexpr (AMODE == TC_A_CONV_ROWS) {
+    const uint64_t rows = (uint64_t)a.img_n * (a.img_h + 2 * a.pad) * (a.img_w + 2 * a.pad);
+    RC_TRY(encode_2d(&tmA, a.A, a.c_in, rows, (uint32_t)a.img_w));
   } else {
     RC_TRY(encode_2d(&tmA, a.A, a.K, a.M, BM));
   }
@@ -434,12 +450,13 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.silu = a.silu;
   p.swiglu_I = (int)(a.N / 2);
   p.out_cols = out_w;
-  if constexpr (AMODE == TC_A_CONV) {
+  if constexpr (AMODE == TC_A_CONV || AMODE == TC_A_CONV_ROWS) {
     p.img_hw = (int)(a.img_h * a.img_w);
     p.img_w = (int)a.img_w;
     p.cblocks = (int)(a.c_in / 64);
     p.ks = (int)a.ks;
-    p.pad = (int)a.pad;
+    p.pad = a.padded ? 0 : (int)a.pad;
+    p.pad_rows = (int)a.pad;
   }
   p.offsets = a.offsets;
   p.groups = a.groups;

@@ -24,9 +24,10 @@ def conv_op(N, H, W, Cin, Cout, flags=rc.EPI_BIAS | rc.EPI_SILU):
                  flags=flags)
 
 
-def sched(op, tile_n, stages, split_k=1, fuse=1, persistent=0):
+def sched(op, tile_n, stages, split_k=1, fuse=1, persistent=0, layout=0):
     return op.schedule(rc.T(rc.T_TILE_SIZE, tile_n, axis=1), rc.T(rc.T_PIPELINE_STAGES, stages),
-                       rc.T(rc.T_SPLIT_K, split_k), rc.T(rc.T_FUSE, fuse), rc.T(rc.T_PARALLEL, persistent))
+                       rc.T(rc.T_SPLIT_K, split_k), rc.T(rc.T_FUSE, fuse), rc.T(rc.T_PARALLEL, persistent),
+                       rc.T(rc.T_LAYOUT, layout))
 
 
 @pytest.mark.parametrize("N,H,W,Cin", [(2, 16, 16, 128), (1, 16, 8, 64), (1, 4, 32, 64), (1, 2, 64, 192),
@@ -37,12 +38,12 @@ def test_conv_geometries(N, H, W, Cin):
     ref = oracle.conv2d_nhwc_bf16(x, w, b)
     op = conv_op(N, H, W, Cin, Cout)
     dx, dw, db = to_dev(x), to_dev(w), to_dev(b)
-    for tn, st in itertools.product((64, 80, 160), (1, 2, 4)):
+    for tn, st, lay in itertools.product((64, 80, 160), (1, 2, 4), (0, 1, 2)):
         dy = empty_bf16(N, H, W, Cout).fill_(0x7FC0)
-        op.run(sched(op, tn, st), [dx, dw, db, dy])
+        op.run(sched(op, tn, st, layout=lay), [dx, dw, db, dy])
         op.check()
         err = rel_err(from_dev_bf16(dy).reshape(-1, Cout), ref)
-        assert err <= TOL, (tn, st, err)
+        assert err <= TOL, (tn, st, lay, err)
 
 
 def test_conv_split_k_and_unfused_epilogue():
@@ -84,7 +85,8 @@ def test_conv_full_size_sampled_pixels():
     pix = np.unique(np.concatenate([corners, rng.integers(0, N * H * W, 120)])).astype(np.int64)
     ref = oracle.conv2d_nhwc_bf16(x, w, b, pix=pix)
     for s in [op.schedule(), sched(op, 160, 4), sched(op, 80, 3, 5, 1), sched(op, 64, 6, 3, 0),
-              sched(op, 160, 3, 1, 1, 1), sched(op, 80, 4, 3, 1, 1)]:
+              sched(op, 160, 3, 1, 1, 1), sched(op, 80, 4, 3, 1, 1), sched(op, 80, 3, 1, 1, 0, 1),
+              sched(op, 160, 4, 3, 0, 1, 1), sched(op, 80, 4, 1, 1, 1, 2), sched(op, 160, 3, 3, 0, 0, 2)]:
         op.run(s, [dx, dw, db, dy])
         op.check()
         got = from_dev_bf16(dy).reshape(-1, C)[pix]
