@@ -149,7 +149,9 @@ void rc_op_destroy(rc_op* op);
 
 typedef enum {
   RC_T_TILE_SIZE = 0,        /* axis 0/1/2 = M/N/K tile; value[0] = extent */
-  RC_T_PARALLEL = 1,         /* value[0]: 0 = one CTA per output tile, 1 = persistent CTAs */
+  RC_T_PARALLEL = 1,         /* value[0]: GEMM-shaped ops: 0 = one CTA per output tile, 1 = persistent
+                              * CTAs; ATTENTION: 0 = one UMMA-issuing warp per CTA, 1 = one per
+                              * query tile (two query tiles, P in TMEM only) */
   RC_T_COMPUTE_LOCATION = 2, /* value[0]: where producer work runs (op specific, see knobs) */
   RC_T_UNROLL = 3,           /* value[0]: unroll factor of the innermost reduction loop */
   RC_T_LOOP_ORDER = 4,       /* value[0]: tile raster 0 = M fastest, 1 = N fastest; value[1] = group */

@@ -127,6 +127,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // V as [keys][d] or transposed to [d][keys]
       v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});  // P stored in shared or tensor memory
       v.push_back({RC_T_UNROLL, 0, {1, 2}, {}});  // key blocks in flight per query tile
+      v.push_back({RC_T_PARALLEL, 0, {0, 1}, {}});  // one UMMA-issuing warp per CTA, or one per query tile
       break;
     case RC_OP_MOE_ROUTE:
       v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
@@ -241,14 +242,19 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
       // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
       const int64_t qt = k.tile_m / 128;
       const int64_t smem = qt * 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 +
-                           (k.location ? 0 : qt * 128 * (int64_t)k.tile_n * 2) + 1024 + 256;
-      if (k.location == 1 && k.tile_m != 256) {
-        if (why) *why = "P in tensor memory is a variant of the two-tile kernel";
+                           (k.location ? 0 : qt * 128 * (int64_t)k.tile_n * 2) + 1024 + 512;
+      if (k.location == 1 && k.tile_m != 256 && k.persistent != 1) {
+        if (why) *why = "P in tensor memory needs two query tiles or split UMMA issue";
         return false;
       }
       if (k.unroll == 2 && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
         // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
         if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
+        return false;
+      }
+      if (k.persistent == 1 && !(k.location == 1 && k.unroll == 1 && k.stages >= 2)) {
+        // two tiles: one issuing warp per tile; one tile: two S buffers, S and P V issued by separate warps
+        if (why) *why = "split UMMA issue needs P in TMEM, one key block in flight per issuer and two stages";
         return false;
       }
       if (smem > kSmemLimit) {

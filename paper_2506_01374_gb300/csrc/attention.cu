@@ -159,6 +159,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = max(0, j - stages); i < j; ++i)
         if (!tc::mbar_wait_drain(&kv_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
     }
+    __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
@@ -347,6 +348,171 @@ constexpr int kThreads2 = 320;
 constexpr float kRescaleLog2 = 8.0f;
 
 
+// Softmax and output of one query tile in the two-tile kernels: one TMEM lane
+// quadrant per warp (qd = warp % 4), one query row per thread. S of key block j
+// sits in TMEM columns [(t * NSB + j % NSB) * BN, + BN) and O_t at o_base + t * D.
+// Pass 1 takes the masked row maximum of the whole S row (one TMEM round trip);
+// O is rescaled in TMEM when the reference maximum moves by more than 2^8; pass 2
+// writes P = 2^(s * scale * log2 e - m) as bf16, over its own S columns (PT) or
+// into the swizzled shared-memory P tile, and accumulates the row sum l.
+template <int BN, bool PT, bool SDB>
+__device__ __forceinline__ void softmax_tile(const Params& p, int t, int qd, int lane, int q0, int nkb, int b, int h,
+                                             uint32_t tmem, uint32_t o_base, uint8_t* sP_tile, uint64_t* s_full,
+                                             uint64_t* p_full, uint64_t* pv_full, volatile int* abort_flag,
+                                             volatile int* status) {
+  constexpr int NSB = SDB ? 2 : 1;
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+  const int row = 32 * qd + lane;
+  const int qi = q0 + row;
+  const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+  const uint32_t tO = tmem + lane_base + o_base + t * D;
+  uint8_t* rowp0 = sP_tile + (row / 8) * 1024 + (row % 8) * 128;
+  float m_ref = -INFINITY, l = 0.f;
+  bool ok = true;
+  for (int j = 0; j < nkb; ++j) {
+    const uint32_t tS = tmem + lane_base + (uint32_t)(t * NSB + (j % NSB)) * BN;
+    if (!tc::mbar_wait(&s_full[j % NSB], (uint32_t)(j / NSB) & 1u, abort_flag, status)) {
+      if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+      ok = false;
+      break;
+    }
+    tc::tc_fence_after();
+    const int k0 = j * BN;
+    // keys [k0, k0 + nvis) of this block are visible to query qi
+    int nvis = min(BN, p.S - k0);
+    if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
+    // the whole S row in registers: one TMEM round trip
+    uint32_t r[BN];
+#pragma unroll
+    for (int q = 0; q < BN; q += 16) tc::tmem_ld16(tS + q, *reinterpret_cast<uint32_t(*)[16]>(&r[q]));
+    tc::tmem_ld_wait();
+    if (nvis < BN) {
+#pragma unroll
+      for (int i = 0; i < BN; ++i)
+        if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
+    }
+    // row maximum: 8 independent partial maxima, then combine
+    float pm[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(r[u]);
+#pragma unroll
+    for (int i = 8; i < BN; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(r[i]));
+    const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                           fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+    const float mxs = mx * p.scale_log2;
+    float factor = 1.f;
+    if (m_ref == -INFINITY) {
+      m_ref = mxs;  // first visible scores: O and l are still zero
+    } else if (mxs > m_ref + kRescaleLog2) {
+      factor = exp2f(m_ref - mxs);
+      m_ref = mxs;
+    }
+    const bool rescale = __any_sync(0xffffffffu, factor != 1.f);
+    // pv_full completes once per key block (P_t V of that block). It is
+    // observed phase by phase, so a parity wait never meets a barrier more
+    // than one phase ahead: phase j-1 is awaited in iteration j, before the
+    // O rescale when there is one (O must hold P_t V of block j-1), before
+    // overwriting P's shared-memory buffer, or else after the probabilities
+    // are written. P V of block j is only issued after this thread's p_full.
+    bool pv_seen = j == 0;
+    auto await_pv = [&]() -> bool {
+      if (pv_seen) return true;
+      pv_seen = true;
+      if (!tc::mbar_wait(pv_full, (uint32_t)(j - 1) & 1u, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        return false;
+      }
+      tc::tc_fence_after();
+      return true;
+    };
+    if (rescale || !PT) {
+      if (!await_pv()) {
+        ok = false;
+        break;
+      }
+    }
+    if (rescale) {
+#pragma unroll 1
+      for (int c = 0; c < D; c += 16) {
+        uint32_t r[16];
+        tc::tmem_ld16(tO + c, r);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
+        tc::tmem_st16(tO + c, r);
+      }
+      tc::tmem_st_wait();
+    }
+    // pass 2: probabilities -> P (bf16) and the row sum
+    const float mref = m_ref == -INFINITY ? 0.f : m_ref;
+    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < BN; c += 32) {
+      uint32_t pk[16];
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        // masked scores are -inf: 2^-inf = +0
+        const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i]), p.scale_log2, -mref));
+        const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i + 1]), p.scale_log2, -mref));
+        ls[(i / 2) % 4] += p0 + p1;
+        pk[i / 2] = pack2(p0, p1);
+      }
+      if constexpr (PT) {
+        // P for keys [c, c + 32) goes to columns [c/2, c/2 + 16) of the S row (already in registers)
+        tc::tmem_st16(tS + c / 2, pk);
+      } else {
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int cc = c + 16 * h2;
+          uint8_t* rowp = rowp0 + (cc / 64) * (BM * 128);
+          const int ch = (cc % 64) / 8;
+          *reinterpret_cast<uint4*>(rowp + ((ch ^ (row % 8)) * 16)) =
+              make_uint4(pk[8 * h2], pk[8 * h2 + 1], pk[8 * h2 + 2], pk[8 * h2 + 3]);
+          *reinterpret_cast<uint4*>(rowp + (((ch + 1) ^ (row % 8)) * 16)) =
+              make_uint4(pk[8 * h2 + 4], pk[8 * h2 + 5], pk[8 * h2 + 6], pk[8 * h2 + 7]);
+        }
+      }
+    }
+    l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+    if constexpr (PT) tc::tmem_st_wait();
+    if (!await_pv()) {
+      ok = false;
+      break;
+    }
+    tc::tc_fence_before();
+    if constexpr (!PT) tc::fence_proxy_async_smem();
+    tc::mbar_arrive(p_full);
+  }
+  if (ok && nkb > 0) {
+    if (tc::mbar_wait(pv_full, (uint32_t)(nkb - 1) & 1u, abort_flag, status)) {
+      tc::tc_fence_after();
+      const float inv_l = l > 0.f ? 1.f / l : 0.f;
+      const bool row_ok = qi < p.S;
+      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < D; c += 16) {
+        uint32_t r[16];
+        tc::tmem_ld16(tO + c, r);
+        tc::tmem_ld_wait();
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 16; i += 2)
+          pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
+        if (row_ok) {
+          *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        }
+      }
+      if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
+    } else if (!*abort_flag) {
+      fail(RC_DEV_TIMEOUT_ACCUM);
+    }
+  }
+}
+
 template <int BN, bool VT, bool PT, bool SDB>
 __global__ void __launch_bounds__(kThreads2, 1)
     attn2_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -370,10 +536,14 @@ __global__ void __launch_bounds__(kThreads2, 1)
   uint8_t* sQ = smem;                                   // [2] tiles
   uint8_t* ring = smem + 2 * Q_BYTES;
   uint8_t* sP = ring + (size_t)stages * 2 * KV_TILE;    // [2] tiles
+  // separate K and V rings of `stages` slots each: K of a block is released
+  // once both tiles' S products are issued, V once both P V products are
   uint64_t* q_full = (uint64_t*)(sP + 2 * P_BYTES);
-  uint64_t* kv_full = q_full + 1;
-  uint64_t* kv_empty = kv_full + stages;
-  uint64_t* s_full = kv_empty + stages;  // [2 tiles][NSB buffers]
+  uint64_t* k_full = q_full + 1;
+  uint64_t* k_empty = k_full + stages;
+  uint64_t* v_full = k_empty + stages;
+  uint64_t* v_empty = v_full + stages;
+  uint64_t* s_full = v_empty + stages;  // [2 tiles][NSB buffers]
   uint64_t* p_full = s_full + 2 * NSB;   // [2]
   uint64_t* pv_full = p_full + 2;        // [2]
   uint64_t* drain = pv_full + 2;
@@ -410,8 +580,10 @@ __global__ void __launch_bounds__(kThreads2, 1)
   if (threadIdx.x == 0) {
     tc::mbar_init(q_full, 1);
     for (int s = 0; s < stages; ++s) {
-      tc::mbar_init(&kv_full[s], 1);
-      tc::mbar_init(&kv_empty[s], 1);
+      tc::mbar_init(&k_full[s], 1);
+      tc::mbar_init(&k_empty[s], 1);
+      tc::mbar_init(&v_full[s], 1);
+      tc::mbar_init(&v_empty[s], 1);
     }
     for (int t = 0; t < 2; ++t) {
       for (int b2 = 0; b2 < NSB; ++b2) tc::mbar_init(&s_full[t * NSB + b2], 1);
@@ -444,40 +616,57 @@ __global__ void __launch_bounds__(kThreads2, 1)
       for (; j < nblk; ++j) {
         const int s = j % stages;
         const uint32_t ph = (uint32_t)(j / stages) & 1u;
-        if (!tc::mbar_wait(&kv_empty[s], ph ^ 1u, abort_flag, status)) {
+        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
+        uint8_t* sv = sk + KV_TILE;
+        const int krow = b * p.S + j * BN;
+        if (!tc::mbar_wait(&k_empty[s], ph ^ 1u, abort_flag, status)) {
           fail(RC_DEV_TIMEOUT_EMPTY);
           break;
         }
-        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
-        uint8_t* sv = sk + KV_TILE;
-        tc::mbar_expect_tx(&kv_full[s], 2 * KV_TILE);
-        const int krow = b * p.S + j * BN;
-        tc::tma_load_2d(sk, &tmK, &kv_full[s], g * D, krow);
-        tc::tma_load_2d(sk + BN * 128, &tmK, &kv_full[s], g * D + 64, krow);
+        tc::mbar_expect_tx(&k_full[s], KV_TILE);
+        tc::tma_load_2d(sk, &tmK, &k_full[s], g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, &k_full[s], g * D + 64, krow);
+        if (!tc::mbar_wait(&v_empty[s], ph ^ 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          // K of this block is in flight: let it land before exit
+          if (!tc::mbar_wait_drain(&k_full[s], ph)) fail(RC_DEV_TIMEOUT_DRAIN);
+          break;
+        }
+        tc::mbar_expect_tx(&v_full[s], KV_TILE);
         if constexpr (VT) {
 #pragma unroll
           for (int a = 0; a < BN / 64; ++a)
-            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &kv_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
+            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &v_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
         } else {
-          tc::tma_load_2d(sv, &tmV, &kv_full[s], g * D, krow);
-          tc::tma_load_2d(sv + BN * 128, &tmV, &kv_full[s], g * D + 64, krow);
+          tc::tma_load_2d(sv, &tmV, &v_full[s], g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, &v_full[s], g * D + 64, krow);
         }
       }
       if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      for (int i = max(0, j - stages); i < j; ++i)
-        if (!tc::mbar_wait_drain(&kv_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+      for (int i = max(0, j - stages); i < j; ++i) {
+        if (!tc::mbar_wait_drain(&k_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+        if (!tc::mbar_wait_drain(&v_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
     }
+    __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
       constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
       bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
       if (!ok) fail(RC_DEV_TIMEOUT_FULL);
-      int loaded = -1;  // highest key block whose K/V arrival was awaited
-      auto await_block = [&](int j) -> bool {
-        if (j <= loaded) return true;
-        if (!tc::mbar_wait(&kv_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status)) return false;
-        loaded = j;
+      int k_seen = -1, v_seen = -1;  // highest key block whose K / V arrival was awaited
+      auto await_k = [&](int j) -> bool {
+        if (j <= k_seen) return true;
+        if (!tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status)) return false;
+        k_seen = j;
+        tc::tc_fence_after();
+        return true;
+      };
+      auto await_v = [&](int j) -> bool {
+        if (j <= v_seen) return true;
+        if (!tc::mbar_wait(&v_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status)) return false;
+        v_seen = j;
         tc::tc_fence_after();
         return true;
       };
@@ -514,24 +703,26 @@ __global__ void __launch_bounds__(kThreads2, 1)
         }
         tc::umma_commit(&pv_full[t]);
       };
-      // prologue: S for the first NSB key blocks of both tiles
+      // prologue: S for the first NSB key blocks of both tiles; their K is then free
       for (int j0 = 0; ok && j0 < NSB && j0 < nblk; ++j0) {
-        ok = await_block(j0);
-        if (ok)
+        ok = await_k(j0);
+        if (ok) {
           for (int t = 0; t < 2; ++t)
             if (j0 < nkb[t]) issue_s(t, j0);
+          tc::umma_commit(&k_empty[j0 % stages]);
+        }
       }
       for (int j = 0; ok && j < nblk; ++j) {
         for (int t = 0; t < 2; ++t) {
           if (j >= nkb[t]) continue;
-          if (!tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status)) {
+          if (!tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status) || !await_v(j)) {
             ok = false;
             break;
           }
           tc::tc_fence_after();
           issue_pv(t, j);
           if (j + NSB < nkb[t]) {
-            if (!await_block(j + NSB)) {
+            if (!await_k(j + NSB)) {
               ok = false;
               break;
             }
@@ -539,7 +730,8 @@ __global__ void __launch_bounds__(kThreads2, 1)
           }
         }
         if (!ok) break;
-        tc::umma_commit(&kv_empty[j % stages]);
+        tc::umma_commit(&v_empty[j % stages]);  // both P V products of block j issued
+        if (j + NSB < nblk) tc::umma_commit(&k_empty[(j + NSB) % stages]);  // both S products of block j+NSB
       }
       if (!ok) {
         fail(RC_DEV_TIMEOUT_FULL);
@@ -550,153 +742,761 @@ __global__ void __launch_bounds__(kThreads2, 1)
     __syncwarp();
   } else if (warp >= 2) {
     const int t = (warp - 2) / 4;  // query tile of this warpgroup
-    const int qd = warp & 3;
-    const int row = 32 * qd + lane;
-    const int qi = q0[t] + row;
-    const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
-    const uint32_t tO = tmem + lane_base + O_BASE + t * D;
-    uint8_t* rowp0 = sP + t * P_BYTES + (row / 8) * 1024 + (row % 8) * 128;
-    float m_ref = -INFINITY, l = 0.f;
-    bool ok = true;
-    for (int j = 0; j < nkb[t]; ++j) {
-      const uint32_t tS = tmem + lane_base + (uint32_t)(t * NSB + (j % NSB)) * BN;
-      if (!tc::mbar_wait(&s_full[t * NSB + (j % NSB)], (uint32_t)(j / NSB) & 1u, abort_flag, status)) {
-        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
-        ok = false;
-        break;
-      }
-      tc::tc_fence_after();
-      const int k0 = j * BN;
-      // keys [k0, k0 + nvis) of this block are visible to query qi
-      int nvis = min(BN, p.S - k0);
-      if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
-      // the whole S row in registers: one TMEM round trip
-      uint32_t r[BN];
-#pragma unroll
-      for (int q = 0; q < BN; q += 16) tc::tmem_ld16(tS + q, *reinterpret_cast<uint32_t(*)[16]>(&r[q]));
-      tc::tmem_ld_wait();
-      if (nvis < BN) {
-#pragma unroll
-        for (int i = 0; i < BN; ++i)
-          if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
-      }
-      // row maximum: 8 independent partial maxima, then combine
-      float pm[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(r[u]);
-#pragma unroll
-      for (int i = 8; i < BN; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(r[i]));
-      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-      const float mxs = mx * p.scale_log2;
-      float factor = 1.f;
-      if (m_ref == -INFINITY) {
-        m_ref = mxs;  // first visible scores: O and l are still zero
-      } else if (mxs > m_ref + kRescaleLog2) {
-        factor = exp2f(m_ref - mxs);
-        m_ref = mxs;
-      }
-      const bool rescale = __any_sync(0xffffffffu, factor != 1.f);
-      // pv_full completes once per key block (P_t V of that block). It is
-      // observed phase by phase, so a parity wait never meets a barrier more
-      // than one phase ahead: phase j-1 is awaited in iteration j, before the
-      // O rescale when there is one (O must hold P_t V of block j-1), before
-      // overwriting P's shared-memory buffer, or else after the probabilities
-      // are written. P V of block j is only issued after this thread's p_full.
-      bool pv_seen = j == 0;
-      auto await_pv = [&]() -> bool {
-        if (pv_seen) return true;
-        pv_seen = true;
-        if (!tc::mbar_wait(&pv_full[t], (uint32_t)(j - 1) & 1u, abort_flag, status)) {
-          if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
-          return false;
-        }
-        tc::tc_fence_after();
-        return true;
-      };
-      if (rescale || !PT) {
-        if (!await_pv()) {
-          ok = false;
-          break;
-        }
-      }
-      if (rescale) {
+    softmax_tile<BN, PT, SDB>(p, t, warp & 3, lane, q0[t], nkb[t], b, h, tmem, O_BASE, sP + t * P_BYTES,
+                              &s_full[t * NSB], &p_full[t], &pv_full[t], abort_flag, status);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+// Compact softmax of one query tile for P in TMEM (one S buffer per tile): the
+// S row is walked twice in chunks of 32 columns by loops that are not
+// unrolled, first for the masked maximum (masked scores are written back as
+// -inf, only in chunks that hold any), then for P and the row sum. It holds 32
+// scores in registers instead of the whole row (68 registers per thread
+// instead of 168) and measures as fast as the whole-row version in the
+// two-issuer kernel, where the tensor pipe, not the softmax, sets the pace.
+// P of keys [c, c + 32) goes to columns [c/2, c/2 + 16), which hold S values
+// already consumed.
+template <int BN>
+__device__ __forceinline__ void softmax_tile_chunked(const Params& p, int t, int qd, int lane, int q0, int nkb, int b,
+                                                     int h, uint32_t tmem, uint32_t o_base, uint64_t* s_full,
+                                                     uint64_t* p_full, uint64_t* pv_full, volatile int* abort_flag,
+                                                     volatile int* status) {
+  constexpr int CH = 32;
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+  const int row = 32 * qd + lane;
+  const int qi = q0 + row;
+  const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+  const uint32_t tO = tmem + lane_base + o_base + t * D;
+  const uint32_t tS = tmem + lane_base + (uint32_t)(t * BN);
+  float m_ref = -INFINITY, l = 0.f;
+  bool ok = true;
+  for (int j = 0; j < nkb; ++j) {
+    if (!tc::mbar_wait(s_full, (uint32_t)j & 1u, abort_flag, status)) {
+      if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+      ok = false;
+      break;
+    }
+    tc::tc_fence_after();
+    const int k0 = j * BN;
+    // keys [k0, k0 + nvis) of this block are visible to query qi
+    int nvis = min(BN, p.S - k0);
+    if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
+    float mx = -INFINITY;
 #pragma unroll 1
-        for (int c = 0; c < D; c += 16) {
-          uint32_t r[16];
-          tc::tmem_ld16(tO + c, r);
-          tc::tmem_ld_wait();
+    for (int c = 0; c < BN; c += CH) {
+      uint32_t r[CH];
+      tc::tmem_ld32(tS + c, r);
+      tc::tmem_ld_wait();
+      if (__any_sync(0xffffffffu, nvis < c + CH)) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
-          tc::tmem_st16(tO + c, r);
-        }
+        for (int i = 0; i < CH; ++i)
+          if (c + i >= nvis) r[i] = __float_as_uint(-INFINITY);
+        tc::tmem_st32(tS + c, r);
         tc::tmem_st_wait();
       }
-      // pass 2: probabilities -> P (bf16) and the row sum
-      const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+      float pm[4];
 #pragma unroll
-      for (int c = 0; c < BN; c += 32) {
-        uint32_t pk[16];
+      for (int u = 0; u < 4; ++u) pm[u] = __uint_as_float(r[u]);
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          // masked scores are -inf: 2^-inf = +0
-          const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i]), p.scale_log2, -mref));
-          const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i + 1]), p.scale_log2, -mref));
-          ls[(i / 2) % 4] += p0 + p1;
-          pk[i / 2] = pack2(p0, p1);
-        }
-        if constexpr (PT) {
-          // P for keys [c, c + 32) goes to columns [c/2, c/2 + 16) of the S row (already in registers)
-          tc::tmem_st16(tS + c / 2, pk);
-        } else {
-#pragma unroll
-          for (int h2 = 0; h2 < 2; ++h2) {
-            const int cc = c + 16 * h2;
-            uint8_t* rowp = rowp0 + (cc / 64) * (BM * 128);
-            const int ch = (cc % 64) / 8;
-            *reinterpret_cast<uint4*>(rowp + ((ch ^ (row % 8)) * 16)) =
-                make_uint4(pk[8 * h2], pk[8 * h2 + 1], pk[8 * h2 + 2], pk[8 * h2 + 3]);
-            *reinterpret_cast<uint4*>(rowp + (((ch + 1) ^ (row % 8)) * 16)) =
-                make_uint4(pk[8 * h2 + 4], pk[8 * h2 + 5], pk[8 * h2 + 6], pk[8 * h2 + 7]);
-          }
-        }
+      for (int i = 4; i < CH; ++i) pm[i % 4] = fmaxf(pm[i % 4], __uint_as_float(r[i]));
+      mx = fmaxf(mx, fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])));
+    }
+    const float mxs = mx * p.scale_log2;
+    float factor = 1.f;
+    if (m_ref == -INFINITY) {
+      m_ref = mxs;  // first visible scores: O and l are still zero
+    } else if (mxs > m_ref + kRescaleLog2) {
+      factor = exp2f(m_ref - mxs);
+      m_ref = mxs;
+    }
+    const bool rescale = __any_sync(0xffffffffu, factor != 1.f);
+    // pv_full phase j-1 (P_t V of block j-1) is observed once per key block:
+    // before the O rescale when there is one, else after P is written
+    bool pv_seen = j == 0;
+    auto await_pv = [&]() -> bool {
+      if (pv_seen) return true;
+      pv_seen = true;
+      if (!tc::mbar_wait(pv_full, (uint32_t)(j - 1) & 1u, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        return false;
       }
-      l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
-      if constexpr (PT) tc::tmem_st_wait();
+      tc::tc_fence_after();
+      return true;
+    };
+    if (rescale) {
       if (!await_pv()) {
         ok = false;
         break;
       }
-      tc::tc_fence_before();
-      if constexpr (!PT) tc::fence_proxy_async_smem();
-      tc::mbar_arrive(&p_full[t]);
-    }
-    if (ok && nkb[t] > 0) {
-      if (tc::mbar_wait(&pv_full[t], (uint32_t)(nkb[t] - 1) & 1u, abort_flag, status)) {
-        tc::tc_fence_after();
-        const float inv_l = l > 0.f ? 1.f / l : 0.f;
-        const bool row_ok = qi < p.S;
-        __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
 #pragma unroll 1
-        for (int c = 0; c < D; c += 16) {
-          uint32_t r[16];
-          tc::tmem_ld16(tO + c, r);
-          tc::tmem_ld_wait();
-          uint32_t pk[8];
+      for (int c = 0; c < D; c += CH) {
+        uint32_t r[CH];
+        tc::tmem_ld32(tO + c, r);
+        tc::tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 16; i += 2)
-            pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
-          if (row_ok) {
-            *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          }
+        for (int i = 0; i < CH; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
+        tc::tmem_st32(tO + c, r);
+      }
+      tc::tmem_st_wait();
+    }
+    const float mref = m_ref == -INFINITY ? 0.f : m_ref;
+    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+    for (int c = 0; c < BN; c += CH) {
+      uint32_t r[CH];
+      tc::tmem_ld32(tS + c, r);
+      tc::tmem_ld_wait();
+      uint32_t pk[CH / 2];
+#pragma unroll
+      for (int i = 0; i < CH; i += 2) {
+        // masked scores are -inf: 2^-inf = +0
+        const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[i]), p.scale_log2, -mref));
+        const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[i + 1]), p.scale_log2, -mref));
+        ls[(i / 2) % 4] += p0 + p1;
+        pk[i / 2] = pack2(p0, p1);
+      }
+      tc::tmem_st16(tS + c / 2, pk);
+    }
+    l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+    tc::tmem_st_wait();
+    if (!await_pv()) {
+      ok = false;
+      break;
+    }
+    tc::tc_fence_before();
+    tc::mbar_arrive(p_full);
+  }
+  if (ok && nkb > 0) {
+    if (tc::mbar_wait(pv_full, (uint32_t)(nkb - 1) & 1u, abort_flag, status)) {
+      tc::tc_fence_after();
+      const float inv_l = l > 0.f ? 1.f / l : 0.f;
+      const bool row_ok = qi < p.S;
+      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < D; c += 16) {
+        uint32_t r[16];
+        tc::tmem_ld16(tO + c, r);
+        tc::tmem_ld_wait();
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 16; i += 2)
+          pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
+        if (row_ok) {
+          *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
-        if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
-      } else if (!*abort_flag) {
-        fail(RC_DEV_TIMEOUT_ACCUM);
+      }
+      if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
+    } else if (!*abort_flag) {
+      fail(RC_DEV_TIMEOUT_ACCUM);
+    }
+  }
+}
+
+// Two query tiles per CTA with one UMMA-issuing warp per tile (Parallel = 1).
+// One thread needs about as long to issue a 128 x 128 x 16 UMMA as the tensor
+// pipe needs to execute it, and its barrier waits and commits come on top, so
+// when a single thread issues both tiles' chains the pipe idles while that
+// thread waits. Here each tile has its own issuer, which checks that V_j and
+// K_{j+1} have landed while the softmax still works on S_j, and releases K_j
+// once S_j is done and V_j once P_j V_j is done, through its own barriers; the
+// producer refills a slot when every tile that read the block held there has
+// released it (under the causal mask tile 0 stops before tile 1).
+// The issuers take turns per chain (tile 0's chain c, then tile 1's chain c,
+// then tile 0's chain c + 1), the UMMA order of the single-issuer kernel:
+// this keeps the tiles half a period apart, so that one tile's softmax runs
+// while the tensor pipe works on the other tile's products.
+//   warp 0       : TMA producer (Q tiles once, then K_j and V_j)
+//   warps 1, 2   : UMMA issue for query tile 0 / 1 (warp 1 also owns TMEM)
+//   warps 3..6   : softmax of tile 0 (TMEM lane quadrant = warp % 4)
+//   warps 7..10  : softmax of tile 1
+// P is kept in TMEM over its S columns.
+constexpr int kThreads3 = 352;
+
+template <int BN, bool VT>
+__global__ void __launch_bounds__(kThreads3, 1)
+    attn3_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  static_assert(BN == 64 || BN == 128, "key block");
+  constexpr int Q_BYTES = BM * D * 2;
+  constexpr int KV_TILE = BN * D * 2;
+  constexpr uint32_t O_BASE = (uint32_t)(2 * BN);  // TMEM: S_0, S_1, then O_0, O_1
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;  // [2] tiles
+  uint8_t* ring = smem + 2 * Q_BYTES;
+  uint64_t* q_full = (uint64_t*)(ring + (size_t)stages * 2 * KV_TILE);
+  uint64_t* k_full = q_full + 1;              // [stages]
+  uint64_t* v_full = k_full + stages;         // [stages]
+  uint64_t* k_empty = v_full + stages;        // [2 tiles][stages]
+  uint64_t* v_empty = k_empty + 2 * stages;   // [2 tiles][stages]
+  uint64_t* s_full = v_empty + 2 * stages;    // [2]
+  uint64_t* p_full = s_full + 2;              // [2]
+  uint64_t* pv_full = p_full + 2;             // [2]
+  uint64_t* drain = pv_full + 2;              // [2]
+  uint32_t* tmem_slot = (uint32_t*)(drain + 2);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* chains = (volatile int*)(tmem_slot + 2);  // [2] UMMA chains issued per tile
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int pairs = (p.q_blocks + 1) / 2;
+  const int BH = p.B * p.Hq;
+  int pb, bh;
+  if (p.raster == 0) {
+    pb = blockIdx.x % pairs;
+    bh = blockIdx.x / pairs;
+  } else {
+    pb = pairs - 1 - (int)(blockIdx.x / BH);
+    bh = blockIdx.x % BH;
+  }
+  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
+  int q0[2], nkb[2];
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    q0[t] = (2 * pb + t) * BM;
+    const int end = p.causal ? min(q0[t] + BM, p.S) : p.S;
+    nkb[t] = q0[t] < p.S ? (end + BN - 1) / BN : 0;
+  }
+  const int nblk = max(nkb[0], nkb[1]);
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&k_full[s], 1);
+      tc::mbar_init(&v_full[s], 1);
+    }
+    for (int i = 0; i < 2 * stages; ++i) {
+      tc::mbar_init(&k_empty[i], 1);
+      tc::mbar_init(&v_empty[i], 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      tc::mbar_init(&s_full[t], 1);
+      tc::mbar_init(&p_full[t], 128);
+      tc::mbar_init(&pv_full[t], 1);
+      tc::mbar_init(&drain[t], 1);
+    }
+    *abort_flag = 0;
+    chains[0] = chains[1] = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(tmem_slot, 512);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::prefetch_tmap(&tmV);
+      tc::mbar_expect_tx(q_full, 2 * Q_BYTES);
+#pragma unroll
+      for (int t = 0; t < 2; ++t) {
+        const int qrow = b * p.S + q0[t];
+        tc::tma_load_2d(sQ + t * Q_BYTES, &tmQ, q_full, h * D, qrow);
+        tc::tma_load_2d(sQ + t * Q_BYTES + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
+      }
+      // Slot s last held key block j - stages. Tile t read that block iff
+      // j - stages < nkb[t]; its release is then the ((j - stages) / stages)-th
+      // phase of its barrier for slot s, of parity ph ^ 1 (for j < stages the
+      // fresh barrier passes that parity at once).
+      auto released = [&](uint64_t* empty, int j, int s, uint32_t ph) -> bool {
+        for (int t = 0; t < 2; ++t)
+          if (j - stages < nkb[t] && !tc::mbar_wait(&empty[t * stages + s], ph ^ 1u, abort_flag, status))
+            return false;
+        return true;
+      };
+      int j = 0;
+      for (; j < nblk; ++j) {
+        const int s = j % stages;
+        const uint32_t ph = (uint32_t)(j / stages) & 1u;
+        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
+        uint8_t* sv = sk + KV_TILE;
+        const int krow = b * p.S + j * BN;
+        if (!released(k_empty, j, s, ph)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          break;
+        }
+        tc::mbar_expect_tx(&k_full[s], KV_TILE);
+        tc::tma_load_2d(sk, &tmK, &k_full[s], g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, &k_full[s], g * D + 64, krow);
+        if (!released(v_empty, j, s, ph)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          if (!tc::mbar_wait_drain(&k_full[s], ph)) fail(RC_DEV_TIMEOUT_DRAIN);  // K of block j is in flight
+          break;
+        }
+        tc::mbar_expect_tx(&v_full[s], KV_TILE);
+        if constexpr (VT) {
+#pragma unroll
+          for (int a = 0; a < BN / 64; ++a)
+            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &v_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
+        } else {
+          tc::tma_load_2d(sv, &tmV, &v_full[s], g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, &v_full[s], g * D + 64, krow);
+        }
+      }
+      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      for (int i = max(0, j - stages); i < j; ++i) {
+        if (!tc::mbar_wait_drain(&k_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+        if (!tc::mbar_wait_drain(&v_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
       }
     }
+    __syncwarp();  // reconverge before the final block barrier
+  } else if (warp <= 2) {
+    const int t = warp - 1;
+    if (lane == 0 && nkb[t] > 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+      const int nk = nkb[t];
+      const int other_chains = nkb[1 - t] > 0 ? nkb[1 - t] + 1 : 0;
+      const uint32_t sq = tc::smem_u32(sQ + t * Q_BYTES);
+      const uint32_t tS = tmem + (uint32_t)(t * BN);
+      const uint32_t tO = tmem + O_BASE + (uint32_t)(t * D);
+      // this thread awaits every key block's K and V exactly once, in order;
+      // a slot's next fill needs this tile's release of the current one
+      auto await_full = [&](uint64_t* full, int j) -> bool {
+        return tc::mbar_wait(&full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status);
+      };
+      // chain c of this tile (c = 0: S_0; c = j + 1: P_j V_j and S_{j+1}) follows
+      // chain c - 1 (tile 0) or chain c (tile 1) of the other tile
+      auto await_turn = [&](int c) -> bool {
+        const int need = min(t == 0 ? c : c + 1, other_chains);
+        const uint64_t t0 = tc::globaltimer();
+        for (uint32_t it = 1; chains[1 - t] < need; ++it)
+          if ((it & 63) == 0 && (*abort_flag || tc::globaltimer() - t0 > tc::kWaitNs)) return false;
+        return true;
+      };
+      auto issue_s = [&](int j) {
+        const uint32_t sk = tc::smem_u32(ring + (size_t)(j % stages) * 2 * KV_TILE);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
+                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&s_full[t]);
+        tc::umma_commit(&k_empty[t * stages + j % stages]);
+      };
+      auto issue_pv = [&](int j) {
+        const int s = j % stages;
+        const uint32_t sv = tc::smem_u32(ring + (size_t)s * 2 * KV_TILE) + KV_TILE;
+#pragma unroll
+        for (int ks = 0; ks < BN / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          uint64_t db;
+          if constexpr (VT)
+            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
+          else
+            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
+          // P aliases S: two bf16 per TMEM column
+          tc::umma_bf16_ts(tO, tS + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        tc::umma_commit(&pv_full[t]);
+        tc::umma_commit(&v_empty[t * stages + s]);
+      };
+      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status) && await_full(k_full, 0) && await_turn(0);
+      if (ok) {
+        tc::tc_fence_after();
+        issue_s(0);
+        chains[t] = 1;
+      }
+      for (int j = 0; ok && j < nk; ++j) {
+        // V_j and K_{j+1} (landed long ago, normally) while the softmax works on S_j
+        ok = await_full(v_full, j) && (j + 1 >= nk || await_full(k_full, j + 1)) &&
+             tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status) && await_turn(j + 1);
+        if (!ok) break;
+        tc::tc_fence_after();
+        issue_pv(j);  // O += P_j V_j
+        if (j + 1 < nk) issue_s(j + 1);
+        chains[t] = j + 2;
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[t]);
+        if (!tc::mbar_wait_drain(&drain[t], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int t = (warp - 3) / 4;
+    softmax_tile_chunked<BN>(p, t, warp & 3, lane, q0[t], nkb[t], b, h, tmem, O_BASE, &s_full[t], &p_full[t],
+                             &pv_full[t], abort_flag, status);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+// One query tile per CTA with two S buffers and a P buffer of its own in TMEM
+// (TileSize M = 128, Parallel = 1). TMEM: S_0, S_1 (BN columns each), O (128),
+// P (BN/2 columns, two bf16 per column). S for key block j + 2 goes into the
+// buffer of block j as soon as the softmax holds S_j in registers, so the
+// tensor pipe computes S two key blocks ahead and the softmax of consecutive
+// blocks runs back to back; the softmax keeps P_j in registers until
+// P_{j-1} V_{j-1} has read the P buffer. The UMMAs come from two warps, one
+// for the S products and one for the P V products (one thread needs about as
+// long to issue a 128 x 128 x 16 UMMA as the pipe needs to run it), and K and
+// V stream through rings of their own, each filled by its own producer warp.
+//   warp 0     : TMA producer of Q and of the K ring
+//   warp 1     : issues S_j = Q K_j^T (and owns TMEM)
+//   warp 2     : issues O += P_j V_j
+//   warp 3     : TMA producer of the V ring
+//   warps 4..7 : softmax (TMEM lane quadrant = warp % 4), one query row per thread
+constexpr int kThreads4 = 256;
+
+template <int BN>
+__device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, int q0, int nkb, int b, int h,
+                                            uint32_t tmem, uint32_t o_col, uint32_t p_col, uint64_t* s_full,
+                                            uint64_t* s_free, uint64_t* p_full, uint64_t* pv_full,
+                                            volatile int* abort_flag, volatile int* status) {
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+  const int row = 32 * qd + lane;
+  const int qi = q0 + row;
+  const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+  const uint32_t tO = tmem + lane_base + o_col;
+  const uint32_t tP = tmem + lane_base + p_col;
+  float m_ref = -INFINITY, l = 0.f;
+  // pv_full completes once per key block (P_j V_j done); its phases are
+  // observed one by one, in order, never more than one behind: phase j - 1
+  // in iteration j (before an O rescale, else before P_j overwrites P_{j-1}),
+  // the last one before the output.
+  int pv_seen = 0;
+  auto await_pv = [&](int upto) -> bool {
+    if (pv_seen > upto) return true;
+    for (; pv_seen <= upto; ++pv_seen)
+      if (!tc::mbar_wait(pv_full, (uint32_t)pv_seen & 1u, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        return false;
+      }
+    tc::tc_fence_after();
+    return true;
+  };
+  bool ok = true;
+  for (int j = 0; j < nkb; ++j) {
+    const int sb = j & 1;
+    const uint32_t tS = tmem + lane_base + (uint32_t)(sb * BN);
+    if (!tc::mbar_wait(&s_full[sb], (uint32_t)(j >> 1) & 1u, abort_flag, status)) {
+      if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+      ok = false;
+      break;
+    }
+    tc::tc_fence_after();
+    uint32_t r[BN];
+#pragma unroll
+    for (int c = 0; c < BN; c += 32) tc::tmem_ld32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&r[c]));
+    tc::tmem_ld_wait();
+    tc::tc_fence_before();
+    tc::mbar_arrive(&s_free[sb]);  // S buffer sb may take S_{j+2}
+    const int k0 = j * BN;
+    int nvis = min(BN, p.S - k0);
+    if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
+    if (nvis < BN) {
+#pragma unroll
+      for (int i = 0; i < BN; ++i)
+        if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
+    }
+    float pm[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(r[u]);
+#pragma unroll
+    for (int i = 8; i < BN; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(r[i]));
+    const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])), fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+    const float mxs = mx * p.scale_log2;
+    float factor = 1.f;
+    if (m_ref == -INFINITY) {
+      m_ref = mxs;  // first visible scores: O and l are still zero
+    } else if (mxs > m_ref + kRescaleLog2) {
+      factor = exp2f(m_ref - mxs);
+      m_ref = mxs;
+    }
+    if (__any_sync(0xffffffffu, factor != 1.f)) {
+      if (!await_pv(j - 1)) {  // O holds P_{j-1} V_{j-1}
+        ok = false;
+        break;
+      }
+#pragma unroll 1
+      for (int c = 0; c < D; c += 32) {
+        uint32_t o[32];
+        tc::tmem_ld32(tO + c, o);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+        tc::tmem_st32(tO + c, o);
+      }
+      tc::tmem_st_wait();
+    }
+    const float mref = m_ref == -INFINITY ? 0.f : m_ref;
+    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+    uint32_t pk[BN / 2];
+#pragma unroll
+    for (int i = 0; i < BN; i += 2) {
+      // masked scores are -inf: 2^-inf = +0
+      const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[i]), p.scale_log2, -mref));
+      const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[i + 1]), p.scale_log2, -mref));
+      ls[(i / 2) % 4] += p0 + p1;
+      pk[i / 2] = pack2(p0, p1);
+    }
+    l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+    if (!await_pv(j - 1)) {  // P_{j-1} V_{j-1} has read the P buffer
+      ok = false;
+      break;
+    }
+#pragma unroll
+    for (int c = 0; c < BN / 2; c += 16) tc::tmem_st16(tP + c, *reinterpret_cast<uint32_t(*)[16]>(&pk[c]));
+    tc::tmem_st_wait();
+    tc::tc_fence_before();
+    tc::mbar_arrive(p_full);
+  }
+  if (ok && nkb > 0) {
+    if (await_pv(nkb - 1)) {
+      const float inv_l = l > 0.f ? 1.f / l : 0.f;
+      const bool row_ok = qi < p.S;
+      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
+#pragma unroll 1
+      for (int c = 0; c < D; c += 16) {
+        uint32_t o[16];
+        tc::tmem_ld16(tO + c, o);
+        tc::tmem_ld_wait();
+        uint32_t pk2[8];
+#pragma unroll
+        for (int i = 0; i < 16; i += 2)
+          pk2[i / 2] = pack2(__uint_as_float(o[i]) * inv_l, __uint_as_float(o[i + 1]) * inv_l);
+        if (row_ok) {
+          *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk2[0], pk2[1], pk2[2], pk2[3]);
+          *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk2[4], pk2[5], pk2[6], pk2[7]);
+        }
+      }
+      if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
+    }
+  }
+}
+
+template <int BN, bool VT>
+__global__ void __launch_bounds__(kThreads4, 1)
+    attn4_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  static_assert(BN == 64 || BN == 128, "key block");
+  constexpr int Q_BYTES = BM * D * 2;
+  constexpr int KV_TILE = BN * D * 2;
+  constexpr uint32_t O_COL = (uint32_t)(2 * BN), P_COL = (uint32_t)(2 * BN + D);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;
+  uint8_t* kring = smem + Q_BYTES;
+  uint8_t* vring = kring + (size_t)stages * KV_TILE;
+  uint64_t* q_full = (uint64_t*)(vring + (size_t)stages * KV_TILE);
+  uint64_t* k_full = q_full + 1;      // [stages]
+  uint64_t* k_empty = k_full + stages;
+  uint64_t* v_full = k_empty + stages;
+  uint64_t* v_empty = v_full + stages;
+  uint64_t* s_full = v_empty + stages;  // [2] S buffers
+  uint64_t* s_free = s_full + 2;        // [2]
+  uint64_t* p_full = s_free + 2;
+  uint64_t* pv_full = p_full + 1;
+  uint64_t* drain = pv_full + 1;        // [2] one per issuing warp
+  uint32_t* tmem_slot = (uint32_t*)(drain + 2);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int BH = p.B * p.Hq;
+  int qb, bh;
+  if (p.raster == 0) {
+    qb = blockIdx.x % p.q_blocks;
+    bh = blockIdx.x / p.q_blocks;
+  } else {  // longest causal rows first
+    qb = p.q_blocks - 1 - (int)(blockIdx.x / BH);
+    bh = blockIdx.x % BH;
+  }
+  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
+  const int q0 = qb * BM;
+  const int kv_end = p.causal ? min(q0 + BM, p.S) : p.S;
+  const int nkb = (kv_end + BN - 1) / BN;
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&k_full[s], 1);
+      tc::mbar_init(&k_empty[s], 1);
+      tc::mbar_init(&v_full[s], 1);
+      tc::mbar_init(&v_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&s_full[i], 1);
+      tc::mbar_init(&s_free[i], 128);
+      tc::mbar_init(&drain[i], 1);
+    }
+    tc::mbar_init(p_full, 128);
+    tc::mbar_init(pv_full, 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(tmem_slot, 512);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // slot s of a ring last held block j - stages; its release is the
+  // ((j - stages) / stages)-th phase of empty[s], parity ph ^ 1 (a fresh
+  // barrier passes that parity at once)
+  auto produce = [&](uint64_t* full, uint64_t* empty, auto load) {
+    int j = 0;
+    for (; j < nkb; ++j) {
+      const int s = j % stages;
+      const uint32_t ph = (uint32_t)(j / stages) & 1u;
+      if (!tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status)) {
+        fail(RC_DEV_TIMEOUT_EMPTY);
+        break;
+      }
+      tc::mbar_expect_tx(&full[s], KV_TILE);
+      load(s, j, &full[s]);
+    }
+    for (int i = max(0, j - stages); i < j; ++i)
+      if (!tc::mbar_wait_drain(&full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::mbar_expect_tx(q_full, Q_BYTES);
+      const int qrow = b * p.S + q0;
+      tc::tma_load_2d(sQ, &tmQ, q_full, h * D, qrow);
+      tc::tma_load_2d(sQ + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
+      produce(k_full, k_empty, [&](int s, int j, uint64_t* bar) {
+        uint8_t* sk = kring + (size_t)s * KV_TILE;
+        const int krow = b * p.S + j * BN;
+        tc::tma_load_2d(sk, &tmK, bar, g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, bar, g * D + 64, krow);
+      });
+      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+    __syncwarp();  // reconverge before the final block barrier
+  } else if (warp == 3) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmV);
+      produce(v_full, v_empty, [&](int s, int j, uint64_t* bar) {
+        uint8_t* sv = vring + (size_t)s * KV_TILE;
+        if constexpr (VT) {
+#pragma unroll
+          for (int a = 0; a < BN / 64; ++a)
+            tc::tma_load_2d(sv + a * (BM * 128), &tmV, bar, j * BN + a * 64, (b * p.Hkv + g) * D);
+        } else {
+          const int krow = b * p.S + j * BN;
+          tc::tma_load_2d(sv, &tmV, bar, g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, bar, g * D + 64, krow);
+        }
+      });
+    }
+    __syncwarp();  // reconverge before the final block barrier
+  } else if (warp == 1) {
+    if (lane == 0 && nkb > 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+      const uint32_t sq = tc::smem_u32(sQ);
+      auto issue_s = [&](int j) {
+        const int s = j % stages;
+        const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
+        const uint32_t tS = tmem + (uint32_t)((j & 1) * BN);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
+                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&s_full[j & 1]);
+        tc::umma_commit(&k_empty[s]);
+      };
+      auto await_k = [&](int j) -> bool {
+        return tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status);
+      };
+      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
+      for (int j = 0; ok && j < 2 && j < nkb; ++j) {
+        if ((ok = await_k(j))) {
+          tc::tc_fence_after();
+          issue_s(j);
+        }
+      }
+      for (int j = 0; ok && j + 2 < nkb; ++j) {
+        // S buffer j & 1 is free once the softmax holds S_j in registers
+        ok = tc::mbar_wait(&s_free[j & 1], (uint32_t)(j >> 1) & 1u, abort_flag, status) && await_k(j + 2);
+        if (!ok) break;
+        tc::tc_fence_after();
+        issue_s(j + 2);
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[0]);
+        if (!tc::mbar_wait_drain(&drain[0], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 2) {
+    if (lane == 0 && nkb > 0) {
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+      const uint32_t tO = tmem + O_COL, tP = tmem + P_COL;
+      bool ok = true;
+      for (int j = 0; ok && j < nkb; ++j) {
+        const int s = j % stages;
+        ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / stages) & 1u, abort_flag, status) &&
+             tc::mbar_wait(p_full, (uint32_t)j & 1u, abort_flag, status);
+        if (!ok) break;
+        tc::tc_fence_after();
+        const uint32_t sv = tc::smem_u32(vring + (size_t)s * KV_TILE);
+#pragma unroll
+        for (int ks = 0; ks < BN / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          uint64_t db;
+          if constexpr (VT)
+            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
+          else
+            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
+          tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        tc::umma_commit(pv_full);
+        tc::umma_commit(&v_empty[s]);
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[1]);
+        if (!tc::mbar_wait_drain(&drain[1], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else {
+    softmax_sdb<BN>(p, warp & 3, lane, q0, nkb, b, h, tmem, O_COL, P_COL, s_full, s_free, p_full, pv_full, abort_flag,
+                    status);
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -728,14 +1528,20 @@ __global__ void transpose_v_kernel(const __nv_bfloat16* __restrict__ V, int S, i
   }
 }
 
+// Q tiles + K/V ring + P tiles + 1 KB alignment slack + barriers (at most
+// 1 + 6 * stages + 8 of them, 8 B each, plus two words: 512 B for stages <= 5)
 size_t smem_bytes(int bn, int stages, int qtiles) {
-  return (size_t)qtiles * BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)qtiles * BM * bn * 2 + 1024 + 256;
+  return (size_t)qtiles * BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)qtiles * BM * bn * 2 + 1024 + 512;
 }
 
-template <int BN, bool VT, bool PINGPONG, bool PT = false, bool SDB = false>
+template <int BN, bool VT, bool PINGPONG, bool PT = false, bool SDB = false, bool PAR = false>
 rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
                  float* lse, const LaunchCtx& c) {
-  auto kern = PINGPONG ? attn2_kernel<BN, VT, PT, SDB> : attn_kernel<BN, VT>;
+  static_assert(!PAR || (PT && !SDB), "split UMMA issue: P in TMEM");
+  // PAR: two query tiles with one issuing warp each (attn3), or one query tile
+  // with two S buffers and separate S and P V issuers (attn4)
+  auto kern = PAR ? (PINGPONG ? attn3_kernel<BN, VT> : attn4_kernel<BN, VT>)
+                  : PINGPONG ? attn2_kernel<BN, VT, PT, SDB> : attn_kernel<BN, VT>;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
@@ -766,10 +1572,21 @@ rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const vo
   p.status = c.status;
   const long long ctas = (long long)p.B * p.Hq * (PINGPONG ? (p.q_blocks + 1) / 2 : p.q_blocks);
   if (ctas > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
-  const size_t smem = smem_bytes(BN, k.stages, PINGPONG ? 2 : 1) - (PT ? (size_t)2 * BM * BN * 2 : 0);
-  kern<<<(unsigned)ctas, PINGPONG ? kThreads2 : kThreads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  const int qtiles = PINGPONG ? 2 : 1;
+  const size_t smem = smem_bytes(BN, k.stages, qtiles) - (PT ? (size_t)qtiles * BM * BN * 2 : 0);
+  const int threads = PAR ? (PINGPONG ? kThreads3 : kThreads4) : PINGPONG ? kThreads2 : kThreads;
+  kern<<<(unsigned)ctas, threads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
   cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention launch: %s", cudaGetErrorString(e));
+  if (e != cudaSuccess) {
+    cudaFuncAttributes fa;
+    memset(&fa, 0, sizeof fa);
+    cudaFuncGetAttributes(&fa, kern);
+    return rc_fail(RC_ERR_CUDA,
+                   "attention launch: %s (%d threads, %zu B dynamic shared memory; kernel: %d registers, %zu B static "
+                   "and at most %d B dynamic shared memory, at most %d threads)",
+                   cudaGetErrorString(e), threads, smem, fa.numRegs, fa.sharedSizeBytes, fa.maxDynamicSharedSizeBytes,
+                   fa.maxThreadsPerBlock);
+  }
   return RC_OK;
 }
 
@@ -793,15 +1610,24 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
   const bool pp = k.tile_m == 256;  // two query tiles per CTA, ping-pong softmax
   if (pp && k.stages < 2) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: ping-pong needs >= 2 stages");
   const bool pt = k.location == 1;  // P kept in tensor memory
-  if (pt && !pp) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: P in TMEM needs the ping-pong kernel");
+  if (pt && !pp && k.persistent != 1)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: P in TMEM needs two query tiles or split UMMA issue");
   if (k.unroll == 2) {  // two key blocks in flight per query tile
-    if (!(pp && pt && k.tile_n == 64 && k.stages >= 4))
+    if (!(pp && pt && k.tile_n == 64 && k.stages >= 4) || k.persistent)
       return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: unroll 2 needs 2 query tiles, P in TMEM, BN 64, 4 stages");
     return vt ? attn::launch<64, true, true, true, true>(k, d, Q, K, Vuse, O, lse, c)
               : attn::launch<64, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c);
   }
+  const bool par = k.persistent == 1;  // UMMA issue split over two warps
+  if (par && !pt) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: split UMMA issue needs P in TMEM");
+  if (par && !pp && k.stages < 2)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: two S buffers need at least two K/V stages");
 #define RC_ATT(BN)                                                                                  \
   if (k.tile_n == BN) {                                                                             \
+    if (par && pp) return vt ? attn::launch<BN, true, true, true, false, true>(k, d, Q, K, Vuse, O, lse, c) \
+                             : attn::launch<BN, false, true, true, false, true>(k, d, Q, K, Vuse, O, lse, c); \
+    if (par) return vt ? attn::launch<BN, true, false, true, false, true>(k, d, Q, K, Vuse, O, lse, c) \
+                       : attn::launch<BN, false, false, true, false, true>(k, d, Q, K, Vuse, O, lse, c); \
     if (pp && pt) return vt ? attn::launch<BN, true, true, true>(k, d, Q, K, Vuse, O, lse, c)       \
                             : attn::launch<BN, false, true, true>(k, d, Q, K, Vuse, O, lse, c);     \
     if (pp) return vt ? attn::launch<BN, true, true>(k, d, Q, K, Vuse, O, lse, c)                   \

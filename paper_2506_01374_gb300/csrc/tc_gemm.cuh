@@ -303,6 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!tc::mbar_wait_drain(&full[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u))
           fail(RC_DEV_TIMEOUT_DRAIN);
     }
+    __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);

@@ -23,10 +23,11 @@ def att_op(B, S, Hq, Hkv, causal=True):
     return rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=128, causal=int(causal))
 
 
-def sched(op, bn, stages, raster, layout, bm=128, p_tmem=0, unroll=1):
+def sched(op, bn, stages, raster, layout, bm=128, p_tmem=0, unroll=1, par=0):
     return op.schedule(rc.T(rc.T_TILE_SIZE, bm, axis=0), rc.T(rc.T_TILE_SIZE, bn, axis=1),
                        rc.T(rc.T_PIPELINE_STAGES, stages), rc.T(rc.T_LOOP_ORDER, raster, group=1),
-                       rc.T(rc.T_LAYOUT, layout), rc.T(rc.T_COMPUTE_LOCATION, p_tmem), rc.T(rc.T_UNROLL, unroll))
+                       rc.T(rc.T_LAYOUT, layout), rc.T(rc.T_COMPUTE_LOCATION, p_tmem), rc.T(rc.T_UNROLL, unroll),
+                       rc.T(rc.T_PARALLEL, par))
 
 
 def run(op, s, Q, K, V):
@@ -45,19 +46,21 @@ def test_attention_schedule_sweep(B, S, Hq, Hkv, causal):
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=causal)
     op = att_op(B, S, Hq, Hkv, causal)
     n = 0
-    for bm, bn, st, ra, lay, pt, un in itertools.product((128, 256), (64, 128), (1, 2, 3, 4), (0, 1), (0, 1), (0, 1),
-                                                         (1, 2)):
+    for bm, bn, st, ra, lay, pt, un, par in itertools.product((128, 256), (64, 128), (1, 2, 3, 4), (0, 1), (0, 1),
+                                                              (0, 1), (1, 2), (0, 1)):
         try:
-            s = sched(op, bn, st, ra, lay, bm, pt, un)
+            s = sched(op, bn, st, ra, lay, bm, pt, un, par)
         except rc.RcError:
             continue  # illegal here (shared memory, S % 8 for the transposed V, variant combinations)
         O, L = run(op, s, Q, K, V)
-        assert rel_err(O, O_ref) <= TOL, (bm, bn, st, ra, lay, pt, un, rel_err(O, O_ref))
-        assert rel_err(L, L_ref) <= TOL_LSE, (bm, bn, st, ra, lay, pt, un)
+        assert rel_err(O, O_ref) <= TOL, (bm, bn, st, ra, lay, pt, un, par, rel_err(O, O_ref))
+        assert rel_err(L, L_ref) <= TOL_LSE, (bm, bn, st, ra, lay, pt, un, par)
         n += 1
-    assert n >= 16
+    assert n >= 24
     with pytest.raises(rc.RcError):  # one K/V stage cannot feed the ping-pong kernel
         sched(op, 64, 1, 0, 0, 256)
+    with pytest.raises(rc.RcError):  # per-tile issuers exist only for two tiles with P in TMEM
+        sched(op, 64, 2, 0, 0, 256, 0, 1, 1)
 
 
 def test_attention_single_token_and_no_lse():
@@ -80,7 +83,10 @@ def test_attention_full_size_sampled_queries():
     op = att_op(B, S, Hq, Hkv)
     for s in [op.schedule(), sched(op, 128, 2, 1, 0), sched(op, 64, 3, 0, 1), sched(op, 64, 3, 1, 0, 256),
               sched(op, 64, 2, 1, 1, 256), sched(op, 128, 2, 1, 0, 256, 1), sched(op, 64, 3, 1, 1, 256, 1),
-              sched(op, 64, 4, 1, 0, 256, 1, 2), sched(op, 64, 5, 0, 1, 256, 1, 2)]:
+              sched(op, 64, 4, 1, 0, 256, 1, 2), sched(op, 64, 5, 0, 1, 256, 1, 2),
+              sched(op, 128, 2, 1, 0, 256, 1, 1, 1), sched(op, 128, 2, 0, 1, 256, 1, 1, 1),
+              sched(op, 64, 5, 1, 0, 256, 1, 1, 1), sched(op, 128, 2, 1, 0, 128, 1, 1, 1),
+              sched(op, 128, 3, 0, 1, 128, 1, 1, 1), sched(op, 64, 4, 1, 0, 128, 1, 1, 1)]:
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
