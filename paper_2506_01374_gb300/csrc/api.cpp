@@ -16,18 +16,23 @@ thread_local std::string g_err;
 
 constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
 
-// Tensor-core GEMM shared-memory footprint: a ring of `stages` A (128 x 64)
-// and B (bn x 64) bf16 tiles plus 1 KB alignment slack and barriers.
-int64_t tc_smem_bytes(int bn_mma, int stages) {
-  return (int64_t)stages * (128 * 64 * 2 + (int64_t)bn_mma * 64 * 2) + 1024 + 256;
+// Tensor-core GEMM shared-memory footprint: a ring of `stages` stages of
+// tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64) bf16 tile,
+// plus 1 KB alignment slack and barriers.
+int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k) {
+  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + (int64_t)bn_mma * 64 * 2) + 1024 + 256;
 }
 
-bool tc_gemm_ok(int bn_mma, int stages, std::string* why) {
+bool tc_gemm_ok(int bn_mma, int stages, int tile_k, std::string* why) {
   if (bn_mma % 16 != 0 || bn_mma < 16 || bn_mma > 256) {
     if (why) *why = "UMMA N must be a multiple of 16 in [16, 256]";
     return false;
   }
-  if (tc_smem_bytes(bn_mma, stages) > kSmemLimit) {
+  if (tile_k != 64 && tile_k != 128) {
+    if (why) *why = "K per stage must be 64 or 128";
+    return false;
+  }
+  if (tc_smem_bytes(bn_mma, stages, tile_k) > kSmemLimit) {
     if (why) *why = "operand ring exceeds 227 KB of shared memory";
     return false;
   }
@@ -84,6 +89,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
   const int kind = op->d.kind;
   auto gemm_common = [&](std::vector<int32_t> tn) {
     v.push_back({RC_T_TILE_SIZE, 1, tn, {}});
+    v.push_back({RC_T_TILE_SIZE, 2, {64, 128}, {}});  // K per ring stage: one or two 64-wide sub-blocks
     v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 6}, {}});
     v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1, 8}});
     v.push_back({RC_T_PARALLEL, 0, {0, 1}, {}});  // one CTA per tile, or persistent CTAs
@@ -224,20 +230,20 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
   const rc_op_desc& o = op->d;
   switch (o.kind) {
     case RC_OP_LINEAR:
-      return tc_gemm_ok(k.tile_n, k.stages, why);
+      return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, why);
     case RC_OP_SWIGLU:
-      return tc_gemm_ok(2 * k.tile_n, k.stages, why);
+      return tc_gemm_ok(2 * k.tile_n, k.stages, k.tile_k, why);
     case RC_OP_MLP:
-      return tc_gemm_ok(stage == 0 ? 2 * k.tile_n : k.tile_n, k.stages, why);
+      return tc_gemm_ok(stage == 0 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, why);
     case RC_OP_CONV2D:
       if (o.c_out % k.tile_n != 0) {
         if (why) *why = "conv N tile must divide Cout";
         return false;
       }
-      return tc_gemm_ok(k.tile_n, k.stages, why);
+      return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, why);
     case RC_OP_MOE:
       if (stage == 0) return true;
-      return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, why);
+      return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, why);
     case RC_OP_ATTENTION: {
       // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
       const int64_t qt = k.tile_m / 128;

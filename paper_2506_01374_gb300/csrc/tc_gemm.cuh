@@ -4,17 +4,25 @@
 // One CTA computes one 128 x BN output tile (cta_group::1, UMMA M = 128):
 //   warp 0     : TMA producer. One elected thread streams 128 x 64 A tiles and
 //                BN x 64 B tiles (128-byte swizzle) into a ring of `stages`
-//                shared-memory buffers, signalling a "full" mbarrier per stage.
+//                shared-memory buffers, one or two such 64-wide K sub-blocks
+//                per stage (TileSize K = 64 or 128), signalling a "full"
+//                mbarrier per stage.
 //   warp 1     : allocates TMEM, and one elected thread issues 4 UMMAs
-//                (K = 16 each) per stage, releasing the stage through
+//                (K = 16 each) per sub-block, releasing the stage through
 //                tcgen05.commit onto its "empty" mbarrier; a final commit
 //                signals the accumulator.
+// Both control threads keep their ring slot, phase and (for convolutions)
+// filter-tap position in counters: a single thread runs dependent integer
+// code at a few cycles per instruction, so a division per k-block costs about
+// as much as the k-block's UMMAs. A stage of two sub-blocks halves the barrier
+// waits and commits per UMMA.
 //   warps 2..5 : epilogue. Warp w reads TMEM lanes 32*(w%4) .. +31 with
 //                tcgen05.ld (one output row per thread), applies the fused
 //                epilogue and stores 16-byte vectors.
 //
 // Schedule knobs that select variants here: the N tile (template BN), the
-// ring depth (runtime `stages`), split-K (grid z), tile raster order and
+// K sub-blocks per stage (runtime `ksub`), the ring depth (runtime
+// `stages`), split-K (work items), tile raster order and
 // group (runtime), and the fused epilogue (template EPI). The A operand is a
 // plain matrix or, for convolutions, an implicit im2col view loaded with a
 // 4-D TMA box whose out-of-range coordinates are zero-filled (the padding).
@@ -56,6 +64,7 @@ struct Params {
   int* status;
   int persistent;       // 1: grid-stride loop over tiles with two TMEM accumulators
   int splits;           // split-K factor (work items = tiles x splits)
+  int ksub;             // 64-wide K sub-blocks per ring stage (1 or 2)
 };
 
 // Linear CTA index -> (m tile, n tile) under the raster order knob.
@@ -202,11 +211,13 @@ template <int BN, int EPI, int AMODE, bool GROUPED>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const Params p,
                 const int stages) {
-  constexpr int A_BYTES = BM * BK * 2;
-  constexpr int B_BYTES = BN * BK * 2;
-  constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  constexpr int A_BYTES = BM * BK * 2;  // one 64-wide K sub-block of A
+  constexpr int B_BYTES = BN * BK * 2;  // and of B
   constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   static_assert(B_BYTES % 1024 == 0, "B tile must keep stage buffers 1024-byte aligned");
+  // stage layout: A sub-blocks [0, ksub), then B sub-blocks [0, ksub)
+  const int ksub = p.ksub;
+  const uint32_t STAGE_BYTES = (uint32_t)ksub * (A_BYTES + B_BYTES);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -252,48 +263,68 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       tc::prefetch_tmap(&tmA);
       tc::prefetch_tmap(&tmB);
-      uint32_t g = 0;  // k-blocks issued so far (ring position)
+      uint32_t g = 0;   // stages filled so far
+      int s = 0;        // ring slot g % stages
+      uint32_t ph = 0;  // its phase parity (g / stages) & 1
       bool ok = true;
       for (long long w = blockIdx.x; ok && w < items; w += gridDim.x) {
         const Item it = resolve_item<GROUPED>(p, w);
         if (!it.valid) continue;
-        for (int i = 0; i < it.nkb; ++i, ++g) {
-          const int s = (int)(g % (uint32_t)stages);
-          const uint32_t ph = (g / (uint32_t)stages) & 1u;
+        // convolutions: image and first output row of the tile; filter tap
+        // (rr, ss) and channel block cb of the current k sub-block
+        int img = 0, prow = 0, rr = 0, ss = 0, cb = 0;
+        if constexpr (AMODE == TC_A_CONV || AMODE == TC_A_CONV_ROWS) {
+          img = it.row0 / p.img_hw;
+          prow = (it.row0 - img * p.img_hw) / p.img_w;
+          const int rs = it.kb0 / p.cblocks;
+          cb = it.kb0 - rs * p.cblocks;
+          rr = rs / p.ks;
+          ss = rs - rr * p.ks;
+        }
+        int kb = it.kb0;
+        for (int i = 0; i < it.nkb; i += ksub, ++g) {
+          const int nsub = min(ksub, it.nkb - i);
           if (!tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status)) {
             fail(RC_DEV_TIMEOUT_EMPTY);
             ok = false;
             break;
           }
-          uint8_t* sa = smem + (size_t)s * STAGE_BYTES;
-          uint8_t* sb = sa + A_BYTES;
-          tc::mbar_expect_tx(&full[s], STAGE_BYTES);
-          const int kb = it.kb0 + i;
-          if constexpr (AMODE == TC_A_CONV) {
-            const int rs = kb / p.cblocks, cb = kb - rs * p.cblocks;
-            const int rr = rs / p.ks, ss = rs - rr * p.ks;
-            const int img = it.row0 / p.img_hw;
-            const int prow = (it.row0 - img * p.img_hw) / p.img_w;
-            tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
-          } else if constexpr (AMODE == TC_A_CONV_ROWS) {
-            // padded input [N][Hp][Wp][C] as rows of pixels: image row i of the tile, shifted by (r, s)
-            const int rs = kb / p.cblocks, cb = kb - rs * p.cblocks;
-            const int rr = rs / p.ks, ss = rs - rr * p.ks;
-            const int img = it.row0 / p.img_hw;
-            const int prow = (it.row0 - img * p.img_hw) / p.img_w;
-            const int wp = p.img_w + 2 * p.pad_rows, hp = p.img_hw / p.img_w + 2 * p.pad_rows;
-            for (int i = 0; i < BM / p.img_w; ++i)
-              tc::tma_load_2d(sa + i * p.img_w * 128, &tmA, &full[s], cb * 64,
-                              (img * hp + prow + i + rr) * wp + ss);
-          } else {
-            tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, it.row0);
+          uint8_t* stage = smem + (size_t)s * STAGE_BYTES;
+          tc::mbar_expect_tx(&full[s], (uint32_t)nsub * (A_BYTES + B_BYTES));
+          for (int q = 0; q < nsub; ++q, ++kb) {
+            uint8_t* sa = stage + q * A_BYTES;
+            uint8_t* sb = stage + ksub * A_BYTES + q * B_BYTES;
+            if constexpr (AMODE == TC_A_CONV) {
+              tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
+            } else if constexpr (AMODE == TC_A_CONV_ROWS) {
+              // padded input [N][Hp][Wp][C] as rows of pixels: image row r of the tile, shifted by (rr, ss)
+              const int wp = p.img_w + 2 * p.pad_rows, hp = p.img_hw / p.img_w + 2 * p.pad_rows;
+              for (int r = 0; r < BM / p.img_w; ++r)
+                tc::tma_load_2d(sa + r * p.img_w * 128, &tmA, &full[s], cb * 64,
+                                (img * hp + prow + r + rr) * wp + ss);
+            } else {
+              tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, it.row0);
+            }
+            if constexpr (AMODE == TC_A_CONV || AMODE == TC_A_CONV_ROWS) {
+              if (++cb == p.cblocks) {
+                cb = 0;
+                if (++ss == p.ks) {
+                  ss = 0;
+                  ++rr;
+                }
+              }
+            }
+            if constexpr (EPI == TC_EPI_SWIGLU) {
+              const int nh = it.nt * (BN / 2);
+              tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + nh);
+              tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], kb * BK, it.brow0 + p.swiglu_I + nh);
+            } else {
+              tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + it.nt * BN);
+            }
           }
-          if constexpr (EPI == TC_EPI_SWIGLU) {
-            const int nh = it.nt * (BN / 2);
-            tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + nh);
-            tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], kb * BK, it.brow0 + p.swiglu_I + nh);
-          } else {
-            tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + it.nt * BN);
+          if (++s == stages) {
+            s = 0;
+            ph ^= 1u;
           }
         }
       }
@@ -307,7 +338,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
-      uint32_t g = 0, li = 0;
+      uint32_t li = 0;
+      int s = 0;        // ring slot, advanced in step with the producer
+      uint32_t ph = 0;  // its phase parity
       bool ok = true;
       for (long long w = blockIdx.x; ok && w < items; w += gridDim.x) {
         const Item it = resolve_item<GROUPED>(p, w);
@@ -321,9 +354,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::tc_fence_after();
         const uint32_t dacc = tmem + buf * ACC_COLS;
-        for (int i = 0; i < it.nkb; ++i, ++g) {
-          const int s = (int)(g % (uint32_t)stages);
-          const uint32_t ph = (g / (uint32_t)stages) & 1u;
+        for (int i = 0; i < it.nkb; i += ksub) {
+          const int nsub = min(ksub, it.nkb - i);
           if (!tc::mbar_wait(&full[s], ph, abort_flag, status)) {
             fail(RC_DEV_TIMEOUT_FULL);
             ok = false;
@@ -331,11 +363,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc::tc_fence_after();
           const uint32_t sa = tc::smem_u32(smem + (size_t)s * STAGE_BYTES);
-          const uint64_t da = tc::sw128_desc(sa), db = tc::sw128_desc(sa + A_BYTES);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, (i > 0 || k > 0) ? 1u : 0u);
+          for (int q = 0; q < 2; ++q) {
+            if (q >= nsub) break;
+            const uint64_t da = tc::sw128_desc(sa + q * A_BYTES);
+            const uint64_t db = tc::sw128_desc(sa + ksub * A_BYTES + q * B_BYTES);
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+              tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, (i > 0 || q > 0 || k > 0) ? 1u : 0u);
+          }
           tc::umma_commit(&empty[s]);
+          if (++s == stages) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (!ok) break;
         tc::umma_commit(&acc_full[buf]);  // accumulator ready (also when nkb == 0)
@@ -403,14 +444,16 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
   return RC_OK;
 }
 
-inline size_t smem_bytes(int bn, int stages) {
-  return (size_t)stages * (BM * BK * 2 + (size_t)bn * BK * 2) + 1024 + 256;
+inline size_t smem_bytes(int bn, int stages, int ksub) {
+  return (size_t)stages * ksub * (BM * BK * 2 + (size_t)bn * BK * 2) + 1024 + 256;
 }
 
 template <int BN, int EPI, int AMODE, bool GROUPED>
 rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED>;
-  const size_t smem = smem_bytes(BN, k.stages);
+  if (k.tile_k != 64 && k.tile_k != 128) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: K tile %d", k.tile_k);
+  const int ksub = k.tile_k / 64;
+  const size_t smem = smem_bytes(BN, k.stages, ksub);
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
@@ -443,6 +486,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.kb_per = (p.kb_total + splits - 1) / splits;
   p.splits = splits;
   p.persistent = k.persistent ? 1 : 0;
+  p.ksub = ksub;
   p.raster = k.raster;
   p.group = k.group > 0 ? k.group : 1;
   p.D = a.D;
