@@ -18,9 +18,10 @@ constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
 
 // Tensor-core GEMM shared-memory footprint: a ring of `stages` stages of
 // tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64) bf16 tile,
-// plus 1 KB alignment slack and barriers.
+// plus 1 KB alignment slack, barriers and four fp32 copies of a bias tile.
 int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k) {
-  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + (int64_t)bn_mma * 64 * 2) + 1024 + 256;
+  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + (int64_t)bn_mma * 64 * 2) + 1024 + 256 +
+         4 * (int64_t)bn_mma * 4;
 }
 
 bool tc_gemm_ok(int bn_mma, int stages, int tile_k, std::string* why) {

@@ -95,9 +95,10 @@ __device__ __forceinline__ uint4 pack8(const float* v) {
   return p.u;
 }
 
+// sbias: this warp's copy of the tile's bias (fp32, BN values; BIAS_SILU only)
 template <int BN, int EPI>
 __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r, int row_end, int nt, int split,
-                                         bool have_acc) {
+                                         bool have_acc, const float* sbias) {
   const bool row_ok = r < row_end;
   if constexpr (EPI == TC_EPI_SWIGLU) {
     constexpr int HALF = BN / 2;
@@ -124,22 +125,34 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
     }
   } else {
     const int n0 = nt * BN;
+    // MoE combine: the routed slot of this row and its weight, once per tile
+    long long orow = 0;
+    float scale = 0.f;
+    if constexpr (EPI == TC_EPI_SCALE_ATOMIC) {
+      if (row_ok) {
+        const int slot = p.row_map[r];
+        scale = p.row_scale[slot];
+        orow = slot / p.row_div;
+      }
+    }
 #pragma unroll 1
     for (int c = 0; c < BN; c += 16) {
+      const int col = n0 + c;
       uint32_t a[16];
       tc::tmem_ld16(taddr + c, a);
       tc::tmem_ld_wait();
       float v[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = have_acc ? __uint_as_float(a[j]) : 0.f;
-      const int col = n0 + c;
       if (!row_ok) continue;
       if constexpr (EPI == TC_EPI_STORE_BF16 || EPI == TC_EPI_BIAS_SILU) {
         if constexpr (EPI == TC_EPI_BIAS_SILU) {
+          float bv[16];
+#pragma unroll
+          for (int j = 0; j < 16; j += 4) *reinterpret_cast<float4*>(&bv[j]) = *reinterpret_cast<const float4*>(&sbias[c + j]);
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
-            float x = v[j];
-            if (p.bias && col + j < p.out_cols) x += __bfloat162float(p.bias[col + j]);
+            const float x = v[j] + bv[j];
             v[j] = p.silu ? tc::silu(x) : x;
           }
         }
@@ -153,9 +166,8 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
           if (col + 4 * q < p.out_cols)
             *reinterpret_cast<float4*>(out + col + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
       } else if constexpr (EPI == TC_EPI_SCALE_ATOMIC) {
-        const int slot = p.row_map[r];
-        const float s = p.row_scale[slot];
-        float* out = (float*)p.D + (long long)(slot / p.row_div) * p.ldd;
+        const float s = scale;
+        float* out = (float*)p.D + orow * p.ldd;
 #pragma unroll
         for (int q = 0; q < 4; ++q)
           if (col + 4 * q < p.out_cols)
@@ -229,6 +241,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = (uint32_t*)(drain + 1);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
   volatile int* status = p.status;
+  // one copy of the tile's bias per epilogue warp (BN floats each, 16-byte aligned)
+  float* sbias_all = (float*)(((uintptr_t)(abort_flag + 1) + 15) & ~(uintptr_t)15);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n_acc = p.persistent ? 2 : 1;  // accumulator buffers in TMEM
@@ -390,10 +404,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     const int q = warp & 3;
+    float* sbias = sbias_all + (warp - 2) * BN;
     uint32_t li = 0;
     for (long long w = blockIdx.x; w < items; w += gridDim.x) {
       const Item it = resolve_item<GROUPED>(p, w);
       if (!it.valid) continue;
+      if constexpr (EPI == TC_EPI_BIAS_SILU) {
+        // the tile's bias, loaded while the accumulator is being computed
+        __syncwarp();  // the previous tile's reads of this copy are done
+        for (int j = lane; j < BN; j += 32) {
+          const int col = it.nt * BN + j;
+          sbias[j] = p.bias && col < p.out_cols ? __bfloat162float(p.bias[col]) : 0.f;
+        }
+        __syncwarp();
+      }
       const uint32_t buf = li % (uint32_t)n_acc;
       const uint32_t aph = (li / (uint32_t)n_acc) & 1u;
       if (!tc::mbar_wait(&acc_full[buf], aph, abort_flag, status)) {
@@ -402,7 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc::tc_fence_after();
       epilogue<BN, EPI>(p, tmem + buf * ACC_COLS + ((uint32_t)(32 * q) << 16), it.row0 + 32 * q + lane,
-                        it.row_end, it.nt, it.split, it.nkb > 0);
+                        it.row_end, it.nt, it.split, it.nkb > 0, sbias);
       tc::tc_fence_before();
       tc::mbar_arrive(&acc_empty[buf]);
       ++li;
@@ -444,8 +468,9 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
   return RC_OK;
 }
 
+// ring + 1 KB alignment slack + barriers and flags (256 B) + four fp32 bias copies
 inline size_t smem_bytes(int bn, int stages, int ksub) {
-  return (size_t)stages * ksub * (BM * BK * 2 + (size_t)bn * BK * 2) + 1024 + 256;
+  return (size_t)stages * ksub * (BM * BK * 2 + (size_t)bn * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4;
 }
 
 template <int BN, int EPI, int AMODE, bool GROUPED>
