@@ -49,7 +49,10 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mlp", choices=["mlp", "attention", "conv2d", "moe", "gemm_f32"])
-    ap.add_argument("--samples", type=int, default=1200, help="schedules the search measures")
+    ap.add_argument("--samples", type=int, default=5000, help="schedules the search measures")
+    ap.add_argument("--branching", type=int, default=4,
+                    help="MCTS children per expansion (the paper's 2 assumes LLM-proposed transformations; with "
+                         "random valid proposals a binary tree of depth 8 fills up at 511 nodes)")
     ap.add_argument("--cpu-sample", type=int, default=0,
                     help="size of the CPU-oracle sample (rows/queries/pixels/tokens; 0 = workload default, "
                          "-1 = skip)")
@@ -58,7 +61,9 @@ def parse():
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--ops", default=None,
                     help="other workloads to search and report ('' = none; default: all others for mlp)")
-    ap.add_argument("--op-samples", type=int, default=160, help="schedules measured per extra op")
+    ap.add_argument("--op-samples", type=int, default=600, help="schedules measured per extra op")
+    ap.add_argument("--restarts", type=int, default=2,
+                    help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
     ap.add_argument("--seed", type=int, default=0)
     return ap.parse_args()
 
@@ -316,11 +321,24 @@ def parse_schedule(op, text, rc):
     return op.schedule(*ts)
 
 
-def search_best(op, io, samples, seed=0):
-    """MCTS over op's schedule space with device-timed candidates; returns (search, best, m, n, cand/s)."""
+def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1):
+    """MCTS over op's schedule space with device-timed candidates; returns (search, best, m, n, cand/s).
+
+    Candidates are timed with 5 repeats while searching; the `finalists` best
+    of them are timed again with 20 repeats and the fastest is returned, so a
+    noisy short measurement does not decide the result.
+    """
     from paper_2506_01374_gb300 import rc
-    search = rc.Search(op, seed=seed)
+    if restarts > 1:  # independent searches; rewards are noisy measurements, so trajectories differ
+        runs = [search_best(op, io, samples, seed + r, branching, finalists) for r in range(restarts)]
+        i = min(range(restarts), key=lambda r: runs[r][2].ms_median if runs[r][2].status == rc.OK else float("inf"))
+        search, best, m, _, _ = runs[i]
+        n = sum(r[3] for r in runs)
+        cps = [r[4] for r in runs if r[4]]
+        return search, best, m, n, (sum(cps) / len(cps) if cps else None)
+    search = rc.Search(op, seed=seed, branching=branching)
     res, n, t, pending = [], 0, 0.0, False
+    seen = []  # (median ms, schedule owned by the search)
     while n < samples:
         nxt = search.step(res)
         pending = False
@@ -330,14 +348,21 @@ def search_best(op, io, samples, seed=0):
         res = op.measure(nxt, io, warmup=2, repeats=5)
         t += time.perf_counter() - t0
         n += len(nxt)
+        seen += [(m.ms_median, s) for s, m in zip(nxt, res) if m.status == rc.OK]
         pending = True
     if pending:  # hand the last batch's measurements to the search
         search.step(res)
     best, m = search.best()
+    seen.sort(key=lambda x: x[0])
+    cands = [best] + [sch for _, sch in seen[:finalists]]
+    final = op.measure(cands, io, warmup=3, repeats=20)
+    i = min(range(len(cands)), key=lambda j: final[j].ms_median if final[j].status == rc.OK else float("inf"))
+    if i > 0:
+        best, m = cands[i].clone(), final[i]
     return search, best, m, n, (n / t if t else None)
 
 
-def extra_ops(names, samples, peak_tf):
+def extra_ops(names, samples, peak_tf, branching=4, restarts=1):
     """Search each other workload briefly and report its best schedule."""
     import torch
 
@@ -346,7 +371,7 @@ def extra_ops(names, samples, peak_tf):
     for name in names:
         wl = Workload(name)
         io = wl.device_io()
-        _, best, _, n, cps = search_best(wl.op, io, samples)
+        _, best, _, n, cps = search_best(wl.op, io, samples, branching=branching, restarts=restarts)
         m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
         if m.status != rc.OK:
             out[name] = {"workload": wl.label, "error": rc.STATUS_NAMES.get(m.status, m.status)}
@@ -426,7 +451,8 @@ def run_ours(args):
     if args.schedule:
         best = parse_schedule(op, args.schedule, rc)
     else:
-        search, best, best_m, n_meas, cps = search_best(op, io, args.samples, seed=args.seed)
+        search, best, best_m, n_meas, cps = search_best(op, io, args.samples, seed=args.seed,
+                                                        branching=args.branching, restarts=args.restarts)
 
     # 2) timed steps of the best schedule
     flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
@@ -507,7 +533,7 @@ def run_ours(args):
         if names:
             del io
             torch.cuda.empty_cache()
-            out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"])
+            out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"], args.branching, args.restarts)
         if args.cpu_sample >= 0:
             cb = wl.cpu_sample(args.cpu_sample)
             cb.pop("seconds", None)

@@ -16,24 +16,38 @@ thread_local std::string g_err;
 
 constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
 
-// Tensor-core GEMM shared-memory footprint: a ring of `stages` stages of
-// tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64) bf16 tile,
-// plus 1 KB alignment slack, barriers and four fp32 copies of a bias tile.
-int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k) {
-  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + (int64_t)bn_mma * 64 * 2) + 1024 + 256 +
-         4 * (int64_t)bn_mma * 4;
+// Tensor-core GEMM shared-memory footprint per CTA: a ring of `stages`
+// stages of tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64,
+// or bn/2 x 64 in each CTA of a pair) bf16 tile, plus 1 KB alignment slack,
+// barriers and four fp32 copies of a bias tile.
+int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k, int tile_m) {
+  const int64_t b_rows = tile_m == 256 ? bn_mma / 2 : bn_mma;
+  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + b_rows * 64 * 2) + 1024 + 256 + 4 * (int64_t)bn_mma * 4;
 }
 
-bool tc_gemm_ok(int bn_mma, int stages, int tile_k, std::string* why) {
+bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, std::string* why) {
   if (bn_mma % 16 != 0 || bn_mma < 16 || bn_mma > 256) {
     if (why) *why = "UMMA N must be a multiple of 16 in [16, 256]";
+    return false;
+  }
+  if (tile_m != 128 && tile_m != 256) {
+    if (why) *why = "M tile must be 128 (one CTA) or 256 (a CTA pair)";
+    return false;
+  }
+  if (tile_m == 256 && bn_mma < 32) {
+    if (why) *why = "a CTA pair splits the N tile: at least 32 columns";
+    return false;
+  }
+  if (tile_m == 256 && persistent && bn_mma > 128) {
+    // a pair holds at most 256 TMEM columns (two accumulators of <= 128)
+    if (why) *why = "persistent CTA pairs need N tiles of at most 128";
     return false;
   }
   if (tile_k != 64 && tile_k != 128) {
     if (why) *why = "K per stage must be 64 or 128";
     return false;
   }
-  if (tc_smem_bytes(bn_mma, stages, tile_k) > kSmemLimit) {
+  if (tc_smem_bytes(bn_mma, stages, tile_k, tile_m) > kSmemLimit) {
     if (why) *why = "operand ring exceeds 227 KB of shared memory";
     return false;
   }
@@ -104,10 +118,12 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       break;
     case RC_OP_LINEAR:
       gemm_common({64, 128, 224, 256});
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // one CTA, or a CTA pair sharing each UMMA
       v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       break;
     case RC_OP_SWIGLU:
       gemm_common({32, 64, 128});
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
       break;
     case RC_OP_MLP:
@@ -118,9 +134,11 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       }
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       break;
     case RC_OP_CONV2D:
       gemm_common({64, 80, 160});
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       v.push_back({RC_T_SPLIT_K, 0, {1, 3, 5}, {}});
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
       // implicit zero padding (one 4-D box), or a padded copy read as one 4-D box or as row boxes
@@ -231,20 +249,24 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
   const rc_op_desc& o = op->d;
   switch (o.kind) {
     case RC_OP_LINEAR:
-      return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, why);
+      return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_SWIGLU:
-      return tc_gemm_ok(2 * k.tile_n, k.stages, k.tile_k, why);
+      return tc_gemm_ok(2 * k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_MLP:
-      return tc_gemm_ok(stage == 0 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, why);
+      return tc_gemm_ok(stage == 0 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_CONV2D:
       if (o.c_out % k.tile_n != 0) {
         if (why) *why = "conv N tile must divide Cout";
         return false;
       }
-      return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, why);
+      if (k.tile_m == 256 && k.layout == 2) {
+        if (why) *why = "a CTA pair loads A as one 4-D box (layouts 0 and 1)";
+        return false;
+      }
+      return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_MOE:
       if (stage == 0) return true;
-      return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, why);
+      return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_ATTENTION: {
       // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
       const int64_t qt = k.tile_m / 128;

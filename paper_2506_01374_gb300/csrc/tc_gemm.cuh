@@ -219,12 +219,21 @@ __device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
   return it;
 }
 
-template <int BN, int EPI, int AMODE, bool GROUPED>
+// PAIR (TileSize M = 256): a cluster of two CTAs computes a 256 x BN tile
+// with cta_group::2 UMMAs. Each CTA loads its own 128 rows of A and half of
+// the B tile (rows [0, BN/2) in the leader, [BN/2, BN) in the peer; for the
+// fused SwiGLU the gate rows and the up rows), and both CTAs' copies complete
+// on the leader's "full" barrier. The leader's MMA thread issues M = 256
+// UMMAs and multicasts its commits to both CTAs' "empty" and "accumulator
+// full" barriers; each CTA's epilogue drains its own TMEM rows and arrives
+// on the leader's "accumulator empty" barrier (one arrival per warp).
+template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const Params p,
                 const int stages) {
-  constexpr int A_BYTES = BM * BK * 2;  // one 64-wide K sub-block of A
-  constexpr int B_BYTES = BN * BK * 2;  // and of B
+  static_assert(!PAIR || !GROUPED, "CTA pairs are for dense and convolution GEMMs");
+  constexpr int A_BYTES = BM * BK * 2;                    // one 64-wide K sub-block of A
+  constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * BK * 2;  // and this CTA's rows of B
   constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   static_assert(B_BYTES % 1024 == 0, "B tile must keep stage buffers 1024-byte aligned");
   // stage layout: A sub-blocks [0, ksub), then B sub-blocks [0, ksub)
@@ -247,7 +256,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n_acc = p.persistent ? 2 : 1;  // accumulator buffers in TMEM
   const uint32_t tmem_cols = ACC_COLS * (uint32_t)n_acc;
-  const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;
+  const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;  // tiles of 128 (PAIR: 256) rows
+  const uint32_t rank = PAIR ? tc::cluster_ctarank() : 0u;              // 0 = leader of the pair
+  const long long w_first = PAIR ? blockIdx.x / 2 : blockIdx.x;
+  const long long w_step = PAIR ? gridDim.x / 2 : gridDim.x;
+  auto item = [&](long long w) -> Item {
+    Item it = resolve_item<GROUPED>(p, w);
+    if constexpr (PAIR) it.row0 = 2 * it.row0 + (int)rank * BM;  // this CTA's half of the 256-row tile
+    return it;
+  };
 
   auto fail = [&](int code) {
     *abort_flag = 1;
@@ -261,15 +278,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       tc::mbar_init(&acc_full[b], 1);
-      tc::mbar_init(&acc_empty[b], 128);
+      tc::mbar_init(&acc_empty[b], PAIR ? 8 : 128);  // PAIR: one arrival per epilogue warp of either CTA
     }
     tc::mbar_init(drain, 1);
     *abort_flag = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 1) tc::tmem_alloc(tmem_slot, tmem_cols);
+  if (warp == 1) {
+    if constexpr (PAIR)
+      tc::tmem_alloc_pair(tmem_slot, tmem_cols);
+    else
+      tc::tmem_alloc(tmem_slot, tmem_cols);
+  }
   tc::tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR)
+    tc::cluster_sync();  // both CTAs' barriers exist before any copy or commit reaches them
+  else
+    __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
@@ -281,8 +306,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int s = 0;        // ring slot g % stages
       uint32_t ph = 0;  // its phase parity (g / stages) & 1
       bool ok = true;
-      for (long long w = blockIdx.x; ok && w < items; w += gridDim.x) {
-        const Item it = resolve_item<GROUPED>(p, w);
+      for (long long w = w_first; ok && w < items; w += w_step) {
+        const Item it = item(w);
         if (!it.valid) continue;
         // convolutions: image and first output row of the tile; filter tap
         // (rr, ss) and channel block cb of the current k sub-block
@@ -304,20 +329,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           uint8_t* stage = smem + (size_t)s * STAGE_BYTES;
-          tc::mbar_expect_tx(&full[s], (uint32_t)nsub * (A_BYTES + B_BYTES));
+          // PAIR: the leader's barrier counts both CTAs' bytes
+          const uint32_t cbar = PAIR ? tc::mapa_shared(tc::smem_u32(&full[s]), 0) : 0u;
+          if (rank == 0) tc::mbar_expect_tx(&full[s], (uint32_t)nsub * (PAIR ? 2 : 1) * (A_BYTES + B_BYTES));
+          auto ld2 = [&](void* dst, const CUtensorMap* m, int x, int y) {
+            if constexpr (PAIR)
+              tc::tma_load_2d_pair(dst, m, cbar, x, y);
+            else
+              tc::tma_load_2d(dst, m, &full[s], x, y);
+          };
           for (int q = 0; q < nsub; ++q, ++kb) {
             uint8_t* sa = stage + q * A_BYTES;
             uint8_t* sb = stage + ksub * A_BYTES + q * B_BYTES;
             if constexpr (AMODE == TC_A_CONV) {
-              tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
+              if constexpr (PAIR)
+                tc::tma_load_4d_pair(sa, &tmA, cbar, cb * 64, ss - p.pad, prow + rr - p.pad, img);
+              else
+                tc::tma_load_4d(sa, &tmA, &full[s], cb * 64, ss - p.pad, prow + rr - p.pad, img);
             } else if constexpr (AMODE == TC_A_CONV_ROWS) {
               // padded input [N][Hp][Wp][C] as rows of pixels: image row r of the tile, shifted by (rr, ss)
               const int wp = p.img_w + 2 * p.pad_rows, hp = p.img_hw / p.img_w + 2 * p.pad_rows;
               for (int r = 0; r < BM / p.img_w; ++r)
-                tc::tma_load_2d(sa + r * p.img_w * 128, &tmA, &full[s], cb * 64,
-                                (img * hp + prow + r + rr) * wp + ss);
+                ld2(sa + r * p.img_w * 128, &tmA, cb * 64, (img * hp + prow + r + rr) * wp + ss);
             } else {
-              tc::tma_load_2d(sa, &tmA, &full[s], kb * BK, it.row0);
+              ld2(sa, &tmA, kb * BK, it.row0);
             }
             if constexpr (AMODE == TC_A_CONV || AMODE == TC_A_CONV_ROWS) {
               if (++cb == p.cblocks) {
@@ -330,10 +365,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if constexpr (EPI == TC_EPI_SWIGLU) {
               const int nh = it.nt * (BN / 2);
-              tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + nh);
-              tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], kb * BK, it.brow0 + p.swiglu_I + nh);
+              if constexpr (PAIR) {  // gate rows in the leader, up rows in the peer
+                ld2(sb, &tmB, kb * BK, it.brow0 + (rank ? p.swiglu_I : 0) + nh);
+              } else {
+                ld2(sb, &tmB, kb * BK, it.brow0 + nh);
+                ld2(sb + (BN / 2) * 128, &tmB, kb * BK, it.brow0 + p.swiglu_I + nh);
+              }
             } else {
-              tc::tma_load_2d(sb, &tmB, &full[s], kb * BK, it.brow0 + it.nt * BN);
+              ld2(sb, &tmB, kb * BK, it.brow0 + it.nt * BN + (int)rank * (BN / 2));
             }
           }
           if (++s == stages) {
@@ -343,21 +382,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       // let the copies issued in the last `stages` ring slots land before exit
+      // (PAIR peer: its copies complete on the leader's barrier; it waits
+      // instead, bounded, for the leader's release of those slots)
       const uint32_t first = g > (uint32_t)stages ? g - (uint32_t)stages : 0u;
-      for (uint32_t j = first; j < g; ++j)
-        if (!tc::mbar_wait_drain(&full[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u))
-          fail(RC_DEV_TIMEOUT_DRAIN);
+      for (uint32_t j = first; j < g; ++j) {
+        if (rank == 0) {
+          if (!tc::mbar_wait_drain(&full[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u))
+            fail(RC_DEV_TIMEOUT_DRAIN);
+        } else {
+          tc::mbar_wait_drain(&empty[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u);
+        }
+      }
     }
     __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idesc = tc::idesc_bf16_f32(BM, BN);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = tc::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN);
       uint32_t li = 0;
       int s = 0;        // ring slot, advanced in step with the producer
       uint32_t ph = 0;  // its phase parity
       bool ok = true;
-      for (long long w = blockIdx.x; ok && w < items; w += gridDim.x) {
-        const Item it = resolve_item<GROUPED>(p, w);
+      for (long long w = w_first; ok && w < items; w += w_step) {
+        const Item it = item(w);
         if (!it.valid) continue;
         const uint32_t buf = li % (uint32_t)n_acc;
         const uint32_t aph = (li / (uint32_t)n_acc) & 1u;
@@ -383,21 +429,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t da = tc::sw128_desc(sa + q * A_BYTES);
             const uint64_t db = tc::sw128_desc(sa + ksub * A_BYTES + q * B_BYTES);
 #pragma unroll
-            for (int k = 0; k < BK / 16; ++k)
-              tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, (i > 0 || q > 0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < BK / 16; ++k) {
+              const uint32_t acc = (i > 0 || q > 0 || k > 0) ? 1u : 0u;
+              if constexpr (PAIR)
+                tc::umma_bf16_pair(dacc, da + 2 * k, db + 2 * k, idesc, acc);
+              else
+                tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, acc);
+            }
           }
-          tc::umma_commit(&empty[s]);
+          if constexpr (PAIR)
+            tc::umma_commit_pair(&empty[s], 3);  // the slot is free in both CTAs
+          else
+            tc::umma_commit(&empty[s]);
           if (++s == stages) {
             s = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        tc::umma_commit(&acc_full[buf]);  // accumulator ready (also when nkb == 0)
+        if constexpr (PAIR)
+          tc::umma_commit_pair(&acc_full[buf], 3);
+        else
+          tc::umma_commit(&acc_full[buf]);  // accumulator ready (also when nkb == 0)
         ++li;
       }
       if (!ok) {
-        tc::umma_commit(drain);  // wait for the MMAs already issued before TMEM is freed
+        if constexpr (PAIR)
+          tc::umma_commit_pair(drain, 1);
+        else
+          tc::umma_commit(drain);  // wait for the MMAs already issued before TMEM is freed
         if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
       }
     }
@@ -406,8 +466,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;
     float* sbias = sbias_all + (warp - 2) * BN;
     uint32_t li = 0;
-    for (long long w = blockIdx.x; w < items; w += gridDim.x) {
-      const Item it = resolve_item<GROUPED>(p, w);
+    for (long long w = w_first; w < items; w += w_step) {
+      const Item it = item(w);
       if (!it.valid) continue;
       if constexpr (EPI == TC_EPI_BIAS_SILU) {
         // the tile's bias, loaded while the accumulator is being computed
@@ -428,16 +488,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       epilogue<BN, EPI>(p, tmem + buf * ACC_COLS + ((uint32_t)(32 * q) << 16), it.row0 + 32 * q + lane,
                         it.row_end, it.nt, it.split, it.nkb > 0, sbias);
       tc::tc_fence_before();
-      tc::mbar_arrive(&acc_empty[buf]);
+      if constexpr (PAIR) {
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive_cluster(tc::mapa_shared(tc::smem_u32(&acc_empty[buf]), 0));
+      } else {
+        tc::mbar_arrive(&acc_empty[buf]);
+      }
       ++li;
     }
   }
   tc::tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR)
+    tc::cluster_sync();  // no copy, commit or arrival may reach a CTA that has exited
+  else
+    __syncthreads();
   if (warp == 1) {
     __syncwarp();
     tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, tmem_cols);
+    if constexpr (PAIR)
+      tc::tmem_dealloc_pair(tmem, tmem_cols);
+    else
+      tc::tmem_dealloc(tmem, tmem_cols);
   }
 }
 
@@ -448,37 +519,57 @@ rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uin
 
 template <typename Kern>
 rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tmB, const Params& p, int stages,
-                        int acc_cols, size_t smem, const LaunchCtx& c) {
+                        int acc_cols, size_t smem, bool pair, const LaunchCtx& c) {
   const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;
-  if (items <= 0 || items > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: %lld work items", items);
-  long long ctas = items;
+  if (items <= 0 || items > 0x3fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: %lld work items", items);
+  const int per_item = pair ? 2 : 1;  // CTAs per work item
+  long long ctas = items * per_item;
   if (p.persistent) {
     // as many CTAs as fit on the SMs at once (shared memory and 512 TMEM columns)
     long long per_sm = 233472 / (long long)(smem + 1024);
     const long long by_tmem = 512 / (2LL * acc_cols);
     if (by_tmem < per_sm) per_sm = by_tmem;
     if (per_sm < 1) per_sm = 1;
-    const long long resident = per_sm * (c.num_sms > 0 ? c.num_sms : 1);
+    long long resident = per_sm * (c.num_sms > 0 ? c.num_sms : 1);
+    resident -= resident % per_item;
     if (resident < ctas) ctas = resident;
   }
-  dim3 grid((unsigned)ctas, 1, 1);
-  kern<<<grid, kThreads, smem, (cudaStream_t)c.stream>>>(tmA, tmB, p, stages);
-  cudaError_t e = cudaGetLastError();
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof cfg);
+  cfg.gridDim = dim3((unsigned)ctas, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = (cudaStream_t)c.stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)per_item;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pair ? 1 : 0;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmA, tmB, p, stages);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
   return RC_OK;
 }
 
-// ring + 1 KB alignment slack + barriers and flags (256 B) + four fp32 bias copies
-inline size_t smem_bytes(int bn, int stages, int ksub) {
-  return (size_t)stages * ksub * (BM * BK * 2 + (size_t)bn * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4;
+// ring of A (128 rows) and this CTA's B rows (bn, or bn / 2 for a CTA pair)
+// per sub-block + 1 KB alignment slack + barriers and flags (256 B) + four
+// fp32 bias copies of the bn-column tile
+inline size_t smem_bytes(int bn, int stages, int ksub, bool pair = false) {
+  const size_t b_rows = pair ? (size_t)bn / 2 : (size_t)bn;
+  return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4;
 }
 
-template <int BN, int EPI, int AMODE, bool GROUPED>
+template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
 rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
-  auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED>;
+  auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED, PAIR>;
   if (k.tile_k != 64 && k.tile_k != 128) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: K tile %d", k.tile_k);
+  constexpr int acc_cols_tile = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  if (PAIR && (k.persistent ? 2 : 1) * acc_cols_tile > 256)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: a CTA pair holds at most 256 TMEM columns");
   const int ksub = k.tile_k / 64;
-  const size_t smem = smem_bytes(BN, k.stages, ksub);
+  const size_t smem = smem_bytes(BN, k.stages, ksub, PAIR);
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
@@ -496,7 +587,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
     RC_TRY(encode_2d(&tmA, a.A, a.K, a.M, BM));
   }
   const int64_t b_rows = GROUPED ? (int64_t)a.groups * a.b_group_rows : a.N;
-  RC_TRY(encode_2d(&tmB, a.B, a.K, b_rows, EPI == TC_EPI_SWIGLU ? BN / 2 : BN));
+  RC_TRY(encode_2d(&tmB, a.B, a.K, b_rows, (PAIR || EPI == TC_EPI_SWIGLU) ? BN / 2 : BN));
   Params p;
   memset(&p, 0, sizeof p);
   p.M = (int)a.M;
@@ -505,7 +596,8 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   const int out_w = EPI == TC_EPI_SWIGLU ? (int)(a.N / 2) : (int)a.N;
   const int tile_out = EPI == TC_EPI_SWIGLU ? BN / 2 : BN;
   p.tiles_n = (out_w + tile_out - 1) / tile_out;
-  p.tiles_m = GROUPED ? (int)a.max_tiles_m : (int)((a.M + BM - 1) / BM);
+  const int64_t tile_rows = PAIR ? 2 * BM : BM;
+  p.tiles_m = GROUPED ? (int)a.max_tiles_m : (int)((a.M + tile_rows - 1) / tile_rows);
   p.kb_total = (int)((a.K + BK - 1) / BK);
   const int splits = EPI == TC_EPI_PARTIAL_F32 ? k.split_k : 1;
   p.kb_per = (p.kb_total + splits - 1) / splits;
@@ -536,7 +628,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.row_div = a.row_div > 0 ? a.row_div : 1;
   p.status = c.status;
   constexpr int acc_cols = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
-  return launch_kernel(kern, tmA, tmB, p, k.stages, acc_cols, smem, c);
+  return launch_kernel(kern, tmA, tmB, p, k.stages, acc_cols, smem, PAIR, c);
 }
 
 }  // namespace tcg

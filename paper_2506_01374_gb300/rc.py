@@ -231,6 +231,12 @@ class Schedule:
     def hash(self) -> int:
         return lib().rc_schedule_hash(self.h)
 
+    def clone(self) -> "Schedule":
+        """An owned copy (outlives the search or op call that produced this handle)."""
+        c = _P()
+        _check(lib().rc_schedule_clone(self.h, C.byref(c)), "rc_schedule_clone")
+        return Schedule(c.value)
+
     def __str__(self):
         need = C.c_size_t(0)
         _check(lib().rc_schedule_to_string(self.h, None, 0, C.byref(need)))

@@ -24,10 +24,11 @@ def conv_op(N, H, W, Cin, Cout, flags=rc.EPI_BIAS | rc.EPI_SILU):
                  flags=flags)
 
 
-def sched(op, tile_n, stages, split_k=1, fuse=1, persistent=0, layout=0, tile_k=64):
+def sched(op, tile_n, stages, split_k=1, fuse=1, persistent=0, layout=0, tile_k=64, tile_m=128):
     return op.schedule(rc.T(rc.T_TILE_SIZE, tile_n, axis=1), rc.T(rc.T_PIPELINE_STAGES, stages),
                        rc.T(rc.T_SPLIT_K, split_k), rc.T(rc.T_FUSE, fuse), rc.T(rc.T_PARALLEL, persistent),
-                       rc.T(rc.T_LAYOUT, layout), rc.T(rc.T_TILE_SIZE, tile_k, axis=2))
+                       rc.T(rc.T_LAYOUT, layout), rc.T(rc.T_TILE_SIZE, tile_k, axis=2),
+                       rc.T(rc.T_TILE_SIZE, tile_m, axis=0))
 
 
 @pytest.mark.parametrize("N,H,W,Cin", [(2, 16, 16, 128), (1, 16, 8, 64), (1, 4, 32, 64), (1, 2, 64, 192),
@@ -38,16 +39,16 @@ def test_conv_geometries(N, H, W, Cin):
     ref = oracle.conv2d_nhwc_bf16(x, w, b)
     op = conv_op(N, H, W, Cin, Cout)
     dx, dw, db = to_dev(x), to_dev(w), to_dev(b)
-    for tn, st, lay, tk in itertools.product((64, 80, 160), (1, 2, 4), (0, 1, 2), (64, 128)):
+    for tn, st, lay, tk, tm in itertools.product((64, 80, 160), (1, 2, 4), (0, 1, 2), (64, 128), (128, 256)):
         try:
-            s = sched(op, tn, st, layout=lay, tile_k=tk)
+            s = sched(op, tn, st, layout=lay, tile_k=tk, tile_m=tm)
         except rc.RcError:
-            continue  # K = 128 per stage with 4 stages at N = 160 exceeds shared memory
+            continue  # shared memory (K = 128, 4 stages, N = 160); CTA pairs read A as one 4-D box only
         dy = empty_bf16(N, H, W, Cout).fill_(0x7FC0)
         op.run(s, [dx, dw, db, dy])
         op.check()
         err = rel_err(from_dev_bf16(dy).reshape(-1, Cout), ref)
-        assert err <= TOL, (tn, st, lay, tk, err)
+        assert err <= TOL, (tn, st, lay, tk, tm, err)
 
 
 def test_conv_split_k_and_unfused_epilogue():
@@ -56,12 +57,16 @@ def test_conv_split_k_and_unfused_epilogue():
     ref = oracle.conv2d_nhwc_bf16(x, w, b)
     op = conv_op(N, H, W, Cin, Cout)
     dx, dw, db = to_dev(x), to_dev(w), to_dev(b)
-    for sk, fuse, tn, pe, tk in itertools.product((1, 3, 5), (0, 1), (80, 160), (0, 1), (64, 128)):
+    for sk, fuse, tn, pe, tk, tm in itertools.product((1, 3, 5), (0, 1), (80, 160), (0, 1), (64, 128), (128, 256)):
+        try:
+            s = sched(op, tn, 3 if tk == 64 else 2, sk, fuse, pe, tile_k=tk, tile_m=tm)
+        except rc.RcError:
+            continue  # persistent CTA pairs hold N tiles of at most 128
         dy = empty_bf16(N, H, W, Cout).fill_(0x7FC0)
-        op.run(sched(op, tn, 3 if tk == 64 else 2, sk, fuse, pe, tile_k=tk), [dx, dw, db, dy])
+        op.run(s, [dx, dw, db, dy])
         op.check()
         err = rel_err(from_dev_bf16(dy).reshape(-1, Cout), ref)
-        assert err <= TOL, (sk, fuse, tn, pe, tk, err)
+        assert err <= TOL, (sk, fuse, tn, pe, tk, tm, err)
 
 
 def test_conv_without_bias_or_silu():
@@ -90,7 +95,8 @@ def test_conv_full_size_sampled_pixels():
     ref = oracle.conv2d_nhwc_bf16(x, w, b, pix=pix)
     for s in [op.schedule(), sched(op, 160, 4), sched(op, 80, 3, 5, 1), sched(op, 64, 6, 3, 0),
               sched(op, 160, 3, 1, 1, 1), sched(op, 80, 4, 3, 1, 1), sched(op, 80, 3, 1, 1, 0, 1),
-              sched(op, 160, 4, 3, 0, 1, 1), sched(op, 80, 4, 1, 1, 1, 2), sched(op, 160, 3, 3, 0, 0, 2)]:
+              sched(op, 160, 4, 3, 0, 1, 1), sched(op, 80, 4, 1, 1, 1, 2), sched(op, 160, 3, 3, 0, 0, 2),
+              sched(op, 160, 3, 1, 1, 0, 0, 128, 256), sched(op, 80, 4, 3, 1, 1, 1, 64, 256)]:
         op.run(s, [dx, dw, db, dy])
         op.check()
         got = from_dev_bf16(dy).reshape(-1, C)[pix]

@@ -21,7 +21,8 @@ TOL = 2e-2
 
 def sched(op, stage=0, base=None, **kv):
     ts = []
-    names = {"tile_n": (rc.T_TILE_SIZE, 1), "tile_k": (rc.T_TILE_SIZE, 2), "stages": (rc.T_PIPELINE_STAGES, 0),
+    names = {"tile_m": (rc.T_TILE_SIZE, 0), "tile_n": (rc.T_TILE_SIZE, 1), "tile_k": (rc.T_TILE_SIZE, 2),
+             "stages": (rc.T_PIPELINE_STAGES, 0),
              "split_k": (rc.T_SPLIT_K, 0),
              "fuse": (rc.T_FUSE, 0), "persistent": (rc.T_PARALLEL, 0)}
     for k, v in kv.items():
@@ -54,6 +55,30 @@ def test_linear_schedule_sweep(M, N, K):
     assert n >= 120
 
 
+@pytest.mark.parametrize("M,N,K", [(300, 384, 520), (256, 256, 64), (1, 64, 8), (513, 224, 1000)])
+def test_linear_cta_pairs(M, N, K):
+    # TileSize M = 256: two CTAs share each UMMA (cta_group::2), each holding
+    # 128 rows of A and half of the B tile; ragged M leaves the second CTA of
+    # the last pair partly or wholly past the end.
+    X, W = inputs.linear_bf16(M, N, K, seed=25)
+    ref = oracle.linear_bf16(X, W)
+    op = rc.Op(rc.OP_LINEAR, m=M, n=N, k=K)
+    dX, dW = to_dev(X), to_dev(W)
+    n = 0
+    for tn, tk, st, sk, pe in itertools.product((64, 128, 224, 256), (64, 128), (1, 2, 4), (1, 2), (0, 1)):
+        try:
+            s = sched(op, tile_m=256, tile_n=tn, tile_k=tk, stages=st, split_k=sk, persistent=pe)
+        except rc.RcError:
+            continue
+        dY = empty_bf16(M, N).fill_(0x7FC0)
+        op.run(s, [dX, dW, dY])
+        op.check()
+        err = rel_err(from_dev_bf16(dY), ref)
+        assert err <= TOL, (tn, tk, st, sk, pe, err)
+        n += 1
+    assert n >= 40
+
+
 def test_linear_raster_orders():
     M, N, K = 640, 1024, 256
     X, W = inputs.linear_bf16(M, N, K, seed=22)
@@ -73,12 +98,16 @@ def test_swiglu_fused_and_unfused(M, I, K):
     ref = oracle.swiglu_bf16(X, W1)
     op = rc.Op(rc.OP_SWIGLU, m=M, n=I, k=K)
     dX, dW = to_dev(X), to_dev(W1)
-    for tn, st, fuse, pe in itertools.product((32, 64, 128), (1, 3), (0, 1), (0, 1)):
+    for tn, st, fuse, pe, tm in itertools.product((32, 64, 128), (1, 3), (0, 1), (0, 1), (128, 256)):
+        try:  # a CTA pair fuses SwiGLU with the gate rows in one CTA and the up rows in the other
+            s = sched(op, tile_m=tm, tile_n=tn, stages=st, fuse=fuse, persistent=pe)
+        except rc.RcError:
+            continue
         dh = empty_bf16(M, I).fill_(0x7FC0)
-        op.run(sched(op, tile_n=tn, stages=st, fuse=fuse, persistent=pe), [dX, dW, dh])
+        op.run(s, [dX, dW, dh])
         op.check()
         err = rel_err(from_dev_bf16(dh), ref)
-        assert err <= TOL, (tn, st, fuse, pe, err)
+        assert err <= TOL, (tn, st, fuse, pe, tm, err)
 
 
 def test_mlp_block_small():
@@ -90,7 +119,11 @@ def test_mlp_block_small():
     cases = [dict(), dict(s0=dict(tile_n=128, stages=4, fuse=1), s1=dict(tile_n=256, stages=3, split_k=2)),
              dict(s0=dict(tile_n=64, stages=2, fuse=0), s1=dict(tile_n=64, stages=6, split_k=4)),
              dict(s0=dict(tile_n=128, stages=4, fuse=1, persistent=1),
-                  s1=dict(tile_n=256, stages=4, split_k=2, persistent=1))]
+                  s1=dict(tile_n=256, stages=4, split_k=2, persistent=1)),
+             dict(s0=dict(tile_m=256, tile_n=128, stages=3, fuse=1, tile_k=128),
+                  s1=dict(tile_m=256, tile_n=224, stages=4, persistent=0)),
+             dict(s0=dict(tile_m=256, tile_n=64, stages=4, fuse=1, persistent=1),
+                  s1=dict(tile_m=256, tile_n=128, stages=4, split_k=2, persistent=1))]
     for c in cases:
         s = op.schedule()
         if c:
