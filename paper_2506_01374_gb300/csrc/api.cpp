@@ -162,9 +162,11 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
       } else if (stage == 1) {
         gemm_common({32, 64, 128});
+        v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256: a CTA pair within one expert's rows
       } else {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+        v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       }
       break;
   }

@@ -10,6 +10,7 @@
 rc_status tc_dispatch_dense(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_dense_pair(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_conv_pair(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
+rc_status tc_dispatch_grouped_pair(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_conv(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_grouped(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 
@@ -81,9 +82,8 @@ rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const Launch
   if (k.stages < 1) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: stages < 1");
   if (k.tile_m != 128 && k.tile_m != 256) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: M tile %d", k.tile_m);
   const bool pair = k.tile_m == 256;  // a CTA pair per 256-row tile
-  if (pair && a.groups > 0) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: grouped GEMMs use 128-row tiles");
   if (a.a_mode == TC_A_CONV || a.a_mode == TC_A_CONV_ROWS)
     return pair ? tc_dispatch_conv_pair(k, a, c) : tc_dispatch_conv(k, a, c);
-  if (a.groups > 0) return tc_dispatch_grouped(k, a, c);
+  if (a.groups > 0) return pair ? tc_dispatch_grouped_pair(k, a, c) : tc_dispatch_grouped(k, a, c);
   return pair ? tc_dispatch_dense_pair(k, a, c) : tc_dispatch_dense(k, a, c);
 }

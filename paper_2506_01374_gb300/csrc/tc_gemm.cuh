@@ -186,7 +186,8 @@ struct Item {
   int row0, row_end, brow0, nt, split, kb0, nkb;
 };
 
-template <bool GROUPED>
+// TR: rows of a tile (128, or 256 for a CTA pair)
+template <bool GROUPED, int TR>
 __device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
   Item it;
   const long long tiles = (long long)p.tiles_m * p.tiles_n;
@@ -200,9 +201,9 @@ __device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
     it.valid = false;
     for (; g < p.groups; ++g) {
       const int lo = p.offsets[g], hi = p.offsets[g + 1];
-      const int n_g = (hi - lo + BM - 1) / BM;
+      const int n_g = (hi - lo + TR - 1) / TR;
       if (mt < acc + n_g) {
-        it.row0 = lo + (mt - acc) * BM;
+        it.row0 = lo + (mt - acc) * TR;
         it.row_end = hi;
         it.valid = true;
         break;
@@ -211,7 +212,7 @@ __device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
     }
     it.brow0 = g * p.b_group_rows;
   } else {
-    it.row0 = mt * BM;
+    it.row0 = mt * TR;
     it.row_end = p.M;
   }
   it.kb0 = it.split * p.kb_per;
@@ -231,7 +232,6 @@ template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const Params p,
                 const int stages) {
-  static_assert(!PAIR || !GROUPED, "CTA pairs are for dense and convolution GEMMs");
   constexpr int A_BYTES = BM * BK * 2;                    // one 64-wide K sub-block of A
   constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * BK * 2;  // and this CTA's rows of B
   constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
@@ -261,8 +261,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const long long w_first = PAIR ? blockIdx.x / 2 : blockIdx.x;
   const long long w_step = PAIR ? gridDim.x / 2 : gridDim.x;
   auto item = [&](long long w) -> Item {
-    Item it = resolve_item<GROUPED>(p, w);
-    if constexpr (PAIR) it.row0 = 2 * it.row0 + (int)rank * BM;  // this CTA's half of the 256-row tile
+    Item it = resolve_item<GROUPED, PAIR ? 2 * BM : BM>(p, w);
+    if constexpr (PAIR) it.row0 += (int)rank * BM;  // this CTA's half of the 256-row tile
     return it;
   };
 
@@ -597,7 +597,9 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   const int tile_out = EPI == TC_EPI_SWIGLU ? BN / 2 : BN;
   p.tiles_n = (out_w + tile_out - 1) / tile_out;
   const int64_t tile_rows = PAIR ? 2 * BM : BM;
-  p.tiles_m = GROUPED ? (int)a.max_tiles_m : (int)((a.M + tile_rows - 1) / tile_rows);
+  // grouped: an upper bound of the tiles the segments need (spare tiles are skipped)
+  p.tiles_m = GROUPED ? (int)(PAIR ? a.M / tile_rows + a.groups : a.max_tiles_m)
+                      : (int)((a.M + tile_rows - 1) / tile_rows);
   p.kb_total = (int)((a.K + BK - 1) / BK);
   const int splits = EPI == TC_EPI_PARTIAL_F32 ? k.split_k : 1;
   p.kb_per = (p.kb_total + splits - 1) / splits;

@@ -60,12 +60,13 @@ def moe_op(T, H, E, I, K):
     return rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
 
 
-def moe_sched(op, tm, tn1, st1, tn2, st2, fuse, persistent=0, tile_k=64):
+def moe_sched(op, tm, tn1, st1, tn2, st2, fuse, persistent=0, tile_k=64, tile_m=128):
     return op.schedule(rc.T(rc.T_TILE_SIZE, tm, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
                        rc.T(rc.T_PIPELINE_STAGES, st1, stage=1), rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2),
                        rc.T(rc.T_PIPELINE_STAGES, st2, stage=2), rc.T(rc.T_FUSE, fuse, stage=2),
                        rc.T(rc.T_PARALLEL, persistent, stage=1), rc.T(rc.T_PARALLEL, persistent, stage=2),
-                       rc.T(rc.T_TILE_SIZE, tile_k, axis=2, stage=1), rc.T(rc.T_TILE_SIZE, tile_k, axis=2, stage=2))
+                       rc.T(rc.T_TILE_SIZE, tile_k, axis=2, stage=1), rc.T(rc.T_TILE_SIZE, tile_k, axis=2, stage=2),
+                       rc.T(rc.T_TILE_SIZE, tile_m, axis=0, stage=1), rc.T(rc.T_TILE_SIZE, tile_m, axis=0, stage=2))
 
 
 def test_moe_layer_schedule_sweep():
@@ -75,12 +76,12 @@ def test_moe_layer_schedule_sweep():
     ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
     op = moe_op(T, H, E, I, K)
     dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
-    for tn1, tn2, fuse, st, pe, tk in itertools.product((32, 64, 128), (64, 128, 224, 256), (0, 1), (1, 3), (0, 1),
-                                                        (64, 128)):
-        try:
-            s = moe_sched(op, 8, tn1, st, tn2, st, fuse, pe, tk)
+    for tn1, tn2, fuse, st, pe, tk, tm in itertools.product((32, 64, 128), (64, 128, 224, 256), (0, 1), (1, 3),
+                                                            (0, 1), (64, 128), (128, 256)):
+        try:  # CTA pairs (tm = 256) take 256 rows of one expert's segment
+            s = moe_sched(op, 8, tn1, st, tn2, st, fuse, pe, tk, tm)
         except rc.RcError:
-            continue  # K = 128 per stage, 3 stages and the widest N tile exceed shared memory
+            continue  # shared memory (K = 128, 3 stages, widest N); TMEM of persistent pairs
         out = empty_bf16(T, H).fill_(0x7FC0)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         gp = torch.empty(T * K, dtype=torch.int32, device="cuda")
@@ -89,7 +90,7 @@ def test_moe_layer_schedule_sweep():
         np.testing.assert_array_equal(gi.cpu().numpy(), ids)
         np.testing.assert_array_equal(gp.cpu().numpy(), perm)
         err = rel_err(from_dev_bf16(out), ref)
-        assert err <= TOL, (tn1, tn2, fuse, st, pe, tk, err)
+        assert err <= TOL, (tn1, tn2, fuse, st, pe, tk, tm, err)
 
 
 def test_moe_layer_imbalanced_and_empty_experts():
@@ -102,11 +103,12 @@ def test_moe_layer_imbalanced_and_empty_experts():
     assert (np.diff(off)[4:] == 0).all() and (np.diff(off)[:4] == T).all()
     ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
     op = moe_op(T, H, E, I, K)
-    for fuse, pe in itertools.product((0, 1), (0, 1)):
+    for fuse, pe, tm in itertools.product((0, 1), (0, 1), (128, 256)):
         out = empty_bf16(T, H).fill_(0x7FC0)
-        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse, pe), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse, pe, tile_m=tm),
+               [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
-        assert rel_err(from_dev_bf16(out), ref) <= TOL, fuse
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm)
 
 
 def test_moe_full_size_sampled_tokens():
