@@ -1166,10 +1166,12 @@ __global__ void __launch_bounds__(kThreads3, 1)
 //   warps 4..7 : softmax (TMEM lane quadrant = warp % 4), one query row per thread
 constexpr int kThreads4 = 256;
 
-template <int BN>
+template <int BN, int NSB>
+// NSB S buffers at TMEM columns s_col + b * BN (block j in buffer j % NSB),
+// O at o_col, P at p_col.
 __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, int q0, int nkb, int b, int h,
-                                            uint32_t tmem, uint32_t o_col, uint32_t p_col, uint64_t* s_full,
-                                            uint64_t* s_free, uint64_t* p_full, uint64_t* pv_full,
+                                            uint32_t tmem, uint32_t s_col, uint32_t o_col, uint32_t p_col,
+                                            uint64_t* s_full, uint64_t* s_free, uint64_t* p_full, uint64_t* pv_full,
                                             volatile int* abort_flag, volatile int* status) {
   auto fail = [&](int code) {
     *abort_flag = 1;
@@ -1198,9 +1200,9 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
   };
   bool ok = true;
   for (int j = 0; j < nkb; ++j) {
-    const int sb = j & 1;
-    const uint32_t tS = tmem + lane_base + (uint32_t)(sb * BN);
-    if (!tc::mbar_wait(&s_full[sb], (uint32_t)(j >> 1) & 1u, abort_flag, status)) {
+    const int sb = j % NSB;
+    const uint32_t tS = tmem + lane_base + s_col + (uint32_t)(sb * BN);
+    if (!tc::mbar_wait(&s_full[sb], (uint32_t)(j / NSB) & 1u, abort_flag, status)) {
       if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
       ok = false;
       break;
@@ -1211,7 +1213,7 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
     for (int c = 0; c < BN; c += 32) tc::tmem_ld32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&r[c]));
     tc::tmem_ld_wait();
     tc::tc_fence_before();
-    tc::mbar_arrive(&s_free[sb]);  // S buffer sb may take S_{j+2}
+    tc::mbar_arrive(&s_free[sb]);  // S buffer sb may take S_{j+NSB}
     const int k0 = j * BN;
     int nvis = min(BN, p.S - k0);
     if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
@@ -1495,12 +1497,243 @@ __global__ void __launch_bounds__(kThreads4, 1)
     }
     __syncwarp();
   } else {
-    softmax_sdb<BN>(p, warp & 3, lane, q0, nkb, b, h, tmem, O_COL, P_COL, s_full, s_free, p_full, pv_full, abort_flag,
-                    status);
+    softmax_sdb<BN, 2>(p, warp & 3, lane, q0, nkb, b, h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full, pv_full,
+                       abort_flag, status);
   }
   tc::tc_fence_before();
   __syncthreads();
   if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
+// Two query tiles per CTA with key blocks of 64 and a P buffer per tile
+// (TileSize M = 256, N = 64, Parallel = 1). TMEM per tile t: S_t (64
+// columns), P_t (32, two bf16 per column) and O_t (128): 448 columns. With P
+// apart from S, S_{j+1} of a tile is issued as soon as its softmax holds S_j
+// in registers, so the tensor pipe computes it while the softmax
+// exponentiates, and the two tiles' softmax warpgroups run independently of
+// each other. The UMMAs come from four warps (the S and the P V products of
+// each tile), K and V from a producer warp each; a ring slot is refilled when
+// every tile that read the block held there has released it.
+//   warp 0      : TMA producer of Q (both tiles) and of the K ring
+//   warp 1      : TMA producer of the V ring
+//   warps 2, 3  : S_t = Q_t K_j^T issue for tile 0 / 1 (warp 2 also owns TMEM)
+//   warps 4, 5  : O_t += P_t V_j issue for tile 0 / 1
+//   warps 6..13 : softmax of tile (warp - 6) / 4, TMEM lane quadrant warp % 4
+constexpr int kThreads5 = 448;
+
+template <bool VT>
+__global__ void __launch_bounds__(kThreads5, 1)
+    attn5_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  constexpr int BN = 64;
+  constexpr int Q_BYTES = BM * D * 2;
+  constexpr int KV_TILE = BN * D * 2;
+  constexpr uint32_t S_COL = 0, P_COL = 2 * BN, O_COL = 3 * BN;  // tile t: + t*BN, + t*BN/2, + t*D
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;  // [2] tiles
+  uint8_t* kring = smem + 2 * Q_BYTES;
+  uint8_t* vring = kring + (size_t)stages * KV_TILE;
+  uint64_t* q_full = (uint64_t*)(vring + (size_t)stages * KV_TILE);
+  uint64_t* k_full = q_full + 1;              // [stages]
+  uint64_t* v_full = k_full + stages;         // [stages]
+  uint64_t* k_empty = v_full + stages;        // [2 tiles][stages]
+  uint64_t* v_empty = k_empty + 2 * stages;   // [2 tiles][stages]
+  uint64_t* s_full = v_empty + 2 * stages;    // [2]
+  uint64_t* s_free = s_full + 2;              // [2]
+  uint64_t* p_full = s_free + 2;              // [2]
+  uint64_t* pv_full = p_full + 2;             // [2]
+  uint64_t* drain = pv_full + 2;              // [4] one per issuing warp
+  uint32_t* tmem_slot = (uint32_t*)(drain + 4);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int pairs = (p.q_blocks + 1) / 2;
+  const int BH = p.B * p.Hq;
+  int pb, bh;
+  if (p.raster == 0) {
+    pb = blockIdx.x % pairs;
+    bh = blockIdx.x / pairs;
+  } else {
+    pb = pairs - 1 - (int)(blockIdx.x / BH);
+    bh = blockIdx.x % BH;
+  }
+  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
+  int q0[2], nkb[2];
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    q0[t] = (2 * pb + t) * BM;
+    const int end = p.causal ? min(q0[t] + BM, p.S) : p.S;
+    nkb[t] = q0[t] < p.S ? (end + BN - 1) / BN : 0;
+  }
+  const int nblk = max(nkb[0], nkb[1]);
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&k_full[s], 1);
+      tc::mbar_init(&v_full[s], 1);
+    }
+    for (int i = 0; i < 2 * stages; ++i) {
+      tc::mbar_init(&k_empty[i], 1);
+      tc::mbar_init(&v_empty[i], 1);
+    }
+    for (int t = 0; t < 2; ++t) {
+      tc::mbar_init(&s_full[t], 1);
+      tc::mbar_init(&s_free[t], 128);
+      tc::mbar_init(&p_full[t], 128);
+      tc::mbar_init(&pv_full[t], 1);
+    }
+    for (int i = 0; i < 4; ++i) tc::mbar_init(&drain[i], 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 2) tc::tmem_alloc(tmem_slot, 512);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // Slot s of a ring last held key block j - stages; tile t read it iff
+  // j - stages < nkb[t], and released it in the ((j - stages) / stages)-th
+  // phase of its barrier for slot s (parity ph ^ 1; a fresh barrier passes).
+  auto produce = [&](uint64_t* full, uint64_t* empty, auto load) {
+    int j = 0;
+    for (; j < nblk; ++j) {
+      const int s = j % stages;
+      const uint32_t ph = (uint32_t)(j / stages) & 1u;
+      bool ok = true;
+      for (int t = 0; t < 2 && ok; ++t)
+        if (j - stages < nkb[t]) ok = tc::mbar_wait(&empty[t * stages + s], ph ^ 1u, abort_flag, status);
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_EMPTY);
+        break;
+      }
+      tc::mbar_expect_tx(&full[s], KV_TILE);
+      load(s, j, &full[s]);
+    }
+    for (int i = max(0, j - stages); i < j; ++i)
+      if (!tc::mbar_wait_drain(&full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::mbar_expect_tx(q_full, 2 * Q_BYTES);
+#pragma unroll
+      for (int t = 0; t < 2; ++t) {
+        const int qrow = b * p.S + q0[t];
+        tc::tma_load_2d(sQ + t * Q_BYTES, &tmQ, q_full, h * D, qrow);
+        tc::tma_load_2d(sQ + t * Q_BYTES + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
+      }
+      produce(k_full, k_empty, [&](int s, int j, uint64_t* bar) {
+        uint8_t* sk = kring + (size_t)s * KV_TILE;
+        const int krow = b * p.S + j * BN;
+        tc::tma_load_2d(sk, &tmK, bar, g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, bar, g * D + 64, krow);
+      });
+      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+    __syncwarp();  // reconverge before the final block barrier
+  } else if (warp == 1) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmV);
+      produce(v_full, v_empty, [&](int s, int j, uint64_t* bar) {
+        uint8_t* sv = vring + (size_t)s * KV_TILE;
+        if constexpr (VT) {
+          tc::tma_load_2d(sv, &tmV, bar, j * BN, (b * p.Hkv + g) * D);
+        } else {
+          const int krow = b * p.S + j * BN;
+          tc::tma_load_2d(sv, &tmV, bar, g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, bar, g * D + 64, krow);
+        }
+      });
+    }
+    __syncwarp();
+  } else if (warp <= 3) {  // S issue of tile warp - 2
+    const int t = warp - 2;
+    if (lane == 0 && nkb[t] > 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+      const uint32_t sq = tc::smem_u32(sQ + t * Q_BYTES);
+      const uint32_t tS = tmem + S_COL + (uint32_t)(t * BN);
+      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
+      for (int j = 0; ok && j < nkb[t]; ++j) {
+        // the S buffer is free once the softmax holds S_{j-1} in registers
+        if (j > 0) ok = tc::mbar_wait(&s_free[t], (uint32_t)(j - 1) & 1u, abort_flag, status);
+        const int s = j % stages;
+        ok = ok && tc::mbar_wait(&k_full[s], (uint32_t)(j / stages) & 1u, abort_flag, status);
+        if (!ok) break;
+        tc::tc_fence_after();
+        const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t off = (uint32_t)(ks % 4) * 32;
+          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
+                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+        }
+        tc::umma_commit(&s_full[t]);
+        tc::umma_commit(&k_empty[t * stages + s]);
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[t]);
+        if (!tc::mbar_wait_drain(&drain[t], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else if (warp <= 5) {  // P V issue of tile warp - 4
+    const int t = warp - 4;
+    if (lane == 0 && nkb[t] > 0) {
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+      const uint32_t tO = tmem + O_COL + (uint32_t)(t * D), tP = tmem + P_COL + (uint32_t)(t * BN / 2);
+      bool ok = true;
+      for (int j = 0; ok && j < nkb[t]; ++j) {
+        const int s = j % stages;
+        ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / stages) & 1u, abort_flag, status) &&
+             tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status);
+        if (!ok) break;
+        tc::tc_fence_after();
+        const uint32_t sv = tc::smem_u32(vring + (size_t)s * KV_TILE);
+#pragma unroll
+        for (int ks = 0; ks < BN / 16; ++ks) {
+          uint64_t db;
+          if constexpr (VT)
+            db = tc::sw128_desc(sv + (uint32_t)(ks % 4) * 32);
+          else
+            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
+          tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        tc::umma_commit(&pv_full[t]);
+        tc::umma_commit(&v_empty[t * stages + s]);
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[2 + t]);
+        if (!tc::mbar_wait_drain(&drain[2 + t], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else {
+    const int t = (warp - 6) / 4;
+    softmax_sdb<BN, 1>(p, warp & 3, lane, q0[t], nkb[t], b, h, tmem, S_COL + (uint32_t)(t * BN),
+                       O_COL + (uint32_t)(t * D), P_COL + (uint32_t)(t * BN / 2), &s_full[t], &s_free[t], &p_full[t],
+                       &pv_full[t], abort_flag, status);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
     __syncwarp();
     tc::tc_fence_after();
     tc::tmem_dealloc(tmem, 512);
@@ -1540,7 +1773,8 @@ rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const vo
   static_assert(!PAR || (PT && !SDB), "split UMMA issue: P in TMEM");
   // PAR: two query tiles with one issuing warp each (attn3), or one query tile
   // with two S buffers and separate S and P V issuers (attn4)
-  auto kern = PAR ? (PINGPONG ? attn3_kernel<BN, VT> : attn4_kernel<BN, VT>)
+  // (two tiles with BN = 64: P apart from S, four issuing warps, attn5)
+  auto kern = PAR ? (PINGPONG ? (BN == 64 ? attn5_kernel<VT> : attn3_kernel<BN, VT>) : attn4_kernel<BN, VT>)
                   : PINGPONG ? attn2_kernel<BN, VT, PT, SDB> : attn_kernel<BN, VT>;
   static bool attr = false;
   if (!attr) {
@@ -1574,7 +1808,7 @@ rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const vo
   if (ctas > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
   const int qtiles = PINGPONG ? 2 : 1;
   const size_t smem = smem_bytes(BN, k.stages, qtiles) - (PT ? (size_t)qtiles * BM * BN * 2 : 0);
-  const int threads = PAR ? (PINGPONG ? kThreads3 : kThreads4) : PINGPONG ? kThreads2 : kThreads;
+  const int threads = PAR ? (PINGPONG ? (BN == 64 ? kThreads5 : kThreads3) : kThreads4) : PINGPONG ? kThreads2 : kThreads;
   kern<<<(unsigned)ctas, threads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
