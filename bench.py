@@ -305,7 +305,7 @@ def parse_schedule(op, text, rc):
     KNOB_T = {"tile_m": (rc.T_TILE_SIZE, 0), "tile_n": (rc.T_TILE_SIZE, 1), "tile_k": (rc.T_TILE_SIZE, 2),
               "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0), "fuse": (rc.T_FUSE, 0),
               "raster": (rc.T_LOOP_ORDER, 0), "persistent": (rc.T_PARALLEL, 0), "layout": (rc.T_LAYOUT, 0),
-              "unroll": (rc.T_UNROLL, 0)}
+              "unroll": (rc.T_UNROLL, 0), "location": (rc.T_COMPUTE_LOCATION, 0)}
     ts = []
     for part in filter(None, text.split(";")):
         stage_s, kvs = part.split(":")

@@ -150,10 +150,15 @@ void rc_op_destroy(rc_op* op);
 typedef enum {
   RC_T_TILE_SIZE = 0,        /* axis 0/1/2 = M/N/K tile; value[0] = extent */
   RC_T_PARALLEL = 1,         /* value[0]: GEMM-shaped ops: 0 = one CTA per output tile, 1 = persistent
-                              * CTAs; ATTENTION: 0 = one UMMA-issuing warp per CTA, 1 = one per
-                              * query tile (two query tiles, P in TMEM only) */
-  RC_T_COMPUTE_LOCATION = 2, /* value[0]: where producer work runs (op specific, see knobs) */
-  RC_T_UNROLL = 3,           /* value[0]: unroll factor of the innermost reduction loop */
+                              * CTAs; ATTENTION: 0 = one UMMA-issuing warp per CTA, 1 = UMMA issue
+                              * split over warps (P in TMEM only): one issuer per query tile for two
+                              * tiles, separate S and P V issuers for one tile */
+  RC_T_COMPUTE_LOCATION = 2, /* value[0]: where producer work runs (op specific, see knobs);
+                              * ATTENTION: 1 = P kept in TMEM, 0 = P in shared memory */
+  RC_T_UNROLL = 3,           /* value[0]: unroll factor of the innermost reduction loop;
+                              * ATTENTION: key blocks in flight per query tile (1 or 2 S buffers);
+                              * one tile with split issue and one S buffer at key blocks of 64
+                              * runs two CTAs per SM */
   RC_T_LOOP_ORDER = 4,       /* value[0]: tile raster 0 = M fastest, 1 = N fastest; value[1] = group */
   RC_T_FUSE = 5,             /* value[0]: 1 = epilogue fused into the producing kernel, 0 = separate pass */
   RC_T_LAYOUT = 6,           /* value[0]: op-specific data layout choice */

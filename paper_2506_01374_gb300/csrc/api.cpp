@@ -278,13 +278,15 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
         if (why) *why = "P in tensor memory needs two query tiles or split UMMA issue";
         return false;
       }
-      if (k.unroll == 2 && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
+      const bool one_tile_split = k.tile_m == 128 && k.persistent == 1;
+      if (k.unroll == 2 && !one_tile_split && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
         // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
         if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
         return false;
       }
-      if (k.persistent == 1 && !(k.location == 1 && k.unroll == 1 && k.stages >= 2)) {
-        // two tiles: one issuing warp per tile; one tile: two S buffers, S and P V issued by separate warps
+      if (k.persistent == 1 && !(k.location == 1 && (k.unroll == 1 || one_tile_split) && k.stages >= 2)) {
+        // two tiles: one issuing warp per tile; one tile: one or two S buffers, S and P V issued by
+        // separate warps
         if (why) *why = "split UMMA issue needs P in TMEM, one key block in flight per issuer and two stages";
         return false;
       }

@@ -57,6 +57,95 @@ __device__ __forceinline__ uint32_t pack2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// Packed fp32 pairs: two floats in one 64-bit register, for the f32x2
+// add / fma instructions of sm_100+ (one issue slot for two lanes' worth;
+// the FMA pipe still takes two cycles per warp, so they save issue slots,
+// which is what the softmax runs short of, not FMA throughput).
+__device__ __forceinline__ uint64_t f2(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Maximum of N raw scores (N even, >= 8): four independent chains of
+// three-input maxima, then a combine.
+template <int N>
+__device__ __forceinline__ float row_max(const uint32_t* r) {
+  float pm[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) pm[u] = __uint_as_float(r[u]);
+#pragma unroll
+  for (int i = 4; i < N; i += 2)
+    pm[(i / 2) % 4] = max3(pm[(i / 2) % 4], __uint_as_float(r[i]), __uint_as_float(r[i + 1]));
+  return fmaxf(max3(pm[0], pm[1], pm[2]), pm[3]);
+}
+
+// p_i = 2^(s_i * scale_log2 - mref) for N raw scores: bf16 pairs into pk and
+// fp32 partial sums into ls2 (two packed accumulators). Masked scores are
+// -inf and give +0.
+template <int N>
+__device__ __forceinline__ void exp_pack(const uint32_t* r, uint64_t sc2, uint64_t nm2, uint32_t* pk,
+                                         uint64_t (&ls2)[2]) {
+#pragma unroll
+  for (int i = 0; i < N; i += 2) {
+    const uint64_t x = f2_fma(f2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), sc2, nm2);
+    float x0, x1;
+    f2_split(x, x0, x1);
+    const float p0 = tc::ex2_approx(x0), p1 = tc::ex2_approx(x1);
+    ls2[(i / 2) % 2] = f2_add(ls2[(i / 2) % 2], f2(p0, p1));
+    pk[i / 2] = pack2(p0, p1);
+  }
+}
+
+__device__ __forceinline__ float sum_pairs(const uint64_t (&ls2)[2]) {
+  float a, b, c, d;
+  f2_split(ls2[0], a, b);
+  f2_split(ls2[1], c, d);
+  return (a + b) + (c + d);
+}
+
+// One normalised output row: O (fp32 in this thread's TMEM lane, columns
+// tO .. tO + D - 1) times 1/l, rounded to bf16, stored as 16-byte vectors.
+// Each 64-column half is fetched with two loads and a single wait.
+__device__ __forceinline__ void store_o_row(uint32_t tO, float inv_l, __nv_bfloat16* orow, bool row_ok) {
+#pragma unroll
+  for (int c = 0; c < D; c += 64) {
+    uint32_t o[64];
+    tc::tmem_ld32(tO + c, *reinterpret_cast<uint32_t(*)[32]>(&o[0]));
+    tc::tmem_ld32(tO + c + 32, *reinterpret_cast<uint32_t(*)[32]>(&o[32]));
+    tc::tmem_ld_wait();
+    if (row_ok) {
+#pragma unroll
+      for (int i = 0; i < 64; i += 8) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          pk[u] = pack2(__uint_as_float(o[i + 2 * u]) * inv_l, __uint_as_float(o[i + 2 * u + 1]) * inv_l);
+        *reinterpret_cast<uint4*>(orow + c + i) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+    }
+  }
+}
+
+
 template <int BN, bool VT>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -394,15 +483,7 @@ __device__ __forceinline__ void softmax_tile(const Params& p, int t, int qd, int
       for (int i = 0; i < BN; ++i)
         if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
     }
-    // row maximum: 8 independent partial maxima, then combine
-    float pm[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(r[u]);
-#pragma unroll
-    for (int i = 8; i < BN; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(r[i]));
-    const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                           fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-    const float mxs = mx * p.scale_log2;
+    const float mxs = row_max<BN>(r) * p.scale_log2;
     float factor = 1.f;
     if (m_ref == -INFINITY) {
       m_ref = mxs;  // first visible scores: O and l are still zero
@@ -448,18 +529,12 @@ __device__ __forceinline__ void softmax_tile(const Params& p, int t, int qd, int
     }
     // pass 2: probabilities -> P (bf16) and the row sum
     const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
+    uint64_t ls2[2] = {0ull, 0ull};
 #pragma unroll
     for (int c = 0; c < BN; c += 32) {
       uint32_t pk[16];
-#pragma unroll
-      for (int i = 0; i < 32; i += 2) {
-        // masked scores are -inf: 2^-inf = +0
-        const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i]), p.scale_log2, -mref));
-        const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[c + i + 1]), p.scale_log2, -mref));
-        ls[(i / 2) % 4] += p0 + p1;
-        pk[i / 2] = pack2(p0, p1);
-      }
+      exp_pack<32>(r + c, sc2, nm2, pk, ls2);
       if constexpr (PT) {
         // P for keys [c, c + 32) goes to columns [c/2, c/2 + 16) of the S row (already in registers)
         tc::tmem_st16(tS + c / 2, pk);
@@ -476,7 +551,7 @@ __device__ __forceinline__ void softmax_tile(const Params& p, int t, int qd, int
         }
       }
     }
-    l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+    l = l * factor + sum_pairs(ls2);
     if constexpr (PT) tc::tmem_st_wait();
     if (!await_pv()) {
       ok = false;
@@ -492,20 +567,7 @@ __device__ __forceinline__ void softmax_tile(const Params& p, int t, int qd, int
       const float inv_l = l > 0.f ? 1.f / l : 0.f;
       const bool row_ok = qi < p.S;
       __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        uint32_t r[16];
-        tc::tmem_ld16(tO + c, r);
-        tc::tmem_ld_wait();
-        uint32_t pk[8];
-#pragma unroll
-        for (int i = 0; i < 16; i += 2)
-          pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
-        if (row_ok) {
-          *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        }
-      }
+      store_o_row(tO, inv_l, orow, row_ok);
       if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
     } else if (!*abort_flag) {
       fail(RC_DEV_TIMEOUT_ACCUM);
@@ -804,12 +866,7 @@ __device__ __forceinline__ void softmax_tile_chunked(const Params& p, int t, int
         tc::tmem_st32(tS + c, r);
         tc::tmem_st_wait();
       }
-      float pm[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) pm[u] = __uint_as_float(r[u]);
-#pragma unroll
-      for (int i = 4; i < CH; ++i) pm[i % 4] = fmaxf(pm[i % 4], __uint_as_float(r[i]));
-      mx = fmaxf(mx, fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])));
+      mx = fmaxf(mx, row_max<CH>(r));
     }
     const float mxs = mx * p.scale_log2;
     float factor = 1.f;
@@ -850,24 +907,18 @@ __device__ __forceinline__ void softmax_tile_chunked(const Params& p, int t, int
       tc::tmem_st_wait();
     }
     const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
+    uint64_t ls2[2] = {0ull, 0ull};
 #pragma unroll 1
     for (int c = 0; c < BN; c += CH) {
       uint32_t r[CH];
       tc::tmem_ld32(tS + c, r);
       tc::tmem_ld_wait();
       uint32_t pk[CH / 2];
-#pragma unroll
-      for (int i = 0; i < CH; i += 2) {
-        // masked scores are -inf: 2^-inf = +0
-        const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[i]), p.scale_log2, -mref));
-        const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[i + 1]), p.scale_log2, -mref));
-        ls[(i / 2) % 4] += p0 + p1;
-        pk[i / 2] = pack2(p0, p1);
-      }
+      exp_pack<CH>(r, sc2, nm2, pk, ls2);
       tc::tmem_st16(tS + c / 2, pk);
     }
-    l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+    l = l * factor + sum_pairs(ls2);
     tc::tmem_st_wait();
     if (!await_pv()) {
       ok = false;
@@ -882,20 +933,7 @@ __device__ __forceinline__ void softmax_tile_chunked(const Params& p, int t, int
       const float inv_l = l > 0.f ? 1.f / l : 0.f;
       const bool row_ok = qi < p.S;
       __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        uint32_t r[16];
-        tc::tmem_ld16(tO + c, r);
-        tc::tmem_ld_wait();
-        uint32_t pk[8];
-#pragma unroll
-        for (int i = 0; i < 16; i += 2)
-          pk[i / 2] = pack2(__uint_as_float(r[i]) * inv_l, __uint_as_float(r[i + 1]) * inv_l);
-        if (row_ok) {
-          *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-        }
-      }
+      store_o_row(tO, inv_l, orow, row_ok);
       if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
     } else if (!*abort_flag) {
       fail(RC_DEV_TIMEOUT_ACCUM);
@@ -1222,13 +1260,7 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
       for (int i = 0; i < BN; ++i)
         if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
     }
-    float pm[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) pm[u] = __uint_as_float(r[u]);
-#pragma unroll
-    for (int i = 8; i < BN; ++i) pm[i % 8] = fmaxf(pm[i % 8], __uint_as_float(r[i]));
-    const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])), fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-    const float mxs = mx * p.scale_log2;
+    const float mxs = row_max<BN>(r) * p.scale_log2;
     float factor = 1.f;
     if (m_ref == -INFINITY) {
       m_ref = mxs;  // first visible scores: O and l are still zero
@@ -1253,17 +1285,11 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
       tc::tmem_st_wait();
     }
     const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-    float ls[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
+    uint64_t ls2[2] = {0ull, 0ull};
     uint32_t pk[BN / 2];
-#pragma unroll
-    for (int i = 0; i < BN; i += 2) {
-      // masked scores are -inf: 2^-inf = +0
-      const float p0 = tc::ex2_approx(fmaf(__uint_as_float(r[i]), p.scale_log2, -mref));
-      const float p1 = tc::ex2_approx(fmaf(__uint_as_float(r[i + 1]), p.scale_log2, -mref));
-      ls[(i / 2) % 4] += p0 + p1;
-      pk[i / 2] = pack2(p0, p1);
-    }
-    l = l * factor + ((ls[0] + ls[1]) + (ls[2] + ls[3]));
+    exp_pack<BN>(r, sc2, nm2, pk, ls2);
+    l = l * factor + sum_pairs(ls2);
     if (!await_pv(j - 1)) {  // P_{j-1} V_{j-1} has read the P buffer
       ok = false;
       break;
@@ -1279,33 +1305,36 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
       const float inv_l = l > 0.f ? 1.f / l : 0.f;
       const bool row_ok = qi < p.S;
       __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        uint32_t o[16];
-        tc::tmem_ld16(tO + c, o);
-        tc::tmem_ld_wait();
-        uint32_t pk2[8];
-#pragma unroll
-        for (int i = 0; i < 16; i += 2)
-          pk2[i / 2] = pack2(__uint_as_float(o[i]) * inv_l, __uint_as_float(o[i + 1]) * inv_l);
-        if (row_ok) {
-          *reinterpret_cast<uint4*>(orow + c) = make_uint4(pk2[0], pk2[1], pk2[2], pk2[3]);
-          *reinterpret_cast<uint4*>(orow + c + 8) = make_uint4(pk2[4], pk2[5], pk2[6], pk2[7]);
-        }
-      }
+      store_o_row(tO, inv_l, orow, row_ok);
       if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
     }
   }
 }
 
-template <int BN, bool VT>
-__global__ void __launch_bounds__(kThreads4, 1)
+// TMEM layout of the one-tile kernel with NSB S buffers: S at 0 (and BN),
+// then P and O. With one S buffer and BN = 64 the tile takes 256 columns
+// (S 64, P 32, O 128 at column 128), so two CTAs share an SM: one CTA's
+// softmax overlaps the other's tensor-core work, and a finishing CTA's tail
+// overlaps its neighbour instead of idling the SM.
+template <int BN, int NSB>
+struct Attn4Cols {
+  static constexpr uint32_t P = NSB == 2 ? 2 * BN + D : BN;
+  static constexpr uint32_t O = NSB == 2 ? 2 * BN : (BN + BN / 2 + 127) / 128 * 128;
+  static constexpr uint32_t END = NSB == 2 ? 2 * BN + D + BN / 2 : O + D;
+  static constexpr uint32_t ALLOC = END <= 256 ? 256 : 512;
+  static constexpr int CTAS_PER_SM = ALLOC == 256 ? 2 : 1;
+};
+
+template <int BN, bool VT, int NSB>
+__global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     attn4_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                  const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
   static_assert(BN == 64 || BN == 128, "key block");
+  static_assert(NSB == 1 || NSB == 2, "S buffers");
   constexpr int Q_BYTES = BM * D * 2;
   constexpr int KV_TILE = BN * D * 2;
-  constexpr uint32_t O_COL = (uint32_t)(2 * BN), P_COL = (uint32_t)(2 * BN + D);
+  constexpr uint32_t O_COL = Attn4Cols<BN, NSB>::O, P_COL = Attn4Cols<BN, NSB>::P;
+  constexpr uint32_t TMEM_COLS = Attn4Cols<BN, NSB>::ALLOC;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -1364,7 +1393,7 @@ __global__ void __launch_bounds__(kThreads4, 1)
     *abort_flag = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 1) tc::tmem_alloc(tmem_slot, 512);
+  if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
@@ -1430,32 +1459,32 @@ __global__ void __launch_bounds__(kThreads4, 1)
       auto issue_s = [&](int j) {
         const int s = j % stages;
         const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
-        const uint32_t tS = tmem + (uint32_t)((j & 1) * BN);
+        const uint32_t tS = tmem + (uint32_t)((j % NSB) * BN);
 #pragma unroll
         for (int ks = 0; ks < D / 16; ++ks) {
           const uint32_t off = (uint32_t)(ks % 4) * 32;
           tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
                         tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
         }
-        tc::umma_commit(&s_full[j & 1]);
+        tc::umma_commit(&s_full[j % NSB]);
         tc::umma_commit(&k_empty[s]);
       };
       auto await_k = [&](int j) -> bool {
         return tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status);
       };
       bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
-      for (int j = 0; ok && j < 2 && j < nkb; ++j) {
+      for (int j = 0; ok && j < NSB && j < nkb; ++j) {
         if ((ok = await_k(j))) {
           tc::tc_fence_after();
           issue_s(j);
         }
       }
-      for (int j = 0; ok && j + 2 < nkb; ++j) {
-        // S buffer j & 1 is free once the softmax holds S_j in registers
-        ok = tc::mbar_wait(&s_free[j & 1], (uint32_t)(j >> 1) & 1u, abort_flag, status) && await_k(j + 2);
+      for (int j = 0; ok && j + NSB < nkb; ++j) {
+        // S buffer j % NSB is free once the softmax holds S_j in registers
+        ok = tc::mbar_wait(&s_free[j % NSB], (uint32_t)(j / NSB) & 1u, abort_flag, status) && await_k(j + NSB);
         if (!ok) break;
         tc::tc_fence_after();
-        issue_s(j + 2);
+        issue_s(j + NSB);
       }
       if (!ok) {
         fail(RC_DEV_TIMEOUT_FULL);
@@ -1497,15 +1526,15 @@ __global__ void __launch_bounds__(kThreads4, 1)
     }
     __syncwarp();
   } else {
-    softmax_sdb<BN, 2>(p, warp & 3, lane, q0, nkb, b, h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full, pv_full,
-                       abort_flag, status);
+    softmax_sdb<BN, NSB>(p, warp & 3, lane, q0, nkb, b, h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full, pv_full,
+                         abort_flag, status);
   }
   tc::tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     __syncwarp();
     tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, 512);
+    tc::tmem_dealloc(tmem, TMEM_COLS);
   }
 }
 
@@ -1770,15 +1799,23 @@ size_t smem_bytes(int bn, int stages, int qtiles) {
 template <int BN, bool VT, bool PINGPONG, bool PT = false, bool SDB = false, bool PAR = false>
 rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
                  float* lse, const LaunchCtx& c) {
-  static_assert(!PAR || (PT && !SDB), "split UMMA issue: P in TMEM");
+  static_assert(!PAR || (PT && !(SDB && PINGPONG)), "split UMMA issue: P in TMEM");
   // PAR: two query tiles with one issuing warp each (attn3), or one query tile
-  // with two S buffers and separate S and P V issuers (attn4)
+  // with one or two (SDB) S buffers and separate S and P V issuers (attn4)
   // (two tiles with BN = 64: P apart from S, four issuing warps, attn5)
-  auto kern = PAR ? (PINGPONG ? (BN == 64 ? attn5_kernel<VT> : attn3_kernel<BN, VT>) : attn4_kernel<BN, VT>)
-                  : PINGPONG ? attn2_kernel<BN, VT, PT, SDB> : attn_kernel<BN, VT>;
+  auto pick = []() {
+    if constexpr (PAR && PINGPONG && BN == 64) return &attn5_kernel<VT>;
+    else if constexpr (PAR && PINGPONG) return &attn3_kernel<BN, VT>;
+    else if constexpr (PAR) return &attn4_kernel<BN, VT, SDB ? 2 : 1>;
+    else if constexpr (PINGPONG) return &attn2_kernel<BN, VT, PT, SDB>;
+    else return &attn_kernel<BN, VT>;
+  };
+  auto kern = pick();
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+    // the largest shared-memory carve-out, so that two 1-tile CTAs can share an SM
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention: smem attribute: %s", cudaGetErrorString(e));
     attr = true;
   }
@@ -1846,13 +1883,14 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
   const bool pt = k.location == 1;  // P kept in tensor memory
   if (pt && !pp && k.persistent != 1)
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: P in TMEM needs two query tiles or split UMMA issue");
-  if (k.unroll == 2) {  // two key blocks in flight per query tile
+  const bool par = k.persistent == 1;  // UMMA issue split over several warps
+  if (k.unroll == 2 && !(par && !pp)) {  // two key blocks in flight per query tile
     if (!(pp && pt && k.tile_n == 64 && k.stages >= 4) || k.persistent)
       return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: unroll 2 needs 2 query tiles, P in TMEM, BN 64, 4 stages");
     return vt ? attn::launch<64, true, true, true, true>(k, d, Q, K, Vuse, O, lse, c)
               : attn::launch<64, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c);
   }
-  const bool par = k.persistent == 1;  // UMMA issue split over two warps
+  const bool sdb = k.unroll == 2;  // one tile, split issue: two S buffers (two key blocks in flight)
   if (par && !pt) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: split UMMA issue needs P in TMEM");
   if (par && !pp && k.stages < 2)
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: two S buffers need at least two K/V stages");
@@ -1860,6 +1898,8 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
   if (k.tile_n == BN) {                                                                             \
     if (par && pp) return vt ? attn::launch<BN, true, true, true, false, true>(k, d, Q, K, Vuse, O, lse, c) \
                              : attn::launch<BN, false, true, true, false, true>(k, d, Q, K, Vuse, O, lse, c); \
+    if (par && sdb) return vt ? attn::launch<BN, true, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c) \
+                              : attn::launch<BN, false, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c); \
     if (par) return vt ? attn::launch<BN, true, false, true, false, true>(k, d, Q, K, Vuse, O, lse, c) \
                        : attn::launch<BN, false, false, true, false, true>(k, d, Q, K, Vuse, O, lse, c); \
     if (pp && pt) return vt ? attn::launch<BN, true, true, true>(k, d, Q, K, Vuse, O, lse, c)       \
