@@ -65,6 +65,9 @@ def parse():
     ap.add_argument("--restarts", type=int, default=2,
                     help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--shape", default="",
+                    help="override workload sizes for a profiling case, e.g. 'tokens=1024,experts=16' (the line "
+                         "then reports that shape, not the benchmark configuration)")
     return ap.parse_args()
 
 
@@ -132,13 +135,21 @@ class Clocks:
 class Workload:
     """One hot-path workload: op, seeded host inputs, output slots, dominant kernel."""
 
-    def __init__(self, name):
+    def __init__(self, name, shape=None):
         import numpy as np
 
         from paper_2506_01374_gb300 import inputs, rc
         self.name = name
+        sh = dict(shape or {})
+
+        def dims(**default):
+            unknown = set(sh) - set(default)
+            if unknown:
+                raise ValueError(f"--shape keys {sorted(unknown)} do not apply to {name}")
+            return [sh.get(k, v) for k, v in default.items()]
+
         if name == "mlp":
-            T, H, I = 2048, 4096, 14336
+            T, H, I = dims(tokens=2048, hidden=4096, inter=14336)
             X, W1, W2 = inputs.mlp(T, H, I, seed=1)
             self.op = rc.Op(rc.OP_MLP, m=T, n=I, k=H)
             self.host = [X, W1, W2, None]
@@ -151,7 +162,8 @@ class Workload:
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "attention":
-            B, S, Hq, Hkv, D = 1, 2048, 32, 8, 128
+            B, S, Hq, Hkv = dims(batch=1, seq=2048, heads_q=32, heads_kv=8)
+            D = 128
             Q, K, V = inputs.attention(B, S, Hq, Hkv, D, seed=4)
             self.op = rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=1)
             self.host = [Q, K, V, None, None]
@@ -164,7 +176,7 @@ class Workload:
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "conv2d":
-            N, H, W, C = 2, 64, 64, 320
+            N, H, W, C = dims(n=2, h=64, w=64, c=320)
             x, w, b = inputs.conv2d(N, H, W, C, C, seed=5)
             self.op = rc.Op(rc.OP_CONV2D, img_n=N, img_h=H, img_w=W, c_in=C, c_out=C, kr=3, ks=3, stride=1, pad=1,
                             flags=rc.EPI_BIAS | rc.EPI_SILU)
@@ -178,7 +190,7 @@ class Workload:
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "moe":
-            T, H, E, I, K = 4096, 7168, 64, 2048, 8
+            T, H, E, I, K = dims(tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
             logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=6)
             self.op = rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
             self.host = [logits, X, W1, W2, None]
@@ -191,7 +203,7 @@ class Workload:
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "gemm_f32":
-            M = N = K = 256
+            M, N, K = dims(m=256, n=256, k=256)
             A, B, bias = inputs.gemm_f32(M, N, K, seed=0)
             self.op = rc.Op(rc.OP_GEMM_F32, m=M, n=N, k=K, flags=rc.EPI_BIAS | rc.EPI_RELU)
             self.host = [A, B, bias, None]
@@ -298,6 +310,15 @@ class Workload:
             what, used = f"{n} full 256^3 GEMMs", min(cores, A.shape[0])
         return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": used, "kind": "oracle",
                 "sample": what + ", fp64 loop nests", "seconds": dt}
+
+
+def parse_shape(text):
+    """'tokens=1024,experts=16' -> {'tokens': 1024, 'experts': 16}"""
+    out = {}
+    for kv in filter(None, text.split(",")):
+        k, v = kv.split("=")
+        out[k.strip()] = int(v)
+    return out
 
 
 def parse_schedule(op, text, rc):
@@ -440,7 +461,10 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     stream = torch.cuda.current_stream()
 
-    wl = Workload(args.workload)
+    wl = Workload(args.workload, parse_shape(args.shape))
+    if args.shape:
+        wl.label += "_shape_" + args.shape.replace("=", "").replace(",", "_")
+        wl.config.update(parse_shape(args.shape))
     op = wl.op
     info = op.info
     io = wl.device_io()

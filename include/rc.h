@@ -269,10 +269,13 @@ typedef struct {
   double tflops;      /* algorithmic flops / median time */
   double gbps;        /* algorithmic bytes / median time */
   uint64_t sched_hash;
+  int32_t n_stages;                 /* stages timed separately (0 = none) */
+  double stage_ms[RC_MAX_STAGES];   /* median device time of each stage (ms) */
 } rc_measurement;
 
 /* Device-timed measurement of n candidates on the caller's stream: per
- * candidate W warm-ups, then R x {L2 flush, event, run, event}; median.
+ * candidate W warm-ups, then R x {L2 flush, event, run with an event after
+ * each stage}; medians of the whole run and of each stage.
  * out[] is caller-allocated. The call synchronises the stream. The batch
  * status is RC_OK if every candidate could be attempted; per-candidate
  * failures are reported in out[i].status. */
@@ -289,6 +292,15 @@ typedef struct {
   int32_t horizon;    /* maximum transformation-sequence length T (default 8) */
   int32_t rollout;    /* random transformations per rollout q (default 2) */
   int32_t max_tries;  /* sampling attempts per expansion (default 64) */
+  int32_t surrogate;  /* 0 (default): rollout programs are measured; 1: once >= 24 programs are
+                       * measured, rollout programs are scored by a surrogate f-hat learned from the
+                       * measurements (Sec. 3.2: reward = t(P0) / f-hat(P_sim)) and only expanded
+                       * nodes are measured. f-hat: ridge regression of log device time on one-hot
+                       * knob values and knob-pair values, one model per op stage when the
+                       * measurements carry per-stage times. */
+  int32_t screen;     /* surrogate = 1 only: an expansion draws up to screen * B distinct legal
+                       * proposals and keeps the B with the lowest predicted time (the cost model
+                       * pruning low-value proposals before they join the tree); <= 1 = off */
 } rc_search_opts;
 
 /* Create an LLM-free MCTS search over op's schedule space (Sec. 3.2 with the
@@ -315,8 +327,16 @@ typedef struct {
   int64_t samples;      /* distinct schedules measured */
   int64_t iterations;   /* rc_search_step calls that expanded */
   double best_reward;
+  int64_t model_samples;   /* measurements the current surrogate fit used (0 = not fitted) */
+  int64_t model_features;  /* columns of the current fit, intercept included */
+  int64_t predicted;       /* rollout rewards taken from the surrogate */
 } rc_search_stats;
 rc_status rc_search_get_stats(const rc_search* s, rc_search_stats* st);
+/* The surrogate's predicted device time (ms) of a schedule of the search's
+ * op: the sum over stages of exp(w . x_stage) (per-stage models) or
+ * exp(w . x) (one model). RC_ERR_INVALID_ARG when the surrogate is off or not
+ * fitted yet. Deterministic given the measurement sequence. */
+rc_status rc_search_predict(rc_search* s, const rc_schedule* sched, double* ms);
 /* Node i (0 = root): parent index (-1 for root), Q (cumulative reward), N (visits). */
 rc_status rc_search_node(const rc_search* s, int64_t i, int64_t* parent, double* q, int64_t* n,
                          uint64_t* sched_hash);

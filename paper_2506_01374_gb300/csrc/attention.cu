@@ -1325,6 +1325,30 @@ struct Attn4Cols {
   static constexpr int CTAS_PER_SM = ALLOC == 256 ? 2 : 1;
 };
 
+// K ring depth = the schedule's stages; V ring depth. V_j is consumed one
+// softmax period after K_j, so two-CTA-per-SM kernels keep at most two V
+// slots and spend the shared memory on the K ring, whose refill latency (a
+// K slot frees only when S_j completes) is what stalls S_{j+2}.
+template <int BN, int NSB>
+__host__ __device__ constexpr int attn4_vstages(int stages) {
+  return Attn4Cols<BN, NSB>::CTAS_PER_SM == 2 && stages > 2 ? 2 : stages;
+}
+// Barrier words of attn4 after the rings: q_full, k_full/empty[stages],
+// v_full/empty[vstages], s_full/s_free[2], p_full, pv_full, drain[2], then
+// the TMEM address and the abort flag.
+__host__ __device__ constexpr size_t attn4_bar_bytes(int stages, int vstages) {
+  return (size_t)(9 + 2 * stages + 2 * vstages) * 8 + 8;
+}
+// Two CTAs per SM need the operands packed without alignment slack: the
+// dynamic shared memory base is then required to be 1024-byte aligned (the
+// kernel checks and reports RC_DEV_MISALIGNED otherwise).
+template <int BN, int NSB>
+size_t attn4_smem(int stages) {
+  const int vst = attn4_vstages<BN, NSB>(stages);
+  const size_t tiles = (size_t)BM * D * 2 + (size_t)(stages + vst) * BN * D * 2;
+  return tiles + attn4_bar_bytes(stages, vst) + (Attn4Cols<BN, NSB>::CTAS_PER_SM == 2 ? 0 : 1024);
+}
+
 template <int BN, bool VT, int NSB>
 __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     attn4_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -1337,16 +1361,24 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
   constexpr uint32_t TMEM_COLS = Attn4Cols<BN, NSB>::ALLOC;
 
   extern __shared__ uint8_t smem_raw[];
+  if constexpr (Attn4Cols<BN, NSB>::CTAS_PER_SM == 2) {
+    // the operands are packed without alignment slack (two CTAs per SM)
+    if (tc::smem_u32(smem_raw) & 1023u) {
+      if (threadIdx.x == 0) tc::record_failure(p.status, RC_DEV_MISALIGNED);
+      return;
+    }
+  }
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int vstages = attn4_vstages<BN, NSB>(stages);
   uint8_t* sQ = smem;
   uint8_t* kring = smem + Q_BYTES;
   uint8_t* vring = kring + (size_t)stages * KV_TILE;
-  uint64_t* q_full = (uint64_t*)(vring + (size_t)stages * KV_TILE);
+  uint64_t* q_full = (uint64_t*)(vring + (size_t)vstages * KV_TILE);
   uint64_t* k_full = q_full + 1;      // [stages]
   uint64_t* k_empty = k_full + stages;
-  uint64_t* v_full = k_empty + stages;
-  uint64_t* v_empty = v_full + stages;
-  uint64_t* s_full = v_empty + stages;  // [2] S buffers
+  uint64_t* v_full = k_empty + stages;  // [vstages]
+  uint64_t* v_empty = v_full + vstages;
+  uint64_t* s_full = v_empty + vstages;  // [2] S buffers
   uint64_t* s_free = s_full + 2;        // [2]
   uint64_t* p_full = s_free + 2;
   uint64_t* pv_full = p_full + 1;
@@ -1380,6 +1412,8 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     for (int s = 0; s < stages; ++s) {
       tc::mbar_init(&k_full[s], 1);
       tc::mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < vstages; ++s) {
       tc::mbar_init(&v_full[s], 1);
       tc::mbar_init(&v_empty[s], 1);
     }
@@ -1402,11 +1436,11 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
   // slot s of a ring last held block j - stages; its release is the
   // ((j - stages) / stages)-th phase of empty[s], parity ph ^ 1 (a fresh
   // barrier passes that parity at once)
-  auto produce = [&](uint64_t* full, uint64_t* empty, auto load) {
+  auto produce = [&](uint64_t* full, uint64_t* empty, int depth, auto load) {
     int j = 0;
     for (; j < nkb; ++j) {
-      const int s = j % stages;
-      const uint32_t ph = (uint32_t)(j / stages) & 1u;
+      const int s = j % depth;
+      const uint32_t ph = (uint32_t)(j / depth) & 1u;
       if (!tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status)) {
         fail(RC_DEV_TIMEOUT_EMPTY);
         break;
@@ -1414,8 +1448,8 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
       tc::mbar_expect_tx(&full[s], KV_TILE);
       load(s, j, &full[s]);
     }
-    for (int i = max(0, j - stages); i < j; ++i)
-      if (!tc::mbar_wait_drain(&full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+    for (int i = max(0, j - depth); i < j; ++i)
+      if (!tc::mbar_wait_drain(&full[i % depth], (uint32_t)(i / depth) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
   };
 
   if (warp == 0) {
@@ -1426,7 +1460,7 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
       const int qrow = b * p.S + q0;
       tc::tma_load_2d(sQ, &tmQ, q_full, h * D, qrow);
       tc::tma_load_2d(sQ + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
-      produce(k_full, k_empty, [&](int s, int j, uint64_t* bar) {
+      produce(k_full, k_empty, stages, [&](int s, int j, uint64_t* bar) {
         uint8_t* sk = kring + (size_t)s * KV_TILE;
         const int krow = b * p.S + j * BN;
         tc::tma_load_2d(sk, &tmK, bar, g * D, krow);
@@ -1438,7 +1472,7 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
   } else if (warp == 3) {
     if (lane == 0) {
       tc::prefetch_tmap(&tmV);
-      produce(v_full, v_empty, [&](int s, int j, uint64_t* bar) {
+      produce(v_full, v_empty, vstages, [&](int s, int j, uint64_t* bar) {
         uint8_t* sv = vring + (size_t)s * KV_TILE;
         if constexpr (VT) {
 #pragma unroll
@@ -1499,8 +1533,8 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
       const uint32_t tO = tmem + O_COL, tP = tmem + P_COL;
       bool ok = true;
       for (int j = 0; ok && j < nkb; ++j) {
-        const int s = j % stages;
-        ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / stages) & 1u, abort_flag, status) &&
+        const int s = j % vstages;
+        ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / vstages) & 1u, abort_flag, status) &&
              tc::mbar_wait(p_full, (uint32_t)j & 1u, abort_flag, status);
         if (!ok) break;
         tc::tc_fence_after();
@@ -1844,7 +1878,8 @@ rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const vo
   const long long ctas = (long long)p.B * p.Hq * (PINGPONG ? (p.q_blocks + 1) / 2 : p.q_blocks);
   if (ctas > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
   const int qtiles = PINGPONG ? 2 : 1;
-  const size_t smem = smem_bytes(BN, k.stages, qtiles) - (PT ? (size_t)qtiles * BM * BN * 2 : 0);
+  size_t smem = smem_bytes(BN, k.stages, qtiles) - (PT ? (size_t)qtiles * BM * BN * 2 : 0);
+  if constexpr (PAR && !PINGPONG) smem = attn4_smem<BN, SDB ? 2 : 1>(k.stages);
   const int threads = PAR ? (PINGPONG ? (BN == 64 ? kThreads5 : kThreads3) : kThreads4) : PINGPONG ? kThreads2 : kThreads;
   kern<<<(unsigned)ctas, threads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
   cudaError_t e = cudaGetLastError();

@@ -27,7 +27,8 @@ enum {
   RC_DEV_TIMEOUT_EMPTY = 2,  // producer gave up waiting for a free stage
   RC_DEV_TIMEOUT_ACCUM = 3,  // epilogue gave up waiting for the accumulator
   RC_DEV_TIMEOUT_DRAIN = 4,  // teardown gave up waiting for in-flight copies / MMAs
-  RC_DEV_BAD_ARG = 5         // a kernel-side argument check failed
+  RC_DEV_BAD_ARG = 5,        // a kernel-side argument check failed
+  RC_DEV_MISALIGNED = 6      // dynamic shared memory not at the alignment a packed layout needs
 };
 
 // ------------------------------------------------------------------ ops --

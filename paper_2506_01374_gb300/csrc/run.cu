@@ -276,6 +276,8 @@ rc_status read_status(const rc_op_s* op) {
   if (st != RC_DEV_OK) {
     cudaMemset(op->d_status, 0, sizeof st);
     if (st == RC_DEV_BAD_ARG) return rc_fail(RC_ERR_INVALID_ARG, "a kernel rejected its arguments");
+    if (st == RC_DEV_MISALIGNED)
+      return rc_fail(RC_ERR_CUDA, "dynamic shared memory was not 1024-byte aligned for a packed kernel layout");
     return rc_fail(RC_ERR_DEVICE_TIMEOUT, "a bounded device wait gave up (code %d)", st);
   }
   return RC_OK;
@@ -407,8 +409,17 @@ extern "C" rc_status rc_candidate_measure(const rc_op* op, const rc_schedule* co
     }
   }
   cudaStream_t st = (cudaStream_t)stream;
-  std::vector<cudaEvent_t> ev(2 * (size_t)o.repeats);
-  for (auto& e : ev) RC_TRY(cuda_err(cudaEventCreate(&e), "cudaEventCreate"));
+  // per repeat: a start event and one event after each stage (the last one ends the run)
+  constexpr int EV = RC_MAX_STAGES + 1;
+  std::vector<cudaEvent_t> ev((size_t)EV * o.repeats, nullptr);
+  for (auto& e : ev) {
+    rc_status cs = cuda_err(cudaEventCreate(&e), "cudaEventCreate");
+    if (cs != RC_OK) {
+      for (auto& x : ev)
+        if (x) cudaEventDestroy(x);
+      return cs;
+    }
+  }
   auto destroy = [&]() {
     for (auto& e : ev) cudaEventDestroy(e);
   };
@@ -433,12 +444,19 @@ extern "C" rc_status rc_candidate_measure(const rc_op* op, const rc_schedule* co
     LaunchCtx c;
     rc_status s = prepare(op, cands[i], &c, stream);
     for (int w = 0; s == RC_OK && w < o.warmup; ++w) s = run_impl(op, cands[i], io, c);
+    int n_marks = 0;  // stage-end events of a run (the same for every repeat)
     for (int r = 0; s == RC_OK && r < o.repeats; ++r) {
+      cudaEvent_t* er = ev.data() + (size_t)EV * r;
       if (o.flush_l2) s = rc_launch_l2_flush(di->flush, di->flush_bytes, stream);
-      if (s == RC_OK) s = cuda_err(cudaEventRecord(ev[2 * r], st), "cudaEventRecord");
+      if (s == RC_OK) s = cuda_err(cudaEventRecord(er[0], st), "cudaEventRecord");
+      c.stage_events = (void**)(er + 1);
+      c.n_stage_events = RC_MAX_STAGES;
+      c.next_event = 0;
       if (s == RC_OK) s = run_impl(op, cands[i], io, c);
-      if (s == RC_OK) s = cuda_err(cudaEventRecord(ev[2 * r + 1], st), "cudaEventRecord");
+      if (s == RC_OK && c.next_event == 0) s = rc_mark_stage(c);  // single-stage ops: mark the end
+      n_marks = c.next_event;
     }
+    c.stage_events = nullptr;
     if (s == RC_OK) s = cuda_err(cudaStreamSynchronize(st), "cudaStreamSynchronize");
     if (s == RC_OK) s = read_status(op);
     if (s == RC_ERR_CUDA) {
@@ -455,16 +473,31 @@ extern "C" rc_status rc_candidate_measure(const rc_op* op, const rc_schedule* co
       m.status = s;
       continue;
     }
+    auto median = [](std::vector<double> v) {
+      std::sort(v.begin(), v.end());
+      const size_t R = v.size();
+      return R % 2 ? v[R / 2] : 0.5 * (v[R / 2 - 1] + v[R / 2]);
+    };
     std::vector<double> t(o.repeats);
     for (int r = 0; r < o.repeats; ++r) {
       float ms = 0.f;
-      cudaEventElapsedTime(&ms, ev[2 * r], ev[2 * r + 1]);
+      cudaEventElapsedTime(&ms, ev[(size_t)EV * r], ev[(size_t)EV * r + n_marks]);
       t[r] = ms;
+    }
+    m.n_stages = n_marks;
+    for (int g = 0; g < n_marks; ++g) {
+      std::vector<double> ts(o.repeats);
+      for (int r = 0; r < o.repeats; ++r) {
+        float ms = 0.f;
+        cudaEventElapsedTime(&ms, ev[(size_t)EV * r + g], ev[(size_t)EV * r + g + 1]);
+        ts[r] = ms;
+      }
+      m.stage_ms[g] = median(ts);
     }
     std::vector<double> srt = t;
     std::sort(srt.begin(), srt.end());
     const size_t R = srt.size();
-    m.ms_median = R % 2 ? srt[R / 2] : 0.5 * (srt[R / 2 - 1] + srt[R / 2]);
+    m.ms_median = median(t);
     m.ms_min = srt[0];
     double sum = 0;
     for (double x : t) sum += x;

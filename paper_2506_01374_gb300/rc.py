@@ -80,20 +80,24 @@ class MeasureOpts(C.Structure):
 
 class Measurement(C.Structure):
     _fields_ = [("status", C.c_int32), ("ms_median", C.c_double), ("ms_min", C.c_double), ("ms_mean", C.c_double),
-                ("tflops", C.c_double), ("gbps", C.c_double), ("sched_hash", C.c_uint64)]
+                ("tflops", C.c_double), ("gbps", C.c_double), ("sched_hash", C.c_uint64), ("n_stages", C.c_int32),
+                ("stage_ms", C.c_double * MAX_STAGES)]
 
     def as_dict(self):
-        return {n: getattr(self, n) for n, _ in self._fields_}
+        d = {n: getattr(self, n) for n, _ in self._fields_ if n != "stage_ms"}
+        d["stage_ms"] = [self.stage_ms[i] for i in range(self.n_stages)]
+        return d
 
 
 class SearchOpts(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("c", C.c_double), ("branching", C.c_int32), ("horizon", C.c_int32),
-                ("rollout", C.c_int32), ("max_tries", C.c_int32)]
+                ("rollout", C.c_int32), ("max_tries", C.c_int32), ("surrogate", C.c_int32), ("screen", C.c_int32)]
 
 
 class SearchStats(C.Structure):
     _fields_ = [("nodes", C.c_int64), ("samples", C.c_int64), ("iterations", C.c_int64),
-                ("best_reward", C.c_double)]
+                ("best_reward", C.c_double), ("model_samples", C.c_int64), ("model_features", C.c_int64),
+                ("predicted", C.c_int64)]
 
 
 class RcError(RuntimeError):
@@ -130,6 +134,7 @@ _PROTOS = {
                                  C.POINTER(C.c_size_t)]),
     "rc_search_best": (C.c_int, [_P, C.POINTER(_P), C.POINTER(Measurement)]),
     "rc_search_get_stats": (C.c_int, [_P, C.POINTER(SearchStats)]),
+    "rc_search_predict": (C.c_int, [_P, _P, C.POINTER(C.c_double)]),
     "rc_search_node": (C.c_int, [_P, C.c_int64, C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                  C.POINTER(C.c_int64), C.POINTER(C.c_uint64)]),
     "rc_search_destroy": (None, [_P]),
@@ -324,9 +329,9 @@ class Search:
     """LLM-free MCTS over an op's schedule space (rc_search_*)."""
 
     def __init__(self, op: Op, seed: int = 0, c: float = math.sqrt(2.0), branching: int = 2, horizon: int = 8,
-                 rollout: int = 2, max_tries: int = 64):
+                 rollout: int = 2, max_tries: int = 64, surrogate: bool = False, screen: int = 1):
         self.op = op
-        o = SearchOpts(seed, c, branching, horizon, rollout, max_tries)
+        o = SearchOpts(seed, c, branching, horizon, rollout, max_tries, int(surrogate), screen)
         h = _P()
         _check(lib().rc_search_create(op.h, C.byref(o), C.byref(h)), "rc_search_create")
         self.h = h.value
@@ -360,7 +365,13 @@ class Search:
     def stats(self) -> dict:
         s = SearchStats()
         _check(lib().rc_search_get_stats(self.h, C.byref(s)))
-        return {"nodes": s.nodes, "samples": s.samples, "iterations": s.iterations, "best_reward": s.best_reward}
+        return {n: getattr(s, n) for n, _ in SearchStats._fields_}
+
+    def predict(self, sched: Schedule) -> float:
+        """The learned surrogate's predicted device time (ms) of sched (rc_search_predict)."""
+        ms = C.c_double()
+        _check(lib().rc_search_predict(self.h, sched.h, C.byref(ms)), "rc_search_predict")
+        return ms.value
 
     def node(self, i: int) -> dict:
         p, q, n, h = C.c_int64(), C.c_double(), C.c_int64(), C.c_uint64()
