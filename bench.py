@@ -65,6 +65,11 @@ def parse():
     ap.add_argument("--restarts", type=int, default=2,
                     help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--surrogate", type=int, default=1, choices=[0, 1],
+                    help="1 = rollouts scored by the search's learned surrogate f-hat (Sec. 3.2), only expanded "
+                         "nodes measured; 0 = rollout programs measured too")
+    ap.add_argument("--screen", type=int, default=4,
+                    help="with --surrogate 1: proposals screened by f-hat per kept child (1 = no screening)")
     ap.add_argument("--shape", default="",
                     help="override workload sizes for a profiling case, e.g. 'tokens=1024,experts=16' (the line "
                          "then reports that shape, not the benchmark configuration)")
@@ -342,22 +347,24 @@ def parse_schedule(op, text, rc):
     return op.schedule(*ts)
 
 
-def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1):
+def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, surrogate=False, screen=1):
     """MCTS over op's schedule space with device-timed candidates; returns (search, best, m, n, cand/s).
 
     Candidates are timed with 5 repeats while searching; the `finalists` best
     of them are timed again with 20 repeats and the fastest is returned, so a
-    noisy short measurement does not decide the result.
+    noisy short measurement does not decide the result. surrogate/screen: the
+    learned rollout surrogate and proposal screening of rc_search_opts.
     """
     from paper_2506_01374_gb300 import rc
     if restarts > 1:  # independent searches; rewards are noisy measurements, so trajectories differ
-        runs = [search_best(op, io, samples, seed + r, branching, finalists) for r in range(restarts)]
+        runs = [search_best(op, io, samples, seed + r, branching, finalists, 1, surrogate, screen)
+                for r in range(restarts)]
         i = min(range(restarts), key=lambda r: runs[r][2].ms_median if runs[r][2].status == rc.OK else float("inf"))
         search, best, m, _, _ = runs[i]
         n = sum(r[3] for r in runs)
         cps = [r[4] for r in runs if r[4]]
         return search, best, m, n, (sum(cps) / len(cps) if cps else None)
-    search = rc.Search(op, seed=seed, branching=branching)
+    search = rc.Search(op, seed=seed, branching=branching, surrogate=surrogate, screen=screen)
     res, n, t, pending = [], 0, 0.0, False
     seen = []  # (median ms, schedule owned by the search)
     while n < samples:
@@ -383,7 +390,7 @@ def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1):
     return search, best, m, n, (n / t if t else None)
 
 
-def extra_ops(names, samples, peak_tf, branching=4, restarts=1):
+def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1):
     """Search each other workload briefly and report its best schedule."""
     import torch
 
@@ -392,7 +399,8 @@ def extra_ops(names, samples, peak_tf, branching=4, restarts=1):
     for name in names:
         wl = Workload(name)
         io = wl.device_io()
-        _, best, _, n, cps = search_best(wl.op, io, samples, branching=branching, restarts=restarts)
+        _, best, _, n, cps = search_best(wl.op, io, samples, branching=branching, restarts=restarts,
+                                         surrogate=surrogate, screen=screen)
         m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
         if m.status != rc.OK:
             out[name] = {"workload": wl.label, "error": rc.STATUS_NAMES.get(m.status, m.status)}
@@ -476,7 +484,8 @@ def run_ours(args):
         best = parse_schedule(op, args.schedule, rc)
     else:
         search, best, best_m, n_meas, cps = search_best(op, io, args.samples, seed=args.seed,
-                                                        branching=args.branching, restarts=args.restarts)
+                                                        branching=args.branching, restarts=args.restarts,
+                                                        surrogate=bool(args.surrogate), screen=args.screen)
 
     # 2) timed steps of the best schedule
     flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
@@ -543,7 +552,8 @@ def run_ours(args):
             "roofline": {"bound": wl.bound, "kernel": kname, "achieved": achieved, "peak": peak,
                          "unit": "TFLOP/s", "frac": achieved / peak, "peak_source": peak_src, "traffic": None},
             "step_frac_of_peak": value / world / peak,
-            "search": {"samples": n_meas, "candidates_per_s": cps,
+            "search": {"samples": n_meas, "candidates_per_s": cps, "surrogate": bool(args.surrogate),
+                       "screen": args.screen,
                        "best_search_tflops": best_m.tflops if best_m else None,
                        "stats": search.stats() if search else None},
             "e2e": None if e2e_s is None else {"value": world * info["flops"] / e2e_s / 1e12, "unit": "TFLOP/s",
@@ -557,7 +567,8 @@ def run_ours(args):
         if names:
             del io
             torch.cuda.empty_cache()
-            out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"], args.branching, args.restarts)
+            out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"], args.branching, args.restarts,
+                                   bool(args.surrogate), args.screen)
         if args.cpu_sample >= 0:
             cb = wl.cpu_sample(args.cpu_sample)
             cb.pop("seconds", None)
