@@ -19,10 +19,11 @@ constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
 // Tensor-core GEMM shared-memory footprint per CTA: a ring of `stages`
 // stages of tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64,
 // or bn/2 x 64 in each CTA of a pair) bf16 tile, plus 1 KB alignment slack,
-// barriers and four fp32 copies of a bias tile.
+// barriers, four fp32 copies of a bias tile and a 128-entry row table.
 int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k, int tile_m) {
   const int64_t b_rows = tile_m == 256 ? bn_mma / 2 : bn_mma;
-  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + b_rows * 64 * 2) + 1024 + 256 + 4 * (int64_t)bn_mma * 4;
+  return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + b_rows * 64 * 2) + 1024 + 256 + 4 * (int64_t)bn_mma * 4 +
+         128 * 4;
 }
 
 bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, std::string* why) {
@@ -163,6 +164,9 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       } else if (stage == 1) {
         gemm_common({32, 64, 128});
         v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256: a CTA pair within one expert's rows
+        // where the token rows are gathered: 0 = a separate pass writes the grouped copy (stage 0),
+        // 1 = the grouped GEMM's producer gathers them from X (M tile 128)
+        v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});
       } else {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
@@ -268,6 +272,10 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
       return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_MOE:
       if (stage == 0) return true;
+      if (stage == 1 && k.location == 1 && k.tile_m != 128) {
+        if (why) *why = "rows gathered in the GEMM producer need one CTA per tile (M tile 128)";
+        return false;
+      }
       return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_ATTENTION: {
       // Q tiles + ring of K and V tiles + P tiles + slack, all bf16

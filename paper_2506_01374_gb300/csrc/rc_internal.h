@@ -110,7 +110,8 @@ enum TcEpilogue {
 enum TcAMode {
   TC_A_2D = 0,         // A is a row-major [M][K] matrix
   TC_A_CONV = 1,       // A rows are output pixels of an NHWC 'same' conv; K = (r, s, c); one 4-D box
-  TC_A_CONV_ROWS = 2   // as TC_A_CONV over an explicitly padded input, one 2-D box per image row
+  TC_A_CONV_ROWS = 2,  // as TC_A_CONV over an explicitly padded input, one 2-D box per image row
+  TC_A_GATHER = 3      // grouped only: A row i is row row_map[i] / row_div of a [a_rows][K] matrix
 };
 struct TcGemmArgs {
   int64_t M, N, K;         // N = UMMA columns of the whole problem (2I for SwiGLU)
@@ -135,7 +136,8 @@ struct TcGemmArgs {
   int64_t max_tiles_m;     // upper bound on m-tiles over all groups
   const float* row_scale;  // TC_EPI_SCALE_ATOMIC
   const int* row_map;      // TC_EPI_SCALE_ATOMIC: A row -> slot; output row = slot / row_div
-  int row_div;
+  int row_div;             // (TC_A_GATHER: A row i is source row row_map[i] / row_div)
+  int64_t a_rows;          // TC_A_GATHER: rows of the source matrix A
 };
 rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 // Split-K reduction: out_bf16[M][N] = sum_z part[z][M][N].

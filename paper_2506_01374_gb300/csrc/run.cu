@@ -214,15 +214,24 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       void* Hb = ws.take(2ull * slots * d.inter);
       void* Yb = ws.take(2ull * slots * d.hidden);
       float* acc = (float*)ws.take(4ull * d.tokens * d.hidden);
+      // gate/up compute location 1: the GEMM's producer gathers X's rows itself (no gathered copy)
+      const bool gather_in_gemm = s->k[1].location == 1;
       RC_TRY(rc_launch_moe_route(s->k[0], d, p[0], ids, w, offsets, perm, inv, counts, c));
-      RC_TRY(rc_launch_moe_gather(p[1], perm, slots, d.hidden, (int)d.top_k, Xp, 16, c));
+      if (!gather_in_gemm) RC_TRY(rc_launch_moe_gather(p[1], perm, slots, d.hidden, (int)d.top_k, Xp, 16, c));
       RC_TRY(rc_mark_stage(c));
       const int64_t max_tiles = slots / 128 + d.experts;
-      TcGemmArgs g1 = gemm_args(slots, 2 * d.inter, d.hidden, Xp, p[2], Hb, d.inter, TC_EPI_SWIGLU);
+      TcGemmArgs g1 =
+          gemm_args(slots, 2 * d.inter, d.hidden, gather_in_gemm ? p[1] : Xp, p[2], Hb, d.inter, TC_EPI_SWIGLU);
       g1.groups = (int)d.experts;
       g1.offsets = offsets;
       g1.b_group_rows = 2 * d.inter;
       g1.max_tiles_m = max_tiles;
+      if (gather_in_gemm) {
+        g1.a_mode = TC_A_GATHER;
+        g1.row_map = perm;
+        g1.row_div = (int)d.top_k;
+        g1.a_rows = d.tokens;
+      }
       RC_TRY(rc_launch_tc_gemm(s->k[1], g1, c));
       RC_TRY(rc_mark_stage(c));
       TcGemmArgs g2 = gemm_args(slots, d.hidden, d.inter, Hb, p[3], Yb, d.hidden, TC_EPI_STORE_BF16);

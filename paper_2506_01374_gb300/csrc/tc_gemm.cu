@@ -84,6 +84,8 @@ rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const Launch
   const bool pair = k.tile_m == 256;  // a CTA pair per 256-row tile
   if (a.a_mode == TC_A_CONV || a.a_mode == TC_A_CONV_ROWS)
     return pair ? tc_dispatch_conv_pair(k, a, c) : tc_dispatch_conv(k, a, c);
+  if (a.a_mode == TC_A_GATHER && (pair || a.groups <= 0))
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: gathered A rows need a grouped GEMM on one CTA (M tile 128)");
   if (a.groups > 0) return pair ? tc_dispatch_grouped_pair(k, a, c) : tc_dispatch_grouped(k, a, c);
   return pair ? tc_dispatch_dense_pair(k, a, c) : tc_dispatch_dense(k, a, c);
 }

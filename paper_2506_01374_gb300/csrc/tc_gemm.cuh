@@ -26,7 +26,14 @@
 // group (runtime), and the fused epilogue (template EPI). The A operand is a
 // plain matrix or, for convolutions, an implicit im2col view loaded with a
 // 4-D TMA box whose out-of-range coordinates are zero-filled (the padding).
-// Grouped mode (MoE) partitions A's rows into segments with their own B.
+// Grouped mode (MoE) partitions A's rows into segments with their own B; its
+// A rows may also be gathered from a source matrix by a row map inside the
+// producer (TC_A_GATHER), which then uses the whole warp 0: each lane copies
+// 16-byte chunks of 32 rows with cp.async, applying the 128-byte swizzle
+// itself, and has the stage's "full" barrier count an arrival of its own once
+// those copies land (cp.async.mbarrier.arrive); lane 0 still loads B by TMA.
+// The MMA thread fences the generic-proxy copies for the tensor cores (async
+// proxy) after the barrier wait.
 #pragma once
 
 #include <cstring>
@@ -61,6 +68,7 @@ struct Params {
   const float* row_scale;
   const int* row_map;
   int row_div;
+  const __nv_bfloat16* a_src;  // TC_A_GATHER: source rows [..][K]
   int* status;
   int persistent;       // 1: grid-stride loop over tiles with two TMEM accumulators
   int splits;           // split-K factor (work items = tiles x splits)
@@ -252,6 +260,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* status = p.status;
   // one copy of the tile's bias per epilogue warp (BN floats each, 16-byte aligned)
   float* sbias_all = (float*)(((uintptr_t)(abort_flag + 1) + 15) & ~(uintptr_t)15);
+  // gathered A: source row of each of the tile's 128 rows (-1 = past the segment)
+  int* s_src = (int*)(sbias_all + 4 * BN);
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n_acc = p.persistent ? 2 : 1;  // accumulator buffers in TMEM
@@ -273,7 +283,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
-      tc::mbar_init(&full[s], 1);
+      // gathered A: lane 0's arrival with the B bytes and one arrival per lane for its A copies
+      tc::mbar_init(&full[s], AMODE == TC_A_GATHER ? 33 : 1);
       tc::mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -298,7 +309,78 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
+  if (warp == 0 && AMODE == TC_A_GATHER) {
+    if constexpr (AMODE == TC_A_GATHER && !PAIR) {
+      if (lane == 0) tc::prefetch_tmap(&tmB);
+      const int chunk = lane & 7;          // this lane's 16-byte chunk of each 128-byte row segment
+      const int rsub = lane >> 3;          // and its rows rsub + 4 i, i < 32
+      uint32_t g = 0;                      // stages filled so far
+      int s = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      for (long long w = w_first; ok && w < items; w += w_step) {
+        const Item it = item(w);
+        if (!it.valid) continue;
+        __syncwarp();  // the previous tile's copies have all been issued
+#pragma unroll
+        for (int i = 0; i < BM / 32; ++i) {
+          const int r = it.row0 + lane + 32 * i;
+          s_src[lane + 32 * i] = r < it.row_end ? p.row_map[r] / p.row_div : -1;
+        }
+        __syncwarp();
+        int kb = it.kb0;
+        for (int i = 0; i < it.nkb; i += ksub, ++g) {
+          const int nsub = min(ksub, it.nkb - i);
+          int okl = 1;
+          if (lane == 0) okl = tc::mbar_wait(&empty[s], ph ^ 1u, abort_flag, status) ? 1 : 0;
+          okl = __shfl_sync(0xffffffffu, okl, 0);
+          if (!okl) {
+            if (lane == 0) fail(RC_DEV_TIMEOUT_EMPTY);
+            ok = false;
+            break;
+          }
+          uint8_t* stage = smem + (size_t)s * STAGE_BYTES;
+          if (lane == 0) {
+            tc::mbar_expect_tx(&full[s], (uint32_t)nsub * B_BYTES);
+            for (int q = 0; q < nsub; ++q) {
+              uint8_t* sb = stage + ksub * A_BYTES + q * B_BYTES;
+              const int nh = it.nt * (BN / 2);
+              tc::tma_load_2d(sb, &tmB, &full[s], (kb + q) * BK, it.brow0 + nh);
+              tc::tma_load_2d(sb + (BN / 2) * 128, &tmB, &full[s], (kb + q) * BK, it.brow0 + p.swiglu_I + nh);
+            }
+          }
+          for (int q = 0; q < nsub; ++q) {
+            const uint32_t sa = tc::smem_u32(stage + q * A_BYTES);
+            const int col = (kb + q) * BK + chunk * 8;
+            const bool col_ok = col < p.K;
+#pragma unroll 8
+            for (int ii = 0; ii < 32; ++ii) {
+              const int row = rsub + 4 * ii;
+              const int src = s_src[row];
+              const uint32_t dst = sa + (uint32_t)row * 128u + ((uint32_t)(chunk ^ (row & 7)) << 4);
+              const bool v = src >= 0 && col_ok;
+              tc::cp_async16(dst, v ? (const void*)(p.a_src + (size_t)src * p.K + col) : (const void*)p.a_src,
+                             v ? 16u : 0u);
+            }
+          }
+          kb += nsub;
+          tc::cp_async_mbar_arrive(&full[s]);  // this lane's arrival, when its copies of the stage land
+          if (++s == stages) {
+            s = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+      tc::cp_async_wait(0);  // no copy of this lane is in flight at exit
+      if (lane == 0) {  // let the B copies of the last stages land before exit
+        const uint32_t first = g > (uint32_t)stages ? g - (uint32_t)stages : 0u;
+        for (uint32_t j = first; j < g; ++j)
+          if (!tc::mbar_wait_drain(&full[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u))
+            fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();  // reconverge before the final block barrier
+  } else if (warp == 0) {
     if (lane == 0) {
       tc::prefetch_tmap(&tmA);
       tc::prefetch_tmap(&tmB);
@@ -421,6 +503,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
           }
+          // gathered A: cp.async wrote the rows through the generic proxy; order them before the UMMA reads
+          if constexpr (AMODE == TC_A_GATHER) tc::fence_proxy_async_smem();
           tc::tc_fence_after();
           const uint32_t sa = tc::smem_u32(smem + (size_t)s * STAGE_BYTES);
 #pragma unroll
@@ -555,10 +639,10 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
 
 // ring of A (128 rows) and this CTA's B rows (bn, or bn / 2 for a CTA pair)
 // per sub-block + 1 KB alignment slack + barriers and flags (256 B) + four
-// fp32 bias copies of the bn-column tile
+// fp32 bias copies of the bn-column tile + the gathered-A row table (512 B)
 inline size_t smem_bytes(int bn, int stages, int ksub, bool pair = false) {
   const size_t b_rows = pair ? (size_t)bn / 2 : (size_t)bn;
-  return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4;
+  return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4 + BM * 4;
 }
 
 template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
@@ -583,6 +667,11 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   } else if constexpr (AMODE == TC_A_CONV_ROWS) {
     const uint64_t rows = (uint64_t)a.img_n * (a.img_h + 2 * a.pad) * (a.img_w + 2 * a.pad);
     RC_TRY(encode_2d(&tmA, a.A, a.c_in, rows, (uint32_t)a.img_w));
+  } else if constexpr (AMODE == TC_A_GATHER) {
+    static_assert(GROUPED && !PAIR && EPI == TC_EPI_SWIGLU, "gathered A: grouped SwiGLU on one CTA");
+    if (a.a_rows <= 0 || !a.row_map || (uintptr_t)a.A % 16 || a.K % 8)
+      return rc_fail(RC_ERR_INVALID_ARG, "tc_gemm: gathered A needs a row map, rows and 16-byte rows");
+    memset(&tmA, 0, sizeof tmA);  // A is copied with cp.async; the map is unused
   } else {
     RC_TRY(encode_2d(&tmA, a.A, a.K, a.M, BM));
   }
@@ -628,6 +717,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.row_scale = a.row_scale;
   p.row_map = a.row_map;
   p.row_div = a.row_div > 0 ? a.row_div : 1;
+  p.a_src = (const __nv_bfloat16*)a.A;
   p.status = c.status;
   constexpr int acc_cols = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   return launch_kernel(kern, tmA, tmB, p, k.stages, acc_cols, smem, PAIR, c);

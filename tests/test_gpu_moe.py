@@ -60,8 +60,10 @@ def moe_op(T, H, E, I, K):
     return rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
 
 
-def moe_sched(op, tm, tn1, st1, tn2, st2, fuse, persistent=0, tile_k=64, tile_m=128):
-    return op.schedule(rc.T(rc.T_TILE_SIZE, tm, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
+def moe_sched(op, tm, tn1, st1, tn2, st2, fuse, persistent=0, tile_k=64, tile_m=128, gather=0):
+    # gather = 1: the grouped gate/up GEMM's producer gathers the token rows itself (compute location 1)
+    return op.schedule(rc.T(rc.T_COMPUTE_LOCATION, gather, stage=1),
+                       rc.T(rc.T_TILE_SIZE, tm, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
                        rc.T(rc.T_PIPELINE_STAGES, st1, stage=1), rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2),
                        rc.T(rc.T_PIPELINE_STAGES, st2, stage=2), rc.T(rc.T_FUSE, fuse, stage=2),
                        rc.T(rc.T_PARALLEL, persistent, stage=1), rc.T(rc.T_PARALLEL, persistent, stage=2),
@@ -76,12 +78,12 @@ def test_moe_layer_schedule_sweep():
     ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
     op = moe_op(T, H, E, I, K)
     dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
-    for tn1, tn2, fuse, st, pe, tk, tm in itertools.product((32, 64, 128), (64, 128, 224, 256), (0, 1), (1, 3),
-                                                            (0, 1), (64, 128), (128, 256)):
+    for tn1, tn2, fuse, st, pe, tk, tm, ga in itertools.product((32, 64, 128), (64, 128, 224, 256), (0, 1), (1, 3),
+                                                                (0, 1), (64, 128), (128, 256), (0, 1)):
         try:  # CTA pairs (tm = 256) take 256 rows of one expert's segment
-            s = moe_sched(op, 8, tn1, st, tn2, st, fuse, pe, tk, tm)
+            s = moe_sched(op, 8, tn1, st, tn2, st, fuse, pe, tk, tm, ga)
         except rc.RcError:
-            continue  # shared memory (K = 128, 3 stages, widest N); TMEM of persistent pairs
+            continue  # shared memory (K = 128, 3 stages, widest N); TMEM of persistent pairs; gather on pairs
         out = empty_bf16(T, H).fill_(0x7FC0)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         gp = torch.empty(T * K, dtype=torch.int32, device="cuda")
@@ -90,7 +92,7 @@ def test_moe_layer_schedule_sweep():
         np.testing.assert_array_equal(gi.cpu().numpy(), ids)
         np.testing.assert_array_equal(gp.cpu().numpy(), perm)
         err = rel_err(from_dev_bf16(out), ref)
-        assert err <= TOL, (tn1, tn2, fuse, st, pe, tk, tm, err)
+        assert err <= TOL, (tn1, tn2, fuse, st, pe, tk, tm, ga, err)
 
 
 def test_moe_layer_imbalanced_and_empty_experts():
@@ -103,12 +105,14 @@ def test_moe_layer_imbalanced_and_empty_experts():
     assert (np.diff(off)[4:] == 0).all() and (np.diff(off)[:4] == T).all()
     ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
     op = moe_op(T, H, E, I, K)
-    for fuse, pe, tm in itertools.product((0, 1), (0, 1), (128, 256)):
+    for fuse, pe, tm, ga in itertools.product((0, 1), (0, 1), (128, 256), (0, 1)):
+        if ga and tm == 256:
+            continue
         out = empty_bf16(T, H).fill_(0x7FC0)
-        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse, pe, tile_m=tm),
+        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse, pe, tile_m=tm, gather=ga),
                [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
-        assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm)
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm, ga)
 
 
 def test_moe_full_size_sampled_tokens():
@@ -122,7 +126,8 @@ def test_moe_full_size_sampled_tokens():
     dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
     del W1, W2
     for s in [op.schedule(), moe_sched(op, 8, 128, 2, 256, 2, 0), moe_sched(op, 16, 64, 4, 128, 3, 1),
-              moe_sched(op, 8, 128, 4, 256, 3, 0, 1)]:
+              moe_sched(op, 8, 128, 4, 256, 3, 0, 1), moe_sched(op, 8, 64, 3, 224, 2, 0, gather=1),
+              moe_sched(op, 8, 128, 2, 224, 2, 1, 1, tile_k=128, gather=1)]:
         out = empty_bf16(T, H)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         go = torch.empty(E + 1, dtype=torch.int32, device="cuda")
