@@ -19,11 +19,12 @@ constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
 // Tensor-core GEMM shared-memory footprint per CTA: a ring of `stages`
 // stages of tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64,
 // or bn/2 x 64 in each CTA of a pair) bf16 tile, plus 1 KB alignment slack,
-// barriers, four fp32 copies of a bias tile and a 128-entry row table.
+// barriers, four fp32 copies of a bias tile, a 128-entry row table and the
+// grouped segment tables (2 x 257 entries + 8 B).
 int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k, int tile_m) {
   const int64_t b_rows = tile_m == 256 ? bn_mma / 2 : bn_mma;
   return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + b_rows * 64 * 2) + 1024 + 256 + 4 * (int64_t)bn_mma * 4 +
-         128 * 4;
+         128 * 4 + 2 * 257 * 4 + 8;
 }
 
 bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, std::string* why) {

@@ -194,9 +194,45 @@ struct Item {
   int row0, row_end, brow0, nt, split, kb0, nkb;
 };
 
-// TR: rows of a tile (128, or 256 for a CTA pair)
+// Grouped mode keeps, per CTA, the segment offsets and the exclusive prefix of
+// the segments' tile counts in shared memory (up to kSmemGroups segments),
+// built once by one warp, so that resolving an m tile is a binary search
+// instead of a scan over every segment in global memory.
+constexpr int kSmemGroups = 256;
+constexpr int kGroupTableBytes = 2 * (kSmemGroups + 1) * 4 + 8;
+
+// TR: rows of a tile (128, or 256 for a CTA pair). One warp, all lanes.
+template <int TR>
+__device__ __forceinline__ void build_group_table(const Params& p, int lane, int* s_goff, int* s_gtile) {
+  const int G = p.groups;
+  const int per = (G + 31) / 32;  // segments per lane, lane-major
+  const int g0 = min(G, lane * per), g1 = min(G, g0 + per);
+  int sum = 0;
+  for (int g = g0; g < g1; ++g) {
+    const int lo = p.offsets[g], hi = p.offsets[g + 1];
+    s_goff[g] = lo;
+    sum += (hi - lo + TR - 1) / TR;
+  }
+  int incl = sum;  // inclusive scan of the lanes' tile counts
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, d);
+    if (lane >= d) incl += v;
+  }
+  int acc = incl - sum;
+  for (int g = g0; g < g1; ++g) {
+    s_gtile[g] = acc;
+    acc += (p.offsets[g + 1] - p.offsets[g] + TR - 1) / TR;
+  }
+  if (lane == 31) {
+    s_gtile[G] = incl;
+    s_goff[G] = p.offsets[G];
+  }
+}
+
 template <bool GROUPED, int TR>
-__device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
+__device__ __forceinline__ Item resolve_item(const Params& p, long long w, const int* s_goff = nullptr,
+                                             const int* s_gtile = nullptr) {
   Item it;
   const long long tiles = (long long)p.tiles_m * p.tiles_n;
   it.split = (int)(w / tiles);
@@ -205,18 +241,37 @@ __device__ __forceinline__ Item resolve_item(const Params& p, long long w) {
   it.valid = true;
   it.brow0 = 0;
   if constexpr (GROUPED) {
-    int acc = 0, g = 0;
+    int g = 0;
     it.valid = false;
-    for (; g < p.groups; ++g) {
-      const int lo = p.offsets[g], hi = p.offsets[g + 1];
-      const int n_g = (hi - lo + TR - 1) / TR;
-      if (mt < acc + n_g) {
-        it.row0 = lo + (mt - acc) * TR;
-        it.row_end = hi;
+    if (s_gtile) {
+      // last segment whose first tile is <= mt (empty segments share their successor's start)
+      if (mt < s_gtile[p.groups]) {
+        int lo = 0, hi = p.groups - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (s_gtile[mid] <= mt)
+            lo = mid;
+          else
+            hi = mid - 1;
+        }
+        g = lo;
+        it.row0 = s_goff[g] + (mt - s_gtile[g]) * TR;
+        it.row_end = s_goff[g + 1];
         it.valid = true;
-        break;
       }
-      acc += n_g;
+    } else {
+      int acc = 0;
+      for (; g < p.groups; ++g) {
+        const int lo = p.offsets[g], hi = p.offsets[g + 1];
+        const int n_g = (hi - lo + TR - 1) / TR;
+        if (mt < acc + n_g) {
+          it.row0 = lo + (mt - acc) * TR;
+          it.row_end = hi;
+          it.valid = true;
+          break;
+        }
+        acc += n_g;
+      }
     }
     it.brow0 = g * p.b_group_rows;
   } else {
@@ -262,6 +317,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* sbias_all = (float*)(((uintptr_t)(abort_flag + 1) + 15) & ~(uintptr_t)15);
   // gathered A: source row of each of the tile's 128 rows (-1 = past the segment)
   int* s_src = (int*)(sbias_all + 4 * BN);
+  // grouped: segment offsets and tile prefix (kSmemGroups + 1 entries each)
+  int* s_goff = s_src + BM;
+  int* s_gtile = s_goff + kSmemGroups + 1;
+  const bool gtable = GROUPED && p.groups <= kSmemGroups;
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int n_acc = p.persistent ? 2 : 1;  // accumulator buffers in TMEM
@@ -271,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const long long w_first = PAIR ? blockIdx.x / 2 : blockIdx.x;
   const long long w_step = PAIR ? gridDim.x / 2 : gridDim.x;
   auto item = [&](long long w) -> Item {
-    Item it = resolve_item<GROUPED, PAIR ? 2 * BM : BM>(p, w);
+    Item it = resolve_item<GROUPED, PAIR ? 2 * BM : BM>(p, w, gtable ? s_goff : nullptr, gtable ? s_gtile : nullptr);
     if constexpr (PAIR) it.row0 += (int)rank * BM;  // this CTA's half of the 256-row tile
     return it;
   };
@@ -300,6 +359,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::tmem_alloc_pair(tmem_slot, tmem_cols);
     else
       tc::tmem_alloc(tmem_slot, tmem_cols);
+  }
+  if constexpr (GROUPED) {
+    if (warp == 2 && gtable) build_group_table<PAIR ? 2 * BM : BM>(p, lane, s_goff, s_gtile);
   }
   tc::tc_fence_before();
   if constexpr (PAIR)
@@ -640,9 +702,11 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
 // ring of A (128 rows) and this CTA's B rows (bn, or bn / 2 for a CTA pair)
 // per sub-block + 1 KB alignment slack + barriers and flags (256 B) + four
 // fp32 bias copies of the bn-column tile + the gathered-A row table (512 B)
+// + the grouped segment tables
 inline size_t smem_bytes(int bn, int stages, int ksub, bool pair = false) {
   const size_t b_rows = pair ? (size_t)bn / 2 : (size_t)bn;
-  return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4 + BM * 4;
+  return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4 + BM * 4 +
+         kGroupTableBytes;
 }
 
 template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
