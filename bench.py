@@ -62,6 +62,8 @@ def parse():
     ap.add_argument("--ops", default=None,
                     help="other workloads to search and report ('' = none; default: all others for mlp)")
     ap.add_argument("--op-samples", type=int, default=600, help="schedules measured per extra op")
+    ap.add_argument("--moe-samples", type=int, default=1000,
+                    help="schedules measured for the MoE layer when it is an extra op (three stages of knobs)")
     ap.add_argument("--restarts", type=int, default=2,
                     help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
     ap.add_argument("--seed", type=int, default=0)
@@ -390,7 +392,7 @@ def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, s
     return search, best, m, n, (n / t if t else None)
 
 
-def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1):
+def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None):
     """Search each other workload briefly and report its best schedule."""
     import torch
 
@@ -399,7 +401,8 @@ def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False,
     for name in names:
         wl = Workload(name)
         io = wl.device_io()
-        _, best, _, n, cps = search_best(wl.op, io, samples, branching=branching, restarts=restarts,
+        n_s = moe_samples if (name == "moe" and moe_samples) else samples
+        _, best, _, n, cps = search_best(wl.op, io, n_s, branching=branching, restarts=restarts,
                                          surrogate=surrogate, screen=screen)
         m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
         if m.status != rc.OK:
@@ -568,7 +571,7 @@ def run_ours(args):
             del io
             torch.cuda.empty_cache()
             out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"], args.branching, args.restarts,
-                                   bool(args.surrogate), args.screen)
+                                   bool(args.surrogate), args.screen, args.moe_samples)
         if args.cpu_sample >= 0:
             cb = wl.cpu_sample(args.cpu_sample)
             cb.pop("seconds", None)

@@ -138,3 +138,18 @@ def test_moe_full_size_sampled_tokens():
         np.testing.assert_array_equal(go.cpu().numpy(), off)
         np.testing.assert_array_equal(gp.cpu().numpy(), perm)
         assert rel_err(from_dev_bf16(out)[tok], ref) <= TOL, str(s)
+
+
+def test_moe_layer_256_experts():
+    # the most segments a grouped GEMM takes (each CTA holds the segment table in shared memory,
+    # eight segments per lane of the building warp); most experts get no or one row
+    T, H, E, I, K = 96, 128, 256, 64, 6
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=44)
+    ids, w, off, _ = oracle.moe_route(logits, K)
+    ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
+    op = moe_op(T, H, E, I, K)
+    for tm, fuse in itertools.product((128, 256), (0, 1)):
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(moe_sched(op, 8, 64, 2, 128, 2, fuse, tile_m=tm), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.check()
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (tm, fuse)
