@@ -62,7 +62,7 @@ def parse():
     ap.add_argument("--ops", default=None,
                     help="other workloads to search and report ('' = none; default: all others for mlp)")
     ap.add_argument("--op-samples", type=int, default=600, help="schedules measured per extra op")
-    ap.add_argument("--moe-samples", type=int, default=1000,
+    ap.add_argument("--moe-samples", type=int, default=2000,
                     help="schedules measured for the MoE layer when it is an extra op (three stages of knobs)")
     ap.add_argument("--restarts", type=int, default=2,
                     help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
@@ -72,6 +72,10 @@ def parse():
                          "nodes measured; 0 = rollout programs measured too")
     ap.add_argument("--screen", type=int, default=4,
                     help="with --surrogate 1: proposals screened by f-hat per kept child (1 = no screening)")
+    ap.add_argument("--study", default="",
+                    help="instead of the benchmark line: 'search' prints best-so-far curves (JSON lines) of the "
+                         "search variants on --workload: MCTS with measured rollouts at B = 2 and 4, MCTS with the "
+                         "learned surrogate and 4x screening, and random search, over seeds --seed .. --seed+1")
     ap.add_argument("--shape", default="",
                     help="override workload sizes for a profiling case, e.g. 'tokens=1024,experts=16' (the line "
                          "then reports that shape, not the benchmark configuration)")
@@ -392,6 +396,73 @@ def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, s
     return search, best, m, n, (n / t if t else None)
 
 
+def random_search(op, io, samples, seed, horizon=8, batch=8):
+    """Uniform random search: each candidate is P0 after up to `horizon` random legal transformations."""
+    import random
+
+    from paper_2506_01374_gb300 import rc
+    rng = random.Random(seed)
+    space = op.transform_space()
+    seen, n, curve, best = set(), 0, [], float("inf")
+    while n < samples:
+        cands = []
+        for _ in range(64 * batch):
+            if len(cands) == batch:
+                break
+            s = op.schedule()
+            for _ in range(rng.randint(1, horizon)):
+                try:
+                    s = op.schedule(rng.choice(space), base=s)
+                except rc.RcError:
+                    pass
+            key = str(s)
+            if key not in seen:
+                seen.add(key)
+                cands.append(s)
+        if not cands:
+            break
+        for m in op.measure(cands, io, warmup=2, repeats=5):
+            n += 1
+            if m.status == rc.OK:
+                best = min(best, m.ms_median)
+            curve.append((n, best))
+    return curve
+
+
+def search_study(wl, io, samples, seed):
+    """Best-so-far (TFLOP/s of the best measured candidate) against measured samples, per search variant."""
+    from paper_2506_01374_gb300 import rc
+    flops = wl.op.info["flops"]
+    marks = [m for m in (50, 100, 250, 500, 1000, 2000, 3000, 5000, 10000) if m <= samples] + [samples]
+    variants = [("mcts_B2_measured", 2, False, 1), ("mcts_B4_measured", 4, False, 1),
+                ("mcts_B4_surrogate_screen4", 4, True, 4), ("random", 0, False, 1)]
+    for sd in (seed, seed + 1):
+        for name, B, sur, scr in variants:
+            t0 = time.perf_counter()
+            if name == "random":
+                curve = random_search(wl.op, io, samples, sd)
+            else:
+                search = rc.Search(wl.op, seed=sd, branching=B, surrogate=sur, screen=scr)
+                res, n, curve, best = [], 0, [], float("inf")
+                while n < samples:
+                    nxt = search.step(res)
+                    if not nxt:
+                        break
+                    res = wl.op.measure(nxt, io, warmup=2, repeats=5)
+                    for m in res:
+                        n += 1
+                        if m.status == rc.OK:
+                            best = min(best, m.ms_median)
+                        curve.append((n, best))
+            pts = []
+            for mk in marks:
+                b = min((c[1] for c in curve if c[0] <= mk), default=float("inf"))
+                pts.append([mk, round(flops / (b * 1e-3) / 1e12, 1) if b < float("inf") else None])
+            print(json.dumps({"study": "search", "workload": wl.label, "variant": name, "seed": sd,
+                              "samples": len(curve), "seconds": round(time.perf_counter() - t0, 1),
+                              "best_tflops_at_samples": pts}), flush=True)
+
+
 def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None):
     """Search each other workload briefly and report its best schedule."""
     import torch
@@ -473,6 +544,11 @@ def run_ours(args):
     stream = torch.cuda.current_stream()
 
     wl = Workload(args.workload, parse_shape(args.shape))
+    if args.study == "search":
+        search_study(wl, wl.device_io(), args.samples, args.seed)
+        return
+    if args.study:
+        raise SystemExit(f"unknown --study {args.study}")
     if args.shape:
         wl.label += "_shape_" + args.shape.replace("=", "").replace(",", "_")
         wl.config.update(parse_shape(args.shape))
