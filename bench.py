@@ -48,7 +48,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="mlp", choices=["mlp", "attention", "conv2d", "moe", "gemm_f32"])
+    ap.add_argument("--workload", default="mlp",
+                    choices=["mlp", "attention", "conv2d", "moe", "gemm_f32", "attention_flux"])
     ap.add_argument("--samples", type=int, default=5000, help="schedules the search measures")
     ap.add_argument("--branching", type=int, default=4,
                     help="MCTS children per expansion (the paper's 2 assumes LLM-proposed transformations; with "
@@ -186,6 +187,21 @@ class Workload:
             self.dom_name = "fused attention kernel"
             self.bound = "tensor"
             self.dtype = "bf16"
+        elif name == "attention_flux":
+            # FLUX-style (DiT) self-attention: non-causal, multi-head, 64 x 64 image tokens
+            B, S, Hq = dims(batch=1, seq=4096, heads=24)
+            Hkv, D = Hq, 128
+            Q, K, V = inputs.attention(B, S, Hq, Hkv, D, seed=7)
+            self.op = rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=0)
+            self.host = [Q, K, V, None, None]
+            self.outs = {3: ((B, S, Hq, D), np.uint16), 4: ((B, Hq, S), np.float32)}
+            self.label = f"flux_attention_B{B}_S{S}_H{Hq}_d128_noncausal_bf16"
+            self.config = {"batch": B, "seq": S, "heads": Hq, "head_dim": D, "causal": False}
+            self.metric = "best-schedule TFLOP/s (non-causal MHA attention, bf16)"
+            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_name = "fused attention kernel"
+            self.bound = "tensor"
+            self.dtype = "bf16"
         elif name == "conv2d":
             N, H, W, C = dims(n=2, h=64, w=64, c=320)
             x, w, b = inputs.conv2d(N, H, W, C, C, seed=5)
@@ -280,15 +296,16 @@ class Workload:
             dt = time.perf_counter() - t0
             flops = 6.0 * n * X.shape[1] * (W1.shape[0] // 2)
             what, used = f"{n} of {X.shape[0]} token rows of the MLP block", min(cores, n)
-        elif self.name == "attention":
+        elif self.name in ("attention", "attention_flux"):
             Q, K, V = self.host[:3]
             S = Q.shape[1]
+            causal = self.name == "attention"
             n = n or 256
             qpos = np.linspace(0, S - 1, n).astype(np.int64)
             t0 = time.perf_counter()
-            oracle.attention_bf16(Q, K, V, causal=True, qpos=qpos)
+            oracle.attention_bf16(Q, K, V, causal=causal, qpos=qpos)
             dt = time.perf_counter() - t0
-            flops = float(sum(4.0 * Q.shape[3] * Q.shape[2] * (int(i) + 1) for i in qpos))
+            flops = float(sum(4.0 * Q.shape[3] * Q.shape[2] * ((int(i) + 1) if causal else S) for i in qpos))
             what, used = f"{n} of {S} query positions (all heads)", min(cores, n)
         elif self.name == "conv2d":
             x, w, b = self.host[:3]
@@ -501,7 +518,7 @@ def run_reference(args):
         return
     wl = Workload(args.workload)
     n = args.cpu_sample if args.cpu_sample > 0 else {"mlp": 16, "attention": 32, "conv2d": 512, "moe": 4,
-                                                     "gemm_f32": 4}[args.workload]
+                                                     "gemm_f32": 4, "attention_flux": 16}[args.workload]
     for _ in range(args.warmup):
         wl.cpu_sample(n)
     samples = [wl.cpu_sample(n) for _ in range(args.steps)]
@@ -521,13 +538,14 @@ def launches_per_step(workload, s):
     k = [s.knobs(i) for i in range(s.num_stages)]
     if workload == "mlp":
         return (1 if k[0]["fuse"] else 2) + (1 if k[1]["split_k"] == 1 else 2)
-    if workload == "attention":
+    if workload in ("attention", "attention_flux"):
         return 1 + (1 if k[0]["layout"] == 1 else 0)
     if workload == "conv2d":
         return 1 + (1 if k[0]["split_k"] > 1 else 0) + (1 if (k[0]["split_k"] > 1 or not k[0]["fuse"]) else 0)
     if workload == "moe":
-        # routing (3 kernels), gather, grouped gate/up, grouped down, combine (or memset + convert)
-        return 3 + 1 + 1 + 1 + 1
+        # routing (3 kernels), gather (unless the gate/up producer gathers), grouped gate/up, grouped
+        # down, combine (or, with the atomic combine, the fp32 -> bf16 conversion; the memset is not ours)
+        return 3 + (0 if k[1]["location"] == 1 else 1) + 1 + 1 + 1
     return 1
 
 
@@ -641,7 +659,7 @@ def run_ours(args):
             "clocks": clk,
         }
         others = args.ops if args.ops is not None else (
-            "gemm_f32,conv2d,attention,moe" if args.workload == "mlp" else "")
+            "gemm_f32,conv2d,attention,attention_flux,moe" if args.workload == "mlp" else "")
         names = [x for x in others.split(",") if x and x != args.workload]
         if names:
             del io

@@ -93,3 +93,18 @@ def test_attention_full_size_sampled_queries():
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
+
+
+def test_flux_shaped_noncausal_attention_sampled_queries():
+    # FLUX-style (DiT) self-attention: batch 1, 4096 image tokens, 24 heads (MHA), d = 128, no mask.
+    B, S, H = 1, 4096, 24
+    Q, K, V = inputs.attention(B, S, H, H, 128, seed=7)
+    qpos = np.array([0, 1, 127, 128, 2047, 2048, 4000, 4095], dtype=np.int64)
+    O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=False, qpos=qpos)
+    op = att_op(B, S, H, H, causal=False)
+    for s in [op.schedule(), sched(op, 128, 2, 1, 0, 256, 1, 1, 1), sched(op, 64, 2, 1, 0, 256, 1, 1, 1),
+              sched(op, 64, 2, 0, 0, 128, 1, 1, 1), sched(op, 64, 3, 1, 1, 128, 1, 1, 1),
+              sched(op, 128, 2, 1, 0, 128, 1, 2, 1)]:
+        O, L = run(op, s, Q, K, V)
+        assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
+        assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
