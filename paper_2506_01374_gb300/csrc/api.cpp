@@ -344,7 +344,7 @@ std::vector<SlotInfo> rc_slots(const rc_op_s* op) {
     case RC_OP_MLP:
       s = {{b2 * d.m * d.k, true, false, false},
            {b2 * 2 * d.n * d.k, true, false, false},
-           {b2 * d.k * d.n, true, false, false},
+           {b2 * d.k * d.n, true, false, false, 1},  // W2: read by the down projection only
            {b2 * d.m * d.k, false, true, false}};
       break;
     case RC_OP_ATTENTION: {
@@ -378,8 +378,8 @@ std::vector<SlotInfo> rc_slots(const rc_op_s* op) {
       const size_t tk = (size_t)d.tokens * d.top_k;
       s = {{lg, true, false, false},
            {b2 * d.tokens * d.hidden, true, false, false},
-           {b2 * d.experts * 2 * d.inter * d.hidden, true, false, false},
-           {b2 * d.experts * d.hidden * d.inter, true, false, false},
+           {b2 * d.experts * 2 * d.inter * d.hidden, true, false, false, 1},  // W1: grouped gate/up
+           {b2 * d.experts * d.hidden * d.inter, true, false, false, 2},      // W2: grouped down
            {b2 * d.tokens * d.hidden, false, true, false},
            {b4 * tk, false, true, true},
            {b4 * tk, false, true, true},

@@ -43,6 +43,11 @@ struct rc_op_s {
   mutable size_t ws_bytes = 0;
   mutable void* stage_buf[RC_MAX_TENSORS] = {};
   mutable size_t stage_bytes[RC_MAX_TENSORS] = {};
+  // rc_run_host: a copy stream for inputs of later stages, and per stage an
+  // event recorded when that stage's inputs have landed
+  mutable void* copy_stream = nullptr;
+  mutable void* input_ready[RC_MAX_STAGES] = {};
+  mutable void* first_inputs_done = nullptr;
   mutable int* d_status = nullptr;
   mutable int device = -1;
 };
@@ -73,6 +78,7 @@ struct SlotInfo {
   bool input;
   bool output;
   bool optional;
+  int first_stage = 0;  // inputs: the first stage of the op that reads the slot
 };
 std::vector<SlotInfo> rc_slots(const rc_op_s* op);
 
@@ -90,8 +96,13 @@ struct LaunchCtx {
   void** stage_events = nullptr;
   int n_stage_events = 0;
   mutable int next_event = 0;
+  // optional (rc_run_host): before stage i > 0 runs, the stream waits on
+  // stage_inputs[i] (NULL = nothing to wait for)
+  void* const* stage_inputs = nullptr;
+  mutable int stages_done = 0;
 };
-// Record the next stage marker on the stream, if markers were requested.
+// End of a stage: record the next stage marker, if markers were requested, and
+// make the stream wait for the next stage's inputs, if given.
 rc_status rc_mark_stage(const LaunchCtx& c);
 
 rc_status rc_launch_gemm_f32(const rc_knobs& k, int64_t M, int64_t N, int64_t K, const float* A,

@@ -300,6 +300,10 @@ extern "C" void rc_op_destroy(rc_op* op) {
   for (int i = 0; i < RC_MAX_TENSORS; ++i)
     if (op->stage_buf[i]) cudaFree(op->stage_buf[i]);
   if (op->d_status) cudaFree(op->d_status);
+  for (int i = 0; i < RC_MAX_STAGES; ++i)
+    if (op->input_ready[i]) cudaEventDestroy((cudaEvent_t)op->input_ready[i]);
+  if (op->first_inputs_done) cudaEventDestroy((cudaEvent_t)op->first_inputs_done);
+  if (op->copy_stream) cudaStreamDestroy((cudaStream_t)op->copy_stream);
   delete op;
 }
 
@@ -312,9 +316,14 @@ extern "C" rc_status rc_run(const rc_op* op, const rc_schedule* s, const rc_tens
 }
 
 rc_status rc_mark_stage(const LaunchCtx& c) {
-  if (!c.stage_events || c.next_event >= c.n_stage_events) return RC_OK;
-  return cuda_err(cudaEventRecord((cudaEvent_t)c.stage_events[c.next_event++], (cudaStream_t)c.stream),
-                  "cudaEventRecord(stage)");
+  const int done = ++c.stages_done;
+  if (c.stage_events && c.next_event < c.n_stage_events)
+    RC_TRY(cuda_err(cudaEventRecord((cudaEvent_t)c.stage_events[c.next_event++], (cudaStream_t)c.stream),
+                    "cudaEventRecord(stage)"));
+  if (c.stage_inputs && done < RC_MAX_STAGES && c.stage_inputs[done])
+    RC_TRY(cuda_err(cudaStreamWaitEvent((cudaStream_t)c.stream, (cudaEvent_t)c.stage_inputs[done], 0),
+                    "cudaStreamWaitEvent(stage inputs)"));
+  return RC_OK;
 }
 
 extern "C" rc_status rc_run_profiled(const rc_op* op, const rc_schedule* s, const rc_tensors* io, void* stream,
@@ -368,6 +377,22 @@ extern "C" rc_status rc_run_host(const rc_op* op, const rc_schedule* s, const rc
   rc_tensors dev;
   memset(&dev, 0, sizeof dev);
   cudaStream_t st = (cudaStream_t)stream;
+  // Inputs first read by a later stage are copied on a second stream after
+  // the first stage's inputs, so that their copy overlaps the earlier stages
+  // (the copy engines are shared: issuing them in parallel would only delay
+  // the first stage). Stage i waits for its inputs at the end of stage i - 1.
+  bool later = false;
+  for (size_t i = 0; i < slots.size(); ++i) later = later || (slots[i].input && slots[i].first_stage > 0);
+  if (later && !op->copy_stream) {
+    cudaStream_t cs = nullptr;
+    RC_TRY(cuda_err(cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking), "cudaStreamCreate(copies)"));
+    op->copy_stream = cs;
+    for (int i = 0; i < RC_MAX_STAGES; ++i)
+      RC_TRY(cuda_err(cudaEventCreateWithFlags((cudaEvent_t*)&op->input_ready[i], cudaEventDisableTiming),
+                      "cudaEventCreate(inputs)"));
+    RC_TRY(cuda_err(cudaEventCreateWithFlags((cudaEvent_t*)&op->first_inputs_done, cudaEventDisableTiming),
+                    "cudaEventCreate(inputs)"));
+  }
   for (size_t i = 0; i < slots.size(); ++i) {
     if (!host_io->p[i]) {
       if (slots[i].optional) continue;
@@ -381,10 +406,35 @@ extern "C" rc_status rc_run_host(const rc_op* op, const rc_schedule* s, const rc
       op->stage_bytes[i] = slots[i].bytes;
     }
     dev.p[i] = op->stage_buf[i];
-    if (slots[i].input && slots[i].bytes)
+    if (slots[i].input && slots[i].bytes && slots[i].first_stage == 0)
       RC_TRY(cuda_err(cudaMemcpyAsync(dev.p[i], host_io->p[i], slots[i].bytes, cudaMemcpyHostToDevice, st), "H2D"));
   }
-  RC_TRY(run_impl(op, s, &dev, c));
+  void* waits[RC_MAX_STAGES] = {};
+  if (later) {
+    cudaStream_t cs = (cudaStream_t)op->copy_stream;
+    RC_TRY(cuda_err(cudaEventRecord((cudaEvent_t)op->first_inputs_done, st), "cudaEventRecord(inputs)"));
+    RC_TRY(cuda_err(cudaStreamWaitEvent(cs, (cudaEvent_t)op->first_inputs_done, 0), "cudaStreamWaitEvent(inputs)"));
+    for (int g = 1; g < RC_MAX_STAGES; ++g) {
+      bool any = false;
+      for (size_t i = 0; i < slots.size(); ++i) {
+        if (!(slots[i].input && slots[i].first_stage == g && dev.p[i] && slots[i].bytes)) continue;
+        RC_TRY(cuda_err(cudaMemcpyAsync(dev.p[i], host_io->p[i], slots[i].bytes, cudaMemcpyHostToDevice, cs), "H2D"));
+        any = true;
+      }
+      if (any) {
+        RC_TRY(cuda_err(cudaEventRecord((cudaEvent_t)op->input_ready[g], cs), "cudaEventRecord(inputs)"));
+        waits[g] = op->input_ready[g];
+      }
+    }
+  }
+  c.stage_inputs = waits;
+  rc_status rs = run_impl(op, s, &dev, c);
+  // a stage whose inputs were never waited for (an error before it) must not outlive the call
+  if (rs != RC_OK) {  // no copy into the caller's buffers may outlive the call
+    if (op->copy_stream) cudaStreamSynchronize((cudaStream_t)op->copy_stream);
+    cudaStreamSynchronize(st);
+    return rs;
+  }
   for (size_t i = 0; i < slots.size(); ++i)
     if (slots[i].output && dev.p[i] && slots[i].bytes)
       RC_TRY(cuda_err(cudaMemcpyAsync(host_io->p[i], dev.p[i], slots[i].bytes, cudaMemcpyDeviceToHost, st), "D2H"));

@@ -153,3 +153,20 @@ def test_moe_layer_256_experts():
         op.run(moe_sched(op, 8, 64, 2, 128, 2, fuse, tile_m=tm), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
         assert rel_err(from_dev_bf16(out), ref) <= TOL, (tm, fuse)
+
+
+def test_moe_host_path_matches_device_path():
+    # rc_run_host copies W1 and W2 on a second stream while routing and the gate/up stage run;
+    # the result must equal the device-buffer run bit for bit
+    T, H, E, I, K = 256, 128, 8, 64, 2
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=45)
+    op = moe_op(T, H, E, I, K)
+    s = moe_sched(op, 8, 64, 2, 128, 2, 0)
+    Yh = np.zeros((T, H), np.uint16)
+    op.run_host(s, [logits, X, W1, W2, Yh])
+    dY = empty_bf16(T, H)
+    op.run(s, [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), dY])
+    op.check()
+    np.testing.assert_array_equal(Yh, dY.cpu().numpy().view(np.uint16))
+    ids, w, _, _ = oracle.moe_route(logits, K)
+    assert rel_err(inputs.bf16_bits_to_f64(Yh), oracle.moe_ffn_bf16(X, W1, W2, ids, w)) <= TOL
