@@ -150,7 +150,9 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256 = two query tiles, ping-pong softmax
       v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});
       v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 5}, {}});
-      v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1}});
+      // 0 = head-major tiles, 1 = longest causal rows first, 2 = persistent CTAs walking the
+      // longest-first tiles in a zigzag (one-tile split-issue kernel)
+      v.push_back({RC_T_LOOP_ORDER, 0, {0, 1, 2}, {1}});
       v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // V as [keys][d] or transposed to [d][keys]
       v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});  // P stored in shared or tensor memory
       v.push_back({RC_T_UNROLL, 0, {1, 2}, {}});  // key blocks in flight per query tile
@@ -291,6 +293,11 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
       if (k.unroll == 2 && !one_tile_split && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
         // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
         if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
+        return false;
+      }
+      if (k.raster == 2 && !(one_tile_split && k.location == 1 && k.tile_n == 64 && k.unroll == 1 &&
+                             k.stages >= 2 && k.stages <= 3)) {
+        if (why) *why = "persistent tiles (loop order 2) need the one-tile split-issue kernel: BN 64, unroll 1, 2-3 stages";
         return false;
       }
       if (k.persistent == 1 && !(k.location == 1 && (k.unroll == 1 || one_tile_split) && k.stages >= 2)) {

@@ -1206,11 +1206,14 @@ constexpr int kThreads4 = 256;
 
 template <int BN, int NSB>
 // NSB S buffers at TMEM columns s_col + b * BN (block j in buffer j % NSB),
-// O at o_col, P at p_col.
+// O at o_col, P at p_col. g0: key blocks this CTA's softmax processed in
+// earlier work items (persistent kernels; the barriers' phases run on across
+// items). o_free (persistent kernels): arrived on once O has been read out.
 __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, int q0, int nkb, int b, int h,
                                             uint32_t tmem, uint32_t s_col, uint32_t o_col, uint32_t p_col,
                                             uint64_t* s_full, uint64_t* s_free, uint64_t* p_full, uint64_t* pv_full,
-                                            volatile int* abort_flag, volatile int* status) {
+                                            volatile int* abort_flag, volatile int* status, int g0 = 0,
+                                            uint64_t* o_free = nullptr) {
   auto fail = [&](int code) {
     *abort_flag = 1;
     tc::record_failure(status, code);
@@ -1224,8 +1227,8 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
   // pv_full completes once per key block (P_j V_j done); its phases are
   // observed one by one, in order, never more than one behind: phase j - 1
   // in iteration j (before an O rescale, else before P_j overwrites P_{j-1}),
-  // the last one before the output.
-  int pv_seen = 0;
+  // the last one before the output. Indices are global (g0 + j).
+  int pv_seen = g0;
   auto await_pv = [&](int upto) -> bool {
     if (pv_seen > upto) return true;
     for (; pv_seen <= upto; ++pv_seen)
@@ -1238,9 +1241,10 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
   };
   bool ok = true;
   for (int j = 0; j < nkb; ++j) {
-    const int sb = j % NSB;
+    const int gj = g0 + j;
+    const int sb = gj % NSB;
     const uint32_t tS = tmem + lane_base + s_col + (uint32_t)(sb * BN);
-    if (!tc::mbar_wait(&s_full[sb], (uint32_t)(j / NSB) & 1u, abort_flag, status)) {
+    if (!tc::mbar_wait(&s_full[sb], (uint32_t)(gj / NSB) & 1u, abort_flag, status)) {
       if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
       ok = false;
       break;
@@ -1269,7 +1273,7 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
       m_ref = mxs;
     }
     if (__any_sync(0xffffffffu, factor != 1.f)) {
-      if (!await_pv(j - 1)) {  // O holds P_{j-1} V_{j-1}
+      if (!await_pv(gj - 1)) {  // O holds P_{j-1} V_{j-1}
         ok = false;
         break;
       }
@@ -1290,7 +1294,7 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
     uint32_t pk[BN / 2];
     exp_pack<BN>(r, sc2, nm2, pk, ls2);
     l = l * factor + sum_pairs(ls2);
-    if (!await_pv(j - 1)) {  // P_{j-1} V_{j-1} has read the P buffer
+    if (!await_pv(gj - 1)) {  // P_{j-1} V_{j-1} has read the P buffer
       ok = false;
       break;
     }
@@ -1301,12 +1305,16 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
     tc::mbar_arrive(p_full);
   }
   if (ok && nkb > 0) {
-    if (await_pv(nkb - 1)) {
+    if (await_pv(g0 + nkb - 1)) {
       const float inv_l = l > 0.f ? 1.f / l : 0.f;
       const bool row_ok = qi < p.S;
       __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
       store_o_row(tO, inv_l, orow, row_ok);
       if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
+      if (o_free) {  // O has been read: the next item's first P V may overwrite it
+        tc::tc_fence_before();
+        tc::mbar_arrive(o_free);
+      }
     }
   }
 }
@@ -1562,6 +1570,293 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
   } else {
     softmax_sdb<BN, NSB>(p, warp & 3, lane, q0, nkb, b, h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full, pv_full,
                          abort_flag, status);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// Persistent form of the one-tile, one-S-buffer kernel with 64-key blocks
+// (Loop order 2). Two CTAs per SM stay resident and walk the query tiles,
+// ordered longest first, in a zigzag over the CTAs (CTA c takes tiles c,
+// 2G - 1 - c, 2G + c, ... of G CTAs), which pairs long causal tiles with
+// short ones. TMEM, barriers and tensor maps are set up once; the K and V
+// rings run on across tiles, so the next tile's keys stream in while the
+// current one finishes; the next Q is loaded as soon as the current tile's
+// last S UMMA has read Q (q_empty), and the next tile's first P V waits until
+// the softmax warps have read O out (o_free). Every barrier's phase counts
+// key blocks (or tiles) over the whole run of the CTA.
+__host__ __device__ constexpr size_t attn4p_bar_bytes(int stages, int vstages) {
+  return (size_t)(11 + 2 * stages + 2 * vstages) * 8 + 8;
+}
+size_t attn4p_smem(int stages) {
+  const int vst = attn4_vstages<64, 1>(stages);
+  return (size_t)BM * D * 2 + (size_t)(stages + vst) * 64 * D * 2 + attn4p_bar_bytes(stages, vst);
+}
+
+template <bool VT>
+__global__ void __launch_bounds__(kThreads4, 2)
+    attn4p_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                  const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  constexpr int BN = 64;
+  constexpr int Q_BYTES = BM * D * 2;
+  constexpr int KV_TILE = BN * D * 2;
+  constexpr uint32_t O_COL = Attn4Cols<BN, 1>::O, P_COL = Attn4Cols<BN, 1>::P;
+  constexpr uint32_t TMEM_COLS = Attn4Cols<BN, 1>::ALLOC;
+  static_assert(TMEM_COLS == 256, "two CTAs per SM");
+
+  extern __shared__ uint8_t smem_raw[];
+  if (tc::smem_u32(smem_raw) & 1023u) {  // operands packed without alignment slack
+    if (threadIdx.x == 0) tc::record_failure(p.status, RC_DEV_MISALIGNED);
+    return;
+  }
+  uint8_t* smem = smem_raw;
+  const int vstages = attn4_vstages<BN, 1>(stages);
+  uint8_t* sQ = smem;
+  uint8_t* kring = smem + Q_BYTES;
+  uint8_t* vring = kring + (size_t)stages * KV_TILE;
+  uint64_t* q_full = (uint64_t*)(vring + (size_t)vstages * KV_TILE);
+  uint64_t* q_empty = q_full + 1;
+  uint64_t* k_full = q_empty + 1;  // [stages]
+  uint64_t* k_empty = k_full + stages;
+  uint64_t* v_full = k_empty + stages;  // [vstages]
+  uint64_t* v_empty = v_full + vstages;
+  uint64_t* s_full = v_empty + vstages;
+  uint64_t* s_free = s_full + 1;
+  uint64_t* p_full = s_free + 1;
+  uint64_t* pv_full = p_full + 1;
+  uint64_t* o_free = pv_full + 1;
+  uint64_t* drain = o_free + 1;  // [2]
+  uint32_t* tmem_slot = (uint32_t*)(drain + 2);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int BH = p.B * p.Hq;
+  const int n_tiles = p.q_blocks * BH;
+  const int G = gridDim.x, c = blockIdx.x;
+  // k-th work item of this CTA: a query tile in longest-first order, zigzag over the CTAs
+  struct Work {
+    bool valid;
+    int q0, nkb, b, h, g;
+  };
+  auto work = [&](int k) -> Work {
+    Work w;
+    const long long t = (long long)k * G + ((k & 1) ? G - 1 - c : c);
+    w.valid = t < n_tiles;
+    if (!w.valid) return w;
+    const int qb = p.q_blocks - 1 - (int)(t / BH), bh = (int)(t % BH);
+    w.b = bh / p.Hq;
+    w.h = bh - w.b * p.Hq;
+    w.g = w.h / p.group;
+    w.q0 = qb * BM;
+    const int kv_end = p.causal ? min(w.q0 + BM, p.S) : p.S;
+    w.nkb = (kv_end + BN - 1) / BN;
+    return w;
+  };
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    tc::mbar_init(q_empty, 1);
+    for (int s = 0; s < stages; ++s) {
+      tc::mbar_init(&k_full[s], 1);
+      tc::mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < vstages; ++s) {
+      tc::mbar_init(&v_full[s], 1);
+      tc::mbar_init(&v_empty[s], 1);
+    }
+    tc::mbar_init(s_full, 1);
+    tc::mbar_init(s_free, 128);
+    tc::mbar_init(p_full, 128);
+    tc::mbar_init(pv_full, 1);
+    tc::mbar_init(o_free, 128);
+    tc::mbar_init(&drain[0], 1);
+    tc::mbar_init(&drain[1], 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // a ring of `depth` slots filled for blocks g = g0 .. g0 + n - 1 of the run
+  auto produce = [&](uint64_t* full, uint64_t* empty, int depth, int g0, int n, auto load) -> bool {
+    for (int j = 0; j < n; ++j) {
+      const int g = g0 + j;
+      const int s = g % depth;
+      if (!tc::mbar_wait(&empty[s], ((uint32_t)(g / depth) & 1u) ^ 1u, abort_flag, status)) {
+        fail(RC_DEV_TIMEOUT_EMPTY);
+        return false;
+      }
+      tc::mbar_expect_tx(&full[s], KV_TILE);
+      load(s, j, &full[s]);
+    }
+    return true;
+  };
+  auto drain_ring = [&](uint64_t* full, int depth, int g_end) {
+    for (int g = max(0, g_end - depth); g < g_end; ++g)
+      if (!tc::mbar_wait_drain(&full[g % depth], (uint32_t)(g / depth) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      int gk = 0, items = 0;
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const Work w = work(k);
+        if (!w.valid) break;
+        if (k > 0 && !tc::mbar_wait(q_empty, (uint32_t)(k - 1) & 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          break;
+        }
+        tc::mbar_expect_tx(q_full, Q_BYTES);
+        const int qrow = w.b * p.S + w.q0;
+        tc::tma_load_2d(sQ, &tmQ, q_full, w.h * D, qrow);
+        tc::tma_load_2d(sQ + Q_BYTES / 2, &tmQ, q_full, w.h * D + 64, qrow);
+        ++items;
+        ok = produce(k_full, k_empty, stages, gk, w.nkb, [&](int s, int j, uint64_t* bar) {
+          uint8_t* sk = kring + (size_t)s * KV_TILE;
+          const int krow = w.b * p.S + j * BN;
+          tc::tma_load_2d(sk, &tmK, bar, w.g * D, krow);
+          tc::tma_load_2d(sk + BN * 128, &tmK, bar, w.g * D + 64, krow);
+        });
+        gk += w.nkb;
+      }
+      drain_ring(k_full, stages, gk);
+      if (items > 0 && !tc::mbar_wait_drain(q_full, (uint32_t)(items - 1) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+    __syncwarp();
+  } else if (warp == 3) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmV);
+      int gv = 0;
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const Work w = work(k);
+        if (!w.valid) break;
+        ok = produce(v_full, v_empty, vstages, gv, w.nkb, [&](int s, int j, uint64_t* bar) {
+          uint8_t* sv = vring + (size_t)s * KV_TILE;
+          if constexpr (VT) {
+            tc::tma_load_2d(sv, &tmV, bar, j * BN, (w.b * p.Hkv + w.g) * D);
+          } else {
+            const int krow = w.b * p.S + j * BN;
+            tc::tma_load_2d(sv, &tmV, bar, w.g * D, krow);
+            tc::tma_load_2d(sv + BN * 128, &tmV, bar, w.g * D + 64, krow);
+          }
+        });
+        gv += w.nkb;
+      }
+      drain_ring(v_full, vstages, gv);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+      const uint32_t sq = tc::smem_u32(sQ);
+      int gs = 0;
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const Work w = work(k);
+        if (!w.valid) break;
+        if (!tc::mbar_wait(q_full, (uint32_t)k & 1u, abort_flag, status)) {
+          ok = false;
+          break;
+        }
+        for (int j = 0; j < w.nkb; ++j) {
+          const int g = gs + j;
+          const int s = g % stages;
+          // the S buffer is free once the softmax holds S_{g-1} in registers
+          ok = (g == 0 || tc::mbar_wait(s_free, (uint32_t)(g - 1) & 1u, abort_flag, status)) &&
+               tc::mbar_wait(&k_full[s], (uint32_t)(g / stages) & 1u, abort_flag, status);
+          if (!ok) break;
+          tc::tc_fence_after();
+          const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const uint32_t off = (uint32_t)(ks % 4) * 32;
+            tc::umma_bf16(tmem, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
+                          tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+          }
+          tc::umma_commit(s_full);
+          tc::umma_commit(&k_empty[s]);
+        }
+        if (!ok) break;
+        tc::umma_commit(q_empty);  // Q may be replaced once this tile's S products are done
+        gs += w.nkb;
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[0]);
+        if (!tc::mbar_wait_drain(&drain[0], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 2) {
+    if (lane == 0) {
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+      const uint32_t tO = tmem + O_COL, tP = tmem + P_COL;
+      int gp = 0;
+      bool ok = true;
+      for (int k = 0; ok; ++k) {
+        const Work w = work(k);
+        if (!w.valid) break;
+        // O still holds the previous tile until its softmax warps have read it out
+        if (k > 0 && !tc::mbar_wait(o_free, (uint32_t)(k - 1) & 1u, abort_flag, status)) {
+          ok = false;
+          break;
+        }
+        for (int j = 0; j < w.nkb; ++j) {
+          const int g = gp + j;
+          const int s = g % vstages;
+          ok = tc::mbar_wait(&v_full[s], (uint32_t)(g / vstages) & 1u, abort_flag, status) &&
+               tc::mbar_wait(p_full, (uint32_t)g & 1u, abort_flag, status);
+          if (!ok) break;
+          tc::tc_fence_after();
+          const uint32_t sv = tc::smem_u32(vring + (size_t)s * KV_TILE);
+#pragma unroll
+          for (int ks = 0; ks < BN / 16; ++ks) {
+            const uint32_t off = (uint32_t)(ks % 4) * 32;
+            uint64_t db;
+            if constexpr (VT)
+              db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
+            else
+              db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
+            tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+          }
+          tc::umma_commit(pv_full);
+          tc::umma_commit(&v_empty[s]);
+        }
+        gp += w.nkb;
+      }
+      if (!ok) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(&drain[1]);
+        if (!tc::mbar_wait_drain(&drain[1], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+    }
+    __syncwarp();
+  } else {
+    int gsm = 0;
+    for (int k = 0; !*abort_flag; ++k) {
+      const Work w = work(k);
+      if (!w.valid) break;
+      softmax_sdb<BN, 1>(p, warp & 3, lane, w.q0, w.nkb, w.b, w.h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full,
+                         pv_full, abort_flag, status, gsm, o_free);
+      gsm += w.nkb;
+    }
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -1896,6 +2191,50 @@ rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const vo
   return RC_OK;
 }
 
+// Persistent one-tile kernel (Loop order 2): grid = two CTAs per SM, at most one per tile.
+template <bool VT>
+rc_status launch_persistent(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V,
+                            void* O, float* lse, const LaunchCtx& c) {
+  auto kern = attn4p_kernel<VT>;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention: smem attribute: %s", cudaGetErrorString(e));
+    attr = true;
+  }
+  const uint64_t BS = (uint64_t)d.batch * d.seq;
+  CUtensorMap tq, tk, tv;
+  RC_TRY(tcg::encode_2d(&tq, Q, (uint64_t)d.heads_q * D, BS, BM));
+  RC_TRY(tcg::encode_2d(&tk, K, (uint64_t)d.heads_kv * D, BS, 64));
+  if (VT)
+    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.seq, (uint64_t)d.batch * d.heads_kv * D, BM));
+  else
+    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.heads_kv * D, BS, 64));
+  Params p;
+  memset(&p, 0, sizeof p);
+  p.B = (int)d.batch;
+  p.S = (int)d.seq;
+  p.Hq = (int)d.heads_q;
+  p.Hkv = (int)d.heads_kv;
+  p.group = (int)(d.heads_q / d.heads_kv);
+  p.q_blocks = (int)((d.seq + BM - 1) / BM);
+  p.causal = d.causal ? 1 : 0;
+  p.scale_log2 = (float)(d.scale * 1.4426950408889634);
+  p.raster = k.raster;
+  p.O = (__nv_bfloat16*)O;
+  p.lse = lse;
+  p.status = c.status;
+  const long long tiles = (long long)p.B * p.Hq * p.q_blocks;
+  if (tiles > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: too many tiles");
+  const int sms = c.num_sms > 0 ? c.num_sms : 1;
+  const int grid = (int)std::min<long long>(tiles, 2LL * sms);
+  kern<<<grid, kThreads4, attn4p_smem(k.stages), (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention (persistent) launch: %s", cudaGetErrorString(e));
+  return RC_OK;
+}
+
 }  // namespace attn
 
 rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V,
@@ -1919,6 +2258,13 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
   if (pt && !pp && k.persistent != 1)
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: P in TMEM needs two query tiles or split UMMA issue");
   const bool par = k.persistent == 1;  // UMMA issue split over several warps
+  if (k.raster == 2) {  // persistent CTAs over longest-first tiles (one-tile kernel, one S buffer, BN 64)
+    if (!(par && pt && !pp && k.tile_n == 64 && k.unroll == 1 && k.stages >= 2 && k.stages <= 3))
+      return rc_fail(RC_ERR_ILLEGAL_SCHEDULE,
+                     "attention: loop order 2 needs one query tile, split issue, P in TMEM, BN 64, unroll 1, 2-3 stages");
+    return vt ? attn::launch_persistent<true>(k, d, Q, K, Vuse, O, lse, c)
+              : attn::launch_persistent<false>(k, d, Q, K, Vuse, O, lse, c);
+  }
   if (k.unroll == 2 && !(par && !pp)) {  // two key blocks in flight per query tile
     if (!(pp && pt && k.tile_n == 64 && k.stages >= 4) || k.persistent)
       return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: unroll 2 needs 2 query tiles, P in TMEM, BN 64, 4 stages");

@@ -46,7 +46,7 @@ def test_attention_schedule_sweep(B, S, Hq, Hkv, causal):
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=causal)
     op = att_op(B, S, Hq, Hkv, causal)
     n = 0
-    for bm, bn, st, ra, lay, pt, un, par in itertools.product((128, 256), (64, 128), (1, 2, 3, 4), (0, 1), (0, 1),
+    for bm, bn, st, ra, lay, pt, un, par in itertools.product((128, 256), (64, 128), (1, 2, 3, 4), (0, 1, 2), (0, 1),
                                                               (0, 1), (1, 2), (0, 1)):
         try:
             s = sched(op, bn, st, ra, lay, bm, pt, un, par)
@@ -89,7 +89,9 @@ def test_attention_full_size_sampled_queries():
               sched(op, 128, 3, 0, 1, 128, 1, 1, 1), sched(op, 64, 4, 1, 0, 128, 1, 1, 1),
               # one tile with split issue: one S buffer (two CTAs per SM at BN 64, stages 2) or two
               sched(op, 64, 2, 1, 0, 128, 1, 1, 1), sched(op, 64, 2, 0, 1, 128, 1, 1, 1),
-              sched(op, 64, 3, 1, 0, 128, 1, 2, 1), sched(op, 128, 2, 1, 0, 128, 1, 2, 1)]:
+              sched(op, 64, 3, 1, 0, 128, 1, 2, 1), sched(op, 128, 2, 1, 0, 128, 1, 2, 1),
+              # persistent CTAs walking longest-first tiles (loop order 2)
+              sched(op, 64, 2, 2, 0, 128, 1, 1, 1), sched(op, 64, 3, 2, 1, 128, 1, 1, 1)]:
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
@@ -104,7 +106,7 @@ def test_flux_shaped_noncausal_attention_sampled_queries():
     op = att_op(B, S, H, H, causal=False)
     for s in [op.schedule(), sched(op, 128, 2, 1, 0, 256, 1, 1, 1), sched(op, 64, 2, 1, 0, 256, 1, 1, 1),
               sched(op, 64, 2, 0, 0, 128, 1, 1, 1), sched(op, 64, 3, 1, 1, 128, 1, 1, 1),
-              sched(op, 128, 2, 1, 0, 128, 1, 2, 1)]:
+              sched(op, 128, 2, 1, 0, 128, 1, 2, 1), sched(op, 64, 3, 2, 0, 128, 1, 1, 1)]:
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
