@@ -45,7 +45,7 @@ FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mlp",
@@ -110,6 +110,15 @@ class Clocks:
                                          stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
+            return
+        # let the sampler emit its first line before the timed region starts (at most 3 s)
+        t0 = time.time()
+        while time.time() - t0 < 3.0 and self.proc.poll() is None:
+            self.f.flush()
+            if os.path.getsize(self.f.name) > 0:
+                break
+            time.sleep(0.02)
+        self.skip = sum(1 for _ in open(self.f.name))  # lines from before the timed region
 
     def stop(self):
         if self.proc is None:
@@ -121,7 +130,9 @@ class Clocks:
             self.proc.kill()
         self.f.flush()
         rows = []
-        for line in open(self.f.name):
+        for i, line in enumerate(open(self.f.name)):
+            if i < getattr(self, "skip", 0):
+                continue
             parts = [x.strip() for x in line.split(",")]
             if len(parts) >= 9:
                 rows.append(parts)
