@@ -10,12 +10,31 @@
 // Mapping: 256 threads as a 16 x 16 grid; thread (ty, tx) owns the
 // (BM/16) x (BN/16) outputs at rows ty + 16 i and columns tx + 16 j, so
 // shared-memory reads along a warp are broadcast (A) or consecutive (B).
-// Ragged M, N and K are handled by zero-filled tile loads and guarded stores.
+// Tiles stream through a ring of shared-memory stages with cp.async, so
+// several k blocks are in flight. Ragged M, N and K are handled by
+// zero-filled tile loads and guarded stores.
 #include <cuda_runtime.h>
 
 #include "rc_internal.h"
 
 namespace {
+
+// Shared-memory ring depth: as many BK-deep stages as fit in 40 KB of static
+// shared memory (at most 8), so that the global-memory latency of a k block is
+// paid once per ring rather than once per block; a single stage (synchronous
+// loads) when two do not fit.
+template <int BM, int BN, int BK>
+constexpr int k0_stages() {
+  constexpr int bytes = (BM * (BK + 1) + BK * BN) * 4;
+  constexpr int n = 40960 / bytes;
+  return n >= 8 ? 8 : n >= 2 ? n : 1;
+}
+
+// 4-byte global -> shared copy (cp.async); src_bytes = 0 zero-fills.
+__device__ __forceinline__ void cp_async4(float* dst, const float* src, uint32_t src_bytes) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(src), "r"(src_bytes) : "memory");
+}
 
 template <int BM, int BN, int BK, int UNROLL>
 __global__ void __launch_bounds__(256) gemm_f32_kernel(int M, int N, int K, const float* __restrict__ A,
@@ -23,42 +42,66 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(int M, int N, int K, cons
                                                        const float* __restrict__ bias, float* __restrict__ C,
                                                        int relu) {
   constexpr int TM = BM / 16, TN = BN / 16;
-  __shared__ float As[BK][BM + 1];  // As[k][m]: A tile transposed
-  __shared__ float Bs[BK][BN];
+  constexpr int S = k0_stages<BM, BN, BK>();
+  __shared__ float As[S][BM][BK + 1];  // As[s][m][k]
+  __shared__ float Bs[S][BK][BN];
   const int tid = threadIdx.x;
   const int tx = tid % 16, ty = tid / 16;
   const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+  const int nkb = (K + BK - 1) / BK;
   float acc[TM][TN];
 #pragma unroll
   for (int i = 0; i < TM; ++i)
 #pragma unroll
     for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
 
-  for (int k0 = 0; k0 < K; k0 += BK) {
+  // one k block into ring slot st (zero-filled outside M, N, K); consecutive threads walk along k for
+  // A and along n for B (coalesced)
+  auto load = [&](int st, int k0) {
     for (int e = tid; e < BM * BK; e += 256) {
-      const int m = e / BK, k = e % BK;  // consecutive threads walk along k (coalesced)
+      const int m = e / BK, k = e % BK;
       const int gm = m0 + m, gk = k0 + k;
-      As[k][m] = (gm < M && gk < K) ? A[(size_t)gm * K + gk] : 0.f;
+      const bool v = gm < M && gk < K;
+      cp_async4(&As[st][m][k], v ? A + (size_t)gm * K + gk : A, v ? 4u : 0u);
     }
     for (int e = tid; e < BK * BN; e += 256) {
       const int k = e / BN, n = e % BN;
       const int gk = k0 + k, gn = n0 + n;
-      Bs[k][n] = (gk < K && gn < N) ? B[(size_t)gk * N + gn] : 0.f;
+      const bool v = gk < K && gn < N;
+      cp_async4(&Bs[st][k][n], v ? B + (size_t)gk * N + gn : B, v ? 4u : 0u);
     }
+  };
+  // prologue: blocks 0 .. S - 2 (block 0 alone for a single stage)
+#pragma unroll
+  for (int st = 0; st < (S > 1 ? S - 1 : 1); ++st) {
+    if (st < nkb) load(st, st * BK);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+  for (int kb = 0; kb < nkb; ++kb) {
+    // block kb has landed (at most S - 2 younger groups pending)
+    asm volatile("cp.async.wait_group %0;" ::"n"(S > 1 ? S - 2 : 0) : "memory");
     __syncthreads();
+    // refill the slot every thread finished reading in iteration kb - 1
+    if (S > 1 && kb + S - 1 < nkb) load((kb + S - 1) % S, (kb + S - 1) * BK);
+    if (S > 1) asm volatile("cp.async.commit_group;" ::: "memory");
+    const int st = kb % S;
 #pragma unroll UNROLL
     for (int kk = 0; kk < BK; ++kk) {
       float a[TM], b[TN];
 #pragma unroll
-      for (int i = 0; i < TM; ++i) a[i] = As[kk][ty + 16 * i];
+      for (int i = 0; i < TM; ++i) a[i] = As[st][ty + 16 * i][kk];
 #pragma unroll
-      for (int j = 0; j < TN; ++j) b[j] = Bs[kk][tx + 16 * j];
+      for (int j = 0; j < TN; ++j) b[j] = Bs[st][kk][tx + 16 * j];
 #pragma unroll
       for (int i = 0; i < TM; ++i)
 #pragma unroll
         for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
     }
-    __syncthreads();
+    if (S == 1) {  // synchronous: the next block overwrites this slot
+      __syncthreads();
+      if (kb + 1 < nkb) load(0, (kb + 1) * BK);
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    }
   }
 #pragma unroll
   for (int i = 0; i < TM; ++i) {
