@@ -49,7 +49,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mlp",
-                    choices=["mlp", "attention", "conv2d", "moe", "gemm_f32", "attention_flux"])
+                    choices=["mlp", "attention", "conv2d", "moe", "gemm_f32", "attention_flux", "decoder_layer"])
     ap.add_argument("--samples", type=int, default=5000, help="schedules the search measures")
     ap.add_argument("--branching", type=int, default=4,
                     help="MCTS children per expansion (the paper's 2 assumes LLM-proposed transformations; with "
@@ -65,6 +65,13 @@ def parse():
     ap.add_argument("--op-samples", type=int, default=600, help="schedules measured per extra op")
     ap.add_argument("--moe-samples", type=int, default=2000,
                     help="schedules measured for the MoE layer when it is an extra op (three stages of knobs)")
+    ap.add_argument("--layer-samples", type=int, default=3000,
+                    help="schedules measured for the decoder layer when it is an extra op (six stages of knobs)")
+    ap.add_argument("--horizon", type=int, default=0,
+                    help="maximum transformation-sequence length T of each search (0 = the workload's: 8)")
+    ap.add_argument("--tasks", type=int, default=-1, choices=[-1, 0, 1],
+                    help="1 = tune a composite op stage by stage, then jointly (search_tasks); 0 = one joint "
+                         "search; -1 = the workload's choice (stage by stage for the decoder layer)")
     ap.add_argument("--restarts", type=int, default=2,
                     help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
     ap.add_argument("--seed", type=int, default=0)
@@ -163,6 +170,8 @@ class Workload:
 
         from paper_2506_01374_gb300 import inputs, rc
         self.name = name
+        self.horizon = 8  # search horizon T
+        self.tasks = False
         sh = dict(shape or {})
 
         def dims(**default):
@@ -238,6 +247,19 @@ class Workload:
             self.metric = "best-schedule TFLOP/s (MoE layer, 64 experts, top-8, bf16)"
             self.dom_stage, self.dom_flops = 1, 2.0 * T * K * (2 * I) * H
             self.dom_name = "grouped gate/up GEMM + SwiGLU (stage 1)"
+            self.bound = "tensor"
+            self.dtype = "bf16"
+        elif name == "decoder_layer":
+            T, H, Hq, Hkv, I = dims(tokens=2048, hidden=4096, heads_q=32, heads_kv=8, inter=14336)
+            self.host = list(inputs.decoder_layer(T, H, Hq, Hkv, I, seed=8)) + [None]
+            self.op = rc.Op(rc.OP_DECODER_LAYER, tokens=T, hidden=H, inter=I, heads_q=Hq, heads_kv=Hkv, head_dim=128)
+            self.outs = {7: ((T, H), np.uint16)}
+            self.label = f"llama3_8b_decoder_layer_T{T}_H{H}_Hq{Hq}_Hkv{Hkv}_I{I}_bf16"
+            self.config = {"tokens": T, "hidden": H, "heads_q": Hq, "heads_kv": Hkv, "inter": I}
+            self.metric = "best-schedule TFLOP/s (Llama-3-8B decoder layer, bf16)"
+            self.dom_stage, self.dom_flops = 4, 2.0 * T * (2 * I) * H
+            self.dom_name = "gate/up GEMM + SwiGLU (stage 4)"
+            self.tasks = True  # tuned stage by stage (search_tasks), then jointly
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "gemm_f32":
@@ -338,6 +360,23 @@ class Workload:
             dt = time.perf_counter() - t0
             flops = 6.0 * n * 8 * X.shape[1] * (W1.shape[1] // 2)
             what, used = f"routing of all tokens + expert FFN of {n} of {X.shape[0]} tokens", min(cores, n)
+        elif self.name == "decoder_layer":
+            from oracle import decoder
+            x = self.host[0]
+            T, H = x.shape
+            Hq, Hkv, I = self.config["heads_q"], self.config["heads_kv"], self.config["inter"]
+            n = n or 8
+            rows = np.linspace(0, T - 1, n).astype(np.int64)
+            t0 = time.perf_counter()
+            decoder.decoder_layer_bf16(*self.host[:7], Hq, Hkv, rows=rows)
+            dt = time.perf_counter() - t0
+            hq, hkv = Hq * 128, Hkv * 128
+            # the QKV projection of every token (keys and values of all positions) + the rows' own work
+            flops = 2.0 * T * H * (hq + 2 * hkv) + float(sum(4.0 * 128 * Hq * (int(r) + 1) for r in rows)) + \
+                n * (2.0 * hq * H + 6.0 * H * I)
+            what = (f"{n} of {T} token rows of the layer, fp64 (QKV projection of all {T} tokens as a numpy "
+                    "matrix product, attention and MLP of the rows as loop nests)")
+            used = cores
         else:
             A, B, bias = self.host[:3]
             n = n or 40
@@ -347,8 +386,10 @@ class Workload:
             dt = time.perf_counter() - t0
             flops = n * 2.0 * A.shape[0] * A.shape[1] * B.shape[1]
             what, used = f"{n} full 256^3 GEMMs", min(cores, A.shape[0])
+        if self.name != "decoder_layer":
+            what += ", fp64 loop nests"
         return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": used, "kind": "oracle",
-                "sample": what + ", fp64 loop nests", "seconds": dt}
+                "sample": what, "seconds": dt}
 
 
 def parse_shape(text):
@@ -366,39 +407,61 @@ def parse_schedule(op, text, rc):
               "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0), "fuse": (rc.T_FUSE, 0),
               "raster": (rc.T_LOOP_ORDER, 0), "persistent": (rc.T_PARALLEL, 0), "layout": (rc.T_LAYOUT, 0),
               "unroll": (rc.T_UNROLL, 0), "location": (rc.T_COMPUTE_LOCATION, 0)}
+    KNOB_T["loc"] = KNOB_T["location"]
+    p0 = op.schedule()
     ts = []
     for part in filter(None, text.split(";")):
+        if part.startswith("op="):  # the canonical form str(schedule) prints
+            continue
         stage_s, kvs = part.split(":")
         stage = int(stage_s.strip()[1:])
+        items = []
         for kv in filter(None, kvs.split(",")):
             k, v = kv.split("=")
-            kind, axis = KNOB_T[k.strip()]
-            if k.strip() == "raster":
+            if k.strip() == "tile":
+                items += list(zip(("tile_m", "tile_n", "tile_k"), v.split("x")))
+            elif k.strip() != "vec":
+                items.append((k.strip(), v))
+        for k, v in items:
+            if str(p0.knobs(stage).get(k if k != "loc" else "location")) == v and k != "raster":
+                continue  # P0's value (also where the knob is not tunable at this stage)
+            kind, axis = KNOB_T[k]
+            if k == "raster":
                 r, g = (v.split("/") + ["1"])[:2]
+                if p0.knobs(stage)["raster"] == int(r) and p0.knobs(stage)["group"] == int(g):
+                    continue
                 ts.append(rc.T(kind, int(r), stage=stage, group=int(g)))
             else:
                 ts.append(rc.T(kind, int(v), axis=axis, stage=stage))
     return op.schedule(*ts)
 
 
-def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, surrogate=False, screen=1):
+def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, surrogate=False, screen=1,
+                horizon=8, root=None, stages=None):
     """MCTS over op's schedule space with device-timed candidates; returns (search, best, m, n, cand/s).
 
     Candidates are timed with 5 repeats while searching; the `finalists` best
     of them are timed again with 20 repeats and the fastest is returned, so a
     noisy short measurement does not decide the result. surrogate/screen: the
     learned rollout surrogate and proposal screening of rc_search_opts.
+    root/stages: start from `root` and tune only `stages` (rc_search_opts.root
+    and stage_mask); the objective is then those stages' summed time.
     """
     from paper_2506_01374_gb300 import rc
+
+    def obj(m):
+        return sum(m.stage_ms[g] for g in stages) if stages else m.ms_median
+
     if restarts > 1:  # independent searches; rewards are noisy measurements, so trajectories differ
-        runs = [search_best(op, io, samples, seed + r, branching, finalists, 1, surrogate, screen)
-                for r in range(restarts)]
-        i = min(range(restarts), key=lambda r: runs[r][2].ms_median if runs[r][2].status == rc.OK else float("inf"))
+        runs = [search_best(op, io, samples, seed + r, branching, finalists, 1, surrogate, screen, horizon, root,
+                            stages) for r in range(restarts)]
+        i = min(range(restarts), key=lambda r: obj(runs[r][2]) if runs[r][2].status == rc.OK else float("inf"))
         search, best, m, _, _ = runs[i]
         n = sum(r[3] for r in runs)
         cps = [r[4] for r in runs if r[4]]
         return search, best, m, n, (sum(cps) / len(cps) if cps else None)
-    search = rc.Search(op, seed=seed, branching=branching, surrogate=surrogate, screen=screen)
+    search = rc.Search(op, seed=seed, branching=branching, horizon=horizon, surrogate=surrogate, screen=screen,
+                       stages=stages, root=root)
     res, n, t, pending = [], 0, 0.0, False
     seen = []  # (median ms, schedule owned by the search)
     while n < samples:
@@ -410,7 +473,7 @@ def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, s
         res = op.measure(nxt, io, warmup=2, repeats=5)
         t += time.perf_counter() - t0
         n += len(nxt)
-        seen += [(m.ms_median, s) for s, m in zip(nxt, res) if m.status == rc.OK]
+        seen += [(obj(m), s) for s, m in zip(nxt, res) if m.status == rc.OK]
         pending = True
     if pending:  # hand the last batch's measurements to the search
         search.step(res)
@@ -418,10 +481,46 @@ def search_best(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, s
     seen.sort(key=lambda x: x[0])
     cands = [best] + [sch for _, sch in seen[:finalists]]
     final = op.measure(cands, io, warmup=3, repeats=20)
-    i = min(range(len(cands)), key=lambda j: final[j].ms_median if final[j].status == rc.OK else float("inf"))
+    i = min(range(len(cands)), key=lambda j: obj(final[j]) if final[j].status == rc.OK else float("inf"))
     if i > 0:
         best, m = cands[i].clone(), final[i]
     return search, best, m, n, (n / t if t else None)
+
+
+def search_tasks(op, io, samples, seed=0, branching=4, finalists=4, restarts=1, surrogate=False, screen=1,
+                 horizon=8, joint=0.2):
+    """Task-wise tuning of a composite op, as a compiler tunes a network's subgraphs one by one.
+
+    Each stage is one task: an MCTS over that stage's transformations only, whose objective is the
+    stage's own device time, starting from the best program of the tasks before it. Stages go in
+    order of their share of P0's time and get samples in proportion (at least 32 each); the last
+    `joint` fraction of the samples is one MCTS over every stage from the composed program (with
+    `restarts`), which can still trade stages against each other (shared L2, launch gaps). Returns
+    what search_best returns, plus the per-task record.
+    """
+    from paper_2506_01374_gb300 import rc
+    root = op.schedule()
+    m0 = op.measure([root], io, warmup=2, repeats=5)[0]
+    if m0.status != rc.OK:
+        raise RuntimeError(f"P0 failed: {rc.STATUS_NAMES.get(m0.status, m0.status)}")
+    S = root.num_stages
+    share = [max(m0.stage_ms[g], 1e-9) for g in range(S)]
+    alloc = [max(32, int(samples * (1.0 - joint) * x / sum(share))) for x in share]
+    n, t, tasks = 1, 0.0, []
+    for g in sorted(range(S), key=lambda g: -share[g]):
+        # one search per task: a stage's space is small enough that restarts mostly re-measure it
+        _, best, m, k, cps = search_best(op, io, alloc[g], seed, branching, finalists, 1, surrogate, screen,
+                                         horizon, root=root, stages=[g])
+        root = best
+        tasks.append({"stage": g, "samples": k, "p0_ms": share[g], "best_ms": m.stage_ms[g]})
+        n += k
+        t += k / cps if cps else 0.0
+    search, best, m, k, cps = search_best(op, io, max(16, (samples - n) // max(1, restarts)), seed, branching,
+                                          finalists, restarts,
+                                          surrogate, screen, horizon, root=root)
+    n += k
+    t += k / cps if cps else 0.0
+    return search, best, m, n, (n / t if t else None), tasks
 
 
 def random_search(op, io, samples, seed, horizon=8, batch=8):
@@ -491,7 +590,8 @@ def search_study(wl, io, samples, seed):
                               "best_tflops_at_samples": pts}), flush=True)
 
 
-def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None):
+def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None,
+              layer_samples=None):
     """Search each other workload briefly and report its best schedule."""
     import torch
 
@@ -500,9 +600,10 @@ def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False,
     for name in names:
         wl = Workload(name)
         io = wl.device_io()
-        n_s = moe_samples if (name == "moe" and moe_samples) else samples
-        _, best, _, n, cps = search_best(wl.op, io, n_s, branching=branching, restarts=restarts,
-                                         surrogate=surrogate, screen=screen)
+        n_s = {"moe": moe_samples, "decoder_layer": layer_samples}.get(name) or samples
+        find = search_tasks if wl.tasks else search_best
+        _, best, _, n, cps = find(wl.op, io, n_s, branching=branching, restarts=restarts, surrogate=surrogate,
+                                  screen=screen, horizon=wl.horizon)[:5]
         m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
         if m.status != rc.OK:
             out[name] = {"workload": wl.label, "error": rc.STATUS_NAMES.get(m.status, m.status)}
@@ -529,7 +630,8 @@ def run_reference(args):
         return
     wl = Workload(args.workload)
     n = args.cpu_sample if args.cpu_sample > 0 else {"mlp": 16, "attention": 32, "conv2d": 512, "moe": 4,
-                                                     "gemm_f32": 4, "attention_flux": 16}[args.workload]
+                                                     "gemm_f32": 4, "attention_flux": 16,
+                                                     "decoder_layer": 8}[args.workload]
     for _ in range(args.warmup):
         wl.cpu_sample(n)
     samples = [wl.cpu_sample(n) for _ in range(args.steps)]
@@ -557,6 +659,10 @@ def launches_per_step(workload, s):
         # routing (3 kernels), gather (unless the gate/up producer gathers), grouped gate/up, grouped
         # down, combine (or, with the atomic combine, the fp32 -> bf16 conversion; the memset is not ours)
         return 3 + (0 if k[1]["location"] == 1 else 1) + 1 + 1 + 1
+    if workload == "decoder_layer":
+        # RMSNorm, QKV GEMM, RoPE, attention (+ V transpose), O GEMM, add + RMSNorm,
+        # gate/up GEMM (+ SwiGLU pass), down GEMM, residual add
+        return 2 + 1 + 1 + (1 if k[2]["layout"] == 1 else 0) + 2 + (1 if k[4]["fuse"] else 2) + 2
     return 1
 
 
@@ -587,11 +693,16 @@ def run_ours(args):
 
     # 1) schedule search, every candidate measured on the device
     n_meas, cps, best_m = 0, None, None
-    search = None
+    search, tasks = None, []
+    if args.tasks >= 0:
+        wl.tasks = bool(args.tasks)
     if args.schedule:
         best = parse_schedule(op, args.schedule, rc)
     else:
-        search, best, best_m, n_meas, cps = search_best(op, io, args.samples, seed=args.seed,
+        if args.horizon > 0:
+            wl.horizon = args.horizon
+        find = search_tasks if wl.tasks else search_best
+        search, best, best_m, n_meas, cps, *tasks = find(op, io, args.samples, seed=args.seed, horizon=wl.horizon,
                                                         branching=args.branching, restarts=args.restarts,
                                                         surrogate=bool(args.surrogate), screen=args.screen)
 
@@ -661,6 +772,7 @@ def run_ours(args):
                          "unit": "TFLOP/s", "frac": achieved / peak, "peak_source": peak_src, "traffic": None},
             "step_frac_of_peak": value / world / peak,
             "search": {"samples": n_meas, "candidates_per_s": cps, "surrogate": bool(args.surrogate),
+                       "horizon": wl.horizon, "tasks": tasks[0] if tasks else None,
                        "screen": args.screen,
                        "best_search_tflops": best_m.tflops if best_m else None,
                        "stats": search.stats() if search else None},
@@ -670,13 +782,13 @@ def run_ours(args):
             "clocks": clk,
         }
         others = args.ops if args.ops is not None else (
-            "gemm_f32,conv2d,attention,attention_flux,moe" if args.workload == "mlp" else "")
+            "gemm_f32,conv2d,attention,attention_flux,moe,decoder_layer" if args.workload == "mlp" else "")
         names = [x for x in others.split(",") if x and x != args.workload]
         if names:
             del io
             torch.cuda.empty_cache()
             out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"], args.branching, args.restarts,
-                                   bool(args.surrogate), args.screen, args.moe_samples)
+                                   bool(args.surrogate), args.screen, args.moe_samples, args.layer_samples)
         if args.cpu_sample >= 0:
             cb = wl.cpu_sample(args.cpu_sample)
             cb.pop("seconds", None)

@@ -100,7 +100,23 @@ typedef enum {
    * tensors: 0 logits, 1 X bf16[T][H], 2 W1 bf16[E][2I][H], 3 W2 bf16[E][H][I],
    *          4 out bf16[T][H]; optional outputs (NULL = library workspace):
    *          5 ids, 6 weights, 7 offsets, 8 perm (as RC_OP_MOE_ROUTE) */
-  RC_OP_MOE = 7
+  RC_OP_MOE = 7,
+  /* Pre-norm decoder layer of the Llama family (the paper's end-to-end model,
+   * Sec. 4), batch 1, T = tokens positions 0 .. T-1:
+   *   a = RMSNorm(x) g1; [q k v] = a Wqkv^T; q, k = RoPE(q, k);
+   *   o = causal GQA attention(q, k, v); h1 = x + o Wo^T;
+   *   y = h1 + W2 (silu(b Wg^T) * (b Wu^T)), b = RMSNorm(h1) g2,
+   * RMSNorm(v) = v / sqrt(mean(v^2) + norm_eps); RoPE turns the pair
+   * (j, j + D/2) of each head by p * rope_theta^(-2j/D). head_dim = 128.
+   * tokens = T, hidden = H, inter = I, heads_q, heads_kv.
+   * tensors: 0 x bf16[T][H], 1 g1 bf16[H], 2 Wqkv bf16[(Hq + 2 Hkv) D][H]
+   *          (query rows, then key rows, then value rows), 3 Wo bf16[H][Hq D],
+   *          4 g2 bf16[H], 5 W1 bf16[2I][H] (gate rows, then up rows),
+   *          6 W2 bf16[H][I], 7 y bf16[T][H].
+   * Stages: 0 RMSNorm + QKV GEMM, 1 RoPE (and the split into Q, K, V),
+   * 2 attention, 3 O GEMM + residual + RMSNorm, 4 gate/up GEMM + SwiGLU,
+   * 5 down GEMM + residual. Intermediates live in library workspace. */
+  RC_OP_DECODER_LAYER = 8
 } rc_op_kind;
 
 enum { RC_EPI_BIAS = 1, RC_EPI_RELU = 2, RC_EPI_SILU = 4 };
@@ -123,6 +139,9 @@ typedef struct {
   int64_t tokens, hidden, experts, inter, top_k;
   int32_t logits_fp32; /* 0 = bf16 logits, 1 = f32 logits */
   int32_t renorm;      /* 1 = renormalise the k weights (default reading) */
+  /* DECODER_LAYER */
+  double rope_theta;   /* 0 = 500000 (Llama 3) */
+  double norm_eps;     /* 0 = 1e-5 */
 } rc_op_desc;
 
 typedef enum { RC_BOUND_TENSOR = 0, RC_BOUND_HBM = 1, RC_BOUND_FP32_SIMT = 2 } rc_bound;
@@ -202,7 +221,7 @@ typedef struct {
  * step or the result is illegal; *out is then NULL. */
 rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base, const rc_transform* seq,
                             size_t n, rc_schedule** out);
-#define RC_MAX_STAGES 3
+#define RC_MAX_STAGES 6
 /* Number of stages of the op the schedule belongs to, and one stage's knobs. */
 rc_status rc_schedule_knobs(const rc_schedule* s, int32_t stage, rc_knobs* out);
 int32_t rc_schedule_num_stages(const rc_schedule* s);
@@ -301,6 +320,16 @@ typedef struct {
   int32_t screen;     /* surrogate = 1 only: an expansion draws up to screen * B distinct legal
                        * proposals and keeps the B with the lowest predicted time (the cost model
                        * pruning low-value proposals before they join the tree); <= 1 = off */
+  uint32_t stage_mask; /* 0 (default): every stage of the op may be transformed and the objective
+                        * is the op's device time. Else only transformations of the stages whose
+                        * bit is set are proposed, and the objective is the sum of those stages'
+                        * medians (rc_measurement.stage_ms; the whole time where a measurement has
+                        * no per-stage times): one task of a composite op tuned on its own, as a
+                        * compiler tunes the subgraphs of a network one by one */
+  const rc_schedule* root; /* NULL (default): the search starts from P0. Else from this program of
+                            * the same op (copied; the caller keeps ownership), and rewards are
+                            * speedups over it: a later task's search starts from the best program
+                            * of the earlier ones. A schedule of another op is RC_ERR_INVALID_ARG */
 } rc_search_opts;
 
 /* Create an LLM-free MCTS search over op's schedule space (Sec. 3.2 with the

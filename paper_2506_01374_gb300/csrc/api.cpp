@@ -66,6 +66,7 @@ const char* kind_name(int k) {
     case RC_OP_CONV2D: return "conv2d";
     case RC_OP_MOE_ROUTE: return "moe_route";
     case RC_OP_MOE: return "moe";
+    case RC_OP_DECODER_LAYER: return "decoder_layer";
   }
   return "?";
 }
@@ -74,6 +75,7 @@ int n_stages_of(int kind) {
   switch (kind) {
     case RC_OP_MLP: return 2;
     case RC_OP_MOE: return 3;
+    case RC_OP_DECODER_LAYER: return 6;
     default: return 1;
   }
 }
@@ -146,6 +148,19 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       // implicit zero padding (one 4-D box), or a padded copy read as one 4-D box or as row boxes
       v.push_back({RC_T_LAYOUT, 0, {0, 1, 2}, {}});
       break;
+    case RC_OP_DECODER_LAYER:
+      if (stage == 1) {  // RoPE and the split of q, k, v: tokens per CTA
+        v.push_back({RC_T_TILE_SIZE, 0, {1, 2, 4, 8}, {}});
+        break;
+      }
+      if (stage != 2) {
+        // 0: QKV projection, 3: O projection, 4: gate/up + SwiGLU, 5: down projection
+        gemm_common(stage == 4 ? std::vector<int32_t>{32, 64, 128} : std::vector<int32_t>{64, 128, 224, 256});
+        v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+        if (stage == 4) v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+        break;
+      }
+      [[fallthrough]];  // 2: the attention core
     case RC_OP_ATTENTION:
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256 = two query tiles, ping-pong softmax
       v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});
@@ -215,6 +230,17 @@ rc_knobs rc_default_knobs(const rc_op_s* op, int stage) {
       if (stage == 0) k.tile_m = 4;
       else k.tile_n = stage == 1 ? 32 : 64;
       break;
+    case RC_OP_DECODER_LAYER:
+      if (stage == 1) {
+        k.tile_m = 1;
+      } else if (stage == 2) {
+        k.tile_n = 64;
+        k.stages = 2;
+        k.layout = 1;
+      } else {
+        k.tile_n = stage == 4 ? 32 : 64;
+      }
+      break;
   }
   return k;
 }
@@ -224,6 +250,8 @@ static bool in(const std::vector<int32_t>& v, int32_t x) {
     if (y == x) return true;
   return false;
 }
+
+static bool attention_knobs_ok(const rc_knobs& k, int64_t seq, std::string* why);
 
 bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string* why) {
   // 1) every tunable knob holds one of its listed values; untunable knobs keep P0's value
@@ -280,50 +308,59 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
         return false;
       }
       return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
-    case RC_OP_ATTENTION: {
-      // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
-      const int64_t qt = k.tile_m / 128;
-      const int64_t smem = qt * 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 +
-                           (k.location ? 0 : qt * 128 * (int64_t)k.tile_n * 2) + 1024 + 512;
-      if (k.location == 1 && k.tile_m != 256 && k.persistent != 1) {
-        if (why) *why = "P in tensor memory needs two query tiles or split UMMA issue";
-        return false;
-      }
-      const bool one_tile_split = k.tile_m == 128 && k.persistent == 1;
-      if (k.unroll == 2 && !one_tile_split && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
-        // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
-        if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
-        return false;
-      }
-      if (k.raster == 2 && !(one_tile_split && k.location == 1 && k.tile_n == 64 && k.unroll == 1 &&
-                             k.stages >= 2 && k.stages <= 3)) {
-        if (why) *why = "persistent tiles (loop order 2) need the one-tile split-issue kernel: BN 64, unroll 1, 2-3 stages";
-        return false;
-      }
-      if (k.persistent == 1 && !(k.location == 1 && (k.unroll == 1 || one_tile_split) && k.stages >= 2)) {
-        // two tiles: one issuing warp per tile; one tile: one or two S buffers, S and P V issued by
-        // separate warps
-        if (why) *why = "split UMMA issue needs P in TMEM, one key block in flight per issuer and two stages";
-        return false;
-      }
-      if (smem > kSmemLimit) {
-        if (why) *why = "attention ring exceeds 227 KB of shared memory";
-        return false;
-      }
-      if (k.tile_m == 256 && k.stages < 2) {
-        // the ping-pong kernel issues S for key block j+1 before releasing block j
-        if (why) *why = "two query tiles per CTA need at least two K/V stages";
-        return false;
-      }
-      if (k.layout == 1 && o.seq % 8) {
-        if (why) *why = "transposed V needs seq % 8 == 0 (16-byte TMA rows)";
-        return false;
-      }
-      return true;
-    }
+    case RC_OP_DECODER_LAYER:
+      if (stage == 1) return true;
+      if (stage == 2) return attention_knobs_ok(k, o.tokens, why);
+      return tc_gemm_ok(stage == 4 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
+    case RC_OP_ATTENTION:
+      return attention_knobs_ok(k, o.seq, why);
     default:
       return true;
   }
+}
+
+// Resource and variant rules of the attention kernels (RC_OP_ATTENTION and the
+// decoder layer's attention stage).
+static bool attention_knobs_ok(const rc_knobs& k, int64_t seq, std::string* why) {
+  // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
+  const int64_t qt = k.tile_m / 128;
+  const int64_t smem = qt * 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 +
+                       (k.location ? 0 : qt * 128 * (int64_t)k.tile_n * 2) + 1024 + 512;
+  if (k.location == 1 && k.tile_m != 256 && k.persistent != 1) {
+    if (why) *why = "P in tensor memory needs two query tiles or split UMMA issue";
+    return false;
+  }
+  const bool one_tile_split = k.tile_m == 128 && k.persistent == 1;
+  if (k.unroll == 2 && !one_tile_split && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
+    // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
+    if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
+    return false;
+  }
+  if (k.raster == 2 && !(one_tile_split && k.location == 1 && k.tile_n == 64 && k.unroll == 1 &&
+                         k.stages >= 2 && k.stages <= 3)) {
+    if (why) *why = "persistent tiles (loop order 2) need the one-tile split-issue kernel: BN 64, unroll 1, 2-3 stages";
+    return false;
+  }
+  if (k.persistent == 1 && !(k.location == 1 && (k.unroll == 1 || one_tile_split) && k.stages >= 2)) {
+    // two tiles: one issuing warp per tile; one tile: one or two S buffers, S and P V issued by
+    // separate warps
+    if (why) *why = "split UMMA issue needs P in TMEM, one key block in flight per issuer and two stages";
+    return false;
+  }
+  if (smem > kSmemLimit) {
+    if (why) *why = "attention ring exceeds 227 KB of shared memory";
+    return false;
+  }
+  if (k.tile_m == 256 && k.stages < 2) {
+    // the ping-pong kernel issues S for key block j+1 before releasing block j
+    if (why) *why = "two query tiles per CTA need at least two K/V stages";
+    return false;
+  }
+  if (k.layout == 1 && seq % 8) {
+    if (why) *why = "transposed V needs seq % 8 == 0 (16-byte TMA rows)";
+    return false;
+  }
+  return true;
 }
 
 // -------------------------------------------------------------- op slots --
@@ -394,6 +431,18 @@ std::vector<SlotInfo> rc_slots(const rc_op_s* op) {
            {b4 * tk, false, true, true}};
       break;
     }
+    case RC_OP_DECODER_LAYER: {
+      const size_t T = d.tokens, H = d.hidden, D = d.head_dim;
+      s = {{b2 * T * H, true, false, false},
+           {b2 * H, true, false, false},
+           {b2 * (d.heads_q + 2 * d.heads_kv) * D * H, true, false, false},
+           {b2 * H * d.heads_q * D, true, false, false, 3},  // Wo: O projection
+           {b2 * H, true, false, false, 3},                  // g2: the second RMSNorm
+           {b2 * 2 * d.inter * H, true, false, false, 4},    // W1: gate/up
+           {b2 * H * d.inter, true, false, false, 5},        // W2: down
+           {b2 * T * H, false, true, false}};
+      break;
+    }
   }
   return s;
 }
@@ -424,6 +473,19 @@ size_t rc_workspace_bytes(const rc_op_s* op, const rc_schedule_s* s) {
     }
     case RC_OP_ATTENTION:
       return (k && k[0].layout == 1) ? align256(2ull * d.batch * d.heads_kv * d.head_dim * d.seq) : 0;
+    case RC_OP_DECODER_LAYER: {
+      const size_t T = d.tokens, H = d.hidden, D = d.head_dim, I = d.inter;
+      const size_t hq = d.heads_q * D, hkv = d.heads_kv * D;
+      size_t b = align256(2 * T * H);                               // a = RMSNorm(x) g1
+      b += align256(2 * T * (hq + 2 * hkv));                        // qkv
+      b += align256(2 * T * hq) + 2 * align256(2 * T * hkv);        // Q, K, V after RoPE
+      b += align256(2 * T * hq);                                    // attention output o
+      b += 3 * align256(2 * T * H);                                 // t (projection), h1, b
+      b += align256(2 * T * I);                                     // SwiGLU output
+      if (k && !k[4].fuse) b += align256(2 * T * 2 * I);            // gate|up before SwiGLU
+      if (k && k[2].layout == 1) b += align256(2 * hkv * T);        // V transposed for attention
+      return b;
+    }
     case RC_OP_MOE_ROUTE:
       return align256(4ull * d.experts);  // per-expert counts
     case RC_OP_MOE: {
@@ -534,6 +596,35 @@ extern "C" rc_status rc_op_describe(const rc_op_desc* desc, rc_op** out) {
         info.bound = info.flops / info.bytes >= ridge ? RC_BOUND_TENSOR : RC_BOUND_HBM;
         info.n_tensors = 9;
       }
+      break;
+    }
+    case RC_OP_DECODER_LAYER: {
+      if (d.tokens <= 0 || d.hidden <= 0 || d.inter <= 0 || d.heads_q <= 0 || d.heads_kv <= 0)
+        return bad("tokens, hidden, inter, heads_q, heads_kv must be positive");
+      if (d.head_dim == 0) d.head_dim = 128;
+      if (d.head_dim != 128) return unsup("head_dim must be 128");
+      if (d.heads_q % d.heads_kv) return bad("heads_q must be a multiple of heads_kv");
+      if (d.hidden % 256 || d.hidden > 32768)
+        return unsup("hidden must be a multiple of 256 and at most 32768 (one RMSNorm row per CTA in registers)");
+      if (d.inter % 64) return unsup("inter must be a multiple of 64");
+      if (d.tokens > 0x7fffffffLL) return unsup("tokens must fit in 31 bits");
+      if (d.rope_theta == 0.0) d.rope_theta = 500000.0;
+      if (d.norm_eps == 0.0) d.norm_eps = 1e-5;
+      if (!(d.rope_theta > 1.0) || !(d.norm_eps > 0.0)) return bad("rope_theta must be > 1 and norm_eps > 0");
+      d.batch = 1;
+      d.seq = d.tokens;
+      d.causal = 1;
+      d.scale = 1.0 / std::sqrt(128.0);
+      const double T = (double)d.tokens, H = (double)d.hidden, I = (double)d.inter, D = 128.0;
+      const double hq = d.heads_q * D, hkv = d.heads_kv * D;
+      const double pairs = 0.5 * T * (T + 1);
+      info.flops = 2.0 * T * H * (hq + 2 * hkv)      // QKV projection
+                   + 4.0 * D * d.heads_q * pairs      // causal attention (QK^T and PV)
+                   + 2.0 * T * hq * H                 // O projection
+                   + 6.0 * T * H * I;                 // gate/up and down projections
+      info.bytes = 2.0 * (2.0 * T * H + 2.0 * H + H * (hq + 2 * hkv) + H * hq + 3.0 * H * I);
+      info.bound = info.flops / info.bytes >= ridge ? RC_BOUND_TENSOR : RC_BOUND_HBM;
+      info.n_tensors = 8;
       break;
     }
     default:

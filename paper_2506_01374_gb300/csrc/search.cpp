@@ -187,7 +187,7 @@ struct rc_search_s {
   std::vector<std::unique_ptr<rc_schedule_s>> owned;     // schedules handed out
   std::vector<Pending> pending;                          // last batch, in order
   std::vector<int64_t> awaiting;                         // nodes waiting for their reward
-  double t0_ms = 0.0;                                    // P0 median time
+  double t0_ms = 0.0;                                    // objective of the root program
   bool root_measured = false;
   int64_t iterations = 0;
   uint64_t best_hash = 0;
@@ -225,12 +225,26 @@ struct rc_search_s {
       n_fit = n_train;
     }
   }
-  // Predicted device time (ms) of a schedule.
+  bool in_task(int g) const { return o.stage_mask == 0 || (g < 32 && ((o.stage_mask >> g) & 1u)); }
+  // The objective of a measurement: the op's median time, or with a stage
+  // mask the sum of the selected stages' medians.
+  double objective(const rc_measurement& m) const {
+    if (!o.stage_mask || m.n_stages != nodes[0].sched->n_stages) return m.ms_median;
+    double t = 0.0;
+    for (int g = 0; g < m.n_stages; ++g) {
+      if (!in_task(g)) continue;
+      if (!(m.stage_ms[g] > 0)) return m.ms_median;
+      t += m.stage_ms[g];
+    }
+    return t;
+  }
+  // Predicted objective (ms) of a schedule.
   double predict_ms(const rc_schedule_s* sc) {
     const int S = sc->n_stages;
     if (per_stage == 1) {
       double t = 0.0;
-      for (int g = 0; g < S; ++g) t += std::exp(models[g].predict(&sc->k[g], 1, g));
+      for (int g = 0; g < S; ++g)
+        if (in_task(g)) t += std::exp(models[g].predict(&sc->k[g], 1, g));
       return t;
     }
     return std::exp(models[0].predict(sc->k, S, 0));
@@ -321,6 +335,8 @@ extern "C" rc_status rc_search_create(const rc_op* op, const rc_search_opts* opt
   o.max_tries = 64;
   o.surrogate = 0;
   o.screen = 1;
+  o.stage_mask = 0;
+  o.root = nullptr;
   if (opts) {
     o.seed = opts->seed;
     if (opts->c > 0) o.c = opts->c;
@@ -332,6 +348,13 @@ extern "C" rc_status rc_search_create(const rc_op* op, const rc_search_opts* opt
       return rc_fail(RC_ERR_INVALID_ARG, "rc_search_create: surrogate must be 0 or 1");
     o.surrogate = opts->surrogate;
     if (opts->screen > 1) o.screen = opts->screen;
+    const int S = op->n_stages;
+    if (S < 32 && (opts->stage_mask >> S) != 0)
+      return rc_fail(RC_ERR_INVALID_ARG, "rc_search_create: stage_mask names a stage the op does not have");
+    o.stage_mask = opts->stage_mask;
+    if (opts->root && (opts->root->op_kind != op->d.kind || opts->root->n_stages != S))
+      return rc_fail(RC_ERR_INVALID_ARG, "rc_search_create: root is a schedule of another op");
+    o.root = opts->root;
   }
   auto* s = new (std::nothrow) rc_search_s;
   if (!s) return rc_fail(RC_ERR_OOM, "rc_search_create: out of host memory");
@@ -342,12 +365,19 @@ extern "C" rc_status rc_search_create(const rc_op* op, const rc_search_opts* opt
   rc_transform_space(op, nullptr, 0, &n);
   s->space.resize(n);
   if (n) rc_transform_space(op, s->space.data(), n, &n);
+  if (o.stage_mask) {  // one task: only the selected stages' transformations
+    std::vector<rc_transform> keep;
+    for (const rc_transform& t : s->space)
+      if (t.stage < 32 && ((o.stage_mask >> t.stage) & 1u)) keep.push_back(t);
+    s->space.swap(keep);
+  }
   rc_schedule* root = nullptr;
-  rc_status st = rc_schedule_apply(op, nullptr, nullptr, 0, &root);
+  rc_status st = rc_schedule_apply(op, o.root, nullptr, 0, &root);
   if (st != RC_OK) {
     delete s;
     return st;
   }
+  s->o.root = nullptr;  // copied above; the caller's schedule is not referenced afterwards
   Node r;
   r.sched.reset(root);
   r.hash = rc_schedule_hash(root);
@@ -374,12 +404,12 @@ extern "C" rc_status rc_search_step(rc_search* s, const rc_measurement* results,
     const Pending& p = s->pending[i];
     const rc_measurement& m = results[i];
     if (!s->root_measured) {
-      if (m.status != RC_OK || !(m.ms_median > 0))
-        return rc_fail(RC_ERR_INVALID_ARG, "rc_search_step: the root program P0 must measure successfully");
-      s->t0_ms = m.ms_median;
+      if (m.status != RC_OK || !(m.ms_median > 0) || !(s->objective(m) > 0))
+        return rc_fail(RC_ERR_INVALID_ARG, "rc_search_step: the root program must measure successfully");
+      s->t0_ms = s->objective(m);
       s->root_measured = true;
     }
-    const double r = (m.status == RC_OK && m.ms_median > 0) ? s->t0_ms / m.ms_median : 0.0;
+    const double r = (m.status == RC_OK && m.ms_median > 0) ? s->t0_ms / s->objective(m) : 0.0;
     s->reward[p.hash] = r;
     s->meas[p.hash] = m;
     s->meas[p.hash].sched_hash = p.hash;

@@ -198,16 +198,17 @@ def attention(B: int, S: int, Hq: int, Hkv: int, D: int, seed: int = 4):
     return Q, Kt, V
 
 
-def decoder_layer(T: int, H: int, Hq: int, Hkv: int, I: int, seed: int = 8, D: int = 128):
+def decoder_layer(T: int, H: int, Hq: int, Hkv: int, I: int, seed: int = 8, D: int = 128, x_std: float = 1.0,
+                  wqkv_std: float = 0.02):
     """Llama-style decoder layer inputs, bf16 bits.
 
-    x[T,H] ~ N(0,1); norm weights g1, g2[H] = 1 + 0.1 N(0,1); Wqkv[(Hq + 2 Hkv) D, H]
-    (query, key, value rows), Wo[H, Hq D], W1[2I, H] (gate rows, then up rows),
-    W2[H, I] ~ N(0, 0.02).
+    x[T,H] ~ N(0, x_std^2); norm weights g1, g2[H] = 1 + 0.1 N(0,1);
+    Wqkv[(Hq + 2 Hkv) D, H] (query, key, value rows) ~ N(0, wqkv_std^2);
+    Wo[H, Hq D], W1[2I, H] (gate rows, then up rows), W2[H, I] ~ N(0, 0.02).
     """
-    x = _bf16_normal(seed, 1, (T, H), 1.0)
+    x = _bf16_normal(seed, 1, (T, H), x_std)
     g1 = to_bf16_bits(1.0 + 0.1 * normal(key(seed, 2), H))
-    Wqkv = _bf16_normal(seed, 3, ((Hq + 2 * Hkv) * D, H), 0.02)
+    Wqkv = _bf16_normal(seed, 3, ((Hq + 2 * Hkv) * D, H), wqkv_std)
     Wo = _bf16_normal(seed, 4, (H, Hq * D), 0.02)
     g2 = to_bf16_bits(1.0 + 0.1 * normal(key(seed, 5), H))
     W1 = _bf16_normal(seed, 6, (2 * I, H), 0.02)

@@ -23,7 +23,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED_OP, ERR_ILLEGAL_SCHEDULE, ERR_DUPLICATE, ER
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED_OP", 3: "ILLEGAL_SCHEDULE", 4: "DUPLICATE",
                 5: "CUDA", 6: "DEVICE_TIMEOUT", 7: "TIMEOUT", 8: "PARITY", 9: "OOM", 10: "EXHAUSTED"}
 
-OP_GEMM_F32, OP_LINEAR, OP_SWIGLU, OP_MLP, OP_ATTENTION, OP_CONV2D, OP_MOE_ROUTE, OP_MOE = range(8)
+OP_GEMM_F32, OP_LINEAR, OP_SWIGLU, OP_MLP, OP_ATTENTION, OP_CONV2D, OP_MOE_ROUTE, OP_MOE, OP_DECODER_LAYER = range(9)
 EPI_BIAS, EPI_RELU, EPI_SILU = 1, 2, 4
 BOUND_NAMES = {0: "tensor", 1: "hbm", 2: "fp32_simt"}
 
@@ -32,7 +32,7 @@ T_TILE_SIZE, T_PARALLEL, T_COMPUTE_LOCATION, T_UNROLL, T_LOOP_ORDER, T_FUSE, T_L
 T_NAMES = ["TileSize", "Parallel", "ComputeLocation", "Unroll", "LoopOrder", "Fuse", "Layout", "Vectorize",
            "PipelineStages", "SplitK"]
 MAX_TENSORS = 10
-MAX_STAGES = 3
+MAX_STAGES = 6
 
 
 class OpDesc(C.Structure):
@@ -44,7 +44,8 @@ class OpDesc(C.Structure):
                 ("c_out", C.c_int64), ("kr", C.c_int64), ("ks", C.c_int64), ("stride", C.c_int64),
                 ("pad", C.c_int64),
                 ("tokens", C.c_int64), ("hidden", C.c_int64), ("experts", C.c_int64), ("inter", C.c_int64),
-                ("top_k", C.c_int64), ("logits_fp32", C.c_int32), ("renorm", C.c_int32)]
+                ("top_k", C.c_int64), ("logits_fp32", C.c_int32), ("renorm", C.c_int32),
+                ("rope_theta", C.c_double), ("norm_eps", C.c_double)]
 
 
 class OpInfo(C.Structure):
@@ -91,7 +92,8 @@ class Measurement(C.Structure):
 
 class SearchOpts(C.Structure):
     _fields_ = [("seed", C.c_uint64), ("c", C.c_double), ("branching", C.c_int32), ("horizon", C.c_int32),
-                ("rollout", C.c_int32), ("max_tries", C.c_int32), ("surrogate", C.c_int32), ("screen", C.c_int32)]
+                ("rollout", C.c_int32), ("max_tries", C.c_int32), ("surrogate", C.c_int32), ("screen", C.c_int32),
+                ("stage_mask", C.c_uint32), ("root", C.c_void_p)]
 
 
 class SearchStats(C.Structure):
@@ -329,9 +331,14 @@ class Search:
     """LLM-free MCTS over an op's schedule space (rc_search_*)."""
 
     def __init__(self, op: Op, seed: int = 0, c: float = math.sqrt(2.0), branching: int = 2, horizon: int = 8,
-                 rollout: int = 2, max_tries: int = 64, surrogate: bool = False, screen: int = 1):
+                 rollout: int = 2, max_tries: int = 64, surrogate: bool = False, screen: int = 1,
+                 stages: Sequence[int] | None = None, root: Schedule | None = None):
+        """stages: tune only these stages of a composite op (objective = their summed time);
+        root: start from this schedule instead of P0 (rewards are speedups over it)."""
         self.op = op
-        o = SearchOpts(seed, c, branching, horizon, rollout, max_tries, int(surrogate), screen)
+        mask = 0 if not stages else sum(1 << int(g) for g in set(stages))
+        o = SearchOpts(seed, c, branching, horizon, rollout, max_tries, int(surrogate), screen, mask,
+                       root.h if root is not None else None)
         h = _P()
         _check(lib().rc_search_create(op.h, C.byref(o), C.byref(h)), "rc_search_create")
         self.h = h.value

@@ -121,3 +121,48 @@ def test_schedule_string_round_trip_size():
     s = op.schedule()
     txt = str(s)
     assert txt.startswith("op=moe;s0:") and ";s2:" in txt
+
+
+def _decoder(**kw):
+    a = dict(tokens=2048, hidden=4096, inter=14336, heads_q=32, heads_kv=8, head_dim=128)
+    a.update(kw)
+    return rc.Op(rc.OP_DECODER_LAYER, **a)
+
+
+def test_decoder_layer_op_work_and_validation():
+    info = _decoder().info
+    T, H, I, hq, hkv = 2048, 4096, 14336, 32 * 128, 8 * 128
+    want = 2 * T * H * (hq + 2 * hkv) + 4 * 128 * 32 * T * (T + 1) // 2 + 2 * T * hq * H + 6 * T * H * I
+    assert info["flops"] == want and info["bound"] == "tensor" and info["n_tensors"] == 8
+    for kw, st in [(dict(hidden=4000), rc.ERR_UNSUPPORTED_OP), (dict(head_dim=64), rc.ERR_UNSUPPORTED_OP),
+                   (dict(heads_q=12, heads_kv=8), rc.ERR_INVALID_ARG), (dict(tokens=0), rc.ERR_INVALID_ARG),
+                   (dict(inter=100), rc.ERR_UNSUPPORTED_OP), (dict(norm_eps=-1.0), rc.ERR_INVALID_ARG)]:
+        with pytest.raises(rc.RcError) as e:
+            _decoder(**kw)
+        assert e.value.status == st, kw
+    # head_dim 0 takes the default of 128
+    assert _decoder(head_dim=0).info["flops"] == want
+
+
+def test_decoder_layer_schedule_has_six_independent_stages():
+    op = _decoder(tokens=256, hidden=512, inter=768, heads_q=4, heads_kv=2)
+    p0 = op.schedule()
+    assert p0.num_stages == 6 and str(p0).startswith("op=decoder_layer;s0:") and ";s5:" in str(p0)
+    s = op.schedule(rc.T(rc.T_TILE_SIZE, 4, axis=0, stage=1), rc.T(rc.T_FUSE, 1, stage=4),
+                    rc.T(rc.T_TILE_SIZE, 128, axis=1, stage=2), rc.T(rc.T_TILE_SIZE, 256, axis=0, stage=5))
+    assert s.knobs(1)["tile_m"] == 4 and s.knobs(4)["fuse"] == 1
+    assert s.knobs(2)["tile_n"] == 128 and s.knobs(5)["tile_m"] == 256 and s.knobs(0) == p0.knobs(0)
+    stages = {t.stage for t in op.transform_space()}
+    assert stages == set(range(6))
+    for t in [rc.T(rc.T_TILE_SIZE, 3, axis=0, stage=1),       # tokens per CTA outside {1, 2, 4, 8}
+              rc.T(rc.T_SPLIT_K, 2, stage=5),                 # no split-K in the layer's GEMMs
+              rc.T(rc.T_FUSE, 1, stage=0),                    # fusion belongs to the gate/up GEMM
+              rc.T(rc.T_LOOP_ORDER, 2, stage=2),              # persistent attention needs its own knobs
+              rc.T(rc.T_TILE_SIZE, 64, axis=1, stage=6)]:     # no seventh stage
+        with pytest.raises(rc.RcError) as e:
+            op.schedule(t)
+        assert e.value.status == rc.ERR_ILLEGAL_SCHEDULE, t
+    # P0's workspace: a, qkv, Q, K, V, o, t, h1, b, the SwiGLU output, gate|up (unfused) and V transposed
+    T, H, I, hq, hkv = 256, 512, 768, 512, 256
+    want = 2 * (T * H + T * (hq + 2 * hkv) + T * hq + 2 * T * hkv + T * hq + 3 * T * H + T * I + 2 * T * I + hkv * T)
+    assert op.info["workspace_bytes"] == want

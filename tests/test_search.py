@@ -167,3 +167,74 @@ def test_best_schedule_outlives_the_search():
     import gc
     gc.collect()
     assert best.knobs() == knobs and best.hash == m.sched_hash
+
+
+# ------------------------------------------------- one task of a composite op --
+
+def _decoder_op():
+    return rc.Op(rc.OP_DECODER_LAYER, tokens=512, hidden=1024, inter=2048, heads_q=8, heads_kv=2, head_dim=128)
+
+
+def _stage_meas(s, noise):
+    """Synthetic per-stage times: stage g's time from its own knobs; `noise` perturbs the others."""
+    m = rc.Measurement()
+    m.status = rc.OK
+    m.n_stages = s.num_stages
+    for g in range(s.num_stages):
+        k = s.knobs(g)
+        t = 1.0 + 0.01 * g + 1.0 / max(k["tile_n"], 1) + 0.1 / max(k["stages"], 1) + 0.05 * k["fuse"]
+        m.stage_ms[g] = t + noise(g)
+    m.ms_median = sum(m.stage_ms[g] for g in range(s.num_stages))
+    return m
+
+
+def _drive(srch, measure, samples):
+    fed, res, pend = [], [], False
+    while len(fed) < samples:
+        nxt = srch.step(res)
+        pend = False
+        if not nxt:
+            break
+        res = [measure(s) for s in nxt]
+        fed += list(zip(nxt, res))
+        pend = True
+    if pend:
+        srch.step(res)
+    return fed
+
+
+def test_stage_mask_tunes_one_task_from_a_given_root():
+    op = _decoder_op()
+    root = op.schedule(rc.T(rc.T_FUSE, 1, stage=4), rc.T(rc.T_TILE_SIZE, 4, axis=0, stage=1))
+    rng = iter(range(10 ** 6))
+
+    def noise(g):  # the untouched stages' times jump around by up to 0.5 ms per measurement
+        return 0.0 if g == 3 else 0.5 * ((next(rng) * 7919) % 101) / 100
+
+    srch = rc.Search(op, seed=3, branching=4, stages=[3], root=root)
+    fed = _drive(srch, lambda s: _stage_meas(s, noise), 120)
+    assert fed[0][0].hash == root.hash  # the root is measured first
+    for s, _ in fed:  # only stage 3 ever changes
+        for g in range(6):
+            if g != 3:
+                assert s.knobs(g) == root.knobs(g)
+    best, m = srch.best()
+    # the objective is stage 3's own time: the best is the fastest stage-3 program seen, whatever the noise
+    t3 = min(r.stage_ms[3] for _, r in fed)
+    assert m.stage_ms[3] == pytest.approx(t3)
+    assert srch.stats()["best_reward"] == pytest.approx(fed[0][1].stage_ms[3] / t3)
+
+
+def test_stage_mask_and_root_are_validated():
+    op = _decoder_op()
+    with pytest.raises(rc.RcError) as e:
+        rc.Search(op, stages=[6])
+    assert e.value.status == rc.ERR_INVALID_ARG
+    other = rc.Op(rc.OP_MLP, m=256, n=512, k=256)
+    with pytest.raises(rc.RcError) as e:
+        rc.Search(op, root=other.schedule())
+    assert e.value.status == rc.ERR_INVALID_ARG
+    # a task with a handful of programs is exhausted, not an error, for the caller
+    srch = rc.Search(op, stages=[1], branching=4)
+    fed = _drive(srch, lambda s: _stage_meas(s, lambda g: 0.0), 100)
+    assert len({s.hash for s, _ in fed}) == 4  # TileSize tokens-per-CTA in {1, 2, 4, 8}
