@@ -71,7 +71,7 @@ def parse():
                     help="maximum transformation-sequence length T of each search (0 = the workload's: 8)")
     ap.add_argument("--tasks", type=int, default=-1, choices=[-1, 0, 1],
                     help="1 = tune a composite op stage by stage, then jointly (search_tasks); 0 = one joint "
-                         "search; -1 = the workload's choice (stage by stage for the decoder layer)")
+                         "search; -1 = the workload's choice (stage by stage for the MLP, MoE and decoder layer)")
     ap.add_argument("--restarts", type=int, default=2,
                     help="independent searches (seeds seed, seed+1, ...) per workload; the fastest result is kept")
     ap.add_argument("--seed", type=int, default=0)
@@ -171,7 +171,7 @@ class Workload:
         from paper_2506_01374_gb300 import inputs, rc
         self.name = name
         self.horizon = 8  # search horizon T
-        self.tasks = False
+        self.tasks = False  # composite ops: tuned stage by stage (search_tasks), then jointly
         sh = dict(shape or {})
 
         def dims(**default):
@@ -181,6 +181,7 @@ class Workload:
             return [sh.get(k, v) for k, v in default.items()]
 
         if name == "mlp":
+            self.tasks = True
             T, H, I = dims(tokens=2048, hidden=4096, inter=14336)
             X, W1, W2 = inputs.mlp(T, H, I, seed=1)
             self.op = rc.Op(rc.OP_MLP, m=T, n=I, k=H)
@@ -237,6 +238,7 @@ class Workload:
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "moe":
+            self.tasks = True
             T, H, E, I, K = dims(tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
             logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=6)
             self.op = rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
@@ -250,6 +252,7 @@ class Workload:
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "decoder_layer":
+            self.tasks = True
             T, H, Hq, Hkv, I = dims(tokens=2048, hidden=4096, heads_q=32, heads_kv=8, inter=14336)
             self.host = list(inputs.decoder_layer(T, H, Hq, Hkv, I, seed=8)) + [None]
             self.op = rc.Op(rc.OP_DECODER_LAYER, tokens=T, hidden=H, inter=I, heads_q=Hq, heads_kv=Hkv, head_dim=128)
@@ -259,7 +262,6 @@ class Workload:
             self.metric = "best-schedule TFLOP/s (Llama-3-8B decoder layer, bf16)"
             self.dom_stage, self.dom_flops = 4, 2.0 * T * (2 * I) * H
             self.dom_name = "gate/up GEMM + SwiGLU (stage 4)"
-            self.tasks = True  # tuned stage by stage (search_tasks), then jointly
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "gemm_f32":
@@ -660,9 +662,9 @@ def launches_per_step(workload, s):
         # down, combine (or, with the atomic combine, the fp32 -> bf16 conversion; the memset is not ours)
         return 3 + (0 if k[1]["location"] == 1 else 1) + 1 + 1 + 1
     if workload == "decoder_layer":
-        # RMSNorm, QKV GEMM, RoPE, attention (+ V transpose), O GEMM, add + RMSNorm,
-        # gate/up GEMM (+ SwiGLU pass), down GEMM, residual add
-        return 2 + 1 + 1 + (1 if k[2]["layout"] == 1 else 0) + 2 + (1 if k[4]["fuse"] else 2) + 2
+        # RMSNorm, QKV GEMM, RoPE, attention (+ V transpose), O GEMM with the residual, RMSNorm,
+        # gate/up GEMM (+ SwiGLU pass), down GEMM with the residual
+        return 2 + 1 + 1 + (1 if k[2]["layout"] == 1 else 0) + 2 + (1 if k[4]["fuse"] else 2) + 1
     return 1
 
 

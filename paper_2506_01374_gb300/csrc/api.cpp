@@ -480,7 +480,7 @@ size_t rc_workspace_bytes(const rc_op_s* op, const rc_schedule_s* s) {
       b += align256(2 * T * (hq + 2 * hkv));                        // qkv
       b += align256(2 * T * hq) + 2 * align256(2 * T * hkv);        // Q, K, V after RoPE
       b += align256(2 * T * hq);                                    // attention output o
-      b += 3 * align256(2 * T * H);                                 // t (projection), h1, b
+      b += 2 * align256(2 * T * H);                                 // h1, b
       b += align256(2 * T * I);                                     // SwiGLU output
       if (k && !k[4].fuse) b += align256(2 * T * 2 * I);            // gate|up before SwiGLU
       if (k && k[2].layout == 1) b += align256(2 * hkv * T);        // V transposed for attention

@@ -1,8 +1,8 @@
 // Memory-bound kernels of the decoder layer (RC_OP_DECODER_LAYER) around its
-// GEMMs and attention: RMSNorm (optionally after a residual add), RoPE with
-// the split of the fused QKV projection into contiguous Q, K, V, and the final
-// residual add. All read and write 16-byte vectors of bf16 and compute in
-// fp32.
+// GEMMs and attention: RMSNorm, and RoPE with the split of the fused QKV
+// projection into contiguous Q, K, V heads. (The residual adds happen in the
+// O and down GEMMs' epilogues.) Both read and write 16-byte vectors of bf16
+// and compute in fp32.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -18,10 +18,11 @@ union V8 {
   __nv_bfloat16 h[8];
 };
 
-// One CTA per row, one 16-byte vector (8 elements) per thread and pass, at
-// most kMaxVec passes kept in registers: h = bf16(x + t) when t is given
-// (written to h_out), then y = h / sqrt(mean(h^2) + eps) * g. H % 256 == 0,
-// blockDim = min(H / 8, 1024) (a multiple of 32).
+// One CTA per row; each thread loads up to kMaxVec 16-byte vectors (8
+// elements each) at once and keeps them in registers between the sum of
+// squares and the scaling: y = x / sqrt(mean(x^2) + eps) * g. H % 256 == 0,
+// blockDim = the multiple of 32 that covers H / 8 in at most kMaxVec
+// vectors per thread (128 threads at H = 4096).
 constexpr int kMaxVec = 4;
 
 __device__ __forceinline__ float block_sum(float v, float* red) {
@@ -35,33 +36,25 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return s;
 }
 
-__global__ void rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ t,
-                               const __nv_bfloat16* __restrict__ g, int H, float eps,
-                               __nv_bfloat16* __restrict__ h_out, __nv_bfloat16* __restrict__ y) {
+__global__ void rmsnorm_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ g, int H,
+                               float eps, __nv_bfloat16* __restrict__ y) {
   __shared__ float red[32];
   const int64_t off = (int64_t)blockIdx.x * H;
   const int nvec = H / 8;
   V8 a[kMaxVec];
+#pragma unroll
+  for (int i = 0; i < kMaxVec; ++i) {  // every load in flight before the first use
+    const int v = threadIdx.x + i * blockDim.x;
+    a[i].u = v < nvec ? reinterpret_cast<const uint4*>(x + off)[v] : make_uint4(0, 0, 0, 0);
+  }
   float ss = 0.f;
 #pragma unroll
-  for (int i = 0; i < kMaxVec; ++i) {
-    const int v = threadIdx.x + i * blockDim.x;
-    if (v >= nvec) break;
-    a[i].u = reinterpret_cast<const uint4*>(x + off)[v];
-    if (t) {
-      V8 b;
-      b.u = reinterpret_cast<const uint4*>(t + off)[v];
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        a[i].h[j] = __float2bfloat16_rn(__bfloat162float(a[i].h[j]) + __bfloat162float(b.h[j]));
-      reinterpret_cast<uint4*>(h_out + off)[v] = a[i].u;
-    }
+  for (int i = 0; i < kMaxVec; ++i)
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const float f = __bfloat162float(a[i].h[j]);
       ss = fmaf(f, f, ss);
     }
-  }
   const float inv = rsqrtf(block_sum(ss, red) / (float)H + eps);
 #pragma unroll
   for (int i = 0; i < kMaxVec; ++i) {
@@ -88,7 +81,8 @@ struct InvFreq {
 // A CTA handles `per` (<= 8) consecutive tokens: their cos/sin are formed once
 // in shared memory (fp32 angle p * inv_freq[j], at most ~2^-13 rad off at
 // p = 2047, far below the bf16 rounding of the output), then each thread
-// rotates 8 pairs at a time with 16-byte loads and stores.
+// rotates 8 pairs per unit with 16-byte loads and stores, several units at a
+// time.
 template <int D>
 __global__ void rope_split_kernel(const __nv_bfloat16* __restrict__ qkv, int T, int Hq, int Hkv,
                                   const InvFreq<D> invf, int per, __nv_bfloat16* __restrict__ Q,
@@ -108,42 +102,48 @@ __global__ void rope_split_kernel(const __nv_bfloat16* __restrict__ qkv, int T, 
   const int width = (Hq + 2 * Hkv) * D;
   const int rot_units = (Hq + Hkv) * G;
   const int units = rot_units + Hkv * D / 8;
-  for (int e = threadIdx.x; e < nt * units; e += blockDim.x) {
-    const int tt = e / units, u = e % units;
-    const int64_t t = t0 + tt;
-    const __nv_bfloat16* row = qkv + t * width;
-    if (u < rot_units) {
-      const int hd = u / G, j0 = (u % G) * 8;
-      V8 lo, hi, olo, ohi;
-      lo.u = *reinterpret_cast<const uint4*>(row + hd * D + j0);
-      hi.u = *reinterpret_cast<const uint4*>(row + hd * D + D / 2 + j0);
+  // kUnits units in flight per thread: all their loads are issued before the first use
+  constexpr int kUnits = 4;
+  const int total = nt * units;
+  for (int base = threadIdx.x; base < total; base += kUnits * blockDim.x) {
+    V8 lo[kUnits], hi[kUnits];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const float c = cs[tt][j0 + i], s = sn[tt][j0 + i];
-        const float l = __bfloat162float(lo.h[i]), h = __bfloat162float(hi.h[i]);
-        olo.h[i] = __float2bfloat16_rn(l * c - h * s);
-        ohi.h[i] = __float2bfloat16_rn(h * c + l * s);
+    for (int q = 0; q < kUnits; ++q) {
+      const int e = base + q * blockDim.x;
+      if (e >= total) break;
+      const int tt = e / units, u = e % units;
+      const __nv_bfloat16* row = qkv + (int64_t)(t0 + tt) * width;
+      if (u < rot_units) {
+        const int hd = u / G, j0 = (u % G) * 8;
+        lo[q].u = *reinterpret_cast<const uint4*>(row + hd * D + j0);
+        hi[q].u = *reinterpret_cast<const uint4*>(row + hd * D + D / 2 + j0);
+      } else {
+        lo[q].u = *reinterpret_cast<const uint4*>(row + (Hq + Hkv) * D + (u - rot_units) * 8);
       }
-      __nv_bfloat16* dst = hd < Hq ? Q + (t * Hq + hd) * D : K + (t * Hkv + (hd - Hq)) * D;
-      *reinterpret_cast<uint4*>(dst + j0) = olo.u;
-      *reinterpret_cast<uint4*>(dst + D / 2 + j0) = ohi.u;
-    } else {
-      const int v = u - rot_units;
-      reinterpret_cast<uint4*>(V + t * Hkv * D)[v] = reinterpret_cast<const uint4*>(row + (Hq + Hkv) * D)[v];
     }
-  }
-}
-
-// y = bf16(a + b), n % 8 == 0.
-__global__ void add_kernel(const __nv_bfloat16* __restrict__ a, const __nv_bfloat16* __restrict__ b, int64_t n8,
-                           __nv_bfloat16* __restrict__ y) {
-  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n8; v += (int64_t)gridDim.x * blockDim.x) {
-    V8 x, z, o;
-    x.u = reinterpret_cast<const uint4*>(a)[v];
-    z.u = reinterpret_cast<const uint4*>(b)[v];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) o.h[j] = __float2bfloat16_rn(__bfloat162float(x.h[j]) + __bfloat162float(z.h[j]));
-    reinterpret_cast<uint4*>(y)[v] = o.u;
+    for (int q = 0; q < kUnits; ++q) {
+      const int e = base + q * blockDim.x;
+      if (e >= total) break;
+      const int tt = e / units, u = e % units;
+      const int64_t t = t0 + tt;
+      if (u < rot_units) {
+        const int hd = u / G, j0 = (u % G) * 8;
+        V8 olo, ohi;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float c = cs[tt][j0 + i], s = sn[tt][j0 + i];
+          const float l = __bfloat162float(lo[q].h[i]), h = __bfloat162float(hi[q].h[i]);
+          olo.h[i] = __float2bfloat16_rn(l * c - h * s);
+          ohi.h[i] = __float2bfloat16_rn(h * c + l * s);
+        }
+        __nv_bfloat16* dst = hd < Hq ? Q + (t * Hq + hd) * D : K + (t * Hkv + (hd - Hq)) * D;
+        *reinterpret_cast<uint4*>(dst + j0) = olo.u;
+        *reinterpret_cast<uint4*>(dst + D / 2 + j0) = ohi.u;
+      } else {
+        reinterpret_cast<uint4*>(V + t * Hkv * D)[u - rot_units] = lo[q].u;
+      }
+    }
   }
 }
 
@@ -155,16 +155,16 @@ rc_status launched(const char* what) {
 
 }  // namespace
 
-rc_status rc_launch_rmsnorm(const void* x, const void* t, const void* g, int64_t rows, int64_t H, double eps,
-                            void* h_out, void* y, const LaunchCtx& c) {
+rc_status rc_launch_rmsnorm(const void* x, const void* g, int64_t rows, int64_t H, double eps, void* y,
+                            const LaunchCtx& c) {
   if (H % 256 || H / 8 > 1024 * kMaxVec)
     return rc_fail(RC_ERR_UNSUPPORTED_OP, "rmsnorm: hidden must be a multiple of 256 and at most 32768");
   if (rows <= 0) return RC_OK;
   if (rows > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "rmsnorm: too many rows");
-  const int threads = (int)std::min<int64_t>(H / 8, 1024);
+  const int64_t per_thread = (H / 8 + kMaxVec - 1) / kMaxVec;
+  const int threads = (int)std::min<int64_t>((per_thread + 31) / 32 * 32, 1024);
   rmsnorm_kernel<<<(unsigned)rows, threads, 0, (cudaStream_t)c.stream>>>(
-      (const __nv_bfloat16*)x, (const __nv_bfloat16*)t, (const __nv_bfloat16*)g, (int)H, (float)eps,
-      (__nv_bfloat16*)h_out, (__nv_bfloat16*)y);
+      (const __nv_bfloat16*)x, (const __nv_bfloat16*)g, (int)H, (float)eps, (__nv_bfloat16*)y);
   return launched("rmsnorm");
 }
 
@@ -183,15 +183,4 @@ rc_status rc_launch_rope_split(const rc_knobs& k, const void* qkv, int64_t T, in
       (const __nv_bfloat16*)qkv, (int)T, (int)Hq, (int)Hkv, f, per, (__nv_bfloat16*)Q, (__nv_bfloat16*)K,
       (__nv_bfloat16*)V);
   return launched("rope");
-}
-
-rc_status rc_launch_add(const void* a, const void* b, int64_t n, void* y, const LaunchCtx& c) {
-  if (n % 8) return rc_fail(RC_ERR_UNSUPPORTED_OP, "add: n %% 8 != 0");
-  const int64_t n8 = n / 8;
-  int64_t g = (n8 + 255) / 256;
-  const int64_t cap = (int64_t)(c.num_sms > 0 ? c.num_sms : 1) * 8;
-  if (g > cap) g = cap;
-  add_kernel<<<(unsigned)(g < 1 ? 1 : g), 256, 0, (cudaStream_t)c.stream>>>(
-      (const __nv_bfloat16*)a, (const __nv_bfloat16*)b, n8, (__nv_bfloat16*)y);
-  return launched("residual add");
 }

@@ -149,6 +149,7 @@ struct TcGemmArgs {
   const int* row_map;      // TC_EPI_SCALE_ATOMIC: A row -> slot; output row = slot / row_div
   int row_div;             // (TC_A_GATHER: A row i is source row row_map[i] / row_div)
   int64_t a_rows;          // TC_A_GATHER: rows of the source matrix A
+  const void* resid;       // TC_EPI_STORE_BF16: bf16 [M][ldd] added to D before the one rounding (NULL = none)
 };
 rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 // Split-K reduction: out_bf16[M][N] = sum_z part[z][M][N].
@@ -180,13 +181,10 @@ rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, const Lau
 rc_status rc_launch_pad_nhwc(const void* x, int64_t N, int64_t H, int64_t W, int64_t C, int64_t pad, void* xp,
                              const LaunchCtx& c);
 // Decoder-layer passes (bf16 storage, fp32 arithmetic). RMSNorm of rows[H]:
-// y = h / sqrt(mean(h^2) + eps) * g with h = x, or h = bf16(x + t) (also
-// stored to h_out) when t is given. H % 256 == 0.
-rc_status rc_launch_rmsnorm(const void* x, const void* t, const void* g, int64_t rows, int64_t H, double eps,
-                            void* h_out, void* y, const LaunchCtx& c);
+// y = x / sqrt(mean(x^2) + eps) * g, H % 256 == 0 and H <= 32768.
+rc_status rc_launch_rmsnorm(const void* x, const void* g, int64_t rows, int64_t H, double eps, void* y,
+                            const LaunchCtx& c);
 // qkv[T][(Hq + 2 Hkv) D] -> Q[T][Hq][D], K[T][Hkv][D] (rotate-half RoPE at
 // positions 0 .. T-1) and V[T][Hkv][D]; k.tile_m tokens per CTA.
 rc_status rc_launch_rope_split(const rc_knobs& k, const void* qkv, int64_t T, int64_t Hq, int64_t Hkv, int64_t D,
                                double theta, void* Q, void* K, void* V, const LaunchCtx& c);
-// y[n] = bf16(a + b), n % 8 == 0.
-rc_status rc_launch_add(const void* a, const void* b, int64_t n, void* y, const LaunchCtx& c);

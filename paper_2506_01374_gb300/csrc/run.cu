@@ -206,14 +206,13 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       void* K = ws.take(2ull * T * hkv);
       void* V = ws.take(2ull * T * hkv);
       void* O = ws.take(2ull * T * hq);
-      void* t = ws.take(2ull * T * H);
       void* h1 = ws.take(2ull * T * H);
       void* b = ws.take(2ull * T * H);
       void* hb = ws.take(2ull * T * I);
       void* gu = s->k[4].fuse ? nullptr : ws.take(2ull * T * 2 * I);
       void* vt = s->k[2].layout == 1 ? ws.take(2ull * hkv * T) : nullptr;
       // 0: a = RMSNorm(x) g1, qkv = a Wqkv^T
-      RC_TRY(rc_launch_rmsnorm(p[0], nullptr, p[1], T, H, d.norm_eps, nullptr, a, c));
+      RC_TRY(rc_launch_rmsnorm(p[0], p[1], T, H, d.norm_eps, a, c));
       RC_TRY(run_linear(s->k[0], T, nqkv, H, a, p[2], qkv, nullptr, c));
       RC_TRY(rc_mark_stage(c));
       // 1: RoPE on q and k, split into contiguous heads
@@ -222,16 +221,19 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       // 2: causal GQA attention over the T positions
       RC_TRY(rc_launch_attention(s->k[2], d, Q, K, V, O, nullptr, vt, c));
       RC_TRY(rc_mark_stage(c));
-      // 3: t = o Wo^T; h1 = x + t; b = RMSNorm(h1) g2
-      RC_TRY(run_linear(s->k[3], T, H, hq, O, p[3], t, nullptr, c));
-      RC_TRY(rc_launch_rmsnorm(p[0], t, p[4], T, H, d.norm_eps, h1, b, c));
+      // 3: h1 = x + o Wo^T (residual added in the GEMM epilogue); b = RMSNorm(h1) g2
+      TcGemmArgs go = gemm_args(T, H, hq, O, p[3], h1, H, TC_EPI_STORE_BF16);
+      go.resid = p[0];
+      RC_TRY(rc_launch_tc_gemm(s->k[3], go, c));
+      RC_TRY(rc_launch_rmsnorm(h1, p[4], T, H, d.norm_eps, b, c));
       RC_TRY(rc_mark_stage(c));
       // 4: SwiGLU of the gate/up projection
       RC_TRY(run_swiglu(s->k[4], T, I, H, b, p[5], hb, gu, c));
       RC_TRY(rc_mark_stage(c));
-      // 5: y = h1 + hb W2^T
-      RC_TRY(run_linear(s->k[5], T, H, I, hb, p[6], t, nullptr, c));
-      RC_TRY(rc_launch_add(h1, t, T * H, p[7], c));
+      // 5: y = h1 + hb W2^T (residual added in the GEMM epilogue)
+      TcGemmArgs gd = gemm_args(T, H, I, hb, p[6], p[7], H, TC_EPI_STORE_BF16);
+      gd.resid = h1;
+      RC_TRY(rc_launch_tc_gemm(s->k[5], gd, c));
       return rc_mark_stage(c);
     }
     case RC_OP_MOE_ROUTE: {

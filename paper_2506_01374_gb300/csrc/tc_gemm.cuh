@@ -73,6 +73,7 @@ struct Params {
   int persistent;       // 1: grid-stride loop over tiles with two TMEM accumulators
   int splits;           // split-K factor (work items = tiles x splits)
   int ksub;             // 64-wide K sub-blocks per ring stage (1 or 2)
+  const __nv_bfloat16* resid;  // STORE_BF16: residual [M][ldd] added before the rounding (NULL = none)
 };
 
 // Linear CTA index -> (m tile, n tile) under the raster order knob.
@@ -162,6 +163,26 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
           for (int j = 0; j < 16; ++j) {
             const float x = v[j] + bv[j];
             v[j] = p.silu ? tc::silu(x) : x;
+          }
+        }
+        if constexpr (EPI == TC_EPI_STORE_BF16) {
+          if (p.resid) {  // residual connection: D = bf16(acc + resid), one rounding
+            const __nv_bfloat16* rr = p.resid + (long long)r * p.ldd + col;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              if (col + 8 * h >= p.out_cols) break;
+              union {
+                uint4 u;
+                __nv_bfloat162 b2[4];
+              } x;
+              x.u = *reinterpret_cast<const uint4*>(rr + 8 * h);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const float2 f = __bfloat1622float2(x.b2[q]);
+                v[8 * h + 2 * q] += f.x;
+                v[8 * h + 2 * q + 1] += f.y;
+              }
+            }
           }
         }
         __nv_bfloat16* out = (__nv_bfloat16*)p.D + (long long)r * p.ldd;
@@ -750,6 +771,9 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.group = k.group > 0 ? k.group : 1;
   p.D = a.D;
   p.ldd = a.ldd;
+  if (a.resid && (EPI != TC_EPI_STORE_BF16 || ((uintptr_t)a.resid % 16) || a.ldd % 8))
+    return rc_fail(RC_ERR_INVALID_ARG, "tc_gemm: a residual needs the bf16 store epilogue and 16-byte rows");
+  p.resid = (const __nv_bfloat16*)a.resid;
   p.bias = (const __nv_bfloat16*)a.bias;
   p.silu = a.silu;
   p.swiglu_I = (int)(a.N / 2);

@@ -162,7 +162,7 @@ def test_decoder_layer_schedule_has_six_independent_stages():
         with pytest.raises(rc.RcError) as e:
             op.schedule(t)
         assert e.value.status == rc.ERR_ILLEGAL_SCHEDULE, t
-    # P0's workspace: a, qkv, Q, K, V, o, t, h1, b, the SwiGLU output, gate|up (unfused) and V transposed
+    # P0's workspace: a, qkv, Q, K, V, o, h1, b, the SwiGLU output, gate|up (unfused) and V transposed
     T, H, I, hq, hkv = 256, 512, 768, 512, 256
-    want = 2 * (T * H + T * (hq + 2 * hkv) + T * hq + 2 * T * hkv + T * hq + 3 * T * H + T * I + 2 * T * I + hkv * T)
+    want = 2 * (T * H + T * (hq + 2 * hkv) + T * hq + 2 * T * hkv + T * hq + 2 * T * H + T * I + 2 * T * I + hkv * T)
     assert op.info["workspace_bytes"] == want
