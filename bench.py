@@ -83,7 +83,10 @@ def parse():
     ap.add_argument("--study", default="",
                     help="instead of the benchmark line: 'search' prints best-so-far curves (JSON lines) of the "
                          "search variants on --workload: MCTS with measured rollouts at B = 2 and 4, MCTS with the "
-                         "learned surrogate and 4x screening, and random search, over seeds --seed .. --seed+1")
+                         "learned surrogate and 4x screening, random search, and (composite ops) stage-by-stage "
+                         "tuning then a joint search, over seeds --seed .. --seed+1")
+    ap.add_argument("--study-variants", default="",
+                    help="with --study search: comma-separated variant names to run (default: all)")
     ap.add_argument("--shape", default="",
                     help="override workload sizes for a profiling case, e.g. 'tokens=1024,experts=16' (the line "
                          "then reports that shape, not the benchmark configuration)")
@@ -558,18 +561,58 @@ def random_search(op, io, samples, seed, horizon=8, batch=8):
     return curve
 
 
-def search_study(wl, io, samples, seed):
+def tasks_curve(op, io, samples, seed, joint=0.2):
+    """search_tasks' sequence of searches (one per stage, then one joint), recording every candidate:
+    returns [(samples so far, best whole-op median ms so far)]."""
+    from paper_2506_01374_gb300 import rc
+    root = op.schedule()
+    m0 = op.measure([root], io, warmup=2, repeats=5)[0]
+    S = root.num_stages
+    share = [max(m0.stage_ms[g], 1e-9) for g in range(S)]
+    alloc = [max(32, int(samples * (1.0 - joint) * x / sum(share))) for x in share]
+    curve = [(1, m0.ms_median)]
+
+    def run(search, budget):
+        res, k, pend = [], 0, False
+        while k < budget and len(curve) < samples:
+            nxt = search.step(res)
+            pend = False
+            if not nxt:
+                break
+            res = op.measure(nxt, io, warmup=2, repeats=5)
+            pend = True
+            for m in res:
+                k += 1
+                t = m.ms_median if m.status == rc.OK else float("inf")
+                curve.append((len(curve) + 1, min(curve[-1][1], t)))
+        if pend:
+            search.step(res)
+        return search.best()[0].clone()
+
+    for g in sorted(range(S), key=lambda g: -share[g]):
+        root = run(rc.Search(op, seed=seed, branching=4, surrogate=True, screen=4, stages=[g], root=root), alloc[g])
+    run(rc.Search(op, seed=seed, branching=4, surrogate=True, screen=4, root=root), samples)
+    return curve
+
+
+def search_study(wl, io, samples, seed, only=""):
     """Best-so-far (TFLOP/s of the best measured candidate) against measured samples, per search variant."""
     from paper_2506_01374_gb300 import rc
     flops = wl.op.info["flops"]
     marks = [m for m in (50, 100, 250, 500, 1000, 2000, 3000, 5000, 10000) if m <= samples] + [samples]
     variants = [("mcts_B2_measured", 2, False, 1), ("mcts_B4_measured", 4, False, 1),
                 ("mcts_B4_surrogate_screen4", 4, True, 4), ("random", 0, False, 1)]
+    if wl.op.schedule().num_stages > 1:
+        variants.append(("tasks_then_joint_B4_surrogate_screen4", 4, True, 4))
+    if only:
+        variants = [v for v in variants if v[0] in only.split(",")]
     for sd in (seed, seed + 1):
         for name, B, sur, scr in variants:
             t0 = time.perf_counter()
             if name == "random":
                 curve = random_search(wl.op, io, samples, sd)
+            elif name.startswith("tasks"):
+                curve = tasks_curve(wl.op, io, samples, sd)
             else:
                 search = rc.Search(wl.op, seed=sd, branching=B, surrogate=sur, screen=scr)
                 res, n, curve, best = [], 0, [], float("inf")
@@ -617,6 +660,22 @@ def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False,
         del io, wl
         torch.cuda.empty_cache()
     return out
+
+
+def max_over_ranks(vals, world, device):
+    """Element-wise maximum of per-rank values over all ranks (the slowest rank's times); one rank: as is."""
+    if world <= 1:
+        return list(vals)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(vals, device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_tflops(world, flops_per_rank, seconds):
+    """Whole-job throughput of `world` replicas that each did `flops_per_rank` in `seconds` (the max over ranks)."""
+    return world * flops_per_rank / seconds / 1e12
 
 
 def dist_setup():
@@ -682,7 +741,7 @@ def run_ours(args):
 
     wl = Workload(args.workload, parse_shape(args.shape))
     if args.study == "search":
-        search_study(wl, wl.device_io(), args.samples, args.seed)
+        search_study(wl, wl.device_io(), args.samples, args.seed, args.study_variants)
         return
     if args.study:
         raise SystemExit(f"unknown --study {args.study}")
@@ -730,11 +789,8 @@ def run_ours(args):
     clk = clocks.stop()
     ms = statistics.fmean(step_ms)
     ms_dom = statistics.fmean(dom_ms)
-    if world > 1:
-        t = torch.tensor([ms, ms_dom], device="cuda", dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, ms_dom = t.tolist()
-    value = world * info["flops"] / (ms * 1e-3) / 1e12
+    ms, ms_dom = max_over_ranks([ms, ms_dom], world, "cuda")
+    value = job_tflops(world, info["flops"], ms * 1e-3)
 
     # 3) end to end through the host-buffer entry point
     e2e_s = None
@@ -747,11 +803,7 @@ def run_ours(args):
             t0 = time.perf_counter()
             op.run_host(best, host_io)
             e2e_t.append(time.perf_counter() - t0)
-        e2e_s = statistics.fmean(e2e_t)
-        if world > 1:
-            t = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e2e_s = t.item()
+        e2e_s = max_over_ranks([statistics.fmean(e2e_t)], world, "cuda")[0]
     h2d, d2h = wl.io_bytes()
 
     if rank == 0:
@@ -778,7 +830,7 @@ def run_ours(args):
                        "screen": args.screen,
                        "best_search_tflops": best_m.tflops if best_m else None,
                        "stats": search.stats() if search else None},
-            "e2e": None if e2e_s is None else {"value": world * info["flops"] / e2e_s / 1e12, "unit": "TFLOP/s",
+            "e2e": None if e2e_s is None else {"value": job_tflops(world, info["flops"], e2e_s), "unit": "TFLOP/s",
                                                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": args.steps * launches_per_step(args.workload, best),
             "clocks": clk,

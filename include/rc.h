@@ -334,7 +334,8 @@ typedef struct {
 
 /* Create an LLM-free MCTS search over op's schedule space (Sec. 3.2 with the
  * random-valid expansion policy the paper falls back to, App. G). opts NULL
- * = defaults. The first rc_search_step call returns the root P0 to measure. */
+ * = defaults. The first rc_search_step call returns the root (P0, or opts->root)
+ * to measure. */
 rc_status rc_search_create(const rc_op* op, const rc_search_opts* opts, rc_search** out);
 
 /* One search iteration. results[0..n_results) are the measurements of the
@@ -362,7 +363,8 @@ typedef struct {
 } rc_search_stats;
 rc_status rc_search_get_stats(const rc_search* s, rc_search_stats* st);
 /* The surrogate's predicted device time (ms) of a schedule of the search's
- * op: the sum over stages of exp(w . x_stage) (per-stage models) or
+ * op: the sum over stages of exp(w . x_stage) (per-stage models; with a
+ * stage_mask, over the selected stages only: the search's objective) or
  * exp(w . x) (one model). RC_ERR_INVALID_ARG when the surrogate is off or not
  * fitted yet. Deterministic given the measurement sequence. */
 rc_status rc_search_predict(rc_search* s, const rc_schedule* sched, double* ms);
