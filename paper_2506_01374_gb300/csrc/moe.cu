@@ -7,12 +7,15 @@
 //      (logit descending, expert id ascending) by comparing the widened
 //      logits only. Weights w_j = exp(l_j - max) / z, renormalised over the k
 //      picks when requested.
-//   2) route_count: one CTA per expert counts the tokens routed to it.
+//   2) route_count: each CTA histograms 4096 slots' expert ids in shared
+//      memory and adds its non-zero bins to the per-expert counts (integer
+//      atomics: the totals do not depend on their order).
 //   3) route_permute: one CTA per expert takes the exclusive prefix of the
-//      counts as its offset and ranks its tokens in token order with a
-//      block-wide ballot scan, so slot s = t*k + j lands at
-//      perm[offset[e] + rank] - the (expert, token, j) order - with no
-//      dependence on thread timing.
+//      counts as its offset and ranks its tokens in token order: each thread
+//      takes 4 consecutive tokens (all their ids loaded up front), and a
+//      block-wide exclusive scan of the per-thread hits gives the ranks, so
+//      slot s = t*k + j lands at perm[offset[e] + rank] - the (expert,
+//      token, j) order - with no dependence on thread timing.
 // Gather: Xp[pos] = X[perm[pos] / k], 16-byte vectors, one warp per row.
 // Combine: out[t] = sum_{j<k} w[t,j] * Y[inv_perm[t*k+j]] in fp32, in j order,
 //   rounded once to bf16.
@@ -108,56 +111,86 @@ __global__ void route_topk_kernel(const void* __restrict__ logits, int T, int E,
   }
 }
 
-__device__ __forceinline__ bool routes_to(const int* __restrict__ ids, int t, int K, int e, int* jpos) {
-  for (int j = 0; j < K; ++j)
-    if (ids[(size_t)t * K + j] == e) {
-      *jpos = j;
-      return true;
-    }
-  return false;
-}
+constexpr int kCountThreads = 256;
+constexpr int kCountSlots = 16;  // slots per thread
 
-__global__ void route_count_kernel(const int* __restrict__ ids, int T, int K, int* __restrict__ counts) {
-  const int e = blockIdx.x;
-  int c = 0;
-  for (int t = threadIdx.x; t < T; t += blockDim.x) {
-    int j;
-    c += routes_to(ids, t, K, e, &j) ? 1 : 0;
+__global__ void __launch_bounds__(kCountThreads)
+    route_count_kernel(const int* __restrict__ ids, int slots, int E, int* __restrict__ counts) {
+  __shared__ int hist[kMaxE];
+  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
+  __syncthreads();
+  const int s0 = blockIdx.x * (kCountThreads * kCountSlots);
+  int id[kCountSlots];
+#pragma unroll
+  for (int q = 0; q < kCountSlots; ++q) {  // loads first, coalesced across the CTA
+    const int s = s0 + q * kCountThreads + threadIdx.x;
+    id[q] = s < slots ? ids[s] : -1;
   }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-  __shared__ int part[32];
-  if (threadIdx.x % 32 == 0) part[threadIdx.x / 32] = c;
+  for (int q = 0; q < kCountSlots; ++q)
+    if (id[q] >= 0) atomicAdd(&hist[id[q]], 1);
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int s = 0;
-    for (int i = 0; i < (int)(blockDim.x / 32); ++i) s += part[i];
-    counts[e] = s;
-  }
+  for (int e = threadIdx.x; e < E; e += blockDim.x)
+    if (hist[e]) atomicAdd(&counts[e], hist[e]);
 }
 
-__global__ void route_permute_kernel(const int* __restrict__ ids, int T, int K, int E,
-                                     const int* __restrict__ counts, int* __restrict__ offsets,
-                                     int* __restrict__ perm, int* __restrict__ inv_perm) {
+constexpr int kPermThreads = 1024;
+constexpr int kPermTokens = 4;  // consecutive tokens per thread and chunk
+
+__global__ void __launch_bounds__(kPermThreads)
+    route_permute_kernel(const int* __restrict__ ids, int T, int K, int E, const int* __restrict__ counts,
+                         int* __restrict__ offsets, int* __restrict__ perm, int* __restrict__ inv_perm) {
   const int e = blockIdx.x;
   __shared__ int base_s;
-  __shared__ int warp_tot[32];
-  if (threadIdx.x == 0) {
-    int off = 0;
-    for (int i = 0; i < e; ++i) off += counts[i];
-    base_s = off;
-    offsets[e] = off;
-    if (e == E - 1) offsets[E] = off + counts[e];
+  __shared__ int warp_tot[kPermThreads / 32];
+  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32, nw = blockDim.x / 32;
+  if (warp == 0) {  // offset of e = sum of the counts before it; all E counts loaded at once
+    int before = 0, mine = 0;
+#pragma unroll
+    for (int r = 0; r < kMaxPerLane; ++r) {
+      const int i = lane + 32 * r;
+      const int c = i < E ? counts[i] : 0;
+      before += i < e ? c : 0;
+      mine += i == e ? c : 0;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      before += __shfl_xor_sync(0xffffffffu, before, o);
+      mine += __shfl_xor_sync(0xffffffffu, mine, o);
+    }
+    if (lane == 0) {
+      base_s = before;
+      offsets[e] = before;
+      if (e == E - 1) offsets[E] = before + mine;
+    }
   }
   __syncthreads();
   int running = base_s;
-  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32, nw = blockDim.x / 32;
-  for (int t0 = 0; t0 < T; t0 += blockDim.x) {
-    const int t = t0 + threadIdx.x;
-    int j = 0;
-    const bool in = t < T && routes_to(ids, t, K, e, &j);
-    const unsigned bal = __ballot_sync(0xffffffffu, in);
-    if (lane == 0) warp_tot[warp] = __popc(bal);
+  for (int c0 = 0; c0 < T; c0 += blockDim.x * kPermTokens) {
+    const int tb = c0 + threadIdx.x * kPermTokens;
+    // which of this thread's tokens route to e, and at which pick j (ids of a token are distinct);
+    // every id is loaded unconditionally so that the loads are in flight together
+    int jpos[kPermTokens];
+    int cnt = 0;
+#pragma unroll
+    for (int q = 0; q < kPermTokens; ++q) {
+      jpos[q] = -1;
+      const int t = tb + q;
+      if (t < T) {
+#pragma unroll
+        for (int j = 0; j < kMaxK; ++j)  // unrolled to the bound: all K loads in flight at once
+          if (j < K && ids[(size_t)t * K + j] == e) jpos[q] = j;
+      }
+      cnt += jpos[q] >= 0 ? 1 : 0;
+    }
+    // block-wide exclusive scan of the hit counts, in thread (= token) order
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    if (lane == 31) warp_tot[warp] = incl;
     __syncthreads();
     int before = 0, total = 0;
     for (int i = 0; i < nw; ++i) {
@@ -165,14 +198,17 @@ __global__ void route_permute_kernel(const int* __restrict__ ids, int T, int K, 
       before += i < warp ? c : 0;
       total += c;
     }
-    if (in) {
-      const int pos = running + before + __popc(bal & ((1u << lane) - 1u));
-      const int slot = t * K + j;
+    int pos = running + before + incl - cnt;
+#pragma unroll
+    for (int q = 0; q < kPermTokens; ++q) {
+      if (jpos[q] < 0) continue;
+      const int slot = (tb + q) * K + jpos[q];
       perm[pos] = slot;
       if (inv_perm) inv_perm[slot] = pos;
+      ++pos;
     }
     running += total;
-    __syncthreads();
+    __syncthreads();  // warp_tot is rewritten by the next chunk
   }
 }
 
@@ -236,18 +272,22 @@ rc_status rc_launch_moe_route(const rc_knobs& k, const rc_op_desc& d, const void
                               int* offsets, int* perm, int* inv_perm, int* counts, const LaunchCtx& c) {
   const int T = (int)d.tokens, E = (int)d.experts, K = (int)d.top_k;
   if (E > kMaxE || K > kMaxK || K > E) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: E <= 256, k <= 16");
-  if ((int64_t)T * K > 0x7fffffff) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: too many slots");
+  if ((int64_t)T * K > 0x7fffffff - 8192 || T > (1 << 30)) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: too many slots");
   cudaStream_t st = (cudaStream_t)c.stream;
   const int warps = k.tile_m > 0 ? k.tile_m : 4;
   const int blocks = (T + warps - 1) / warps;
+  cudaError_t me = cudaMemsetAsync(counts, 0, sizeof(int) * (size_t)E, st);
+  if (me != cudaSuccess) return rc_fail(RC_ERR_CUDA, "routing counts memset: %s", cudaGetErrorString(me));
   if (d.logits_fp32)
     route_topk_kernel<true><<<blocks, 32 * warps, 0, st>>>(logits, T, E, K, d.renorm, ids, w);
   else
     route_topk_kernel<false><<<blocks, 32 * warps, 0, st>>>(logits, T, E, K, d.renorm, ids, w);
   RC_TRY(launched("route_topk"));
-  route_count_kernel<<<E, 256, 0, st>>>(ids, T, K, counts);
+  const int slots = T * K;
+  const int cblocks = (slots + kCountThreads * kCountSlots - 1) / (kCountThreads * kCountSlots);
+  route_count_kernel<<<cblocks > 0 ? cblocks : 1, kCountThreads, 0, st>>>(ids, slots, E, counts);
   RC_TRY(launched("route_count"));
-  route_permute_kernel<<<E, 256, 0, st>>>(ids, T, K, E, counts, offsets, perm, inv_perm);
+  route_permute_kernel<<<E, kPermThreads, 0, st>>>(ids, T, K, E, counts, offsets, perm, inv_perm);
   return launched("route_permute");
 }
 
