@@ -11,11 +11,11 @@
 //      memory and adds its non-zero bins to the per-expert counts (integer
 //      atomics: the totals do not depend on their order).
 //   3) route_permute: one CTA per expert takes the exclusive prefix of the
-//      counts as its offset and ranks its tokens in token order: each thread
-//      takes 4 consecutive tokens (all their ids loaded up front), and a
-//      block-wide exclusive scan of the per-thread hits gives the ranks, so
-//      slot s = t*k + j lands at perm[offset[e] + rank] - the (expert,
-//      token, j) order - with no dependence on thread timing.
+//      counts as its offset and ranks the slots whose id is e in slot order
+//      (coalesced striped loads, warp ballots, one block-wide scan of the
+//      per-warp hit counts per chunk), so slot s = t*k + j lands at
+//      perm[offset[e] + rank] - the (expert, token, j) order - with no
+//      dependence on thread timing.
 // Gather: Xp[pos] = X[perm[pos] / k], 16-byte vectors, one warp per row.
 // Combine: out[t] = sum_{j<k} w[t,j] * Y[inv_perm[t*k+j]] in fp32, in j order,
 //   rounded once to bf16.
@@ -134,16 +134,22 @@ __global__ void __launch_bounds__(kCountThreads)
     if (hist[e]) atomicAdd(&counts[e], hist[e]);
 }
 
-constexpr int kPermThreads = 1024;
-constexpr int kPermTokens = 4;  // consecutive tokens per thread and chunk
+constexpr int kPermThreads = 1024;  // 32 warps
+constexpr int kPermRounds = 16;     // slots per thread and chunk: a chunk is 16384 consecutive slots
 
+// Slots are read striped (slot c0 + q*1024 + warp*32 + lane), so every load is
+// coalesced. A slot is a hit when its id is e; since a token's k ids are
+// distinct, ranking hits by slot index ranks them by token.
 __global__ void __launch_bounds__(kPermThreads)
     route_permute_kernel(const int* __restrict__ ids, int T, int K, int E, const int* __restrict__ counts,
                          int* __restrict__ offsets, int* __restrict__ perm, int* __restrict__ inv_perm) {
+  constexpr int NW = kPermThreads / 32;
+  constexpr int NV = kPermRounds * NW;  // per-(round, warp) hit counts of a chunk
   const int e = blockIdx.x;
   __shared__ int base_s;
-  __shared__ int warp_tot[kPermThreads / 32];
-  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32, nw = blockDim.x / 32;
+  __shared__ int scan[NV];
+  __shared__ int warp_tot[NW];
+  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
   if (warp == 0) {  // offset of e = sum of the counts before it; all E counts loaded at once
     int before = 0, mine = 0;
 #pragma unroll
@@ -166,25 +172,25 @@ __global__ void __launch_bounds__(kPermThreads)
   }
   __syncthreads();
   int running = base_s;
-  for (int c0 = 0; c0 < T; c0 += blockDim.x * kPermTokens) {
-    const int tb = c0 + threadIdx.x * kPermTokens;
-    // which of this thread's tokens route to e, and at which pick j (ids of a token are distinct);
-    // every id is loaded unconditionally so that the loads are in flight together
-    int jpos[kPermTokens];
-    int cnt = 0;
+  const int slots = T * K;
+  for (int c0 = 0; c0 < slots; c0 += kPermThreads * kPermRounds) {
+    int v[kPermRounds];
 #pragma unroll
-    for (int q = 0; q < kPermTokens; ++q) {
-      jpos[q] = -1;
-      const int t = tb + q;
-      if (t < T) {
-#pragma unroll
-        for (int j = 0; j < kMaxK; ++j)  // unrolled to the bound: all K loads in flight at once
-          if (j < K && ids[(size_t)t * K + j] == e) jpos[q] = j;
-      }
-      cnt += jpos[q] >= 0 ? 1 : 0;
+    for (int q = 0; q < kPermRounds; ++q) {  // every load of the chunk in flight before any use
+      const int sl = c0 + q * kPermThreads + warp * 32 + lane;
+      v[q] = sl < slots ? ids[sl] : -1;
     }
-    // block-wide exclusive scan of the hit counts, in thread (= token) order
-    int incl = cnt;
+    unsigned bal[kPermRounds];
+#pragma unroll
+    for (int q = 0; q < kPermRounds; ++q) bal[q] = __ballot_sync(0xffffffffu, v[q] == e);
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < kPermRounds; ++q) scan[q * NW + warp] = __popc(bal[q]);
+    }
+    __syncthreads();
+    // exclusive scan of the NV counts in (round, warp) order = slot order, one count per thread
+    const int x = threadIdx.x < NV ? scan[threadIdx.x] : 0;
+    int incl = x;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int n = __shfl_up_sync(0xffffffffu, incl, o);
@@ -193,22 +199,24 @@ __global__ void __launch_bounds__(kPermThreads)
     if (lane == 31) warp_tot[warp] = incl;
     __syncthreads();
     int before = 0, total = 0;
-    for (int i = 0; i < nw; ++i) {
+    for (int i = 0; i < NW; ++i) {
       const int c = warp_tot[i];
       before += i < warp ? c : 0;
       total += c;
     }
-    int pos = running + before + incl - cnt;
+    __syncthreads();  // every thread has its count and the warp totals before scan[] is overwritten
+    if (threadIdx.x < NV) scan[threadIdx.x] = before + incl - x;
+    __syncthreads();
 #pragma unroll
-    for (int q = 0; q < kPermTokens; ++q) {
-      if (jpos[q] < 0) continue;
-      const int slot = (tb + q) * K + jpos[q];
-      perm[pos] = slot;
-      if (inv_perm) inv_perm[slot] = pos;
-      ++pos;
+    for (int q = 0; q < kPermRounds; ++q) {
+      if (!((bal[q] >> lane) & 1u)) continue;
+      const int sl = c0 + q * kPermThreads + warp * 32 + lane;
+      const int pos = running + scan[q * NW + warp] + __popc(bal[q] & ((1u << lane) - 1u));
+      perm[pos] = sl;
+      if (inv_perm) inv_perm[sl] = pos;
     }
     running += total;
-    __syncthreads();  // warp_tot is rewritten by the next chunk
+    __syncthreads();  // scan[] and warp_tot[] are rewritten by the next chunk
   }
 }
 
@@ -272,7 +280,7 @@ rc_status rc_launch_moe_route(const rc_knobs& k, const rc_op_desc& d, const void
                               int* offsets, int* perm, int* inv_perm, int* counts, const LaunchCtx& c) {
   const int T = (int)d.tokens, E = (int)d.experts, K = (int)d.top_k;
   if (E > kMaxE || K > kMaxK || K > E) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: E <= 256, k <= 16");
-  if ((int64_t)T * K > 0x7fffffff - 8192 || T > (1 << 30)) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: too many slots");
+  if ((int64_t)T * K > 0x7fffffff - 32768) return rc_fail(RC_ERR_UNSUPPORTED_OP, "routing: too many slots");
   cudaStream_t st = (cudaStream_t)c.stream;
   const int warps = k.tile_m > 0 ? k.tile_m : 4;
   const int blocks = (T + warps - 1) / warps;
