@@ -1,0 +1,121 @@
+"""Host logic of bench.py that needs no GPU: schedule text round trips, the
+stage-by-stage search driver on a synthetic separable landscape, and the
+launch counts the bench reports."""
+import math
+import os
+import random
+import sys
+
+import pytest
+
+from paper_2506_01374_gb300 import rc
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def _ops():
+    return [rc.Op(rc.OP_GEMM_F32, m=256, n=256, k=256, flags=rc.EPI_BIAS | rc.EPI_RELU),
+            rc.Op(rc.OP_MLP, m=2048, n=14336, k=4096),
+            rc.Op(rc.OP_ATTENTION, batch=1, seq=2048, heads_q=32, heads_kv=8, head_dim=128, causal=1),
+            rc.Op(rc.OP_CONV2D, img_n=2, img_h=64, img_w=64, c_in=320, c_out=320, kr=3, ks=3, stride=1, pad=1,
+                  flags=rc.EPI_BIAS | rc.EPI_SILU),
+            rc.Op(rc.OP_MOE, tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8),
+            rc.Op(rc.OP_DECODER_LAYER, tokens=2048, hidden=4096, inter=14336, heads_q=32, heads_kv=8,
+                  head_dim=128)]
+
+
+def _random_schedule(op, rng, n=12):
+    space = op.transform_space()
+    s = op.schedule()
+    for _ in range(n):
+        t = space[rng.randrange(len(space))]
+        try:
+            s = op.schedule(t, base=s)
+        except rc.RcError:
+            pass
+    return s
+
+
+def test_canonical_schedule_text_round_trips_through_parse_schedule():
+    rng = random.Random(5)
+    for op in _ops():
+        for _ in range(25):
+            s = _random_schedule(op, rng)
+            back = bench.parse_schedule(op, str(s), rc)
+            assert back.hash == s.hash and str(back) == str(s)
+
+
+class _SeparableOp:
+    """An op whose device time is a sum of per-stage times, each a function of that stage's knobs."""
+
+    def __init__(self, op):
+        self.op = op
+        self.h = op.h
+
+    def __getattr__(self, name):
+        return getattr(self.op, name)
+
+    @staticmethod
+    def stage_ms(g, k):
+        t = 1.0 + g
+        t *= {32: 1.9, 64: 1.4, 128: 1.0, 224: 0.93, 256: 0.9}.get(k["tile_n"], 1.2)
+        t *= 0.8 if k["tile_m"] == 256 else 1.0
+        t *= {1: 1.7, 2: 1.2, 3: 1.0, 4: 1.02, 6: 1.1}.get(k["stages"], 1.05)
+        t *= 0.85 if k["fuse"] else 1.0
+        return t
+
+    def measure(self, scheds, io, **kw):
+        out = []
+        for s in scheds:
+            m = rc.Measurement()
+            m.status = rc.OK
+            m.n_stages = s.num_stages
+            for g in range(s.num_stages):
+                m.stage_ms[g] = self.stage_ms(g, s.knobs(g))
+            m.ms_median = sum(m.stage_ms[g] for g in range(s.num_stages))
+            out.append(m)
+        return out
+
+
+def test_stage_by_stage_driver_reaches_each_stage_optimum_within_budget():
+    op = _SeparableOp(rc.Op(rc.OP_MLP, m=2048, n=14336, k=4096))
+    search, best, m, n, cps, tasks = bench.search_tasks(op, None, 1500, seed=1, surrogate=True, screen=4)
+    assert [t["stage"] for t in tasks] == [1, 0]  # the larger stage of P0 first
+    assert n <= 1500 + 64  # the budget, up to the last batch and the final re-timing
+    # each stage of the result is as fast as that stage can be on this landscape
+    for g in range(2):
+        space_best = min(op.stage_ms(g, s.knobs(g)) for s in _stage_programs(op.op, g))
+        assert m.stage_ms[g] == pytest.approx(space_best)
+    assert m.ms_median == pytest.approx(sum(m.stage_ms[g] for g in range(2)))
+
+
+def _stage_programs(op, g):
+    """Every legal program that differs from P0 in stage g only (enumerated knob by knob)."""
+    space = [t for t in op.transform_space() if t.stage == g]
+    seen, frontier = {}, [op.schedule()]
+    while frontier:
+        s = frontier.pop()
+        if s.hash in seen:
+            continue
+        seen[s.hash] = s
+        for t in space:
+            try:
+                frontier.append(op.schedule(t, base=s))
+            except rc.RcError:
+                pass
+    return list(seen.values())
+
+
+def test_launch_counts_follow_the_schedule():
+    mlp = rc.Op(rc.OP_MLP, m=2048, n=14336, k=4096)
+    assert bench.launches_per_step("mlp", mlp.schedule()) == 2 + 1  # unfused gate/up + SwiGLU pass, down
+    fused = mlp.schedule(rc.T(rc.T_FUSE, 1, stage=0), rc.T(rc.T_SPLIT_K, 2, stage=1))
+    assert bench.launches_per_step("mlp", fused) == 1 + 2  # fused gate/up, split-K down + reduce
+    dec = _ops()[-1]
+    # RMSNorm, QKV, RoPE, V transpose + attention, O, RMSNorm, gate/up + SwiGLU pass, down
+    assert bench.launches_per_step("decoder_layer", dec.schedule()) == 10
+    tuned = dec.schedule(rc.T(rc.T_LAYOUT, 0, stage=2), rc.T(rc.T_FUSE, 1, stage=4))
+    assert bench.launches_per_step("decoder_layer", tuned) == 8
+    assert math.isclose(bench.job_tflops(4, 2e12, 0.5), 16.0)
