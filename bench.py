@@ -318,13 +318,32 @@ class Workload:
         d2h = sum(int(np.prod(s)) * np.dtype(dt).itemsize for s, dt in self.outs.values())
         return h2d, d2h
 
-    def cpu_sample(self, n):
-        """Time the fp64 oracle on a bounded sample; returns the cpu_baseline dict."""
+    def cpu_sample(self, n, single_thread=True):
+        """Time the fp64 oracle on a bounded sample with all its threads; returns the cpu_baseline dict.
+
+        single_thread: also time a sample 1/threads the size with one thread (the oracle's
+        results do not depend on its thread count), reported under "single_thread". The decoder
+        layer's numpy matrix product is threaded by numpy's BLAS, outside the oracle's control,
+        so it gets no single-thread figure."""
+        import oracle
+        oracle.build()
+        out = self._oracle_sample(n)
+        if single_thread and self.name != "decoder_layer":
+            prev = oracle.threads()
+            oracle.threads(1)
+            try:
+                one = self._oracle_sample(max(1, out["n"] // max(1, prev)))
+            finally:
+                oracle.threads(prev)
+            out["single_thread"] = {"value": one["value"], "sample": one["sample"], "seconds": one["seconds"]}
+        out.pop("n")
+        return out
+
+    def _oracle_sample(self, n):
         import numpy as np
 
         import oracle
-        oracle.build()
-        cores = os.cpu_count() or 1
+        cores = oracle.threads()
         if self.name == "mlp":
             X, W1, W2 = self.host[:3]
             n = n or 2048
@@ -394,7 +413,7 @@ class Workload:
         if self.name != "decoder_layer":
             what += ", fp64 loop nests"
         return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": used, "kind": "oracle",
-                "sample": what, "seconds": dt}
+                "sample": what, "seconds": dt, "n": n}
 
 
 def parse_shape(text):
@@ -694,8 +713,8 @@ def run_reference(args):
                                                      "gemm_f32": 4, "attention_flux": 16,
                                                      "decoder_layer": 8}[args.workload]
     for _ in range(args.warmup):
-        wl.cpu_sample(n)
-    samples = [wl.cpu_sample(n) for _ in range(args.steps)]
+        wl.cpu_sample(n, single_thread=False)
+    samples = [wl.cpu_sample(n, single_thread=False) for _ in range(args.steps)]
     secs = statistics.fmean(s["seconds"] for s in samples)
     val = statistics.fmean(s["value"] for s in samples)
     cb = {k: v for k, v in samples[0].items() if k != "seconds"}

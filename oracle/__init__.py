@@ -71,6 +71,13 @@ def _rows(rows):
     return None if rows is None else _c(rows, np.int64)
 
 
+def threads(n=0):
+    """Thread count of the oracle's OpenMP loops; n > 0 sets it. Results do not depend on it."""
+    lib = _load()
+    lib.oracle_threads.restype = ctypes.c_int
+    return int(lib.oracle_threads(ctypes.c_int(int(n))))
+
+
 def gemm_bias_relu_f32(A, B, bias=None, relu=True):
     """K0: C = max(0, A B + bias) in fp64 (App. A loop nest plus bias/ReLU). A[M,K], B[K,N]."""
     A = _c(A, np.float32)

@@ -23,7 +23,23 @@
 #include <stdlib.h>
 #include <string.h>
 
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
 #define EXPORT __attribute__((visibility("default")))
+
+/* Thread count of the OpenMP loops (n > 0 sets it); returns the count now in
+ * effect, 1 when built without OpenMP. Results do not depend on it. */
+EXPORT int oracle_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+  return omp_get_max_threads();
+#else
+  (void)n;
+  return 1;
+#endif
+}
 
 static double bf(uint16_t b) {
   uint32_t u = (uint32_t)b << 16;

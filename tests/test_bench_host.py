@@ -119,3 +119,17 @@ def test_launch_counts_follow_the_schedule():
     tuned = dec.schedule(rc.T(rc.T_LAYOUT, 0, stage=2), rc.T(rc.T_FUSE, 1, stage=4))
     assert bench.launches_per_step("decoder_layer", tuned) == 8
     assert math.isclose(bench.job_tflops(4, 2e12, 0.5), 16.0)
+
+
+def test_cpu_baseline_reports_all_threads_and_one_thread():
+    import oracle
+    wl = bench.Workload("mlp", {"tokens": 64, "hidden": 256, "inter": 256})
+    before = oracle.threads()
+    cb = wl.cpu_sample(32)
+    assert oracle.threads() == before  # the one-thread leg restores the thread count
+    assert cb["kind"] == "oracle" and cb["value"] > 0 and cb["cores"] == min(before, 32)
+    assert "32 of 64 token rows" in cb["sample"] and "n" not in cb
+    one = cb["single_thread"]
+    assert one["value"] > 0 and f"{max(1, 32 // before)} of 64 token rows" in one["sample"]
+    ref = bench.Workload("attention", {"seq": 64, "heads_q": 2, "heads_kv": 1}).cpu_sample(8, single_thread=False)
+    assert "single_thread" not in ref and "8 of 64 query positions" in ref["sample"]
