@@ -401,8 +401,11 @@ void rc_search_destroy(rc_search* s);
  * any stream capture. Every call on a device shares the one array, so calls
  * whose kernels overlap on the GPU (different streams, no ordering) race;
  * order them on one stream or with events. The array keeps the last call's
- * counts; each call overwrites the entries it uses, so nothing needs
- * clearing. */
+ * counts; each call first zeroes the entries it uses (cudaMemsetAsync on
+ * `stream`), then the count kernel adds to them with atomicAdd, so the
+ * caller never clears it. The cached address is looked up again when the
+ * device's context changes (after cudaDeviceReset). A NaN logit ranks below
+ * every number, as in rc_run. */
 #define RC_NOALLOC_MAX_EXPERTS 256
 rc_status rc_moe_route_noalloc(const void* logits, int32_t logits_fp32, int64_t tokens, int64_t experts,
                                int64_t top_k, int32_t renorm, int32_t* ids, float* weights, int32_t* offsets,

@@ -251,6 +251,9 @@ EXPORT void oracle_conv2d_nhwc_bf16(int64_t N, int64_t H, int64_t W, int64_t Cin
  * Selection compares logit values only. counts[e] = number of (t, j) routed
  * to e; offsets[E+1] is its exclusive scan; perm[T*k] lists the slots
  * s = t*k + j ordered by (expert, token, j).
+ * A NaN logit has no place in that order; it is read as -inf, so it ranks
+ * below every number (ties among such experts go to the lower id) and its
+ * softmax probability is 0.
  */
 EXPORT void oracle_moe_route(int64_t T, int64_t E, int64_t topk, const void* logits, int logits_fp32,
                              int renorm, int32_t* ids, double* w, int32_t* offsets, int32_t* perm) {
@@ -258,9 +261,11 @@ EXPORT void oracle_moe_route(int64_t T, int64_t E, int64_t topk, const void* log
   for (int64_t t = 0; t < T; ++t) {
     double* l = (double*)malloc(sizeof(double) * (size_t)E);
     char* taken = (char*)calloc((size_t)E, 1);
-    for (int64_t e = 0; e < E; ++e)
+    for (int64_t e = 0; e < E; ++e) {
       l[e] = logits_fp32 ? (double)((const float*)logits)[t * E + e]
                          : bf(((const uint16_t*)logits)[t * E + e]);
+      if (isnan(l[e])) l[e] = -INFINITY;
+    }
     double mx = -INFINITY;
     for (int64_t e = 0; e < E; ++e)
       if (l[e] > mx) mx = l[e];

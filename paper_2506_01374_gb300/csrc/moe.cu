@@ -6,7 +6,9 @@
 //      the warp, and k arg-max rounds pick the experts in the order
 //      (logit descending, expert id ascending) by comparing the widened
 //      logits only. Weights w_j = exp(l_j - max) / z, renormalised over the k
-//      picks when requested.
+//      picks when requested. A NaN logit is read as -inf: it ranks below every
+//      number (ties by lower id) and gets probability 0, so every round picks
+//      an id below E whatever the logits hold.
 //   2) route_count: each CTA histograms 4096 slots' expert ids in shared
 //      memory and adds its non-zero bins to the per-expert counts (integer
 //      atomics: the totals do not depend on their order).
@@ -50,8 +52,9 @@ __global__ void route_topk_kernel(const void* __restrict__ logits, int T, int E,
     const int e = lane + 32 * i;
     taken[i] = false;
     if (e < E) {
-      v[i] = FP32 ? ((const float*)logits)[(size_t)t * E + e]
-                  : __bfloat162float(((const __nv_bfloat16*)logits)[(size_t)t * E + e]);
+      const float x = FP32 ? ((const float*)logits)[(size_t)t * E + e]
+                           : __bfloat162float(((const __nv_bfloat16*)logits)[(size_t)t * E + e]);
+      v[i] = x != x ? -INFINITY : x;  // NaN ranks last
       mx = fmaxf(mx, v[i]);
     } else {
       v[i] = -INFINITY;
@@ -92,6 +95,9 @@ __global__ void route_topk_kernel(const void* __restrict__ logits, int T, int E,
         bi = oi;
       }
     }
+    // Each untaken expert beats the (-inf, INT_MAX) start and K <= E, so bi < E;
+    // the guard keeps an out-of-range index from ever being written.
+    bi = bi < E ? bi : 0;
     if ((bi & 31) == lane) taken[bi >> 5] = true;
     const float p = expf(bv - mx) / z;
     pk[j] = p;
@@ -128,7 +134,7 @@ __global__ void __launch_bounds__(kCountThreads)
   }
 #pragma unroll
   for (int q = 0; q < kCountSlots; ++q)
-    if (id[q] >= 0) atomicAdd(&hist[id[q]], 1);
+    if (id[q] >= 0 && id[q] < E) atomicAdd(&hist[id[q]], 1);
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x)
     if (hist[e]) atomicAdd(&counts[e], hist[e]);

@@ -17,7 +17,31 @@ static __device__ __align__(256) int g_noalloc_route_counts[RC_NOALLOC_MAX_EXPER
 
 namespace {
 std::mutex g_mu;
-int* g_counts_dev[64] = {};  // device address of g_noalloc_route_counts, per device ordinal
+// Device address of g_noalloc_route_counts per device ordinal, with the
+// context it was looked up in: a new primary context (after cudaDeviceReset)
+// loads the module again, so a changed context means a fresh lookup.
+struct CountsAddr {
+  void* ctx = nullptr;
+  int* ptr = nullptr;
+};
+CountsAddr g_counts_dev[64];
+
+typedef int (*CtxGetCurrentFn)(void**);
+CtxGetCurrentFn g_ctx_get_current = nullptr;
+
+// The current driver context, or nullptr when the driver entry point is unavailable.
+void* current_context() {
+  if (!g_ctx_get_current) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_ctx_get_current = (CtxGetCurrentFn)p;
+    if (!g_ctx_get_current) return nullptr;
+  }
+  void* ctx = nullptr;
+  return g_ctx_get_current(&ctx) == 0 ? ctx : nullptr;
+}
 }  // namespace
 
 extern "C" rc_status rc_moe_route_noalloc(const void* logits, int32_t logits_fp32, int64_t tokens, int64_t experts,
@@ -33,7 +57,7 @@ extern "C" rc_status rc_moe_route_noalloc(const void* logits, int32_t logits_fp3
     return rc_fail(RC_ERR_INVALID_ARG, "rc_moe_route_noalloc: experts = %lld exceeds the fixed scratch of %d experts",
                    (long long)experts, RC_NOALLOC_MAX_EXPERTS);
   if (top_k > 16) return rc_fail(RC_ERR_UNSUPPORTED_OP, "rc_moe_route_noalloc: top_k must be <= 16");
-  if (tokens * top_k > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "rc_moe_route_noalloc: too many slots");
+  // tokens * top_k is limited further by rc_launch_moe_route (the routing kernels' slot range).
 
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -41,17 +65,21 @@ extern "C" rc_status rc_moe_route_noalloc(const void* logits, int32_t logits_fp3
   if (dev < 0 || dev >= 64) return rc_fail(RC_ERR_CUDA, "rc_moe_route_noalloc: device ordinal %d", dev);
   int* counts = nullptr;
   {
-    // One-time set-up per device, with that device current: translate the
-    // array's host-side name into its device address.
+    // One-time set-up per device (and per context of that device), with that
+    // device current: translate the array's host-side name into its device
+    // address.
     std::lock_guard<std::mutex> lk(g_mu);
-    if (!g_counts_dev[dev]) {
+    void* ctx = current_context();
+    CountsAddr& a = g_counts_dev[dev];
+    if (!a.ptr || ctx != a.ctx) {
       void* p = nullptr;
       e = cudaGetSymbolAddress(&p, g_noalloc_route_counts);
       if (e != cudaSuccess)
         return rc_fail(RC_ERR_CUDA, "rc_moe_route_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
-      g_counts_dev[dev] = (int*)p;
+      a.ptr = (int*)p;
+      a.ctx = current_context();  // the lookup may have created the primary context
     }
-    counts = g_counts_dev[dev];
+    counts = a.ptr;
   }
 
   rc_knobs k;
@@ -69,7 +97,8 @@ extern "C" rc_status rc_moe_route_noalloc(const void* logits, int32_t logits_fp3
   c.stream = stream;
   c.status = nullptr;
   c.num_sms = 0;
-  // The count kernel overwrites counts[0, experts) on every call, so nothing
-  // needs clearing between calls.
+  // rc_launch_moe_route zeroes counts[0, experts) with cudaMemsetAsync on
+  // `stream` before the count kernel adds to them with atomicAdd, so the
+  // previous call's counts left in the array do not matter.
   return rc_launch_moe_route(k, d, logits, ids, weights, offsets, perm, nullptr, counts, c);
 }

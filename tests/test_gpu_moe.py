@@ -56,6 +56,30 @@ def test_routing_ties_and_imbalance():
     assert list(g[0][0]) == list(range(8))  # all-equal row: lowest ids first
 
 
+@pytest.mark.parametrize("fp32", [False, True])
+def test_routing_nan_logits(fp32):
+    # a NaN logit ranks below every number (read as -inf, ties by lower id) and gets weight 0;
+    # rows with fewer than k numbers still route to k distinct experts below E
+    T, E, K = 64, 64, 8
+    logits, _, _, _ = inputs.moe(T, 8, E, 8, seed=46, logits_fp32=True)
+    L = logits.astype(np.float64)
+    rng = np.random.default_rng(3)
+    L[0, :] = np.nan  # no number at all: ids 0..7
+    L[1, 3:] = np.nan  # three numbers, then the five lowest NaN ids
+    for t in range(2, T, 3):
+        L[t, rng.choice(E, size=rng.integers(1, E), replace=False)] = np.nan
+    lg = L.astype(np.float32) if fp32 else inputs.to_bf16_bits(L)
+    r_ids, r_w, r_off, r_perm = oracle.moe_route(lg, K)
+    assert list(r_ids[0]) == list(range(8))
+    ids, w, off, perm = run_route(lg, E, K)
+    np.testing.assert_array_equal(ids, r_ids)
+    np.testing.assert_array_equal(off, r_off)
+    np.testing.assert_array_equal(perm, r_perm)
+    ok = np.isfinite(r_w).all(axis=1)  # the all-NaN row has no softmax
+    assert ok.sum() == T - 1
+    np.testing.assert_allclose(w[ok], r_w[ok], rtol=2e-6, atol=1e-7)
+
+
 def moe_op(T, H, E, I, K):
     return rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
 

@@ -313,6 +313,28 @@ def test_route_ties_prefer_lower_id():
     assert list(ids[2]) == [2, 63, 0, 1, 3, 4, 5, 6]
 
 
+@pytest.mark.parametrize("fp32", [False, True])
+def test_route_nan_logits_rank_last(fp32):
+    # NaN has no order; the routing reads it as -inf: below every number, ties by lower id, weight 0
+    E, k = 8, 4
+    L = np.full((3, E), np.nan)
+    L[0, [1, 3]] = [1.0, 0.5]  # two numbers, six NaNs: the numbers first, then the lowest NaN ids
+    L[1, :] = np.arange(E)[::-1]  # no NaN: plain order
+    L[1, 0] = np.nan  # the largest value replaced by NaN drops to the end
+    L[2, [6]] = -30.0  # one number, far below zero, still ranks above every NaN
+    logits = L.astype(np.float32) if fp32 else bf(L)
+    ids, w, offsets, perm = oracle.moe_route(logits, k)
+    assert list(ids[0]) == [1, 3, 0, 2]
+    e5 = np.exp(-0.5)
+    np.testing.assert_allclose(w[0], [1 / (1 + e5), e5 / (1 + e5), 0, 0], rtol=1e-15, atol=0)
+    assert list(ids[1]) == [1, 2, 3, 4]
+    assert list(ids[2]) == [6, 0, 1, 2]
+    np.testing.assert_allclose(w[2], [1, 0, 0, 0], rtol=1e-15, atol=0)
+    counts = np.bincount(ids.ravel(), minlength=E)
+    np.testing.assert_array_equal(offsets, np.concatenate([[0], np.cumsum(counts)]))
+    np.testing.assert_array_equal(perm, np.argsort(ids.ravel(), kind="stable"))
+
+
 # ------------------------------------------------------------------- MoE FFN
 
 def _np_expert(x, W1e, W2e):

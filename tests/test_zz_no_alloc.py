@@ -12,6 +12,7 @@ stopping at its first failure has already run every other test.
 import numpy as np
 import pytest
 
+import oracle
 from paper_2506_01374_gb300 import inputs, rc
 
 from .gpu_util import to_dev, torch
@@ -46,6 +47,12 @@ def test_noalloc_routing_matches_regular_entry_point_two_calls():
         np.testing.assert_array_equal(n_perm, r_perm)
         np.testing.assert_allclose(n_w, r_w, rtol=2e-6, atol=1e-7)
         assert n_off[-1] == T * K
+        # and against the fp64 oracle's routing, so the check does not rest on the shared kernels alone
+        o_ids, o_w, o_off, o_perm = oracle.moe_route(logits, K)
+        np.testing.assert_array_equal(n_ids, o_ids)
+        np.testing.assert_array_equal(n_off, o_off)
+        np.testing.assert_array_equal(n_perm, o_perm)
+        np.testing.assert_allclose(n_w, o_w, rtol=2e-6, atol=1e-7)
 
 
 def test_noalloc_routing_rejects_too_many_experts():
