@@ -162,16 +162,17 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       }
       [[fallthrough]];  // 2: the attention core
     case RC_OP_ATTENTION:
-      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256 = two query tiles, ping-pong softmax
-      v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});
+      v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});  // key block BN
       v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 5}, {}});
-      // 0 = head-major tiles, 1 = longest causal rows first, 2 = persistent CTAs walking the
-      // longest-first tiles in a zigzag (one-tile split-issue kernel)
-      v.push_back({RC_T_LOOP_ORDER, 0, {0, 1, 2}, {1}});
-      v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // V as [keys][d] or transposed to [d][keys]
-      v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});  // P stored in shared or tensor memory
-      v.push_back({RC_T_UNROLL, 0, {1, 2}, {}});  // key blocks in flight per query tile
-      v.push_back({RC_T_PARALLEL, 0, {0, 1}, {}});  // one UMMA-issuing warp per CTA, or one per query tile
+      v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1}});  // 0 = head-major tiles, 1 = longest causal rows first
+      v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});        // V as [keys][d] or transposed to [d][keys]
+      // P stored in shared (0) or tensor memory (1); 2: P in tensor memory and the row sums of P
+      // formed by the tensor core (a block of ones appended to V)
+      v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1, 2}, {}});
+      v.push_back({RC_T_UNROLL, 0, {1, 2}, {}});  // S buffers: key blocks in flight per query tile
+      // 0: one UMMA-issuing warp; 1: the S and P V products issued by warps of their own;
+      // 2: as 1 with two softmax threads per query row
+      v.push_back({RC_T_PARALLEL, 0, {0, 1, 2}, {}});
       break;
     case RC_OP_MOE_ROUTE:
       v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
@@ -322,44 +323,33 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
 // Resource and variant rules of the attention kernels (RC_OP_ATTENTION and the
 // decoder layer's attention stage).
 static bool attention_knobs_ok(const rc_knobs& k, int64_t seq, std::string* why) {
-  // Q tiles + ring of K and V tiles + P tiles + slack, all bf16
-  const int64_t qt = k.tile_m / 128;
-  const int64_t smem = qt * 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 +
-                       (k.location ? 0 : qt * 128 * (int64_t)k.tile_n * 2) + 1024 + 512;
-  if (k.location == 1 && k.tile_m != 256 && k.persistent != 1) {
-    if (why) *why = "P in tensor memory needs two query tiles or split UMMA issue";
+  auto no = [&](const char* m) {
+    if (why) *why = m;
     return false;
+  };
+  if (k.persistent == 0) {
+    if (k.location != 0 || k.unroll != 1) return no("one UMMA-issuing warp keeps P in shared memory and one S buffer");
+  } else {
+    if (k.location == 0) return no("split UMMA issue keeps P in tensor memory");
+    if (k.stages < 2) return no("split UMMA issue needs two K/V stages");
   }
-  const bool one_tile_split = k.tile_m == 128 && k.persistent == 1;
-  if (k.unroll == 2 && !one_tile_split && !(k.tile_m == 256 && k.location == 1 && k.tile_n == 64 && k.stages >= 4)) {
-    // two S buffers per tile fill TMEM only at BN = 64; S(j+2) is issued while V(j) is in use
-    if (why) *why = "two key blocks in flight need two query tiles, P in TMEM, BN 64 and 4 stages";
-    return false;
+  if (k.location == 2 && k.layout != 0) return no("row sums on the tensor core need V as given");
+  if (k.layout == 1 && seq % 8) return no("transposed V needs seq % 8 == 0 (16-byte TMA rows)");
+  int64_t smem;
+  if (k.persistent == 0) {
+    // Q tile, K/V ring, P tile, slack and barriers
+    smem = 128 * 128 * 2 + (int64_t)k.stages * 2 * k.tile_n * 128 * 2 + 128 * (int64_t)k.tile_n * 2 + 1024 + 512;
+  } else {
+    // Q, the K ring and a V ring (two slots when two CTAs share an SM), the row-exchange area with two
+    // softmax threads per row, barriers, and alignment slack when one CTA holds the SM
+    const bool split = k.persistent == 2, sumc = k.location == 2;
+    const bool two_ctas = k.tile_n == 64 && !(k.unroll == 2 && sumc);  // TMEM <= 256 columns
+    const int64_t vst = two_ctas && k.stages > 2 ? 2 : k.stages;
+    const int64_t vslot = k.tile_n * 128 * 2 + (sumc ? k.tile_n * 128 : 0);  // + the ones atom
+    smem = 128 * 128 * 2 + k.stages * k.tile_n * 128 * 2 + vst * vslot + (split ? 2048 : 0) +
+           (11 + 2 * k.stages + 2 * vst + (split ? 8 : 0)) * 8 + 8 + (two_ctas ? 0 : 1024);
   }
-  if (k.raster == 2 && !(one_tile_split && k.location == 1 && k.tile_n == 64 && k.unroll == 1 &&
-                         k.stages >= 2 && k.stages <= 3)) {
-    if (why) *why = "persistent tiles (loop order 2) need the one-tile split-issue kernel: BN 64, unroll 1, 2-3 stages";
-    return false;
-  }
-  if (k.persistent == 1 && !(k.location == 1 && (k.unroll == 1 || one_tile_split) && k.stages >= 2)) {
-    // two tiles: one issuing warp per tile; one tile: one or two S buffers, S and P V issued by
-    // separate warps
-    if (why) *why = "split UMMA issue needs P in TMEM, one key block in flight per issuer and two stages";
-    return false;
-  }
-  if (smem > kSmemLimit) {
-    if (why) *why = "attention ring exceeds 227 KB of shared memory";
-    return false;
-  }
-  if (k.tile_m == 256 && k.stages < 2) {
-    // the ping-pong kernel issues S for key block j+1 before releasing block j
-    if (why) *why = "two query tiles per CTA need at least two K/V stages";
-    return false;
-  }
-  if (k.layout == 1 && seq % 8) {
-    if (why) *why = "transposed V needs seq % 8 == 0 (16-byte TMA rows)";
-    return false;
-  }
+  if (smem > kSmemLimit) return no("attention ring exceeds 227 KB of shared memory");
   return true;
 }
 

@@ -2,25 +2,24 @@
 // heads, on the sm_103a tensor cores (tcgen05, TMEM accumulators, TMA).
 //
 // One CTA owns one (batch, query head h, block of 128 queries); the KV head is
-// g = h / (Hq / Hkv). Per key block j of BN keys:
-//   warp 0     : TMA producer - Q once, then K_j (2 x [BN][64] swizzled
-//                halves of the head dimension) and V_j into a ring of stages.
-//   warp 1     : one thread issues S = Q K_j^T into TMEM columns [0, BN)
-//                (8 UMMAs of K = 16 over the 128-wide head dimension), then,
-//                once P_j is in shared memory, O += P_j V_j into TMEM columns
-//                [BN, BN + 128).
-//   warps 2..5 : softmax, one query row per thread (TMEM lane = row). Pass 1
-//                reads S and takes the masked row maximum; the running maximum
-//                m and sum l follow the online softmax in the log2 domain
-//                (p = 2^(s * scale * log2 e - m)); O is rescaled in TMEM by
-//                2^(m_old - m_new) when the maximum moved; pass 2 writes P as
-//                bf16 in the 128-byte-swizzled K-major layout the UMMA reads.
-// The epilogue divides O by l, stores bf16 O and LSE = ln 2 * (m + log2 l).
+// g = h / (Hq / Hkv). Per key block j of BN keys, S_j = Q K_j^T is computed
+// into TMEM, the softmax threads read it (one query row per thread, or per
+// two threads), keep the running row maximum m and sum l in the log2 domain
+// (p = 2^(s * scale * log2 e - m)), rescale O in TMEM when m grows by more
+// than 2^8, and write P_j as bf16; the tensor core then adds P_j V_j to O.
+// The epilogue divides O by l and stores bf16 O and LSE = ln 2 * (m + log2 l).
 //
-// Schedule knobs: BN (template), ring depth (runtime), query-block order
-// (natural or longest-first for the causal triangle), and the layout of V:
-// as given ([keys][d], an MN-major UMMA B operand) or pre-transposed by a pass
-// into [d][keys] (K-major). Masking: key j is visible to query i when j < S and
+// Two kernel families, chosen by the schedule's Parallel knob:
+//   0: attn_kernel - one warp issues every UMMA, P goes through shared
+//      memory (the unoptimised program P0);
+//   1, 2: attn4_kernel - S and P V issued by warps of their own, P in TMEM,
+//      one or two S buffers (Unroll), one or two softmax threads per row
+//      (Parallel 2), and optionally the row sums formed by the tensor core
+//      (ComputeLocation 2).
+// Other knobs: BN (TileSize N), ring depth (PipelineStages), query-block
+// order (natural or longest causal rows first), and the layout of V: as given
+// ([keys][d], an MN-major UMMA B operand) or pre-transposed by a pass into
+// [d][keys] (K-major). Masking: key j is visible to query i when j < S and
 // (not causal or j <= i). Every wait is bounded as in the GEMM kernels.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -112,6 +111,26 @@ __device__ __forceinline__ void exp_pack(const uint32_t* r, uint64_t sc2, uint64
     const float p0 = tc::ex2_approx(x0), p1 = tc::ex2_approx(x1);
     ls2[(i / 2) % 2] = f2_add(ls2[(i / 2) % 2], f2(p0, p1));
     pk[i / 2] = pack2(p0, p1);
+  }
+}
+
+// p_i = 2^(s_i * scale_log2 - mref) for N raw scores, two at a time: the
+// exponent pair is formed in fp32 (packed FMA), rounded to bf16 and raised by
+// one ex2.approx.ftz.bf16x2, which yields the packed bf16 pair the P V UMMA
+// reads. No row sum is kept here: the tensor core forms it (a block of ones
+// appended to V). Rounding the exponent to bf16 moves p by at most
+// ln 2 * |x| * 2^-9 relative, i.e. at most about 2.7e-3 * 2^x absolutely,
+// within about 1.4 times the bf16 rounding of p itself.
+template <int N>
+__device__ __forceinline__ void exp_pack_bf16(const uint32_t* r, uint64_t sc2, uint64_t nm2, uint32_t* pk) {
+#pragma unroll
+  for (int i = 0; i < N; i += 2) {
+    const uint64_t x = f2_fma(f2(__uint_as_float(r[i]), __uint_as_float(r[i + 1])), sc2, nm2);
+    float x0, x1;
+    f2_split(x, x0, x1);
+    uint32_t e;
+    asm("ex2.approx.ftz.bf16x2 %0, %1;" : "=r"(e) : "r"(pack2(x0, x1)));
+    pk[i / 2] = e;
   }
 }
 
@@ -423,797 +442,94 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Two query tiles per CTA (TileSize M = 256), ping-pong between two softmax
-// warpgroups: the MMA warp issues S_0 = Q_0 K^T, S_1 = Q_1 K^T, then
-// O_0 += P_0 V as soon as P_0 is ready and the next S_0 right after it, so
-// one tile's softmax overlaps the other tile's tensor-core work. TMEM holds
-// S_0, S_1 (BN columns each) and O_0, O_1 (128 each). Each softmax thread
-// loads its whole S row with one wait. O is rescaled only when the running
-// maximum grows by more than 2^8 (kRescaleLog2); the exponents use that same
-// reference maximum, and so does the row sum l, so the result is exact.
-// S for key block j+1 is issued before block j's ring slot is released, so
-// this kernel needs a ring of at least two stages.
-constexpr int kThreads2 = 320;
-constexpr float kRescaleLog2 = 8.0f;
-
-
-// Softmax and output of one query tile in the two-tile kernels: one TMEM lane
-// quadrant per warp (qd = warp % 4), one query row per thread. S of key block j
-// sits in TMEM columns [(t * NSB + j % NSB) * BN, + BN) and O_t at o_base + t * D.
-// Pass 1 takes the masked row maximum of the whole S row (one TMEM round trip);
-// O is rescaled in TMEM when the reference maximum moves by more than 2^8; pass 2
-// writes P = 2^(s * scale * log2 e - m) as bf16, over its own S columns (PT) or
-// into the swizzled shared-memory P tile, and accumulates the row sum l.
-template <int BN, bool PT, bool SDB>
-__device__ __forceinline__ void softmax_tile(const Params& p, int t, int qd, int lane, int q0, int nkb, int b, int h,
-                                             uint32_t tmem, uint32_t o_base, uint8_t* sP_tile, uint64_t* s_full,
-                                             uint64_t* p_full, uint64_t* pv_full, volatile int* abort_flag,
-                                             volatile int* status) {
-  constexpr int NSB = SDB ? 2 : 1;
-  auto fail = [&](int code) {
-    *abort_flag = 1;
-    tc::record_failure(status, code);
-  };
-  const int row = 32 * qd + lane;
-  const int qi = q0 + row;
-  const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
-  const uint32_t tO = tmem + lane_base + o_base + t * D;
-  uint8_t* rowp0 = sP_tile + (row / 8) * 1024 + (row % 8) * 128;
-  float m_ref = -INFINITY, l = 0.f;
-  bool ok = true;
-  for (int j = 0; j < nkb; ++j) {
-    const uint32_t tS = tmem + lane_base + (uint32_t)(t * NSB + (j % NSB)) * BN;
-    if (!tc::mbar_wait(&s_full[j % NSB], (uint32_t)(j / NSB) & 1u, abort_flag, status)) {
-      if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
-      ok = false;
-      break;
-    }
-    tc::tc_fence_after();
-    const int k0 = j * BN;
-    // keys [k0, k0 + nvis) of this block are visible to query qi
-    int nvis = min(BN, p.S - k0);
-    if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
-    // the whole S row in registers: one TMEM round trip
-    uint32_t r[BN];
-#pragma unroll
-    for (int q = 0; q < BN; q += 16) tc::tmem_ld16(tS + q, *reinterpret_cast<uint32_t(*)[16]>(&r[q]));
-    tc::tmem_ld_wait();
-    if (nvis < BN) {
-#pragma unroll
-      for (int i = 0; i < BN; ++i)
-        if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
-    }
-    const float mxs = row_max<BN>(r) * p.scale_log2;
-    float factor = 1.f;
-    if (m_ref == -INFINITY) {
-      m_ref = mxs;  // first visible scores: O and l are still zero
-    } else if (mxs > m_ref + kRescaleLog2) {
-      factor = exp2f(m_ref - mxs);
-      m_ref = mxs;
-    }
-    const bool rescale = __any_sync(0xffffffffu, factor != 1.f);
-    // pv_full completes once per key block (P_t V of that block). It is
-    // observed phase by phase, so a parity wait never meets a barrier more
-    // than one phase ahead: phase j-1 is awaited in iteration j, before the
-    // O rescale when there is one (O must hold P_t V of block j-1), before
-    // overwriting P's shared-memory buffer, or else after the probabilities
-    // are written. P V of block j is only issued after this thread's p_full.
-    bool pv_seen = j == 0;
-    auto await_pv = [&]() -> bool {
-      if (pv_seen) return true;
-      pv_seen = true;
-      if (!tc::mbar_wait(pv_full, (uint32_t)(j - 1) & 1u, abort_flag, status)) {
-        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
-        return false;
-      }
-      tc::tc_fence_after();
-      return true;
-    };
-    if (rescale || !PT) {
-      if (!await_pv()) {
-        ok = false;
-        break;
-      }
-    }
-    if (rescale) {
-#pragma unroll 1
-      for (int c = 0; c < D; c += 16) {
-        uint32_t r[16];
-        tc::tmem_ld16(tO + c, r);
-        tc::tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
-        tc::tmem_st16(tO + c, r);
-      }
-      tc::tmem_st_wait();
-    }
-    // pass 2: probabilities -> P (bf16) and the row sum
-    const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-    const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
-    uint64_t ls2[2] = {0ull, 0ull};
-#pragma unroll
-    for (int c = 0; c < BN; c += 32) {
-      uint32_t pk[16];
-      exp_pack<32>(r + c, sc2, nm2, pk, ls2);
-      if constexpr (PT) {
-        // P for keys [c, c + 32) goes to columns [c/2, c/2 + 16) of the S row (already in registers)
-        tc::tmem_st16(tS + c / 2, pk);
-      } else {
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
-          const int cc = c + 16 * h2;
-          uint8_t* rowp = rowp0 + (cc / 64) * (BM * 128);
-          const int ch = (cc % 64) / 8;
-          *reinterpret_cast<uint4*>(rowp + ((ch ^ (row % 8)) * 16)) =
-              make_uint4(pk[8 * h2], pk[8 * h2 + 1], pk[8 * h2 + 2], pk[8 * h2 + 3]);
-          *reinterpret_cast<uint4*>(rowp + (((ch + 1) ^ (row % 8)) * 16)) =
-              make_uint4(pk[8 * h2 + 4], pk[8 * h2 + 5], pk[8 * h2 + 6], pk[8 * h2 + 7]);
-        }
-      }
-    }
-    l = l * factor + sum_pairs(ls2);
-    if constexpr (PT) tc::tmem_st_wait();
-    if (!await_pv()) {
-      ok = false;
-      break;
-    }
-    tc::tc_fence_before();
-    if constexpr (!PT) tc::fence_proxy_async_smem();
-    tc::mbar_arrive(p_full);
-  }
-  if (ok && nkb > 0) {
-    if (tc::mbar_wait(pv_full, (uint32_t)(nkb - 1) & 1u, abort_flag, status)) {
-      tc::tc_fence_after();
-      const float inv_l = l > 0.f ? 1.f / l : 0.f;
-      const bool row_ok = qi < p.S;
-      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
-      store_o_row(tO, inv_l, orow, row_ok);
-      if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
-    } else if (!*abort_flag) {
-      fail(RC_DEV_TIMEOUT_ACCUM);
-    }
-  }
-}
-
-template <int BN, bool VT, bool PT, bool SDB>
-__global__ void __launch_bounds__(kThreads2, 1)
-    attn2_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
-  static_assert(BN == 64 || BN == 128, "key block");
-  constexpr int Q_BYTES = BM * D * 2;   // one query tile: two [128][64] halves
-  constexpr int KV_TILE = BN * D * 2;
-  // P tiles live in shared memory (BN/64 atoms of [128][64]) or, when PT, in
-  // the first BN/2 TMEM columns of their S tile (two bf16 per column).
-  constexpr int P_BYTES = PT ? 0 : BM * BN * 2;
-  // SDB: two S buffers per query tile, so S for key block j+1 is computed
-  // while the softmax works on block j (two key blocks in flight per tile).
-  static_assert(!SDB || (PT && BN == 64), "double-buffered S needs P in TMEM and BN = 64");
-  // (SDB also needs >= 4 ring stages: S of block j+2 is issued while V of
-  // block j is still in use, and the next block should already be loading.)
-  constexpr int NSB = SDB ? 2 : 1;                     // S buffers per tile
-  constexpr uint32_t O_BASE = (uint32_t)(2 * NSB * BN);  // TMEM column of O_0
-
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;                                   // [2] tiles
-  uint8_t* ring = smem + 2 * Q_BYTES;
-  uint8_t* sP = ring + (size_t)stages * 2 * KV_TILE;    // [2] tiles
-  // separate K and V rings of `stages` slots each: K of a block is released
-  // once both tiles' S products are issued, V once both P V products are
-  uint64_t* q_full = (uint64_t*)(sP + 2 * P_BYTES);
-  uint64_t* k_full = q_full + 1;
-  uint64_t* k_empty = k_full + stages;
-  uint64_t* v_full = k_empty + stages;
-  uint64_t* v_empty = v_full + stages;
-  uint64_t* s_full = v_empty + stages;  // [2 tiles][NSB buffers]
-  uint64_t* p_full = s_full + 2 * NSB;   // [2]
-  uint64_t* pv_full = p_full + 2;        // [2]
-  uint64_t* drain = pv_full + 2;
-  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
-  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
-  volatile int* status = p.status;
-
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int pairs = (p.q_blocks + 1) / 2;
-  const int BH = p.B * p.Hq;
-  int pb, bh;
-  if (p.raster == 0) {
-    pb = blockIdx.x % pairs;
-    bh = blockIdx.x / pairs;
-  } else {
-    pb = pairs - 1 - (int)(blockIdx.x / BH);
-    bh = blockIdx.x % BH;
-  }
-  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
-  int q0[2], nkb[2];
-#pragma unroll
-  for (int t = 0; t < 2; ++t) {
-    q0[t] = (2 * pb + t) * BM;
-    const int end = p.causal ? min(q0[t] + BM, p.S) : p.S;
-    nkb[t] = q0[t] < p.S ? (end + BN - 1) / BN : 0;
-  }
-  const int nblk = max(nkb[0], nkb[1]);
-
-  auto fail = [&](int code) {
-    *abort_flag = 1;
-    tc::record_failure(status, code);
-  };
-
-  if (threadIdx.x == 0) {
-    tc::mbar_init(q_full, 1);
-    for (int s = 0; s < stages; ++s) {
-      tc::mbar_init(&k_full[s], 1);
-      tc::mbar_init(&k_empty[s], 1);
-      tc::mbar_init(&v_full[s], 1);
-      tc::mbar_init(&v_empty[s], 1);
-    }
-    for (int t = 0; t < 2; ++t) {
-      for (int b2 = 0; b2 < NSB; ++b2) tc::mbar_init(&s_full[t * NSB + b2], 1);
-      tc::mbar_init(&p_full[t], 128);
-      tc::mbar_init(&pv_full[t], 1);
-    }
-    tc::mbar_init(drain, 1);
-    *abort_flag = 0;
-    tc::fence_mbar_init();
-  }
-  if (warp == 1) tc::tmem_alloc(tmem_slot, 512);
-  tc::tc_fence_before();
-  __syncthreads();
-  tc::tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmQ);
-      tc::prefetch_tmap(&tmK);
-      tc::prefetch_tmap(&tmV);
-      tc::mbar_expect_tx(q_full, 2 * Q_BYTES);
-#pragma unroll
-      for (int t = 0; t < 2; ++t) {
-        const int qrow = b * p.S + q0[t];
-        tc::tma_load_2d(sQ + t * Q_BYTES, &tmQ, q_full, h * D, qrow);
-        tc::tma_load_2d(sQ + t * Q_BYTES + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
-      }
-      int j = 0;
-      for (; j < nblk; ++j) {
-        const int s = j % stages;
-        const uint32_t ph = (uint32_t)(j / stages) & 1u;
-        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
-        uint8_t* sv = sk + KV_TILE;
-        const int krow = b * p.S + j * BN;
-        if (!tc::mbar_wait(&k_empty[s], ph ^ 1u, abort_flag, status)) {
-          fail(RC_DEV_TIMEOUT_EMPTY);
-          break;
-        }
-        tc::mbar_expect_tx(&k_full[s], KV_TILE);
-        tc::tma_load_2d(sk, &tmK, &k_full[s], g * D, krow);
-        tc::tma_load_2d(sk + BN * 128, &tmK, &k_full[s], g * D + 64, krow);
-        if (!tc::mbar_wait(&v_empty[s], ph ^ 1u, abort_flag, status)) {
-          fail(RC_DEV_TIMEOUT_EMPTY);
-          // K of this block is in flight: let it land before exit
-          if (!tc::mbar_wait_drain(&k_full[s], ph)) fail(RC_DEV_TIMEOUT_DRAIN);
-          break;
-        }
-        tc::mbar_expect_tx(&v_full[s], KV_TILE);
-        if constexpr (VT) {
-#pragma unroll
-          for (int a = 0; a < BN / 64; ++a)
-            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &v_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
-        } else {
-          tc::tma_load_2d(sv, &tmV, &v_full[s], g * D, krow);
-          tc::tma_load_2d(sv + BN * 128, &tmV, &v_full[s], g * D + 64, krow);
-        }
-      }
-      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      for (int i = max(0, j - stages); i < j; ++i) {
-        if (!tc::mbar_wait_drain(&k_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-        if (!tc::mbar_wait_drain(&v_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();  // reconverge before the final block barrier
-  } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
-      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
-      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
-      if (!ok) fail(RC_DEV_TIMEOUT_FULL);
-      int k_seen = -1, v_seen = -1;  // highest key block whose K / V arrival was awaited
-      auto await_k = [&](int j) -> bool {
-        if (j <= k_seen) return true;
-        if (!tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status)) return false;
-        k_seen = j;
-        tc::tc_fence_after();
-        return true;
-      };
-      auto await_v = [&](int j) -> bool {
-        if (j <= v_seen) return true;
-        if (!tc::mbar_wait(&v_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status)) return false;
-        v_seen = j;
-        tc::tc_fence_after();
-        return true;
-      };
-      auto issue_s = [&](int t, int j) {
-        const uint32_t sq = tc::smem_u32(sQ + t * Q_BYTES);
-        const uint32_t sk = tc::smem_u32(ring + (size_t)(j % stages) * 2 * KV_TILE);
-        const int sb = t * NSB + (j % NSB);
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          tc::umma_bf16(tmem + (uint32_t)sb * BN, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
-                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
-        }
-        tc::umma_commit(&s_full[sb]);
-      };
-      auto issue_pv = [&](int t, int j) {
-        const uint32_t sp = tc::smem_u32(sP + t * P_BYTES);
-        const uint32_t sv = tc::smem_u32(ring + (size_t)(j % stages) * 2 * KV_TILE) + KV_TILE;
-        const uint32_t tO = tmem + O_BASE + t * D;
-        const uint32_t tP = tmem + (uint32_t)(t * NSB + (j % NSB)) * BN;  // P aliases its S buffer
-#pragma unroll
-        for (int ks = 0; ks < BN / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          uint64_t db;
-          if constexpr (VT)
-            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
-          else
-            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
-          if constexpr (PT)
-            tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
-          else
-            tc::umma_bf16(tO, tc::sw128_desc(sp + (ks / 4) * (BM * 128) + off), db, idO,
-                          (j > 0 || ks > 0) ? 1u : 0u);
-        }
-        tc::umma_commit(&pv_full[t]);
-      };
-      // prologue: S for the first NSB key blocks of both tiles; their K is then free
-      for (int j0 = 0; ok && j0 < NSB && j0 < nblk; ++j0) {
-        ok = await_k(j0);
-        if (ok) {
-          for (int t = 0; t < 2; ++t)
-            if (j0 < nkb[t]) issue_s(t, j0);
-          tc::umma_commit(&k_empty[j0 % stages]);
-        }
-      }
-      for (int j = 0; ok && j < nblk; ++j) {
-        for (int t = 0; t < 2; ++t) {
-          if (j >= nkb[t]) continue;
-          if (!tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status) || !await_v(j)) {
-            ok = false;
-            break;
-          }
-          tc::tc_fence_after();
-          issue_pv(t, j);
-          if (j + NSB < nkb[t]) {
-            if (!await_k(j + NSB)) {
-              ok = false;
-              break;
-            }
-            issue_s(t, j + NSB);
-          }
-        }
-        if (!ok) break;
-        tc::umma_commit(&v_empty[j % stages]);  // both P V products of block j issued
-        if (j + NSB < nblk) tc::umma_commit(&k_empty[(j + NSB) % stages]);  // both S products of block j+NSB
-      }
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_FULL);
-        tc::umma_commit(drain);
-        if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();
-  } else if (warp >= 2) {
-    const int t = (warp - 2) / 4;  // query tile of this warpgroup
-    softmax_tile<BN, PT, SDB>(p, t, warp & 3, lane, q0[t], nkb[t], b, h, tmem, O_BASE, sP + t * P_BYTES,
-                              &s_full[t * NSB], &p_full[t], &pv_full[t], abort_flag, status);
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    __syncwarp();
-    tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, 512);
-  }
-}
-
-// Compact softmax of one query tile for P in TMEM (one S buffer per tile): the
-// S row is walked twice in chunks of 32 columns by loops that are not
-// unrolled, first for the masked maximum (masked scores are written back as
-// -inf, only in chunks that hold any), then for P and the row sum. It holds 32
-// scores in registers instead of the whole row (68 registers per thread
-// instead of 168) and measures as fast as the whole-row version in the
-// two-issuer kernel, where the tensor pipe, not the softmax, sets the pace.
-// P of keys [c, c + 32) goes to columns [c/2, c/2 + 16), which hold S values
-// already consumed.
-template <int BN>
-__device__ __forceinline__ void softmax_tile_chunked(const Params& p, int t, int qd, int lane, int q0, int nkb, int b,
-                                                     int h, uint32_t tmem, uint32_t o_base, uint64_t* s_full,
-                                                     uint64_t* p_full, uint64_t* pv_full, volatile int* abort_flag,
-                                                     volatile int* status) {
-  constexpr int CH = 32;
-  auto fail = [&](int code) {
-    *abort_flag = 1;
-    tc::record_failure(status, code);
-  };
-  const int row = 32 * qd + lane;
-  const int qi = q0 + row;
-  const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
-  const uint32_t tO = tmem + lane_base + o_base + t * D;
-  const uint32_t tS = tmem + lane_base + (uint32_t)(t * BN);
-  float m_ref = -INFINITY, l = 0.f;
-  bool ok = true;
-  for (int j = 0; j < nkb; ++j) {
-    if (!tc::mbar_wait(s_full, (uint32_t)j & 1u, abort_flag, status)) {
-      if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
-      ok = false;
-      break;
-    }
-    tc::tc_fence_after();
-    const int k0 = j * BN;
-    // keys [k0, k0 + nvis) of this block are visible to query qi
-    int nvis = min(BN, p.S - k0);
-    if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
-    float mx = -INFINITY;
-#pragma unroll 1
-    for (int c = 0; c < BN; c += CH) {
-      uint32_t r[CH];
-      tc::tmem_ld32(tS + c, r);
-      tc::tmem_ld_wait();
-      if (__any_sync(0xffffffffu, nvis < c + CH)) {
-#pragma unroll
-        for (int i = 0; i < CH; ++i)
-          if (c + i >= nvis) r[i] = __float_as_uint(-INFINITY);
-        tc::tmem_st32(tS + c, r);
-        tc::tmem_st_wait();
-      }
-      mx = fmaxf(mx, row_max<CH>(r));
-    }
-    const float mxs = mx * p.scale_log2;
-    float factor = 1.f;
-    if (m_ref == -INFINITY) {
-      m_ref = mxs;  // first visible scores: O and l are still zero
-    } else if (mxs > m_ref + kRescaleLog2) {
-      factor = exp2f(m_ref - mxs);
-      m_ref = mxs;
-    }
-    const bool rescale = __any_sync(0xffffffffu, factor != 1.f);
-    // pv_full phase j-1 (P_t V of block j-1) is observed once per key block:
-    // before the O rescale when there is one, else after P is written
-    bool pv_seen = j == 0;
-    auto await_pv = [&]() -> bool {
-      if (pv_seen) return true;
-      pv_seen = true;
-      if (!tc::mbar_wait(pv_full, (uint32_t)(j - 1) & 1u, abort_flag, status)) {
-        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
-        return false;
-      }
-      tc::tc_fence_after();
-      return true;
-    };
-    if (rescale) {
-      if (!await_pv()) {
-        ok = false;
-        break;
-      }
-#pragma unroll 1
-      for (int c = 0; c < D; c += CH) {
-        uint32_t r[CH];
-        tc::tmem_ld32(tO + c, r);
-        tc::tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < CH; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
-        tc::tmem_st32(tO + c, r);
-      }
-      tc::tmem_st_wait();
-    }
-    const float mref = m_ref == -INFINITY ? 0.f : m_ref;
-    const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
-    uint64_t ls2[2] = {0ull, 0ull};
-#pragma unroll 1
-    for (int c = 0; c < BN; c += CH) {
-      uint32_t r[CH];
-      tc::tmem_ld32(tS + c, r);
-      tc::tmem_ld_wait();
-      uint32_t pk[CH / 2];
-      exp_pack<CH>(r, sc2, nm2, pk, ls2);
-      tc::tmem_st16(tS + c / 2, pk);
-    }
-    l = l * factor + sum_pairs(ls2);
-    tc::tmem_st_wait();
-    if (!await_pv()) {
-      ok = false;
-      break;
-    }
-    tc::tc_fence_before();
-    tc::mbar_arrive(p_full);
-  }
-  if (ok && nkb > 0) {
-    if (tc::mbar_wait(pv_full, (uint32_t)(nkb - 1) & 1u, abort_flag, status)) {
-      tc::tc_fence_after();
-      const float inv_l = l > 0.f ? 1.f / l : 0.f;
-      const bool row_ok = qi < p.S;
-      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
-      store_o_row(tO, inv_l, orow, row_ok);
-      if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
-    } else if (!*abort_flag) {
-      fail(RC_DEV_TIMEOUT_ACCUM);
-    }
-  }
-}
-
-// Two query tiles per CTA with one UMMA-issuing warp per tile (Parallel = 1).
-// One thread needs about as long to issue a 128 x 128 x 16 UMMA as the tensor
-// pipe needs to execute it, and its barrier waits and commits come on top, so
-// when a single thread issues both tiles' chains the pipe idles while that
-// thread waits. Here each tile has its own issuer, which checks that V_j and
-// K_{j+1} have landed while the softmax still works on S_j, and releases K_j
-// once S_j is done and V_j once P_j V_j is done, through its own barriers; the
-// producer refills a slot when every tile that read the block held there has
-// released it (under the causal mask tile 0 stops before tile 1).
-// The issuers take turns per chain (tile 0's chain c, then tile 1's chain c,
-// then tile 0's chain c + 1), the UMMA order of the single-issuer kernel:
-// this keeps the tiles half a period apart, so that one tile's softmax runs
-// while the tensor pipe works on the other tile's products.
-//   warp 0       : TMA producer (Q tiles once, then K_j and V_j)
-//   warps 1, 2   : UMMA issue for query tile 0 / 1 (warp 1 also owns TMEM)
-//   warps 3..6   : softmax of tile 0 (TMEM lane quadrant = warp % 4)
-//   warps 7..10  : softmax of tile 1
-// P is kept in TMEM over its S columns.
-constexpr int kThreads3 = 352;
-
-template <int BN, bool VT>
-__global__ void __launch_bounds__(kThreads3, 1)
-    attn3_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
-  static_assert(BN == 64 || BN == 128, "key block");
-  constexpr int Q_BYTES = BM * D * 2;
-  constexpr int KV_TILE = BN * D * 2;
-  constexpr uint32_t O_BASE = (uint32_t)(2 * BN);  // TMEM: S_0, S_1, then O_0, O_1
-
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;  // [2] tiles
-  uint8_t* ring = smem + 2 * Q_BYTES;
-  uint64_t* q_full = (uint64_t*)(ring + (size_t)stages * 2 * KV_TILE);
-  uint64_t* k_full = q_full + 1;              // [stages]
-  uint64_t* v_full = k_full + stages;         // [stages]
-  uint64_t* k_empty = v_full + stages;        // [2 tiles][stages]
-  uint64_t* v_empty = k_empty + 2 * stages;   // [2 tiles][stages]
-  uint64_t* s_full = v_empty + 2 * stages;    // [2]
-  uint64_t* p_full = s_full + 2;              // [2]
-  uint64_t* pv_full = p_full + 2;             // [2]
-  uint64_t* drain = pv_full + 2;              // [2]
-  uint32_t* tmem_slot = (uint32_t*)(drain + 2);
-  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
-  volatile int* chains = (volatile int*)(tmem_slot + 2);  // [2] UMMA chains issued per tile
-  volatile int* status = p.status;
-
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int pairs = (p.q_blocks + 1) / 2;
-  const int BH = p.B * p.Hq;
-  int pb, bh;
-  if (p.raster == 0) {
-    pb = blockIdx.x % pairs;
-    bh = blockIdx.x / pairs;
-  } else {
-    pb = pairs - 1 - (int)(blockIdx.x / BH);
-    bh = blockIdx.x % BH;
-  }
-  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
-  int q0[2], nkb[2];
-#pragma unroll
-  for (int t = 0; t < 2; ++t) {
-    q0[t] = (2 * pb + t) * BM;
-    const int end = p.causal ? min(q0[t] + BM, p.S) : p.S;
-    nkb[t] = q0[t] < p.S ? (end + BN - 1) / BN : 0;
-  }
-  const int nblk = max(nkb[0], nkb[1]);
-
-  auto fail = [&](int code) {
-    *abort_flag = 1;
-    tc::record_failure(status, code);
-  };
-
-  if (threadIdx.x == 0) {
-    tc::mbar_init(q_full, 1);
-    for (int s = 0; s < stages; ++s) {
-      tc::mbar_init(&k_full[s], 1);
-      tc::mbar_init(&v_full[s], 1);
-    }
-    for (int i = 0; i < 2 * stages; ++i) {
-      tc::mbar_init(&k_empty[i], 1);
-      tc::mbar_init(&v_empty[i], 1);
-    }
-    for (int t = 0; t < 2; ++t) {
-      tc::mbar_init(&s_full[t], 1);
-      tc::mbar_init(&p_full[t], 128);
-      tc::mbar_init(&pv_full[t], 1);
-      tc::mbar_init(&drain[t], 1);
-    }
-    *abort_flag = 0;
-    chains[0] = chains[1] = 0;
-    tc::fence_mbar_init();
-  }
-  if (warp == 1) tc::tmem_alloc(tmem_slot, 512);
-  tc::tc_fence_before();
-  __syncthreads();
-  tc::tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmQ);
-      tc::prefetch_tmap(&tmK);
-      tc::prefetch_tmap(&tmV);
-      tc::mbar_expect_tx(q_full, 2 * Q_BYTES);
-#pragma unroll
-      for (int t = 0; t < 2; ++t) {
-        const int qrow = b * p.S + q0[t];
-        tc::tma_load_2d(sQ + t * Q_BYTES, &tmQ, q_full, h * D, qrow);
-        tc::tma_load_2d(sQ + t * Q_BYTES + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
-      }
-      // Slot s last held key block j - stages. Tile t read that block iff
-      // j - stages < nkb[t]; its release is then the ((j - stages) / stages)-th
-      // phase of its barrier for slot s, of parity ph ^ 1 (for j < stages the
-      // fresh barrier passes that parity at once).
-      auto released = [&](uint64_t* empty, int j, int s, uint32_t ph) -> bool {
-        for (int t = 0; t < 2; ++t)
-          if (j - stages < nkb[t] && !tc::mbar_wait(&empty[t * stages + s], ph ^ 1u, abort_flag, status))
-            return false;
-        return true;
-      };
-      int j = 0;
-      for (; j < nblk; ++j) {
-        const int s = j % stages;
-        const uint32_t ph = (uint32_t)(j / stages) & 1u;
-        uint8_t* sk = ring + (size_t)s * 2 * KV_TILE;
-        uint8_t* sv = sk + KV_TILE;
-        const int krow = b * p.S + j * BN;
-        if (!released(k_empty, j, s, ph)) {
-          fail(RC_DEV_TIMEOUT_EMPTY);
-          break;
-        }
-        tc::mbar_expect_tx(&k_full[s], KV_TILE);
-        tc::tma_load_2d(sk, &tmK, &k_full[s], g * D, krow);
-        tc::tma_load_2d(sk + BN * 128, &tmK, &k_full[s], g * D + 64, krow);
-        if (!released(v_empty, j, s, ph)) {
-          fail(RC_DEV_TIMEOUT_EMPTY);
-          if (!tc::mbar_wait_drain(&k_full[s], ph)) fail(RC_DEV_TIMEOUT_DRAIN);  // K of block j is in flight
-          break;
-        }
-        tc::mbar_expect_tx(&v_full[s], KV_TILE);
-        if constexpr (VT) {
-#pragma unroll
-          for (int a = 0; a < BN / 64; ++a)
-            tc::tma_load_2d(sv + a * (BM * 128), &tmV, &v_full[s], j * BN + a * 64, (b * p.Hkv + g) * D);
-        } else {
-          tc::tma_load_2d(sv, &tmV, &v_full[s], g * D, krow);
-          tc::tma_load_2d(sv + BN * 128, &tmV, &v_full[s], g * D + 64, krow);
-        }
-      }
-      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      for (int i = max(0, j - stages); i < j; ++i) {
-        if (!tc::mbar_wait_drain(&k_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-        if (!tc::mbar_wait_drain(&v_full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();  // reconverge before the final block barrier
-  } else if (warp <= 2) {
-    const int t = warp - 1;
-    if (lane == 0 && nkb[t] > 0) {
-      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
-      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
-      const int nk = nkb[t];
-      const int other_chains = nkb[1 - t] > 0 ? nkb[1 - t] + 1 : 0;
-      const uint32_t sq = tc::smem_u32(sQ + t * Q_BYTES);
-      const uint32_t tS = tmem + (uint32_t)(t * BN);
-      const uint32_t tO = tmem + O_BASE + (uint32_t)(t * D);
-      // this thread awaits every key block's K and V exactly once, in order;
-      // a slot's next fill needs this tile's release of the current one
-      auto await_full = [&](uint64_t* full, int j) -> bool {
-        return tc::mbar_wait(&full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status);
-      };
-      // chain c of this tile (c = 0: S_0; c = j + 1: P_j V_j and S_{j+1}) follows
-      // chain c - 1 (tile 0) or chain c (tile 1) of the other tile
-      auto await_turn = [&](int c) -> bool {
-        const int need = min(t == 0 ? c : c + 1, other_chains);
-        const uint64_t t0 = tc::globaltimer();
-        for (uint32_t it = 1; chains[1 - t] < need; ++it)
-          if ((it & 63) == 0 && (*abort_flag || tc::globaltimer() - t0 > tc::kWaitNs)) return false;
-        return true;
-      };
-      auto issue_s = [&](int j) {
-        const uint32_t sk = tc::smem_u32(ring + (size_t)(j % stages) * 2 * KV_TILE);
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
-                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
-        }
-        tc::umma_commit(&s_full[t]);
-        tc::umma_commit(&k_empty[t * stages + j % stages]);
-      };
-      auto issue_pv = [&](int j) {
-        const int s = j % stages;
-        const uint32_t sv = tc::smem_u32(ring + (size_t)s * 2 * KV_TILE) + KV_TILE;
-#pragma unroll
-        for (int ks = 0; ks < BN / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          uint64_t db;
-          if constexpr (VT)
-            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
-          else
-            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
-          // P aliases S: two bf16 per TMEM column
-          tc::umma_bf16_ts(tO, tS + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
-        }
-        tc::umma_commit(&pv_full[t]);
-        tc::umma_commit(&v_empty[t * stages + s]);
-      };
-      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status) && await_full(k_full, 0) && await_turn(0);
-      if (ok) {
-        tc::tc_fence_after();
-        issue_s(0);
-        chains[t] = 1;
-      }
-      for (int j = 0; ok && j < nk; ++j) {
-        // V_j and K_{j+1} (landed long ago, normally) while the softmax works on S_j
-        ok = await_full(v_full, j) && (j + 1 >= nk || await_full(k_full, j + 1)) &&
-             tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status) && await_turn(j + 1);
-        if (!ok) break;
-        tc::tc_fence_after();
-        issue_pv(j);  // O += P_j V_j
-        if (j + 1 < nk) issue_s(j + 1);
-        chains[t] = j + 2;
-      }
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_FULL);
-        tc::umma_commit(&drain[t]);
-        if (!tc::mbar_wait_drain(&drain[t], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();
-  } else {
-    const int t = (warp - 3) / 4;
-    softmax_tile_chunked<BN>(p, t, warp & 3, lane, q0[t], nkb[t], b, h, tmem, O_BASE, &s_full[t], &p_full[t],
-                             &pv_full[t], abort_flag, status);
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    __syncwarp();
-    tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, 512);
-  }
-}
-
-// One query tile per CTA with two S buffers and a P buffer of its own in TMEM
-// (TileSize M = 128, Parallel = 1). TMEM: S_0, S_1 (BN columns each), O (128),
-// P (BN/2 columns, two bf16 per column). S for key block j + 2 goes into the
-// buffer of block j as soon as the softmax holds S_j in registers, so the
-// tensor pipe computes S two key blocks ahead and the softmax of consecutive
-// blocks runs back to back; the softmax keeps P_j in registers until
-// P_{j-1} V_{j-1} has read the P buffer. The UMMAs come from two warps, one
-// for the S products and one for the P V products (one thread needs about as
-// long to issue a 128 x 128 x 16 UMMA as the pipe needs to run it), and K and
-// V stream through rings of their own, each filled by its own producer warp.
-//   warp 0     : TMA producer of Q and of the K ring
-//   warp 1     : issues S_j = Q K_j^T (and owns TMEM)
-//   warp 2     : issues O += P_j V_j
-//   warp 3     : TMA producer of the V ring
-//   warps 4..7 : softmax (TMEM lane quadrant = warp % 4), one query row per thread
+// One query tile per CTA with the UMMAs issued by warps of their own
+// (Parallel 1 and 2). The S and the P V products come from two issuing warps
+// (one thread needs about as long to issue a 128 x 128 x 16 UMMA as the pipe
+// needs to run it), and K and V stream through rings of their own, each
+// filled by its own producer warp.
+//   warp 0          : TMA producer of Q and of the K ring
+//   warp 1          : issues S_j = Q K_j^T (and owns TMEM)
+//   warp 2          : issues O += P_j V_j
+//   warp 3          : TMA producer of the V ring
+//   warps 4..4+4S-1 : softmax (TMEM lane quadrant = warp % 4), S = 1 or 2 threads per query row
+// With one S buffer (Unroll 1) S_{j+1} is issued as soon as the softmax holds
+// S_j in registers and P has columns of its own; with two (Unroll 2) S_{j+1}
+// is computed while the softmax works on S_j and P_j is written over its own
+// S buffer, which takes S_{j+2} once P_j V_j has completed. At BN = 64 both
+// fit 256 TMEM columns, so two CTAs share an SM and one CTA's softmax
+// overlaps the other's UMMAs. ComputeLocation 2 lets the P V UMMA also form
+// the row sums of P (a block of ones appended to V) and takes the
+// exponentials in bf16 pairs.
+constexpr float kRescaleLog2 = 8.0f;  // O is rescaled only when the row maximum grows by more than 2^8
 constexpr int kThreads4 = 256;
 
-template <int BN, int NSB>
-// NSB S buffers at TMEM columns s_col + b * BN (block j in buffer j % NSB),
-// O at o_col, P at p_col. g0: key blocks this CTA's softmax processed in
-// earlier work items (persistent kernels; the barriers' phases run on across
-// items). o_free (persistent kernels): arrived on once O has been read out.
-__device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, int q0, int nkb, int b, int h,
+// Normalised output columns [c0, c0 + NC) of one row, 32 columns per TMEM load.
+template <int NC>
+__device__ __forceinline__ void store_o_cols(uint32_t tO, float inv_l, __nv_bfloat16* orow, bool row_ok) {
+#pragma unroll
+  for (int c = 0; c < NC; c += 32) {
+    uint32_t o[32];
+    tc::tmem_ld32(tO + c, o);
+    tc::tmem_ld_wait();
+    if (row_ok) {
+#pragma unroll
+      for (int i = 0; i < 32; i += 8) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          pk[u] = pack2(__uint_as_float(o[i + 2 * u]) * inv_l, __uint_as_float(o[i + 2 * u + 1]) * inv_l);
+        *reinterpret_cast<uint4*>(orow + c + i) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+    }
+  }
+}
+
+// Row exchange between the two softmax threads of a row (SPLIT = 2): warps
+// 4 + qd and 8 + qd read the same TMEM lanes, one half of the key columns
+// each. Each block they swap their half-row maxima through `xch`
+// ([2 parities][2 halves][128 rows] floats) and an mbarrier per lane
+// quadrant and block parity (64 arrivals), whose waits are bounded like every
+// other wait; at the end they swap their half-row sums the same way.
+struct RowXchg {
+  float* xch;
+  uint64_t* xbar;  // [4 quadrants][2 parities]
+  // Publish v for (row, half) in exchange number n and return the partner's.
+  __device__ __forceinline__ bool swap(int n, int qd, int half, int row, float& v, volatile int* abort_flag,
+                                       volatile int* status) const {
+    float* slot = xch + (n & 1) * 256;
+    slot[half * 128 + row] = v;
+    uint64_t* bar = xbar + qd * 2 + (n & 1);
+    tc::mbar_arrive(bar);  // release: the store above is visible to the partner after its wait
+    if (!tc::mbar_wait(bar, (uint32_t)(n >> 1) & 1u, abort_flag, status)) return false;
+    v = slot[(half ^ 1) * 128 + row];
+    return true;
+  }
+};
+
+// Softmax of the one-tile kernel. NSB S buffers at TMEM columns s_col + b * BN
+// (block j in buffer j % NSB), O at o_col. With one S buffer P has columns of
+// its own at p_col; with two, P_j is written over the first BN / 2 columns of
+// its own S buffer (S_j is in registers by then), so the tile needs no P
+// columns and S_{j+1} is computed while the softmax works on S_j. SPLIT
+// threads share a row: thread `half` exponentiates keys
+// [half * BN / SPLIT, + BN / SPLIT) of every block and owns O columns
+// [half * D / SPLIT, + D / SPLIT); the row maximum is exchanged every block
+// (both threads then take the same rescale decisions) and the row sum once at
+// the end. p_full / pv_full: one barrier per S buffer with two buffers (block
+// i completes phase i / 2 of barrier i % 2), else one. SUMC: the row sums of
+// P come from the tensor core (O's columns D .. D + 15) and the exponentials
+// are taken in bf16 pairs.
+template <int BN, int NSB, int SPLIT, bool SUMC = false>
+__device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int half, int lane, int q0, int nkb, int b, int h,
                                             uint32_t tmem, uint32_t s_col, uint32_t o_col, uint32_t p_col,
                                             uint64_t* s_full, uint64_t* s_free, uint64_t* p_full, uint64_t* pv_full,
-                                            volatile int* abort_flag, volatile int* status, int g0 = 0,
-                                            uint64_t* o_free = nullptr) {
+                                            RowXchg xc, volatile int* abort_flag, volatile int* status) {
+  static_assert(SPLIT == 1 || SPLIT == 2, "threads per row");
+
+  constexpr bool PA = NSB == 2;     // P written over its S buffer
+  constexpr int NPV = PA ? 2 : 1;   // P and P V barriers
+  constexpr int KN = BN / SPLIT;  // keys per block and thread
+  constexpr int OC = D / SPLIT;   // O columns per thread
   auto fail = [&](int code) {
     *abort_flag = 1;
     tc::record_failure(status, code);
@@ -1221,18 +537,18 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
   const int row = 32 * qd + lane;
   const int qi = q0 + row;
   const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
-  const uint32_t tO = tmem + lane_base + o_col;
-  const uint32_t tP = tmem + lane_base + p_col;
+  const uint32_t tO = tmem + lane_base + o_col + (uint32_t)(half * OC);
   float m_ref = -INFINITY, l = 0.f;
-  // pv_full completes once per key block (P_j V_j done); its phases are
-  // observed one by one, in order, never more than one behind: phase j - 1
-  // in iteration j (before an O rescale, else before P_j overwrites P_{j-1}),
-  // the last one before the output. Indices are global (g0 + j).
-  int pv_seen = g0;
+  // P V of block i completes phase i / NPV of pv_full[i % NPV]; the phases are
+  // observed one by one, in block order, never more than one behind on either
+  // barrier: block j - 1 in iteration j (before an O rescale; with one S
+  // buffer also before P_j overwrites P_{j-1}), the last one before the
+  // output.
+  int pv_seen = 0;
   auto await_pv = [&](int upto) -> bool {
     if (pv_seen > upto) return true;
     for (; pv_seen <= upto; ++pv_seen)
-      if (!tc::mbar_wait(pv_full, (uint32_t)pv_seen & 1u, abort_flag, status)) {
+      if (!tc::mbar_wait(&pv_full[pv_seen % NPV], (uint32_t)(pv_seen / NPV) & 1u, abort_flag, status)) {
         if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
         return false;
       }
@@ -1241,30 +557,49 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
   };
   bool ok = true;
   for (int j = 0; j < nkb; ++j) {
-    const int gj = g0 + j;
+    const int gj = j;
     const int sb = gj % NSB;
-    const uint32_t tS = tmem + lane_base + s_col + (uint32_t)(sb * BN);
+    const uint32_t tS = tmem + lane_base + s_col + (uint32_t)(sb * BN + half * KN);
     if (!tc::mbar_wait(&s_full[sb], (uint32_t)(gj / NSB) & 1u, abort_flag, status)) {
       if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
       ok = false;
       break;
     }
     tc::tc_fence_after();
-    uint32_t r[BN];
+    // two S buffers: S_j went into the buffer once P_{j-2} V_{j-2} had completed, so
+    // observing that completion here never stalls and keeps the softmax at most one
+    // phase behind on each P V barrier
+    if (PA && !await_pv(gj - 2)) {
+      ok = false;
+      break;
+    }
+    uint32_t r[KN];
 #pragma unroll
-    for (int c = 0; c < BN; c += 32) tc::tmem_ld32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&r[c]));
+    for (int c = 0; c < KN; c += 32) tc::tmem_ld32(tS + c, *reinterpret_cast<uint32_t(*)[32]>(&r[c]));
     tc::tmem_ld_wait();
-    tc::tc_fence_before();
-    tc::mbar_arrive(&s_free[sb]);  // S buffer sb may take S_{j+NSB}
-    const int k0 = j * BN;
-    int nvis = min(BN, p.S - k0);
+    if constexpr (!PA) {
+      tc::tc_fence_before();
+      tc::mbar_arrive(&s_free[sb]);  // S buffer sb may take S_{j+NSB}
+    }
+    const int k0 = j * BN + half * KN;
+    int nvis = min(KN, p.S - k0);
     if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
-    if (nvis < BN) {
+    if (nvis < KN) {
 #pragma unroll
-      for (int i = 0; i < BN; ++i)
+      for (int i = 0; i < KN; ++i)
         if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
     }
-    const float mxs = row_max<BN>(r) * p.scale_log2;
+    float mx = row_max<KN>(r);
+    if constexpr (SPLIT == 2) {
+      float other = mx;
+      if (!xc.swap(gj, qd, half, row, other, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        ok = false;
+        break;
+      }
+      mx = fmaxf(mx, other);  // the same row maximum in both threads of the row
+    }
+    const float mxs = mx * p.scale_log2;
     float factor = 1.f;
     if (m_ref == -INFINITY) {
       m_ref = mxs;  // first visible scores: O and l are still zero
@@ -1277,58 +612,101 @@ __device__ __forceinline__ void softmax_sdb(const Params& p, int qd, int lane, i
         ok = false;
         break;
       }
-#pragma unroll 1
-      for (int c = 0; c < D; c += 32) {
-        uint32_t o[32];
-        tc::tmem_ld32(tO + c, o);
+      constexpr int RC = SPLIT == 1 ? 32 : 16;  // columns per TMEM round trip (registers)
+      if (SUMC && half == 0) {  // the row-sum columns after O (rescaled once per row)
+        uint32_t o[16];
+        tc::tmem_ld16(tO + D, o);  // half 0: tO is the row's first O column
         tc::tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
-        tc::tmem_st32(tO + c, o);
+        for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+        tc::tmem_st16(tO + D, o);
+      }
+#pragma unroll 1
+      for (int c = 0; c < OC; c += RC) {
+        uint32_t o[RC];
+        if constexpr (RC == 32) {
+          tc::tmem_ld32(tO + c, o);
+        } else {
+          tc::tmem_ld16(tO + c, o);
+        }
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < RC; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+        if constexpr (RC == 32) {
+          tc::tmem_st32(tO + c, o);
+        } else {
+          tc::tmem_st16(tO + c, o);
+        }
       }
       tc::tmem_st_wait();
     }
     const float mref = m_ref == -INFINITY ? 0.f : m_ref;
     const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
-    uint64_t ls2[2] = {0ull, 0ull};
-    uint32_t pk[BN / 2];
-    exp_pack<BN>(r, sc2, nm2, pk, ls2);
-    l = l * factor + sum_pairs(ls2);
-    if (!await_pv(gj - 1)) {  // P_{j-1} V_{j-1} has read the P buffer
+    uint32_t pk[KN / 2];
+    if constexpr (SUMC) {
+      exp_pack_bf16<KN>(r, sc2, nm2, pk);  // the sum of P accumulates in O's last columns
+    } else {
+      uint64_t ls2[2] = {0ull, 0ull};
+      exp_pack<KN>(r, sc2, nm2, pk, ls2);
+      l = l * factor + sum_pairs(ls2);
+    }
+    // P_j goes over S_j (already in registers; the P V that last read this
+    // buffer completed before S_j was computed into it), else into the P
+    // columns once P_{j-1} V_{j-1} has read them
+    if (!PA && !await_pv(gj - 1)) {
       ok = false;
       break;
     }
+    const uint32_t tP = tmem + lane_base + (PA ? s_col + (uint32_t)(sb * BN) : p_col) + (uint32_t)(half * KN / 2);
 #pragma unroll
-    for (int c = 0; c < BN / 2; c += 16) tc::tmem_st16(tP + c, *reinterpret_cast<uint32_t(*)[16]>(&pk[c]));
+    for (int c = 0; c < KN / 2; c += 16) tc::tmem_st16(tP + c, *reinterpret_cast<uint32_t(*)[16]>(&pk[c]));
     tc::tmem_st_wait();
     tc::tc_fence_before();
-    tc::mbar_arrive(p_full);
+    tc::mbar_arrive(&p_full[PA ? sb : 0]);
   }
   if (ok && nkb > 0) {
-    if (await_pv(g0 + nkb - 1)) {
+    if constexpr (SPLIT == 2 && !SUMC) {  // the row sum is the two halves' sums
+      float lp = l;
+      if (!xc.swap(nkb, qd, half, row, lp, abort_flag, status)) {
+        if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+        ok = false;
+      }
+      l += lp;
+    }
+    if (ok && await_pv(nkb - 1)) {
+      if constexpr (SUMC) {  // l = the row sum the P V UMMAs accumulated next to O
+        uint32_t o[16];
+        tc::tmem_ld16(tO - half * OC + D, o);
+        tc::tmem_ld_wait();
+        l = __uint_as_float(o[0]);
+      }
       const float inv_l = l > 0.f ? 1.f / l : 0.f;
       const bool row_ok = qi < p.S;
-      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
-      store_o_row(tO, inv_l, orow, row_ok);
-      if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
-      if (o_free) {  // O has been read: the next item's first P V may overwrite it
-        tc::tc_fence_before();
-        tc::mbar_arrive(o_free);
+      __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D + half * OC;
+      if constexpr (SPLIT == 1) {
+        store_o_row(tO, inv_l, orow, row_ok);
+      } else {
+        store_o_cols<OC>(tO, inv_l, orow, row_ok);
       }
+      if (p.lse && row_ok && half == 0)
+        p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
     }
   }
 }
 
 // TMEM layout of the one-tile kernel with NSB S buffers: S at 0 (and BN),
-// then P and O. With one S buffer and BN = 64 the tile takes 256 columns
-// (S 64, P 32, O 128 at column 128), so two CTAs share an SM: one CTA's
-// softmax overlaps the other's tensor-core work, and a finishing CTA's tail
-// overlaps its neighbour instead of idling the SM.
-template <int BN, int NSB>
+// then P (one S buffer) and O. With BN = 64 the tile takes 256 columns (one S
+// buffer: S 64, P 32, O 128 at column 128; two: S 2 x 64, O 128), so two
+// CTAs share an SM: one CTA's softmax overlaps the other's tensor-core work,
+// and a finishing CTA's tail overlaps its neighbour instead of idling the SM.
+template <int BN, int NSB, bool SUMC = false>
 struct Attn4Cols {
-  static constexpr uint32_t P = NSB == 2 ? 2 * BN + D : BN;
-  static constexpr uint32_t O = NSB == 2 ? 2 * BN : (BN + BN / 2 + 127) / 128 * 128;
-  static constexpr uint32_t END = NSB == 2 ? 2 * BN + D + BN / 2 : O + D;
+  // SUMC (one S buffer): O has D + 16 columns, the last 16 holding the row
+  // sums of P; S at 0, O at BN, P after O
+  static constexpr uint32_t OW = SUMC ? D + 16 : D;
+  static constexpr uint32_t P = NSB == 2 ? 0 : SUMC ? BN + OW : BN;  // two S buffers: P over its S buffer
+  static constexpr uint32_t O = NSB == 2 ? 2 * BN : SUMC ? BN : (BN + BN / 2 + 127) / 128 * 128;
+  static constexpr uint32_t END = NSB == 2 ? O + OW : SUMC ? P + BN / 2 : O + D;
   static constexpr uint32_t ALLOC = END <= 256 ? 256 : 512;
   static constexpr int CTAS_PER_SM = ALLOC == 256 ? 2 : 1;
 };
@@ -1337,39 +715,59 @@ struct Attn4Cols {
 // softmax period after K_j, so two-CTA-per-SM kernels keep at most two V
 // slots and spend the shared memory on the K ring, whose refill latency (a
 // K slot frees only when S_j completes) is what stalls S_{j+2}.
-template <int BN, int NSB>
+template <int BN, int NSB, bool SUMC = false>
 __host__ __device__ constexpr int attn4_vstages(int stages) {
-  return Attn4Cols<BN, NSB>::CTAS_PER_SM == 2 && stages > 2 ? 2 : stages;
+  return Attn4Cols<BN, NSB, SUMC>::CTAS_PER_SM == 2 && stages > 2 ? 2 : stages;
+}
+// Bytes of a V ring slot: the BN x 128 tile, and with row sums on the tensor
+// core a third 64-column atom of ones (N = 128 + 16 for the P V UMMA).
+template <int BN, bool SUMC>
+__host__ __device__ constexpr size_t attn4_vslot() {
+  return (size_t)BN * D * 2 + (SUMC ? (size_t)BN * 128 : 0);
 }
 // Barrier words of attn4 after the rings: q_full, k_full/empty[stages],
-// v_full/empty[vstages], s_full/s_free[2], p_full, pv_full, drain[2], then
-// the TMEM address and the abort flag.
-__host__ __device__ constexpr size_t attn4_bar_bytes(int stages, int vstages) {
-  return (size_t)(9 + 2 * stages + 2 * vstages) * 8 + 8;
+// v_full/empty[vstages], s_full/s_free[2], p_full[2], pv_full[2], drain[2],
+// the row-exchange barriers [4][2] with two softmax threads per row, then the
+// TMEM address and the abort flag.
+__host__ __device__ constexpr size_t attn4_bar_bytes(int stages, int vstages, int split) {
+  return (size_t)(11 + 2 * stages + 2 * vstages + (split == 2 ? 8 : 0)) * 8 + 8;
 }
+// Row-exchange area of the two-threads-per-row softmax: [2][2][128] floats.
+__host__ __device__ constexpr size_t attn4_xch_bytes(int split) { return split == 2 ? 2048 : 0; }
 // Two CTAs per SM need the operands packed without alignment slack: the
 // dynamic shared memory base is then required to be 1024-byte aligned (the
 // kernel checks and reports RC_DEV_MISALIGNED otherwise).
-template <int BN, int NSB>
+template <int BN, int NSB, int SPLIT = 1, bool SUMC = false>
 size_t attn4_smem(int stages) {
-  const int vst = attn4_vstages<BN, NSB>(stages);
-  const size_t tiles = (size_t)BM * D * 2 + (size_t)(stages + vst) * BN * D * 2;
-  return tiles + attn4_bar_bytes(stages, vst) + (Attn4Cols<BN, NSB>::CTAS_PER_SM == 2 ? 0 : 1024);
+  const int vst = attn4_vstages<BN, NSB, SUMC>(stages);
+  const size_t tiles = (size_t)BM * D * 2 + (size_t)stages * BN * D * 2 + (size_t)vst * attn4_vslot<BN, SUMC>();
+  return tiles + attn4_xch_bytes(SPLIT) + attn4_bar_bytes(stages, vst, SPLIT) +
+         (Attn4Cols<BN, NSB, SUMC>::CTAS_PER_SM == 2 ? 0 : 1024);
 }
 
-template <int BN, bool VT, int NSB>
-__global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
+// Threads of the one-tile kernel: four producer / UMMA warps and 4 * SPLIT softmax warps.
+template <int SPLIT>
+constexpr int attn4_threads() {
+  return kThreads4 + 128 * (SPLIT - 1);
+}
+
+template <int BN, bool VT, int NSB, int SPLIT = 1, bool SUMC = false>
+__global__ void __launch_bounds__(attn4_threads<SPLIT>(), (Attn4Cols<BN, NSB, SUMC>::CTAS_PER_SM))
     attn4_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                  const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
   static_assert(BN == 64 || BN == 128, "key block");
   static_assert(NSB == 1 || NSB == 2, "S buffers");
+  static_assert(SPLIT == 1 || SPLIT == 2, "softmax threads per row");
+  static_assert(!SUMC || !VT, "row sums on the tensor core: V as given");
   constexpr int Q_BYTES = BM * D * 2;
   constexpr int KV_TILE = BN * D * 2;
-  constexpr uint32_t O_COL = Attn4Cols<BN, NSB>::O, P_COL = Attn4Cols<BN, NSB>::P;
-  constexpr uint32_t TMEM_COLS = Attn4Cols<BN, NSB>::ALLOC;
+  constexpr size_t VSLOT = attn4_vslot<BN, SUMC>();
+  using Cols = Attn4Cols<BN, NSB, SUMC>;
+  constexpr uint32_t O_COL = Cols::O, P_COL = Cols::P;
+  constexpr uint32_t TMEM_COLS = Cols::ALLOC;
 
   extern __shared__ uint8_t smem_raw[];
-  if constexpr (Attn4Cols<BN, NSB>::CTAS_PER_SM == 2) {
+  if constexpr (Cols::CTAS_PER_SM == 2) {
     // the operands are packed without alignment slack (two CTAs per SM)
     if (tc::smem_u32(smem_raw) & 1023u) {
       if (threadIdx.x == 0) tc::record_failure(p.status, RC_DEV_MISALIGNED);
@@ -1377,21 +775,23 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     }
   }
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  const int vstages = attn4_vstages<BN, NSB>(stages);
+  const int vstages = attn4_vstages<BN, NSB, SUMC>(stages);
   uint8_t* sQ = smem;
   uint8_t* kring = smem + Q_BYTES;
   uint8_t* vring = kring + (size_t)stages * KV_TILE;
-  uint64_t* q_full = (uint64_t*)(vring + (size_t)vstages * KV_TILE);
+  float* xch = (float*)(vring + (size_t)vstages * VSLOT);  // SPLIT == 2: [2][2][128]
+  uint64_t* q_full = (uint64_t*)((uint8_t*)xch + attn4_xch_bytes(SPLIT));
   uint64_t* k_full = q_full + 1;      // [stages]
   uint64_t* k_empty = k_full + stages;
   uint64_t* v_full = k_empty + stages;  // [vstages]
   uint64_t* v_empty = v_full + vstages;
   uint64_t* s_full = v_empty + vstages;  // [2] S buffers
   uint64_t* s_free = s_full + 2;        // [2]
-  uint64_t* p_full = s_free + 2;
-  uint64_t* pv_full = p_full + 1;
-  uint64_t* drain = pv_full + 1;        // [2] one per issuing warp
-  uint32_t* tmem_slot = (uint32_t*)(drain + 2);
+  uint64_t* p_full = s_free + 2;        // [2] one per S buffer with two (P over S)
+  uint64_t* pv_full = p_full + 2;       // [2]
+  uint64_t* drain = pv_full + 2;        // [2] one per issuing warp
+  uint64_t* xbar = drain + 2;           // SPLIT == 2: [4][2]
+  uint32_t* tmem_slot = (uint32_t*)(xbar + (SPLIT == 2 ? 8 : 0));
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
   volatile int* status = p.status;
 
@@ -1427,13 +827,25 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     }
     for (int i = 0; i < 2; ++i) {
       tc::mbar_init(&s_full[i], 1);
-      tc::mbar_init(&s_free[i], 128);
+      tc::mbar_init(&s_free[i], 128 * SPLIT);
+      tc::mbar_init(&p_full[i], 128 * SPLIT);
+      tc::mbar_init(&pv_full[i], 1);
       tc::mbar_init(&drain[i], 1);
     }
-    tc::mbar_init(p_full, 128);
-    tc::mbar_init(pv_full, 1);
+    if constexpr (SPLIT == 2)
+      for (int i = 0; i < 8; ++i) tc::mbar_init(&xbar[i], 64);
     *abort_flag = 0;
     tc::fence_mbar_init();
+  }
+  if constexpr (SUMC) {
+    // the ones atom of every V slot (bf16 1.0): P V then also accumulates sum_j P_j in O's
+    // columns D .. D + 15; written once, through the generic proxy, before any UMMA reads it
+    for (int s = 0; s < vstages; ++s) {
+      uint4* ones = (uint4*)(vring + (size_t)s * VSLOT + (size_t)KV_TILE);
+      for (int i = threadIdx.x; i < BN * 128 / 16; i += blockDim.x)
+        ones[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+    }
+    tc::fence_proxy_async_smem();
   }
   if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
   tc::tc_fence_before();
@@ -1481,7 +893,7 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     if (lane == 0) {
       tc::prefetch_tmap(&tmV);
       produce(v_full, v_empty, vstages, [&](int s, int j, uint64_t* bar) {
-        uint8_t* sv = vring + (size_t)s * KV_TILE;
+        uint8_t* sv = vring + (size_t)s * VSLOT;
         if constexpr (VT) {
 #pragma unroll
           for (int a = 0; a < BN / 64; ++a)
@@ -1522,8 +934,13 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
         }
       }
       for (int j = 0; ok && j + NSB < nkb; ++j) {
-        // S buffer j % NSB is free once the softmax holds S_j in registers
-        ok = tc::mbar_wait(&s_free[j % NSB], (uint32_t)(j / NSB) & 1u, abort_flag, status) && await_k(j + NSB);
+        // one S buffer: free once the softmax holds S_j in registers; two: S buffer j % 2
+        // holds P_j, free once P_j V_j has completed
+        if constexpr (NSB == 1)
+          ok = tc::mbar_wait(&s_free[0], (uint32_t)j & 1u, abort_flag, status);
+        else
+          ok = tc::mbar_wait(&pv_full[j % 2], (uint32_t)(j / 2) & 1u, abort_flag, status);
+        ok = ok && await_k(j + NSB);
         if (!ok) break;
         tc::tc_fence_after();
         issue_s(j + NSB);
@@ -1537,16 +954,18 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     __syncwarp();
   } else if (warp == 2) {
     if (lane == 0 && nkb > 0) {
-      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
-      const uint32_t tO = tmem + O_COL, tP = tmem + P_COL;
+      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, (int)Cols::OW, !VT);
+      const uint32_t tO = tmem + O_COL;
       bool ok = true;
       for (int j = 0; ok && j < nkb; ++j) {
         const int s = j % vstages;
+        const int pb = NSB == 2 ? j % 2 : 0;  // P over S buffer j % 2, or the P columns
+        const uint32_t tP = tmem + (NSB == 2 ? (uint32_t)(pb * BN) : P_COL);
         ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / vstages) & 1u, abort_flag, status) &&
-             tc::mbar_wait(p_full, (uint32_t)j & 1u, abort_flag, status);
+             tc::mbar_wait(&p_full[pb], (uint32_t)(j / (NSB == 2 ? 2 : 1)) & 1u, abort_flag, status);
         if (!ok) break;
         tc::tc_fence_after();
-        const uint32_t sv = tc::smem_u32(vring + (size_t)s * KV_TILE);
+        const uint32_t sv = tc::smem_u32(vring + (size_t)s * VSLOT);
 #pragma unroll
         for (int ks = 0; ks < BN / 16; ++ks) {
           const uint32_t off = (uint32_t)(ks % 4) * 32;
@@ -1557,7 +976,7 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
             db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
           tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
         }
-        tc::umma_commit(pv_full);
+        tc::umma_commit(&pv_full[pb]);
         tc::umma_commit(&v_empty[s]);
       }
       if (!ok) {
@@ -1568,8 +987,8 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     }
     __syncwarp();
   } else {
-    softmax_sdb<BN, NSB>(p, warp & 3, lane, q0, nkb, b, h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full, pv_full,
-                         abort_flag, status);
+    softmax_sdb<BN, NSB, SPLIT, SUMC>(p, warp & 3, (warp - 4) >> 2, lane, q0, nkb, b, h, tmem, 0u, O_COL, P_COL, s_full,
+                                s_free, p_full, pv_full, RowXchg{xch, xbar}, abort_flag, status);
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -1577,524 +996,6 @@ __global__ void __launch_bounds__(kThreads4, (Attn4Cols<BN, NSB>::CTAS_PER_SM))
     __syncwarp();
     tc::tc_fence_after();
     tc::tmem_dealloc(tmem, TMEM_COLS);
-  }
-}
-
-// Persistent form of the one-tile, one-S-buffer kernel with 64-key blocks
-// (Loop order 2). Two CTAs per SM stay resident and walk the query tiles,
-// ordered longest first, in a zigzag over the CTAs (CTA c takes tiles c,
-// 2G - 1 - c, 2G + c, ... of G CTAs), which pairs long causal tiles with
-// short ones. TMEM, barriers and tensor maps are set up once; the K and V
-// rings run on across tiles, so the next tile's keys stream in while the
-// current one finishes; the next Q is loaded as soon as the current tile's
-// last S UMMA has read Q (q_empty), and the next tile's first P V waits until
-// the softmax warps have read O out (o_free). Every barrier's phase counts
-// key blocks (or tiles) over the whole run of the CTA.
-__host__ __device__ constexpr size_t attn4p_bar_bytes(int stages, int vstages) {
-  return (size_t)(11 + 2 * stages + 2 * vstages) * 8 + 8;
-}
-size_t attn4p_smem(int stages) {
-  const int vst = attn4_vstages<64, 1>(stages);
-  return (size_t)BM * D * 2 + (size_t)(stages + vst) * 64 * D * 2 + attn4p_bar_bytes(stages, vst);
-}
-
-template <bool VT>
-__global__ void __launch_bounds__(kThreads4, 2)
-    attn4p_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                  const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
-  constexpr int BN = 64;
-  constexpr int Q_BYTES = BM * D * 2;
-  constexpr int KV_TILE = BN * D * 2;
-  constexpr uint32_t O_COL = Attn4Cols<BN, 1>::O, P_COL = Attn4Cols<BN, 1>::P;
-  constexpr uint32_t TMEM_COLS = Attn4Cols<BN, 1>::ALLOC;
-  static_assert(TMEM_COLS == 256, "two CTAs per SM");
-
-  extern __shared__ uint8_t smem_raw[];
-  if (tc::smem_u32(smem_raw) & 1023u) {  // operands packed without alignment slack
-    if (threadIdx.x == 0) tc::record_failure(p.status, RC_DEV_MISALIGNED);
-    return;
-  }
-  uint8_t* smem = smem_raw;
-  const int vstages = attn4_vstages<BN, 1>(stages);
-  uint8_t* sQ = smem;
-  uint8_t* kring = smem + Q_BYTES;
-  uint8_t* vring = kring + (size_t)stages * KV_TILE;
-  uint64_t* q_full = (uint64_t*)(vring + (size_t)vstages * KV_TILE);
-  uint64_t* q_empty = q_full + 1;
-  uint64_t* k_full = q_empty + 1;  // [stages]
-  uint64_t* k_empty = k_full + stages;
-  uint64_t* v_full = k_empty + stages;  // [vstages]
-  uint64_t* v_empty = v_full + vstages;
-  uint64_t* s_full = v_empty + vstages;
-  uint64_t* s_free = s_full + 1;
-  uint64_t* p_full = s_free + 1;
-  uint64_t* pv_full = p_full + 1;
-  uint64_t* o_free = pv_full + 1;
-  uint64_t* drain = o_free + 1;  // [2]
-  uint32_t* tmem_slot = (uint32_t*)(drain + 2);
-  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
-  volatile int* status = p.status;
-
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int BH = p.B * p.Hq;
-  const int n_tiles = p.q_blocks * BH;
-  const int G = gridDim.x, c = blockIdx.x;
-  // k-th work item of this CTA: a query tile in longest-first order, zigzag over the CTAs
-  struct Work {
-    bool valid;
-    int q0, nkb, b, h, g;
-  };
-  auto work = [&](int k) -> Work {
-    Work w;
-    const long long t = (long long)k * G + ((k & 1) ? G - 1 - c : c);
-    w.valid = t < n_tiles;
-    if (!w.valid) return w;
-    const int qb = p.q_blocks - 1 - (int)(t / BH), bh = (int)(t % BH);
-    w.b = bh / p.Hq;
-    w.h = bh - w.b * p.Hq;
-    w.g = w.h / p.group;
-    w.q0 = qb * BM;
-    const int kv_end = p.causal ? min(w.q0 + BM, p.S) : p.S;
-    w.nkb = (kv_end + BN - 1) / BN;
-    return w;
-  };
-  auto fail = [&](int code) {
-    *abort_flag = 1;
-    tc::record_failure(status, code);
-  };
-
-  if (threadIdx.x == 0) {
-    tc::mbar_init(q_full, 1);
-    tc::mbar_init(q_empty, 1);
-    for (int s = 0; s < stages; ++s) {
-      tc::mbar_init(&k_full[s], 1);
-      tc::mbar_init(&k_empty[s], 1);
-    }
-    for (int s = 0; s < vstages; ++s) {
-      tc::mbar_init(&v_full[s], 1);
-      tc::mbar_init(&v_empty[s], 1);
-    }
-    tc::mbar_init(s_full, 1);
-    tc::mbar_init(s_free, 128);
-    tc::mbar_init(p_full, 128);
-    tc::mbar_init(pv_full, 1);
-    tc::mbar_init(o_free, 128);
-    tc::mbar_init(&drain[0], 1);
-    tc::mbar_init(&drain[1], 1);
-    *abort_flag = 0;
-    tc::fence_mbar_init();
-  }
-  if (warp == 1) tc::tmem_alloc(tmem_slot, TMEM_COLS);
-  tc::tc_fence_before();
-  __syncthreads();
-  tc::tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  // a ring of `depth` slots filled for blocks g = g0 .. g0 + n - 1 of the run
-  auto produce = [&](uint64_t* full, uint64_t* empty, int depth, int g0, int n, auto load) -> bool {
-    for (int j = 0; j < n; ++j) {
-      const int g = g0 + j;
-      const int s = g % depth;
-      if (!tc::mbar_wait(&empty[s], ((uint32_t)(g / depth) & 1u) ^ 1u, abort_flag, status)) {
-        fail(RC_DEV_TIMEOUT_EMPTY);
-        return false;
-      }
-      tc::mbar_expect_tx(&full[s], KV_TILE);
-      load(s, j, &full[s]);
-    }
-    return true;
-  };
-  auto drain_ring = [&](uint64_t* full, int depth, int g_end) {
-    for (int g = max(0, g_end - depth); g < g_end; ++g)
-      if (!tc::mbar_wait_drain(&full[g % depth], (uint32_t)(g / depth) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-  };
-
-  if (warp == 0) {
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmQ);
-      tc::prefetch_tmap(&tmK);
-      int gk = 0, items = 0;
-      bool ok = true;
-      for (int k = 0; ok; ++k) {
-        const Work w = work(k);
-        if (!w.valid) break;
-        if (k > 0 && !tc::mbar_wait(q_empty, (uint32_t)(k - 1) & 1u, abort_flag, status)) {
-          fail(RC_DEV_TIMEOUT_EMPTY);
-          break;
-        }
-        tc::mbar_expect_tx(q_full, Q_BYTES);
-        const int qrow = w.b * p.S + w.q0;
-        tc::tma_load_2d(sQ, &tmQ, q_full, w.h * D, qrow);
-        tc::tma_load_2d(sQ + Q_BYTES / 2, &tmQ, q_full, w.h * D + 64, qrow);
-        ++items;
-        ok = produce(k_full, k_empty, stages, gk, w.nkb, [&](int s, int j, uint64_t* bar) {
-          uint8_t* sk = kring + (size_t)s * KV_TILE;
-          const int krow = w.b * p.S + j * BN;
-          tc::tma_load_2d(sk, &tmK, bar, w.g * D, krow);
-          tc::tma_load_2d(sk + BN * 128, &tmK, bar, w.g * D + 64, krow);
-        });
-        gk += w.nkb;
-      }
-      drain_ring(k_full, stages, gk);
-      if (items > 0 && !tc::mbar_wait_drain(q_full, (uint32_t)(items - 1) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-    }
-    __syncwarp();
-  } else if (warp == 3) {
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmV);
-      int gv = 0;
-      bool ok = true;
-      for (int k = 0; ok; ++k) {
-        const Work w = work(k);
-        if (!w.valid) break;
-        ok = produce(v_full, v_empty, vstages, gv, w.nkb, [&](int s, int j, uint64_t* bar) {
-          uint8_t* sv = vring + (size_t)s * KV_TILE;
-          if constexpr (VT) {
-            tc::tma_load_2d(sv, &tmV, bar, j * BN, (w.b * p.Hkv + w.g) * D);
-          } else {
-            const int krow = w.b * p.S + j * BN;
-            tc::tma_load_2d(sv, &tmV, bar, w.g * D, krow);
-            tc::tma_load_2d(sv + BN * 128, &tmV, bar, w.g * D + 64, krow);
-          }
-        });
-        gv += w.nkb;
-      }
-      drain_ring(v_full, vstages, gv);
-    }
-    __syncwarp();
-  } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
-      const uint32_t sq = tc::smem_u32(sQ);
-      int gs = 0;
-      bool ok = true;
-      for (int k = 0; ok; ++k) {
-        const Work w = work(k);
-        if (!w.valid) break;
-        if (!tc::mbar_wait(q_full, (uint32_t)k & 1u, abort_flag, status)) {
-          ok = false;
-          break;
-        }
-        for (int j = 0; j < w.nkb; ++j) {
-          const int g = gs + j;
-          const int s = g % stages;
-          // the S buffer is free once the softmax holds S_{g-1} in registers
-          ok = (g == 0 || tc::mbar_wait(s_free, (uint32_t)(g - 1) & 1u, abort_flag, status)) &&
-               tc::mbar_wait(&k_full[s], (uint32_t)(g / stages) & 1u, abort_flag, status);
-          if (!ok) break;
-          tc::tc_fence_after();
-          const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
-#pragma unroll
-          for (int ks = 0; ks < D / 16; ++ks) {
-            const uint32_t off = (uint32_t)(ks % 4) * 32;
-            tc::umma_bf16(tmem, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
-                          tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
-          }
-          tc::umma_commit(s_full);
-          tc::umma_commit(&k_empty[s]);
-        }
-        if (!ok) break;
-        tc::umma_commit(q_empty);  // Q may be replaced once this tile's S products are done
-        gs += w.nkb;
-      }
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_FULL);
-        tc::umma_commit(&drain[0]);
-        if (!tc::mbar_wait_drain(&drain[0], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();
-  } else if (warp == 2) {
-    if (lane == 0) {
-      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
-      const uint32_t tO = tmem + O_COL, tP = tmem + P_COL;
-      int gp = 0;
-      bool ok = true;
-      for (int k = 0; ok; ++k) {
-        const Work w = work(k);
-        if (!w.valid) break;
-        // O still holds the previous tile until its softmax warps have read it out
-        if (k > 0 && !tc::mbar_wait(o_free, (uint32_t)(k - 1) & 1u, abort_flag, status)) {
-          ok = false;
-          break;
-        }
-        for (int j = 0; j < w.nkb; ++j) {
-          const int g = gp + j;
-          const int s = g % vstages;
-          ok = tc::mbar_wait(&v_full[s], (uint32_t)(g / vstages) & 1u, abort_flag, status) &&
-               tc::mbar_wait(p_full, (uint32_t)g & 1u, abort_flag, status);
-          if (!ok) break;
-          tc::tc_fence_after();
-          const uint32_t sv = tc::smem_u32(vring + (size_t)s * KV_TILE);
-#pragma unroll
-          for (int ks = 0; ks < BN / 16; ++ks) {
-            const uint32_t off = (uint32_t)(ks % 4) * 32;
-            uint64_t db;
-            if constexpr (VT)
-              db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
-            else
-              db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
-            tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
-          }
-          tc::umma_commit(pv_full);
-          tc::umma_commit(&v_empty[s]);
-        }
-        gp += w.nkb;
-      }
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_FULL);
-        tc::umma_commit(&drain[1]);
-        if (!tc::mbar_wait_drain(&drain[1], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();
-  } else {
-    int gsm = 0;
-    for (int k = 0; !*abort_flag; ++k) {
-      const Work w = work(k);
-      if (!w.valid) break;
-      softmax_sdb<BN, 1>(p, warp & 3, lane, w.q0, w.nkb, w.b, w.h, tmem, 0u, O_COL, P_COL, s_full, s_free, p_full,
-                         pv_full, abort_flag, status, gsm, o_free);
-      gsm += w.nkb;
-    }
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    __syncwarp();
-    tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, TMEM_COLS);
-  }
-}
-
-// Two query tiles per CTA with key blocks of 64 and a P buffer per tile
-// (TileSize M = 256, N = 64, Parallel = 1). TMEM per tile t: S_t (64
-// columns), P_t (32, two bf16 per column) and O_t (128): 448 columns. With P
-// apart from S, S_{j+1} of a tile is issued as soon as its softmax holds S_j
-// in registers, so the tensor pipe computes it while the softmax
-// exponentiates, and the two tiles' softmax warpgroups run independently of
-// each other. The UMMAs come from four warps (the S and the P V products of
-// each tile), K and V from a producer warp each; a ring slot is refilled when
-// every tile that read the block held there has released it.
-//   warp 0      : TMA producer of Q (both tiles) and of the K ring
-//   warp 1      : TMA producer of the V ring
-//   warps 2, 3  : S_t = Q_t K_j^T issue for tile 0 / 1 (warp 2 also owns TMEM)
-//   warps 4, 5  : O_t += P_t V_j issue for tile 0 / 1
-//   warps 6..13 : softmax of tile (warp - 6) / 4, TMEM lane quadrant warp % 4
-constexpr int kThreads5 = 448;
-
-template <bool VT>
-__global__ void __launch_bounds__(kThreads5, 1)
-    attn5_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                 const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
-  constexpr int BN = 64;
-  constexpr int Q_BYTES = BM * D * 2;
-  constexpr int KV_TILE = BN * D * 2;
-  constexpr uint32_t S_COL = 0, P_COL = 2 * BN, O_COL = 3 * BN;  // tile t: + t*BN, + t*BN/2, + t*D
-
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;  // [2] tiles
-  uint8_t* kring = smem + 2 * Q_BYTES;
-  uint8_t* vring = kring + (size_t)stages * KV_TILE;
-  uint64_t* q_full = (uint64_t*)(vring + (size_t)stages * KV_TILE);
-  uint64_t* k_full = q_full + 1;              // [stages]
-  uint64_t* v_full = k_full + stages;         // [stages]
-  uint64_t* k_empty = v_full + stages;        // [2 tiles][stages]
-  uint64_t* v_empty = k_empty + 2 * stages;   // [2 tiles][stages]
-  uint64_t* s_full = v_empty + 2 * stages;    // [2]
-  uint64_t* s_free = s_full + 2;              // [2]
-  uint64_t* p_full = s_free + 2;              // [2]
-  uint64_t* pv_full = p_full + 2;             // [2]
-  uint64_t* drain = pv_full + 2;              // [4] one per issuing warp
-  uint32_t* tmem_slot = (uint32_t*)(drain + 4);
-  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
-  volatile int* status = p.status;
-
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int pairs = (p.q_blocks + 1) / 2;
-  const int BH = p.B * p.Hq;
-  int pb, bh;
-  if (p.raster == 0) {
-    pb = blockIdx.x % pairs;
-    bh = blockIdx.x / pairs;
-  } else {
-    pb = pairs - 1 - (int)(blockIdx.x / BH);
-    bh = blockIdx.x % BH;
-  }
-  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
-  int q0[2], nkb[2];
-#pragma unroll
-  for (int t = 0; t < 2; ++t) {
-    q0[t] = (2 * pb + t) * BM;
-    const int end = p.causal ? min(q0[t] + BM, p.S) : p.S;
-    nkb[t] = q0[t] < p.S ? (end + BN - 1) / BN : 0;
-  }
-  const int nblk = max(nkb[0], nkb[1]);
-
-  auto fail = [&](int code) {
-    *abort_flag = 1;
-    tc::record_failure(status, code);
-  };
-
-  if (threadIdx.x == 0) {
-    tc::mbar_init(q_full, 1);
-    for (int s = 0; s < stages; ++s) {
-      tc::mbar_init(&k_full[s], 1);
-      tc::mbar_init(&v_full[s], 1);
-    }
-    for (int i = 0; i < 2 * stages; ++i) {
-      tc::mbar_init(&k_empty[i], 1);
-      tc::mbar_init(&v_empty[i], 1);
-    }
-    for (int t = 0; t < 2; ++t) {
-      tc::mbar_init(&s_full[t], 1);
-      tc::mbar_init(&s_free[t], 128);
-      tc::mbar_init(&p_full[t], 128);
-      tc::mbar_init(&pv_full[t], 1);
-    }
-    for (int i = 0; i < 4; ++i) tc::mbar_init(&drain[i], 1);
-    *abort_flag = 0;
-    tc::fence_mbar_init();
-  }
-  if (warp == 2) tc::tmem_alloc(tmem_slot, 512);
-  tc::tc_fence_before();
-  __syncthreads();
-  tc::tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-
-  // Slot s of a ring last held key block j - stages; tile t read it iff
-  // j - stages < nkb[t], and released it in the ((j - stages) / stages)-th
-  // phase of its barrier for slot s (parity ph ^ 1; a fresh barrier passes).
-  auto produce = [&](uint64_t* full, uint64_t* empty, auto load) {
-    int j = 0;
-    for (; j < nblk; ++j) {
-      const int s = j % stages;
-      const uint32_t ph = (uint32_t)(j / stages) & 1u;
-      bool ok = true;
-      for (int t = 0; t < 2 && ok; ++t)
-        if (j - stages < nkb[t]) ok = tc::mbar_wait(&empty[t * stages + s], ph ^ 1u, abort_flag, status);
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_EMPTY);
-        break;
-      }
-      tc::mbar_expect_tx(&full[s], KV_TILE);
-      load(s, j, &full[s]);
-    }
-    for (int i = max(0, j - stages); i < j; ++i)
-      if (!tc::mbar_wait_drain(&full[i % stages], (uint32_t)(i / stages) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
-  };
-
-  if (warp == 0) {
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmQ);
-      tc::prefetch_tmap(&tmK);
-      tc::mbar_expect_tx(q_full, 2 * Q_BYTES);
-#pragma unroll
-      for (int t = 0; t < 2; ++t) {
-        const int qrow = b * p.S + q0[t];
-        tc::tma_load_2d(sQ + t * Q_BYTES, &tmQ, q_full, h * D, qrow);
-        tc::tma_load_2d(sQ + t * Q_BYTES + Q_BYTES / 2, &tmQ, q_full, h * D + 64, qrow);
-      }
-      produce(k_full, k_empty, [&](int s, int j, uint64_t* bar) {
-        uint8_t* sk = kring + (size_t)s * KV_TILE;
-        const int krow = b * p.S + j * BN;
-        tc::tma_load_2d(sk, &tmK, bar, g * D, krow);
-        tc::tma_load_2d(sk + BN * 128, &tmK, bar, g * D + 64, krow);
-      });
-      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-    }
-    __syncwarp();  // reconverge before the final block barrier
-  } else if (warp == 1) {
-    if (lane == 0) {
-      tc::prefetch_tmap(&tmV);
-      produce(v_full, v_empty, [&](int s, int j, uint64_t* bar) {
-        uint8_t* sv = vring + (size_t)s * KV_TILE;
-        if constexpr (VT) {
-          tc::tma_load_2d(sv, &tmV, bar, j * BN, (b * p.Hkv + g) * D);
-        } else {
-          const int krow = b * p.S + j * BN;
-          tc::tma_load_2d(sv, &tmV, bar, g * D, krow);
-          tc::tma_load_2d(sv + BN * 128, &tmV, bar, g * D + 64, krow);
-        }
-      });
-    }
-    __syncwarp();
-  } else if (warp <= 3) {  // S issue of tile warp - 2
-    const int t = warp - 2;
-    if (lane == 0 && nkb[t] > 0) {
-      constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
-      const uint32_t sq = tc::smem_u32(sQ + t * Q_BYTES);
-      const uint32_t tS = tmem + S_COL + (uint32_t)(t * BN);
-      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
-      for (int j = 0; ok && j < nkb[t]; ++j) {
-        // the S buffer is free once the softmax holds S_{j-1} in registers
-        if (j > 0) ok = tc::mbar_wait(&s_free[t], (uint32_t)(j - 1) & 1u, abort_flag, status);
-        const int s = j % stages;
-        ok = ok && tc::mbar_wait(&k_full[s], (uint32_t)(j / stages) & 1u, abort_flag, status);
-        if (!ok) break;
-        tc::tc_fence_after();
-        const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
-#pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
-                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
-        }
-        tc::umma_commit(&s_full[t]);
-        tc::umma_commit(&k_empty[t * stages + s]);
-      }
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_FULL);
-        tc::umma_commit(&drain[t]);
-        if (!tc::mbar_wait_drain(&drain[t], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();
-  } else if (warp <= 5) {  // P V issue of tile warp - 4
-    const int t = warp - 4;
-    if (lane == 0 && nkb[t] > 0) {
-      constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
-      const uint32_t tO = tmem + O_COL + (uint32_t)(t * D), tP = tmem + P_COL + (uint32_t)(t * BN / 2);
-      bool ok = true;
-      for (int j = 0; ok && j < nkb[t]; ++j) {
-        const int s = j % stages;
-        ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / stages) & 1u, abort_flag, status) &&
-             tc::mbar_wait(&p_full[t], (uint32_t)j & 1u, abort_flag, status);
-        if (!ok) break;
-        tc::tc_fence_after();
-        const uint32_t sv = tc::smem_u32(vring + (size_t)s * KV_TILE);
-#pragma unroll
-        for (int ks = 0; ks < BN / 16; ++ks) {
-          uint64_t db;
-          if constexpr (VT)
-            db = tc::sw128_desc(sv + (uint32_t)(ks % 4) * 32);
-          else
-            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
-          tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
-        }
-        tc::umma_commit(&pv_full[t]);
-        tc::umma_commit(&v_empty[t * stages + s]);
-      }
-      if (!ok) {
-        fail(RC_DEV_TIMEOUT_FULL);
-        tc::umma_commit(&drain[2 + t]);
-        if (!tc::mbar_wait_drain(&drain[2 + t], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
-      }
-    }
-    __syncwarp();
-  } else {
-    const int t = (warp - 6) / 4;
-    softmax_sdb<BN, 1>(p, warp & 3, lane, q0[t], nkb[t], b, h, tmem, S_COL + (uint32_t)(t * BN),
-                       O_COL + (uint32_t)(t * D), P_COL + (uint32_t)(t * BN / 2), &s_full[t], &s_free[t], &p_full[t],
-                       &pv_full[t], abort_flag, status);
-  }
-  tc::tc_fence_before();
-  __syncthreads();
-  if (warp == 2) {
-    __syncwarp();
-    tc::tc_fence_after();
-    tc::tmem_dealloc(tmem, 512);
   }
 }
 
@@ -2119,120 +1020,114 @@ __global__ void transpose_v_kernel(const __nv_bfloat16* __restrict__ V, int S, i
   }
 }
 
-// Q tiles + K/V ring + P tiles + 1 KB alignment slack + barriers (at most
-// 1 + 6 * stages + 8 of them, 8 B each, plus two words: 512 B for stages <= 5)
-size_t smem_bytes(int bn, int stages, int qtiles) {
-  return (size_t)qtiles * BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)qtiles * BM * bn * 2 + 1024 + 512;
+// P0 kernel: Q tile + K/V ring + P tile + 1 KB alignment slack + barriers
+// (1 + 2 * stages + 4 of them, 8 B each, plus two words: 512 B for stages <= 5)
+size_t smem_bytes(int bn, int stages) {
+  return (size_t)BM * D * 2 + (size_t)stages * 2 * bn * D * 2 + (size_t)BM * bn * 2 + 1024 + 512;
 }
 
-template <int BN, bool VT, bool PINGPONG, bool PT = false, bool SDB = false, bool PAR = false>
-rc_status launch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
-                 float* lse, const LaunchCtx& c) {
-  static_assert(!PAR || (PT && !(SDB && PINGPONG)), "split UMMA issue: P in TMEM");
-  // PAR: two query tiles with one issuing warp each (attn3), or one query tile
-  // with one or two (SDB) S buffers and separate S and P V issuers (attn4)
-  // (two tiles with BN = 64: P apart from S, four issuing warps, attn5)
-  auto pick = []() {
-    if constexpr (PAR && PINGPONG && BN == 64) return &attn5_kernel<VT>;
-    else if constexpr (PAR && PINGPONG) return &attn3_kernel<BN, VT>;
-    else if constexpr (PAR) return &attn4_kernel<BN, VT, SDB ? 2 : 1>;
-    else if constexpr (PINGPONG) return &attn2_kernel<BN, VT, PT, SDB>;
-    else return &attn_kernel<BN, VT>;
-  };
-  auto kern = pick();
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
-    // the largest shared-memory carve-out, so that two 1-tile CTAs can share an SM
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention: smem attribute: %s", cudaGetErrorString(e));
-    attr = true;
-  }
-  const uint64_t BS = (uint64_t)d.batch * d.seq;
-  CUtensorMap tq, tk, tv;
-  RC_TRY(tcg::encode_2d(&tq, Q, (uint64_t)d.heads_q * D, BS, BM));
-  RC_TRY(tcg::encode_2d(&tk, K, (uint64_t)d.heads_kv * D, BS, BN));
-  if (VT)
-    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.seq, (uint64_t)d.batch * d.heads_kv * D, BM));
-  else
-    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.heads_kv * D, BS, BN));
-  Params p;
-  memset(&p, 0, sizeof p);
-  p.B = (int)d.batch;
-  p.S = (int)d.seq;
-  p.Hq = (int)d.heads_q;
-  p.Hkv = (int)d.heads_kv;
-  p.group = (int)(d.heads_q / d.heads_kv);
-  p.q_blocks = (int)((d.seq + BM - 1) / BM);
-  p.causal = d.causal ? 1 : 0;
-  p.scale_log2 = (float)(d.scale * 1.4426950408889634);
-  p.raster = k.raster;
-  p.O = (__nv_bfloat16*)O;
-  p.lse = lse;
-  p.status = c.status;
-  const long long ctas = (long long)p.B * p.Hq * (PINGPONG ? (p.q_blocks + 1) / 2 : p.q_blocks);
-  if (ctas > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
-  const int qtiles = PINGPONG ? 2 : 1;
-  size_t smem = smem_bytes(BN, k.stages, qtiles) - (PT ? (size_t)qtiles * BM * BN * 2 : 0);
-  if constexpr (PAR && !PINGPONG) smem = attn4_smem<BN, SDB ? 2 : 1>(k.stages);
-  const int threads = PAR ? (PINGPONG ? (BN == 64 ? kThreads5 : kThreads3) : kThreads4) : PINGPONG ? kThreads2 : kThreads;
-  kern<<<(unsigned)ctas, threads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) {
-    cudaFuncAttributes fa;
-    memset(&fa, 0, sizeof fa);
-    cudaFuncGetAttributes(&fa, kern);
-    return rc_fail(RC_ERR_CUDA,
-                   "attention launch: %s (%d threads, %zu B dynamic shared memory; kernel: %d registers, %zu B static "
-                   "and at most %d B dynamic shared memory, at most %d threads)",
-                   cudaGetErrorString(e), threads, smem, fa.numRegs, fa.sharedSizeBytes, fa.maxDynamicSharedSizeBytes,
-                   fa.maxThreadsPerBlock);
-  }
+template <typename Kern>
+rc_status smem_attributes(Kern kern, bool& done) {
+  if (done) return RC_OK;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+  // the largest shared-memory carve-out, so that two one-tile CTAs can share an SM
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention: smem attribute: %s", cudaGetErrorString(e));
+  done = true;
   return RC_OK;
 }
 
-// Persistent one-tile kernel (Loop order 2): grid = two CTAs per SM, at most one per tile.
-template <bool VT>
-rc_status launch_persistent(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V,
-                            void* O, float* lse, const LaunchCtx& c) {
-  auto kern = attn4p_kernel<VT>;
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention: smem attribute: %s", cudaGetErrorString(e));
-    attr = true;
-  }
+// Tensor maps and kernel parameters shared by both kernel families.
+template <int BN, bool VT>
+rc_status prepare(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
+                  float* lse, const LaunchCtx& c, CUtensorMap* tq, CUtensorMap* tk, CUtensorMap* tv, Params* p) {
   const uint64_t BS = (uint64_t)d.batch * d.seq;
-  CUtensorMap tq, tk, tv;
-  RC_TRY(tcg::encode_2d(&tq, Q, (uint64_t)d.heads_q * D, BS, BM));
-  RC_TRY(tcg::encode_2d(&tk, K, (uint64_t)d.heads_kv * D, BS, 64));
+  RC_TRY(tcg::encode_2d(tq, Q, (uint64_t)d.heads_q * D, BS, BM));
+  RC_TRY(tcg::encode_2d(tk, K, (uint64_t)d.heads_kv * D, BS, BN));
   if (VT)
-    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.seq, (uint64_t)d.batch * d.heads_kv * D, BM));
+    RC_TRY(tcg::encode_2d(tv, V, (uint64_t)d.seq, (uint64_t)d.batch * d.heads_kv * D, BM));
   else
-    RC_TRY(tcg::encode_2d(&tv, V, (uint64_t)d.heads_kv * D, BS, 64));
-  Params p;
-  memset(&p, 0, sizeof p);
-  p.B = (int)d.batch;
-  p.S = (int)d.seq;
-  p.Hq = (int)d.heads_q;
-  p.Hkv = (int)d.heads_kv;
-  p.group = (int)(d.heads_q / d.heads_kv);
-  p.q_blocks = (int)((d.seq + BM - 1) / BM);
-  p.causal = d.causal ? 1 : 0;
-  p.scale_log2 = (float)(d.scale * 1.4426950408889634);
-  p.raster = k.raster;
-  p.O = (__nv_bfloat16*)O;
-  p.lse = lse;
-  p.status = c.status;
-  const long long tiles = (long long)p.B * p.Hq * p.q_blocks;
-  if (tiles > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: too many tiles");
-  const int sms = c.num_sms > 0 ? c.num_sms : 1;
-  const int grid = (int)std::min<long long>(tiles, 2LL * sms);
-  kern<<<grid, kThreads4, attn4p_smem(k.stages), (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "attention (persistent) launch: %s", cudaGetErrorString(e));
+    RC_TRY(tcg::encode_2d(tv, V, (uint64_t)d.heads_kv * D, BS, BN));
+  memset(p, 0, sizeof *p);
+  p->B = (int)d.batch;
+  p->S = (int)d.seq;
+  p->Hq = (int)d.heads_q;
+  p->Hkv = (int)d.heads_kv;
+  p->group = (int)(d.heads_q / d.heads_kv);
+  p->q_blocks = (int)((d.seq + BM - 1) / BM);
+  p->causal = d.causal ? 1 : 0;
+  p->scale_log2 = (float)(d.scale * 1.4426950408889634);
+  p->raster = k.raster;
+  p->O = (__nv_bfloat16*)O;
+  p->lse = lse;
+  p->status = c.status;
+  if ((long long)p->B * p->Hq * p->q_blocks > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: grid too large");
   return RC_OK;
+}
+
+template <typename Kern>
+rc_status launched(Kern kern, int threads, size_t smem) {
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) return RC_OK;
+  cudaFuncAttributes fa;
+  memset(&fa, 0, sizeof fa);
+  cudaFuncGetAttributes(&fa, kern);
+  return rc_fail(RC_ERR_CUDA,
+                 "attention launch: %s (%d threads, %zu B dynamic shared memory; kernel: %d registers, %zu B static "
+                 "and at most %d B dynamic shared memory, at most %d threads)",
+                 cudaGetErrorString(e), threads, smem, fa.numRegs, fa.sharedSizeBytes, fa.maxDynamicSharedSizeBytes,
+                 fa.maxThreadsPerBlock);
+}
+
+// The P0 kernel: one UMMA-issuing warp, P in shared memory.
+template <int BN, bool VT>
+rc_status launch_basic(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
+                       float* lse, const LaunchCtx& c) {
+  auto kern = attn_kernel<BN, VT>;
+  static bool attr = false;
+  RC_TRY(smem_attributes(kern, attr));
+  CUtensorMap tq, tk, tv;
+  Params p;
+  RC_TRY((prepare<BN, VT>(k, d, Q, K, V, O, lse, c, &tq, &tk, &tv, &p)));
+  const size_t smem = smem_bytes(BN, k.stages);
+  kern<<<(unsigned)(p.B * p.Hq * p.q_blocks), kThreads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  return launched(kern, kThreads, smem);
+}
+
+// The split-issue kernel: NSB S buffers, SPLIT softmax threads per row, row sums on the tensor core.
+template <int BN, bool VT, int NSB, int SPLIT, bool SUMC>
+rc_status launch_split(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
+                       float* lse, const LaunchCtx& c) {
+  auto kern = attn4_kernel<BN, VT, NSB, SPLIT, SUMC>;
+  static bool attr = false;
+  RC_TRY(smem_attributes(kern, attr));
+  CUtensorMap tq, tk, tv;
+  Params p;
+  RC_TRY((prepare<BN, VT>(k, d, Q, K, V, O, lse, c, &tq, &tk, &tv, &p)));
+  const size_t smem = attn4_smem<BN, NSB, SPLIT, SUMC>(k.stages);
+  constexpr int threads = attn4_threads<SPLIT>();
+  kern<<<(unsigned)(p.B * p.Hq * p.q_blocks), threads, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  return launched(kern, threads, smem);
+}
+
+template <int BN, bool VT>
+rc_status dispatch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
+                   float* lse, const LaunchCtx& c) {
+  if (k.persistent == 0) return launch_basic<BN, VT>(k, d, Q, K, V, O, lse, c);
+  const bool two_sb = k.unroll == 2, split = k.persistent == 2;
+  if (k.location == 2) {
+    if constexpr (!VT) {
+      if (two_sb) return split ? launch_split<BN, false, 2, 2, true>(k, d, Q, K, V, O, lse, c)
+                               : launch_split<BN, false, 2, 1, true>(k, d, Q, K, V, O, lse, c);
+      return split ? launch_split<BN, false, 1, 2, true>(k, d, Q, K, V, O, lse, c)
+                   : launch_split<BN, false, 1, 1, true>(k, d, Q, K, V, O, lse, c);
+    }
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: row sums on the tensor core need V as given");
+  }
+  if (two_sb) return split ? launch_split<BN, VT, 2, 2, false>(k, d, Q, K, V, O, lse, c)
+                           : launch_split<BN, VT, 2, 1, false>(k, d, Q, K, V, O, lse, c);
+  return split ? launch_split<BN, VT, 1, 2, false>(k, d, Q, K, V, O, lse, c)
+               : launch_split<BN, VT, 1, 1, false>(k, d, Q, K, V, O, lse, c);
 }
 
 }  // namespace attn
@@ -2241,6 +1136,15 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
                               void* O, float* lse, void* workspace, const LaunchCtx& c) {
   if (d.head_dim != attn::D) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: head_dim must be 128");
   if (d.batch * d.seq > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: B*S too large");
+  // the same rules as the schedule legality check, so a launch never gets a kernel it cannot run
+  if (k.tile_m != attn::BM || k.raster > 1 || (k.tile_n != 64 && k.tile_n != 128))
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: 128-row query tiles, 64- or 128-key blocks, loop order 0 or 1");
+  if (k.persistent == 0 && (k.location != 0 || k.unroll != 1))
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: one issuing warp keeps P in shared memory, one S buffer");
+  if (k.persistent > 0 && (k.location == 0 || k.stages < 2))
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: split UMMA issue needs P in TMEM and two stages");
+  if (k.location == 2 && k.layout != 0)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: row sums on the tensor core need V as given");
   const void* Vuse = V;
   if (k.layout == 1) {
     if (d.seq % 8) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: transposed V needs seq %% 8 == 0");
@@ -2252,46 +1156,7 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
     Vuse = workspace;
   }
   const bool vt = k.layout == 1;
-  const bool pp = k.tile_m == 256;  // two query tiles per CTA, ping-pong softmax
-  if (pp && k.stages < 2) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: ping-pong needs >= 2 stages");
-  const bool pt = k.location == 1;  // P kept in tensor memory
-  if (pt && !pp && k.persistent != 1)
-    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: P in TMEM needs two query tiles or split UMMA issue");
-  const bool par = k.persistent == 1;  // UMMA issue split over several warps
-  if (k.raster == 2) {  // persistent CTAs over longest-first tiles (one-tile kernel, one S buffer, BN 64)
-    if (!(par && pt && !pp && k.tile_n == 64 && k.unroll == 1 && k.stages >= 2 && k.stages <= 3))
-      return rc_fail(RC_ERR_ILLEGAL_SCHEDULE,
-                     "attention: loop order 2 needs one query tile, split issue, P in TMEM, BN 64, unroll 1, 2-3 stages");
-    return vt ? attn::launch_persistent<true>(k, d, Q, K, Vuse, O, lse, c)
-              : attn::launch_persistent<false>(k, d, Q, K, Vuse, O, lse, c);
-  }
-  if (k.unroll == 2 && !(par && !pp)) {  // two key blocks in flight per query tile
-    if (!(pp && pt && k.tile_n == 64 && k.stages >= 4) || k.persistent)
-      return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: unroll 2 needs 2 query tiles, P in TMEM, BN 64, 4 stages");
-    return vt ? attn::launch<64, true, true, true, true>(k, d, Q, K, Vuse, O, lse, c)
-              : attn::launch<64, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c);
-  }
-  const bool sdb = k.unroll == 2;  // one tile, split issue: two S buffers (two key blocks in flight)
-  if (par && !pt) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: split UMMA issue needs P in TMEM");
-  if (par && !pp && k.stages < 2)
-    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: two S buffers need at least two K/V stages");
-#define RC_ATT(BN)                                                                                  \
-  if (k.tile_n == BN) {                                                                             \
-    if (par && pp) return vt ? attn::launch<BN, true, true, true, false, true>(k, d, Q, K, Vuse, O, lse, c) \
-                             : attn::launch<BN, false, true, true, false, true>(k, d, Q, K, Vuse, O, lse, c); \
-    if (par && sdb) return vt ? attn::launch<BN, true, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c) \
-                              : attn::launch<BN, false, false, true, true, true>(k, d, Q, K, Vuse, O, lse, c); \
-    if (par) return vt ? attn::launch<BN, true, false, true, false, true>(k, d, Q, K, Vuse, O, lse, c) \
-                       : attn::launch<BN, false, false, true, false, true>(k, d, Q, K, Vuse, O, lse, c); \
-    if (pp && pt) return vt ? attn::launch<BN, true, true, true>(k, d, Q, K, Vuse, O, lse, c)       \
-                            : attn::launch<BN, false, true, true>(k, d, Q, K, Vuse, O, lse, c);     \
-    if (pp) return vt ? attn::launch<BN, true, true>(k, d, Q, K, Vuse, O, lse, c)                   \
-                      : attn::launch<BN, false, true>(k, d, Q, K, Vuse, O, lse, c);                 \
-    return vt ? attn::launch<BN, true, false>(k, d, Q, K, Vuse, O, lse, c)                          \
-              : attn::launch<BN, false, false>(k, d, Q, K, Vuse, O, lse, c);                        \
-  }
-  RC_ATT(64)
-  RC_ATT(128)
-#undef RC_ATT
-  return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: key block %d", k.tile_n);
+  if (k.tile_n == 64)
+    return vt ? attn::dispatch<64, true>(k, d, Q, K, Vuse, O, lse, c) : attn::dispatch<64, false>(k, d, Q, K, Vuse, O, lse, c);
+  return vt ? attn::dispatch<128, true>(k, d, Q, K, Vuse, O, lse, c) : attn::dispatch<128, false>(k, d, Q, K, Vuse, O, lse, c);
 }

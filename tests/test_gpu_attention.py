@@ -23,11 +23,12 @@ def att_op(B, S, Hq, Hkv, causal=True):
     return rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=128, causal=int(causal))
 
 
-def sched(op, bn, stages, raster, layout, bm=128, p_tmem=0, unroll=1, par=0):
-    return op.schedule(rc.T(rc.T_TILE_SIZE, bm, axis=0), rc.T(rc.T_TILE_SIZE, bn, axis=1),
-                       rc.T(rc.T_PIPELINE_STAGES, stages), rc.T(rc.T_LOOP_ORDER, raster, group=1),
-                       rc.T(rc.T_LAYOUT, layout), rc.T(rc.T_COMPUTE_LOCATION, p_tmem), rc.T(rc.T_UNROLL, unroll),
-                       rc.T(rc.T_PARALLEL, par))
+def sched(op, bn, stages, raster, layout, loc=0, unroll=1, par=0):
+    """loc: P in shared (0) or tensor memory (1), or row sums on the tensor core (2); unroll: S buffers;
+    par: one issuing warp (0), issue split over warps (1), and two softmax threads per row (2)."""
+    return op.schedule(rc.T(rc.T_TILE_SIZE, bn, axis=1), rc.T(rc.T_PIPELINE_STAGES, stages),
+                       rc.T(rc.T_LOOP_ORDER, raster, group=1), rc.T(rc.T_LAYOUT, layout),
+                       rc.T(rc.T_COMPUTE_LOCATION, loc), rc.T(rc.T_UNROLL, unroll), rc.T(rc.T_PARALLEL, par))
 
 
 def run(op, s, Q, K, V):
@@ -46,21 +47,23 @@ def test_attention_schedule_sweep(B, S, Hq, Hkv, causal):
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=causal)
     op = att_op(B, S, Hq, Hkv, causal)
     n = 0
-    for bm, bn, st, ra, lay, pt, un, par in itertools.product((128, 256), (64, 128), (1, 2, 3, 4), (0, 1, 2), (0, 1),
-                                                              (0, 1), (1, 2), (0, 1)):
+    for bn, st, ra, lay, loc, un, par in itertools.product((64, 128), (1, 2, 3, 4), (0, 1), (0, 1), (0, 1, 2), (1, 2),
+                                                          (0, 1, 2)):
         try:
-            s = sched(op, bn, st, ra, lay, bm, pt, un, par)
+            s = sched(op, bn, st, ra, lay, loc, un, par)
         except rc.RcError:
             continue  # illegal here (shared memory, S % 8 for the transposed V, variant combinations)
         O, L = run(op, s, Q, K, V)
-        assert rel_err(O, O_ref) <= TOL, (bm, bn, st, ra, lay, pt, un, par, rel_err(O, O_ref))
-        assert rel_err(L, L_ref) <= TOL_LSE, (bm, bn, st, ra, lay, pt, un, par)
+        assert rel_err(O, O_ref) <= TOL, (bn, st, ra, lay, loc, un, par, rel_err(O, O_ref))
+        assert rel_err(L, L_ref) <= TOL_LSE, (bn, st, ra, lay, loc, un, par)
         n += 1
-    assert n >= 24
-    with pytest.raises(rc.RcError):  # one K/V stage cannot feed the ping-pong kernel
-        sched(op, 64, 1, 0, 0, 256)
-    with pytest.raises(rc.RcError):  # per-tile issuers exist only for two tiles with P in TMEM
-        sched(op, 64, 2, 0, 0, 256, 0, 1, 1)
+    assert n >= 40
+    with pytest.raises(rc.RcError):  # split UMMA issue keeps P in tensor memory
+        sched(op, 64, 2, 0, 0, 0, 1, 1)
+    with pytest.raises(rc.RcError):  # row sums on the tensor core read V as given
+        sched(op, 64, 2, 0, 1, 2, 1, 1)
+    with pytest.raises(rc.RcError):  # one issuing warp: one S buffer
+        sched(op, 64, 2, 0, 0, 0, 2, 0)
 
 
 def test_attention_single_token_and_no_lse():
@@ -81,17 +84,17 @@ def test_attention_full_size_sampled_queries():
     qpos = np.array([0, 1, 63, 64, 127, 128, 129, 1000, 1023, 1024, 2000, 2046, 2047], dtype=np.int64)
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=True, qpos=qpos)
     op = att_op(B, S, Hq, Hkv)
-    for s in [op.schedule(), sched(op, 128, 2, 1, 0), sched(op, 64, 3, 0, 1), sched(op, 64, 3, 1, 0, 256),
-              sched(op, 64, 2, 1, 1, 256), sched(op, 128, 2, 1, 0, 256, 1), sched(op, 64, 3, 1, 1, 256, 1),
-              sched(op, 64, 4, 1, 0, 256, 1, 2), sched(op, 64, 5, 0, 1, 256, 1, 2),
-              sched(op, 128, 2, 1, 0, 256, 1, 1, 1), sched(op, 128, 2, 0, 1, 256, 1, 1, 1),
-              sched(op, 64, 5, 1, 0, 256, 1, 1, 1), sched(op, 128, 2, 1, 0, 128, 1, 1, 1),
-              sched(op, 128, 3, 0, 1, 128, 1, 1, 1), sched(op, 64, 4, 1, 0, 128, 1, 1, 1),
-              # one tile with split issue: one S buffer (two CTAs per SM at BN 64, stages 2) or two
-              sched(op, 64, 2, 1, 0, 128, 1, 1, 1), sched(op, 64, 2, 0, 1, 128, 1, 1, 1),
-              sched(op, 64, 3, 1, 0, 128, 1, 2, 1), sched(op, 128, 2, 1, 0, 128, 1, 2, 1),
-              # persistent CTAs walking longest-first tiles (loop order 2)
-              sched(op, 64, 2, 2, 0, 128, 1, 1, 1), sched(op, 64, 3, 2, 1, 128, 1, 1, 1)]:
+    for s in [op.schedule(), sched(op, 128, 2, 1, 0), sched(op, 64, 3, 0, 1), sched(op, 64, 1, 1, 0),
+              # split issue, one S buffer (two CTAs per SM at BN 64) or two, V as given or transposed
+              sched(op, 64, 2, 1, 0, 1, 1, 1), sched(op, 64, 2, 0, 1, 1, 1, 1), sched(op, 64, 3, 1, 0, 1, 1, 1),
+              sched(op, 128, 2, 1, 0, 1, 1, 1), sched(op, 128, 3, 0, 1, 1, 1, 1),
+              sched(op, 64, 2, 1, 0, 1, 2, 1), sched(op, 64, 4, 1, 1, 1, 2, 1), sched(op, 128, 2, 1, 0, 1, 2, 1),
+              # two softmax threads per row
+              sched(op, 64, 2, 1, 0, 1, 1, 2), sched(op, 64, 3, 0, 1, 1, 1, 2), sched(op, 128, 2, 1, 0, 1, 1, 2),
+              sched(op, 64, 2, 1, 0, 1, 2, 2),
+              # row sums of P on the tensor core
+              sched(op, 64, 2, 1, 0, 2, 1, 1), sched(op, 64, 3, 0, 0, 2, 1, 1), sched(op, 128, 2, 1, 0, 2, 1, 1),
+              sched(op, 64, 2, 1, 0, 2, 2, 1), sched(op, 128, 2, 1, 0, 2, 1, 2)]:
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
@@ -104,9 +107,9 @@ def test_flux_shaped_noncausal_attention_sampled_queries():
     qpos = np.array([0, 1, 127, 128, 2047, 2048, 4000, 4095], dtype=np.int64)
     O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=False, qpos=qpos)
     op = att_op(B, S, H, H, causal=False)
-    for s in [op.schedule(), sched(op, 128, 2, 1, 0, 256, 1, 1, 1), sched(op, 64, 2, 1, 0, 256, 1, 1, 1),
-              sched(op, 64, 2, 0, 0, 128, 1, 1, 1), sched(op, 64, 3, 1, 1, 128, 1, 1, 1),
-              sched(op, 128, 2, 1, 0, 128, 1, 2, 1), sched(op, 64, 3, 2, 0, 128, 1, 1, 1)]:
+    for s in [op.schedule(), sched(op, 64, 2, 0, 0, 1, 1, 1), sched(op, 64, 3, 1, 1, 1, 1, 1),
+              sched(op, 128, 2, 1, 0, 1, 2, 1), sched(op, 64, 2, 1, 0, 1, 1, 2), sched(op, 64, 2, 0, 0, 2, 1, 1),
+              sched(op, 128, 2, 0, 0, 2, 1, 1)]:
         O, L = run(op, s, Q, K, V)
         assert rel_err(O[:, qpos], O_ref) <= TOL, str(s)
         assert rel_err(L[:, :, qpos], L_ref) <= TOL_LSE, str(s)
