@@ -49,7 +49,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mlp",
-                    choices=["mlp", "attention", "conv2d", "moe", "gemm_f32", "attention_flux", "decoder_layer"])
+                    choices=["mlp", "attention", "conv2d", "moe", "gemm_f32", "attention_flux", "decoder_layer",
+                             "linear"])
     ap.add_argument("--samples", type=int, default=5000, help="schedules the search measures")
     ap.add_argument("--branching", type=int, default=4,
                     help="MCTS children per expansion (the paper's 2 assumes LLM-proposed transformations; with "
@@ -173,6 +174,8 @@ class Workload:
 
         from paper_2506_01374_gb300 import inputs, rc
         self.name = name
+        self._op = None
+        self.dom_bytes = None  # algorithmic DRAM bytes of the dominant kernel, where stated
         self.horizon = 8  # search horizon T
         self.tasks = False  # composite ops: tuned stage by stage (search_tasks), then jointly
         sh = dict(shape or {})
@@ -187,13 +190,14 @@ class Workload:
             self.tasks = True
             T, H, I = dims(tokens=2048, hidden=4096, inter=14336)
             X, W1, W2 = inputs.mlp(T, H, I, seed=1)
-            self.op = rc.Op(rc.OP_MLP, m=T, n=I, k=H)
+            self._op_spec = (rc.OP_MLP, dict(m=T, n=I, k=H))
             self.host = [X, W1, W2, None]
             self.outs = {3: ((T, H), np.uint16)}
             self.label = "llama3_8b_mlp_swiglu_bf16_T2048_H4096_I14336"
             self.config = {"tokens": T, "hidden": H, "inter": I}
             self.metric = "best-schedule TFLOP/s (Llama-3-8B MLP block, bf16)"
             self.dom_stage, self.dom_flops = 0, 2.0 * T * (2 * I) * H
+            self.dom_bytes = 2.0 * (T * H + 2 * I * H + T * I)  # X and W1 read once, h written once
             self.dom_name = "gate/up GEMM{} (stage 0)"
             self.bound = "tensor"
             self.dtype = "bf16"
@@ -201,13 +205,14 @@ class Workload:
             B, S, Hq, Hkv = dims(batch=1, seq=2048, heads_q=32, heads_kv=8)
             D = 128
             Q, K, V = inputs.attention(B, S, Hq, Hkv, D, seed=4)
-            self.op = rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=1)
+            self._op_spec = (rc.OP_ATTENTION,
+                             dict(batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=1))
             self.host = [Q, K, V, None, None]
             self.outs = {3: ((B, S, Hq, D), np.uint16), 4: ((B, Hq, S), np.float32)}
             self.label = "causal_gqa_attention_B1_S2048_Hq32_Hkv8_d128_bf16"
             self.config = {"batch": B, "seq": S, "heads_q": Hq, "heads_kv": Hkv, "head_dim": D, "causal": True}
             self.metric = "best-schedule TFLOP/s (causal GQA attention, bf16)"
-            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_stage, self.dom_flops = 0, None  # the op's flops
             self.dom_name = "fused attention kernel"
             self.bound = "tensor"
             self.dtype = "bf16"
@@ -216,27 +221,28 @@ class Workload:
             B, S, Hq = dims(batch=1, seq=4096, heads=24)
             Hkv, D = Hq, 128
             Q, K, V = inputs.attention(B, S, Hq, Hkv, D, seed=7)
-            self.op = rc.Op(rc.OP_ATTENTION, batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=0)
+            self._op_spec = (rc.OP_ATTENTION,
+                             dict(batch=B, seq=S, heads_q=Hq, heads_kv=Hkv, head_dim=D, causal=0))
             self.host = [Q, K, V, None, None]
             self.outs = {3: ((B, S, Hq, D), np.uint16), 4: ((B, Hq, S), np.float32)}
             self.label = f"flux_attention_B{B}_S{S}_H{Hq}_d128_noncausal_bf16"
             self.config = {"batch": B, "seq": S, "heads": Hq, "head_dim": D, "causal": False}
             self.metric = "best-schedule TFLOP/s (non-causal MHA attention, bf16)"
-            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_stage, self.dom_flops = 0, None  # the op's flops
             self.dom_name = "fused attention kernel"
             self.bound = "tensor"
             self.dtype = "bf16"
         elif name == "conv2d":
             N, H, W, C = dims(n=2, h=64, w=64, c=320)
             x, w, b = inputs.conv2d(N, H, W, C, C, seed=5)
-            self.op = rc.Op(rc.OP_CONV2D, img_n=N, img_h=H, img_w=W, c_in=C, c_out=C, kr=3, ks=3, stride=1, pad=1,
-                            flags=rc.EPI_BIAS | rc.EPI_SILU)
+            self._op_spec = (rc.OP_CONV2D, dict(img_n=N, img_h=H, img_w=W, c_in=C, c_out=C, kr=3, ks=3, stride=1, pad=1,
+                            flags=rc.EPI_BIAS | rc.EPI_SILU))
             self.host = [x, w, b, None]
             self.outs = {3: ((N, H, W, C), np.uint16)}
             self.label = "conv2d_nhwc_3x3_N2_64x64_C320_bias_silu_bf16"
             self.config = {"n": N, "h": H, "w": W, "c_in": C, "c_out": C, "kernel": 3}
             self.metric = "best-schedule TFLOP/s (UNet conv2d 3x3 + bias + SiLU, bf16)"
-            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_stage, self.dom_flops = 0, None  # the op's flops
             self.dom_name = "implicit-GEMM conv kernel"
             self.bound = "tensor"
             self.dtype = "bf16"
@@ -244,7 +250,7 @@ class Workload:
             self.tasks = True
             T, H, E, I, K = dims(tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
             logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=6)
-            self.op = rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
+            self._op_spec = (rc.OP_MOE, dict(tokens=T, hidden=H, experts=E, inter=I, top_k=K))
             self.host = [logits, X, W1, W2, None]
             self.outs = {4: ((T, H), np.uint16)}
             self.label = "moe_T4096_H7168_E64_I2048_top8_bf16"
@@ -258,7 +264,8 @@ class Workload:
             self.tasks = True
             T, H, Hq, Hkv, I = dims(tokens=2048, hidden=4096, heads_q=32, heads_kv=8, inter=14336)
             self.host = list(inputs.decoder_layer(T, H, Hq, Hkv, I, seed=8)) + [None]
-            self.op = rc.Op(rc.OP_DECODER_LAYER, tokens=T, hidden=H, inter=I, heads_q=Hq, heads_kv=Hkv, head_dim=128)
+            self._op_spec = (rc.OP_DECODER_LAYER,
+                             dict(tokens=T, hidden=H, inter=I, heads_q=Hq, heads_kv=Hkv, head_dim=128))
             self.outs = {7: ((T, H), np.uint16)}
             self.label = f"llama3_8b_decoder_layer_T{T}_H{H}_Hq{Hq}_Hkv{Hkv}_I{I}_bf16"
             self.config = {"tokens": T, "hidden": H, "heads_q": Hq, "heads_kv": Hkv, "inter": I}
@@ -267,21 +274,47 @@ class Workload:
             self.dom_name = "gate/up GEMM + SwiGLU (stage 4)"
             self.bound = "tensor"
             self.dtype = "bf16"
+        elif name == "linear":
+            # the MLP block's down projection as a plain bf16 GEMM: Y = h W2^T, M = 2048, N = 4096, K = 14336
+            M, N, K = dims(m=2048, n=4096, k=14336)
+            X, Wt = inputs.linear_bf16(M, N, K, seed=3)
+            self._op_spec = (rc.OP_LINEAR, dict(m=M, n=N, k=K))
+            self.host = [X, Wt, None]
+            self.outs = {2: ((M, N), np.uint16)}
+            self.label = f"linear_bf16_M{M}_N{N}_K{K}"
+            self.config = {"m": M, "n": N, "k": K}
+            self.metric = "best-schedule TFLOP/s (bf16 GEMM at the MLP down-projection shape)"
+            self.dom_stage, self.dom_flops = 0, 2.0 * M * N * K
+            self.dom_bytes = 2.0 * (M * K + N * K + M * N)
+            self.dom_name = "tensor-core GEMM"
+            self.bound = "tensor"
+            self.dtype = "bf16"
         elif name == "gemm_f32":
             M, N, K = dims(m=256, n=256, k=256)
             A, B, bias = inputs.gemm_f32(M, N, K, seed=0)
-            self.op = rc.Op(rc.OP_GEMM_F32, m=M, n=N, k=K, flags=rc.EPI_BIAS | rc.EPI_RELU)
+            self._op_spec = (rc.OP_GEMM_F32, dict(m=M, n=N, k=K, flags=rc.EPI_BIAS | rc.EPI_RELU))
             self.host = [A, B, bias, None]
             self.outs = {3: ((M, N), np.float32)}
             self.label = "gemm_bias_relu_f32_256^3"
             self.config = {"m": M, "n": N, "k": K}
             self.metric = "best-schedule TFLOP/s (fp32 GEMM + bias + ReLU, 256^3)"
-            self.dom_stage, self.dom_flops = 0, self.op.info["flops"]
+            self.dom_stage, self.dom_flops = 0, None  # the op's flops
             self.dom_name = "fp32 SIMT GEMM"
             self.bound = "alu"
             self.dtype = "f32"
         else:
             raise ValueError(name)
+
+    @property
+    def op(self):
+        """The library's op (created on first use: the oracle arm never loads the library)."""
+        if self._op is None:
+            from paper_2506_01374_gb300 import rc
+            kind, kw = self._op_spec
+            self._op = rc.Op(kind, **kw)
+            if self.dom_flops is None:
+                self.dom_flops = self._op.info["flops"]
+        return self._op
 
     def device_io(self):
         import numpy as np
@@ -317,6 +350,96 @@ class Workload:
         h2d = sum(a.nbytes for a in self.host if a is not None)
         d2h = sum(int(np.prod(s)) * np.dtype(dt).itemsize for s, dt in self.outs.values())
         return h2d, d2h
+
+    def parity(self, sched, io):
+        """Run `sched` once on the device buffers (outside every timed region) and compare sampled outputs
+        with the fp64 oracle at the op's tolerance: 1e-4 normwise for fp32, 2e-2 for bf16, routing
+        bit-exact. Returns {"max_rel_err", "tol", "sample", "ok"}; a schedule whose check fails is not
+        reported."""
+        import numpy as np
+        import torch
+
+        import oracle
+        oracle.build()
+        op = self.op
+
+        def bf(t):
+            u = t.cpu().numpy().view(np.uint16).astype(np.uint32) << np.uint32(16)
+            return u.view(np.float32).astype(np.float64)
+
+        def rel(got, ref):
+            return float(np.max(np.abs(got - ref)) / max(float(np.max(np.abs(ref))), 1e-30))
+
+        tol = 1e-4 if self.dtype == "f32" else 2e-2
+        extra = {}
+        if self.name == "mlp":
+            X, W1, W2 = self.host[:3]
+            rows = np.linspace(0, X.shape[0] - 1, 16).astype(np.int64)
+            op.run(sched, io)
+            op.check()
+            err = rel(bf(io[3])[rows], oracle.mlp_bf16(X, W1, W2, rows=rows))
+            what = f"{len(rows)} of {X.shape[0]} token rows"
+        elif self.name == "linear":
+            X, Wt = self.host[:2]
+            rows = np.linspace(0, X.shape[0] - 1, 16).astype(np.int64)
+            op.run(sched, io)
+            op.check()
+            err = rel(bf(io[2])[rows], oracle.linear_bf16(X, Wt, rows=rows))
+            what = f"{len(rows)} of {X.shape[0]} rows"
+        elif self.name in ("attention", "attention_flux"):
+            Q, K, V = self.host[:3]
+            qpos = np.linspace(0, Q.shape[1] - 1, 16).astype(np.int64)
+            O_ref, L_ref = oracle.attention_bf16(Q, K, V, causal=self.name == "attention", qpos=qpos)
+            op.run(sched, io)
+            op.check()
+            err = rel(bf(io[3])[:, qpos], O_ref)
+            if io[4] is not None:
+                lse = io[4].cpu().numpy().astype(np.float64)[:, :, qpos]
+                extra["lse_rel_err"] = rel(lse, L_ref)
+                extra["lse_ok"] = extra["lse_rel_err"] <= 1e-3
+            what = f"{len(qpos)} of {Q.shape[1]} query positions, all heads"
+        elif self.name == "conv2d":
+            x, w, b = self.host[:3]
+            total = x.shape[0] * x.shape[1] * x.shape[2]
+            pix = np.linspace(0, total - 1, 256).astype(np.int64)
+            op.run(sched, io)
+            op.check()
+            err = rel(bf(io[3]).reshape(total, -1)[pix], oracle.conv2d_nhwc_bf16(x, w, b, pix=pix))
+            what = f"{len(pix)} of {total} output pixels"
+        elif self.name == "moe":
+            logits, X, W1, W2 = self.host[:4]
+            T, K, E = X.shape[0], self.config["top_k"], self.config["experts"]
+            ids, wts, off, perm = oracle.moe_route(logits, K)
+            tok = np.linspace(0, T - 1, 16).astype(np.int64)
+            gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
+            go = torch.empty(E + 1, dtype=torch.int32, device="cuda")
+            gp = torch.empty(T * K, dtype=torch.int32, device="cuda")
+            op.run(sched, list(io[:5]) + [gi, None, go, gp])
+            op.check()
+            extra["routing_exact"] = bool(np.array_equal(gi.cpu().numpy(), ids) and
+                                          np.array_equal(go.cpu().numpy(), off) and
+                                          np.array_equal(gp.cpu().numpy(), perm))
+            err = rel(bf(io[4])[tok], oracle.moe_ffn_bf16(X, W1, W2, ids, wts, tok=tok))
+            what = f"routing of all {T} tokens (bit-exact) + the layer output of {len(tok)} tokens"
+        elif self.name == "decoder_layer":
+            from oracle import decoder
+            x = self.host[0]
+            rows = np.linspace(0, x.shape[0] - 1, 4).astype(np.int64)
+            ref = decoder.decoder_layer_bf16(*self.host[:7], self.config["heads_q"], self.config["heads_kv"],
+                                             rows=rows)
+            op.run(sched, io)
+            op.check()
+            x0 = decoder.widen(x[rows])
+            err = rel(bf(io[7])[rows] - x0, ref - x0)  # the layer's increment, not the residual copy of x
+            what = f"increment y - x of {len(rows)} of {x.shape[0]} token rows"
+        else:
+            A, B, bias = self.host[:3]
+            op.run(sched, io)
+            op.check()
+            err = rel(io[3].cpu().numpy().astype(np.float64), oracle.gemm_bias_relu_f32(A, B, bias))
+            what = "every output"
+        ok = err <= tol and extra.get("routing_exact", True) and extra.get("lse_ok", True)
+        return dict(max_rel_err=err, tol=tol, sample=what, ok=bool(ok), **extra)
 
     def cpu_sample(self, n, single_thread=True):
         """Time the fp64 oracle on a bounded sample with all its threads; returns the cpu_baseline dict.
@@ -374,6 +497,15 @@ class Workload:
             dt = time.perf_counter() - t0
             flops = 2.0 * n * w.shape[0] * w.shape[1] * w.shape[2] * w.shape[3]
             what, used = f"{n} of {total} output pixels", min(cores, n)
+        elif self.name == "linear":
+            X, Wt = self.host[:2]
+            n = n or 64
+            rows = np.linspace(0, X.shape[0] - 1, n).astype(np.int64)
+            t0 = time.perf_counter()
+            oracle.linear_bf16(X, Wt, rows=rows)
+            dt = time.perf_counter() - t0
+            flops = 2.0 * n * Wt.shape[0] * X.shape[1]
+            what, used = f"{n} of {X.shape[0]} rows", min(cores, n)
         elif self.name == "moe":
             logits, X, W1, W2 = self.host[:4]
             n = n or 32
@@ -413,7 +545,67 @@ class Workload:
         if self.name != "decoder_layer":
             what += ", fp64 loop nests"
         return {"value": flops / dt / 1e12, "unit": "TFLOP/s", "cores": used, "kind": "oracle",
-                "sample": what, "seconds": dt, "n": n}
+                "sample": what, "seconds": dt, "n": n, "cpu_model": cpu_model(), "nproc": os.cpu_count()}
+
+
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.json")
+
+
+def source_digest(paths):
+    """sha256 over the given repository files (the sources a measured kernel was built from)."""
+    import hashlib
+    h = hashlib.sha256()
+    for rel in sorted(paths):
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(rel.encode() + b"\0" + f.read())
+    return h.hexdigest()
+
+
+def measured_traffic(label, stage_knobs):
+    """DRAM bytes per launch of a workload's dominant kernel, from the committed ncu capture
+    (profiles/dram_traffic.json), keyed by the workload and the dominant stage's knobs. None when no
+    capture covers this schedule or the kernel's sources have changed since the capture."""
+    try:
+        table = json.load(open(TRAFFIC_FILE))
+    except (OSError, ValueError):
+        return None
+    for rec in table.get("captures", []):
+        if rec.get("workload") != label or rec.get("stage_knobs") != stage_knobs:
+            continue
+        try:
+            if source_digest(rec["sources"]) != rec["sources_sha256"]:
+                return None
+        except OSError:
+            return None
+        return rec
+    return None
+
+
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), for the CPU-baseline record."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu model")):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def knob_text(sched, stage):
+    """One stage's canonical knob text, e.g. 'tile=256x128x64,unroll=1,...' (the schedule's s<stage> part)."""
+    for part in str(sched).split(";"):
+        if part.startswith(f"s{stage}:"):
+            return part.split(":", 1)[1]
+    return ""
 
 
 def parse_shape(text):
@@ -430,7 +622,7 @@ def parse_schedule(op, text, rc):
     KNOB_T = {"tile_m": (rc.T_TILE_SIZE, 0), "tile_n": (rc.T_TILE_SIZE, 1), "tile_k": (rc.T_TILE_SIZE, 2),
               "stages": (rc.T_PIPELINE_STAGES, 0), "split_k": (rc.T_SPLIT_K, 0), "fuse": (rc.T_FUSE, 0),
               "raster": (rc.T_LOOP_ORDER, 0), "persistent": (rc.T_PARALLEL, 0), "layout": (rc.T_LAYOUT, 0),
-              "unroll": (rc.T_UNROLL, 0), "location": (rc.T_COMPUTE_LOCATION, 0)}
+              "unroll": (rc.T_UNROLL, 0), "location": (rc.T_COMPUTE_LOCATION, 0), "vec": (rc.T_VECTORIZE, 0)}
     KNOB_T["loc"] = KNOB_T["location"]
     p0 = op.schedule()
     ts = []
@@ -444,7 +636,7 @@ def parse_schedule(op, text, rc):
             k, v = kv.split("=")
             if k.strip() == "tile":
                 items += list(zip(("tile_m", "tile_n", "tile_k"), v.split("x")))
-            elif k.strip() != "vec":
+            else:
                 items.append((k.strip(), v))
         for k, v in items:
             if str(p0.knobs(stage).get(k if k != "loc" else "location")) == v and k != "raster":
@@ -614,6 +806,35 @@ def tasks_curve(op, io, samples, seed, joint=0.2):
     return curve
 
 
+def sample_efficiency(speedup, samples):
+    """The paper's sample efficiency: speedup over the untuned program per evaluated sample (Table 1)."""
+    return speedup / samples
+
+
+def efficiency_gain(base_speedup, base_samples, speedup, samples):
+    """Sample-efficiency gain of a search over a baseline search (Table 1's last column)."""
+    return sample_efficiency(speedup, samples) / sample_efficiency(base_speedup, base_samples)
+
+
+def sample_reduction(base_samples, samples):
+    """Samples the baseline search needed per sample of the other (Table 1's sample reduction)."""
+    return base_samples / samples
+
+
+def geomean(xs):
+    import math
+    xs = list(xs)
+    return math.exp(sum(math.log(x) for x in xs) / len(xs))
+
+
+def reach(curve, p0_ms):
+    """(samples, speedup): the first sample count at which a best-so-far curve [(n, best ms)] reached its
+    final best, and that best's speedup over P0 (the reading of Table 1's '# Samples' and 'Speedup')."""
+    final = min(b for _, b in curve)
+    n = next(n for n, b in curve if b <= final)
+    return n, p0_ms / final
+
+
 def search_study(wl, io, samples, seed, only=""):
     """Best-so-far (TFLOP/s of the best measured candidate) against measured samples, per search variant."""
     from paper_2506_01374_gb300 import rc
@@ -625,6 +846,8 @@ def search_study(wl, io, samples, seed, only=""):
         variants.append(("tasks_then_joint_B4_surrogate_screen4", 4, True, 4))
     if only:
         variants = [v for v in variants if v[0] in only.split(",")]
+    p0 = wl.op.measure([wl.op.schedule()], io, warmup=3, repeats=20)[0].ms_median
+    reached = {}
     for sd in (seed, seed + 1):
         for name, B, sur, scr in variants:
             t0 = time.perf_counter()
@@ -649,17 +872,37 @@ def search_study(wl, io, samples, seed, only=""):
             for mk in marks:
                 b = min((c[1] for c in curve if c[0] <= mk), default=float("inf"))
                 pts.append([mk, round(flops / (b * 1e-3) / 1e12, 1) if b < float("inf") else None])
+            n_reach, speedup = reach(curve, p0) if curve else (None, None)
+            reached[(name, sd)] = (n_reach, speedup)
             print(json.dumps({"study": "search", "workload": wl.label, "variant": name, "seed": sd,
                               "samples": len(curve), "seconds": round(time.perf_counter() - t0, 1),
-                              "best_tflops_at_samples": pts}), flush=True)
+                              "p0_ms": p0, "best_tflops_at_samples": pts,
+                              "samples_to_best": n_reach, "speedup_over_p0": speedup,
+                              "sample_efficiency": sample_efficiency(speedup, n_reach) if curve else None}),
+                  flush=True)
+    # each variant against unguided random search, as Table 1 sets the LLM-guided MCTS against evolution
+    for name, *_ in variants:
+        if name == "random":
+            continue
+        rows = [(reached[(name, sd)], reached[("random", sd)]) for sd in (seed, seed + 1)
+                if (name, sd) in reached and ("random", sd) in reached and reached[("random", sd)][0]]
+        if not rows:
+            continue
+        print(json.dumps({"study": "search_summary", "workload": wl.label, "variant": name, "baseline": "random",
+                          "speedup_geomean": geomean(v[1] for v, _ in rows),
+                          "baseline_speedup_geomean": geomean(r[1] for _, r in rows),
+                          "sample_reduction_geomean": geomean(sample_reduction(r[0], v[0]) for v, r in rows),
+                          "efficiency_gain_geomean": geomean(efficiency_gain(r[1], r[0], v[1], v[0])
+                                                             for v, r in rows)}), flush=True)
 
 
 def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None,
-              layer_samples=None):
+              layer_samples=None, hbm_gbs=None):
     """Search each other workload briefly and report its best schedule."""
     import torch
 
     from paper_2506_01374_gb300 import rc
+    hbm_gbs = hbm_gbs or peaks()["hbm_gbs"]
     out = {}
     for name in names:
         wl = Workload(name)
@@ -672,10 +915,21 @@ def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False,
         if m.status != rc.OK:
             out[name] = {"workload": wl.label, "error": rc.STATUS_NAMES.get(m.status, m.status)}
             continue
+        par = wl.parity(best, io)
+        if not par["ok"]:  # a schedule whose output disagrees with the oracle is not reported
+            out[name] = {"workload": wl.label, "error": "parity check failed", "parity": par,
+                         "schedule": str(best)}
+            continue
         tf = wl.op.info["flops"] / (m.ms_median * 1e-3) / 1e12
         peak = FP32_ALU_TFLOPS if wl.bound == "alu" else peak_tf
+        gbs = wl.op.info["bytes"] / (m.ms_median * 1e-3) / 1e9
+        tr = measured_traffic(wl.label, knob_text(best, wl.dom_stage))
         out[name] = {"workload": wl.label, "tflops": tf, "ms": m.ms_median, "bound": wl.bound, "peak": peak,
-                     "frac": tf / peak, "samples": n, "candidates_per_s": cps, "schedule": str(best)}
+                     "frac": tf / peak, "samples": n, "candidates_per_s": cps, "schedule": str(best),
+                     "hbm": {"algorithmic_bytes": wl.op.info["bytes"], "achieved_gbs": gbs,
+                             "frac_of_hbm_peak": gbs / hbm_gbs,
+                             "dominant_kernel_dram_bytes": tr["dram_bytes_per_launch"] if tr else None},
+                     "parity": par}
         del io, wl
         torch.cuda.empty_cache()
     return out
@@ -711,7 +965,7 @@ def run_reference(args):
     wl = Workload(args.workload)
     n = args.cpu_sample if args.cpu_sample > 0 else {"mlp": 16, "attention": 32, "conv2d": 512, "moe": 4,
                                                      "gemm_f32": 4, "attention_flux": 16,
-                                                     "decoder_layer": 8}[args.workload]
+                                                     "decoder_layer": 8, "linear": 16}[args.workload]
     for _ in range(args.warmup):
         wl.cpu_sample(n, single_thread=False)
     samples = [wl.cpu_sample(n, single_thread=False) for _ in range(args.steps)]
@@ -733,6 +987,8 @@ def launches_per_step(workload, s):
         return (1 if k[0]["fuse"] else 2) + (1 if k[1]["split_k"] == 1 else 2)
     if workload in ("attention", "attention_flux"):
         return 1 + (1 if k[0]["layout"] == 1 else 0)
+    if workload == "linear":
+        return 1 if k[0]["split_k"] == 1 else 2
     if workload == "conv2d":
         return 1 + (1 if k[0]["split_k"] > 1 else 0) + (1 if (k[0]["split_k"] > 1 or not k[0]["fuse"]) else 0)
     if workload == "moe":
@@ -811,6 +1067,11 @@ def run_ours(args):
     ms, ms_dom = max_over_ranks([ms, ms_dom], world, "cuda")
     value = job_tflops(world, info["flops"], ms * 1e-3)
 
+    # the best schedule's output against the oracle, outside the timed regions
+    parity = wl.parity(best, io) if rank == 0 else None
+    if parity is not None and not parity["ok"]:
+        raise SystemExit(f"parity check of the best schedule failed: {parity} ({best})")
+
     # 3) end to end through the host-buffer entry point
     e2e_s = None
     if not args.skip_e2e:
@@ -831,6 +1092,7 @@ def run_ours(args):
         peak_src = ("derived: 152 SMs x 128 FP32 lanes x 2 x 2.07 GHz" if wl.bound == "alu"
                     else pk["source"] + " bf16 burst")
         achieved = wl.dom_flops / (ms_dom * 1e-3) / 1e12
+        traffic = measured_traffic(wl.label, knob_text(best, wl.dom_stage))
         kname = wl.dom_name
         if args.workload == "mlp":
             kname = kname.format(" + fused SwiGLU epilogue" if best.knobs(0)["fuse"] else " + SwiGLU pass")
@@ -842,7 +1104,11 @@ def run_ours(args):
                            parallelism="replicas" if world > 1 else "single",
                            l2="flushed between steps (flush outside the timed events)", schedule=str(best)),
             "roofline": {"bound": wl.bound, "kernel": kname, "achieved": achieved, "peak": peak,
-                         "unit": "TFLOP/s", "frac": achieved / peak, "peak_source": peak_src, "traffic": None},
+                         "unit": "TFLOP/s", "frac": achieved / peak, "peak_source": peak_src,
+                         "traffic": traffic["dram_bytes_per_launch"] if traffic else None,
+                         "traffic_source": traffic["profile"] if traffic else
+                         "no ncu capture of this kernel, schedule and source",
+                         "algorithmic_bytes": wl.dom_bytes},
             "step_frac_of_peak": value / world / peak,
             "search": {"samples": n_meas, "candidates_per_s": cps, "surrogate": bool(args.surrogate),
                        "horizon": wl.horizon, "tasks": tasks[0] if tasks else None,
@@ -853,15 +1119,17 @@ def run_ours(args):
                                                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": args.steps * launches_per_step(args.workload, best),
             "clocks": clk,
+            "parity": parity,
         }
         others = args.ops if args.ops is not None else (
-            "gemm_f32,conv2d,attention,attention_flux,moe,decoder_layer" if args.workload == "mlp" else "")
+            "gemm_f32,linear,conv2d,attention,attention_flux,moe,decoder_layer" if args.workload == "mlp" else "")
         names = [x for x in others.split(",") if x and x != args.workload]
         if names:
             del io
             torch.cuda.empty_cache()
             out["ops"] = extra_ops(names, args.op_samples, pk["bf16_tflops"], args.branching, args.restarts,
-                                   bool(args.surrogate), args.screen, args.moe_samples, args.layer_samples)
+                                   bool(args.surrogate), args.screen, args.moe_samples, args.layer_samples,
+                                   pk["hbm_gbs"])
         if args.cpu_sample >= 0:
             cb = wl.cpu_sample(args.cpu_sample)
             cb.pop("seconds", None)

@@ -106,6 +106,9 @@ extern "C" const char* rc_version(void) { return "rc 0.1 (sm_103a)"; }
 std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
   std::vector<KnobSpec> v;
   const int kind = op->d.kind;
+  // bytes per access of the memory-bound pass a stage may run after its GEMM (SwiGLU, bias/SiLU,
+  // split-K reduce, MoE gather and combine); normalised to the default where the stage runs none
+  auto vectorize = [&]() { v.push_back({RC_T_VECTORIZE, 0, {4, 8, 16}, {}}); };
   auto gemm_common = [&](std::vector<int32_t> tn) {
     v.push_back({RC_T_TILE_SIZE, 1, tn, {}});
     v.push_back({RC_T_TILE_SIZE, 2, {64, 128}, {}});  // K per ring stage: one or two 64-wide sub-blocks
@@ -124,11 +127,13 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       gemm_common({64, 128, 224, 256});
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // one CTA, or a CTA pair sharing each UMMA
       v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
+      vectorize();
       break;
     case RC_OP_SWIGLU:
       gemm_common({32, 64, 128});
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      vectorize();
       break;
     case RC_OP_MLP:
       if (stage == 0) {
@@ -139,12 +144,14 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       }
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+      vectorize();
       break;
     case RC_OP_CONV2D:
       gemm_common({64, 80, 160});
       v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       v.push_back({RC_T_SPLIT_K, 0, {1, 3, 5}, {}});
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+      vectorize();
       // implicit zero padding (one 4-D box), or a padded copy read as one 4-D box or as row boxes
       v.push_back({RC_T_LAYOUT, 0, {0, 1, 2}, {}});
       break;
@@ -157,7 +164,10 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         // 0: QKV projection, 3: O projection, 4: gate/up + SwiGLU, 5: down projection
         gemm_common(stage == 4 ? std::vector<int32_t>{32, 64, 128} : std::vector<int32_t>{64, 128, 224, 256});
         v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
-        if (stage == 4) v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+        if (stage == 4) {
+          v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
+          vectorize();  // the SwiGLU pass of the unfused gate/up GEMM
+        }
         break;
       }
       [[fallthrough]];  // 2: the attention core
@@ -180,6 +190,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
     case RC_OP_MOE:
       if (stage == 0) {
         v.push_back({RC_T_TILE_SIZE, 0, {4, 8, 16}, {}});
+        vectorize();  // the row gather
       } else if (stage == 1) {
         gemm_common({32, 64, 128});
         v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // 256: a CTA pair within one expert's rows
@@ -190,6 +201,7 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
         v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+        vectorize();  // the combine (or the fp32 -> bf16 pass of the atomic combine)
       }
       break;
   }
@@ -327,11 +339,11 @@ static bool attention_knobs_ok(const rc_knobs& k, int64_t seq, std::string* why)
     if (why) *why = m;
     return false;
   };
+  // (rc_schedule_apply canonicalises location and unroll per kernel family before this check)
   if (k.persistent == 0) {
     if (k.location != 0 || k.unroll != 1) return no("one UMMA-issuing warp keeps P in shared memory and one S buffer");
-  } else {
-    if (k.location == 0) return no("split UMMA issue keeps P in tensor memory");
-    if (k.stages < 2) return no("split UMMA issue needs two K/V stages");
+  } else if (k.location == 0) {
+    return no("split UMMA issue keeps P in tensor memory");
   }
   if (k.location == 2 && k.layout != 0) return no("row sums on the tensor core need V as given");
   if (k.layout == 1 && seq % 8) return no("transposed V needs seq % 8 == 0 (16-byte TMA rows)");
@@ -643,6 +655,20 @@ extern "C" rc_status rc_op_info(const rc_op* op, rc_op_info_t* info) {
 // rc_op_destroy lives in run.cu (it frees device memory).
 
 // -------------------------------------------------------------- schedules --
+// Whether stage `g` of schedule s runs a memory-bound pass whose access width is the Vectorize knob.
+static bool vectorize_used(const rc_op_s* op, const rc_schedule_s& s, int g) {
+  const rc_knobs& k = s.k[g];
+  switch (op->d.kind) {
+    case RC_OP_LINEAR: return k.split_k > 1;
+    case RC_OP_SWIGLU: return !k.fuse;
+    case RC_OP_MLP: return g == 0 ? !k.fuse : k.split_k > 1;
+    case RC_OP_CONV2D: return k.split_k > 1 || (!k.fuse && (op->d.flags & (RC_EPI_BIAS | RC_EPI_SILU)));
+    case RC_OP_MOE: return g == 0 ? s.k[1].location == 0 : g == 2;
+    case RC_OP_DECODER_LAYER: return g == 4 && !k.fuse;
+    default: return false;
+  }
+}
+
 static rc_status apply_one(const rc_op_s* op, rc_schedule_s* s, const rc_transform& t) {
   if (t.stage < 0 || t.stage >= s->n_stages)
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "transform stage %d out of range", t.stage);
@@ -691,6 +717,23 @@ extern "C" rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base,
     for (int i = 0; i < op->n_stages; ++i) s.k[i] = rc_default_knobs(op, i);
   }
   for (size_t i = 0; i < n; ++i) RC_TRY(apply_one(op, &s, seq[i]));
+  // Vectorize acts only on the memory-bound pass a stage runs; where the chosen knobs run none it
+  // leaves the program unchanged, so the canonical form keeps the default
+  for (int i = 0; i < s.n_stages; ++i)
+    if (!vectorize_used(op, s, i)) s.k[i].vec = rc_default_knobs(op, i).vec;
+  // attention: the one-issuing-warp kernel keeps P in shared memory and one S buffer, and the
+  // split-issue kernels keep P in tensor memory, so each family's canonical form fixes the knobs it
+  // does not offer (a single Parallel transformation then moves between the families)
+  for (int i = 0; i < s.n_stages; ++i) {
+    if (!(op->d.kind == RC_OP_ATTENTION || (op->d.kind == RC_OP_DECODER_LAYER && i == 2))) continue;
+    rc_knobs& k = s.k[i];
+    if (k.persistent == 0) {
+      k.location = 0;
+      k.unroll = 1;
+    } else if (k.location == 0) {
+      k.location = 1;
+    }
+  }
   for (int i = 0; i < s.n_stages; ++i) {
     std::string why;
     if (!rc_knobs_legal(op, i, s.k[i], &why))

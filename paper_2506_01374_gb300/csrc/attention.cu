@@ -1141,8 +1141,8 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: 128-row query tiles, 64- or 128-key blocks, loop order 0 or 1");
   if (k.persistent == 0 && (k.location != 0 || k.unroll != 1))
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: one issuing warp keeps P in shared memory, one S buffer");
-  if (k.persistent > 0 && (k.location == 0 || k.stages < 2))
-    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: split UMMA issue needs P in TMEM and two stages");
+  if (k.persistent > 0 && k.location == 0)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: split UMMA issue keeps P in TMEM");
   if (k.location == 2 && k.layout != 0)
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: row sums on the tensor core need V as given");
   const void* Vuse = V;

@@ -1,6 +1,7 @@
 // Memory-bound passes that unfused schedules run after a GEMM, plus the L2
-// flush used between timed runs. Every pass moves 16-byte vectors (8 bf16 or
-// 4 fp32) per thread with a grid-stride loop sized to the SM count.
+// flush used between timed runs. Each pass moves VB-byte vectors per thread
+// access (the Vectorize knob: 4, 8 or 16 bytes, i.e. 2, 4 or 8 bf16) with a
+// grid-stride loop sized to the SM count.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -10,9 +11,25 @@ namespace {
 
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + __expf(-x)); }
 
-union V8 {
-  uint4 u;
-  __nv_bfloat16 h[8];
+// VB bytes of bf16 elements, loaded and stored as one access.
+template <int VB>
+struct BVec;
+template <>
+struct BVec<16> {
+  using T = uint4;
+};
+template <>
+struct BVec<8> {
+  using T = uint2;
+};
+template <>
+struct BVec<4> {
+  using T = uint32_t;
+};
+template <int VB>
+union VecB {
+  typename BVec<VB>::T u;
+  __nv_bfloat16 h[VB / 2];
 };
 
 int grid_for(int64_t work, const LaunchCtx& c, int threads = 256) {
@@ -23,63 +40,103 @@ int grid_for(int64_t work, const LaunchCtx& c, int threads = 256) {
 }
 
 // h[m, n] = silu(gu[m, n]) * gu[m, I + n]; I % 8 == 0.
+template <int VB>
 __global__ void swiglu_pass_kernel(const __nv_bfloat16* __restrict__ gu, int64_t M, int64_t I,
                                    __nv_bfloat16* __restrict__ h) {
-  const int64_t per_row = I / 8;
+  constexpr int E = VB / 2;
+  const int64_t per_row = I / E;
   const int64_t total = M * per_row;
   for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < total;
        v += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t m = v / per_row, c = (v % per_row) * 8;
-    V8 g, u, o;
-    g.u = *reinterpret_cast<const uint4*>(gu + m * 2 * I + c);
-    u.u = *reinterpret_cast<const uint4*>(gu + m * 2 * I + I + c);
+    const int64_t m = v / per_row, c = (v % per_row) * E;
+    VecB<VB> g, u, o;
+    g.u = *reinterpret_cast<const typename BVec<VB>::T*>(gu + m * 2 * I + c);
+    u.u = *reinterpret_cast<const typename BVec<VB>::T*>(gu + m * 2 * I + I + c);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < E; ++i) {
       const float gf = __bfloat162float(g.h[i]);
       o.h[i] = __float2bfloat16_rn(silu_f(gf) * __bfloat162float(u.h[i]));
     }
-    *reinterpret_cast<uint4*>(h + m * I + c) = o.u;
+    *reinterpret_cast<typename BVec<VB>::T*>(h + m * I + c) = o.u;
   }
 }
 
 // out[r, c] = act(y[r, c] + bias[c]); C % 8 == 0.
+template <int VB>
 __global__ void bias_silu_pass_kernel(const __nv_bfloat16* __restrict__ y, const __nv_bfloat16* __restrict__ bias,
                                       int64_t rows, int64_t C, int silu, __nv_bfloat16* __restrict__ out) {
-  const int64_t per_row = C / 8;
+  constexpr int E = VB / 2;
+  const int64_t per_row = C / E;
   const int64_t total = rows * per_row;
   for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < total;
        v += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t c = (v % per_row) * 8;
-    V8 a, o;
-    a.u = *reinterpret_cast<const uint4*>(y + v * 8);
+    const int64_t c = (v % per_row) * E;
+    VecB<VB> a, o;
+    a.u = *reinterpret_cast<const typename BVec<VB>::T*>(y + v * E);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
+    for (int i = 0; i < E; ++i) {
       float f = __bfloat162float(a.h[i]) + (bias ? __bfloat162float(bias[c + i]) : 0.f);
       o.h[i] = __float2bfloat16_rn(silu ? silu_f(f) : f);
     }
-    *reinterpret_cast<uint4*>(out + v * 8) = o.u;
+    *reinterpret_cast<typename BVec<VB>::T*>(out + v * E) = o.u;
   }
 }
 
+// VB bytes of fp32 partials (VB / 4 floats) per access: load, sum, store as bf16.
+template <int VB>
+struct FVec;
+template <>
+struct FVec<16> {
+  using T = float4;
+};
+template <>
+struct FVec<8> {
+  using T = float2;
+};
+template <>
+struct FVec<4> {
+  using T = float;
+};
+template <int VB>
+union VecF {
+  typename FVec<VB>::T v;
+  float f[VB / 4];
+};
+template <int VB>
+__device__ __forceinline__ void store_bf16(__nv_bfloat16* out, const float (&f)[VB / 4]) {
+#pragma unroll
+  for (int i = 0; i < VB / 4; ++i) out[i] = __float2bfloat16_rn(f[i]);
+}
+template <>
+__device__ __forceinline__ void store_bf16<16>(__nv_bfloat16* out, const float (&f)[4]) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(f[0], f[1]), hi = __floats2bfloat162_rn(f[2], f[3]);
+  uint2 pk;
+  pk.x = *reinterpret_cast<uint32_t*>(&lo);
+  pk.y = *reinterpret_cast<uint32_t*>(&hi);
+  *reinterpret_cast<uint2*>(out) = pk;
+}
+template <>
+__device__ __forceinline__ void store_bf16<8>(__nv_bfloat16* out, const float (&f)[2]) {
+  *reinterpret_cast<__nv_bfloat162*>(out) = __floats2bfloat162_rn(f[0], f[1]);
+}
+
 // out[m, n] = bf16(sum_z part[z, m, n]); N % 4 == 0.
+template <int VB>
 __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits, int64_t MN,
                                      __nv_bfloat16* __restrict__ out) {
-  const int64_t total = MN / 4;
+  constexpr int E = VB / 4;
+  const int64_t total = MN / E;
   for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < total;
        v += (int64_t)gridDim.x * blockDim.x) {
-    float4 s = reinterpret_cast<const float4*>(part)[v];
+    VecF<VB> s;
+    s.v = reinterpret_cast<const typename FVec<VB>::T*>(part)[v];
     for (int z = 1; z < splits; ++z) {
-      const float4 p = reinterpret_cast<const float4*>(part + (int64_t)z * MN)[v];
-      s.x += p.x;
-      s.y += p.y;
-      s.z += p.z;
-      s.w += p.w;
+      VecF<VB> p;
+      p.v = reinterpret_cast<const typename FVec<VB>::T*>(part + (int64_t)z * MN)[v];
+#pragma unroll
+      for (int i = 0; i < E; ++i) s.f[i] += p.f[i];
     }
-    __nv_bfloat162 lo = __floats2bfloat162_rn(s.x, s.y), hi = __floats2bfloat162_rn(s.z, s.w);
-    uint2 pk;
-    pk.x = *reinterpret_cast<uint32_t*>(&lo);
-    pk.y = *reinterpret_cast<uint32_t*>(&hi);
-    reinterpret_cast<uint2*>(out)[v] = pk;
+    store_bf16<VB>(out + v * E, s.f);
   }
 }
 
@@ -97,14 +154,13 @@ __global__ void pad_nhwc_kernel(const uint4* __restrict__ x, int64_t N, int64_t 
   }
 }
 
-__global__ void f32_to_bf16_kernel(const float* __restrict__ in, int64_t n4, __nv_bfloat16* __restrict__ out) {
-  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n4; v += (int64_t)gridDim.x * blockDim.x) {
-    const float4 s = reinterpret_cast<const float4*>(in)[v];
-    __nv_bfloat162 lo = __floats2bfloat162_rn(s.x, s.y), hi = __floats2bfloat162_rn(s.z, s.w);
-    uint2 pk;
-    pk.x = *reinterpret_cast<uint32_t*>(&lo);
-    pk.y = *reinterpret_cast<uint32_t*>(&hi);
-    reinterpret_cast<uint2*>(out)[v] = pk;
+template <int VB>
+__global__ void f32_to_bf16_kernel(const float* __restrict__ in, int64_t n, __nv_bfloat16* __restrict__ out) {
+  constexpr int E = VB / 4;
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n / E; v += (int64_t)gridDim.x * blockDim.x) {
+    VecF<VB> s;
+    s.v = reinterpret_cast<const typename FVec<VB>::T*>(in)[v];
+    store_bf16<VB>(out + v * E, s.f);
   }
 }
 
@@ -122,35 +178,59 @@ rc_status launched(const char* what) {
 
 }  // namespace
 
+// Bytes per access of the Vectorize knob: 4, 8 or 16.
+static bool vec_ok(int vec) { return vec == 4 || vec == 8 || vec == 16; }
+
 rc_status rc_launch_swiglu_pass(const void* gu, int64_t M, int64_t I, void* h, int vec, const LaunchCtx& c) {
-  (void)vec;
   if (I % 8) return rc_fail(RC_ERR_UNSUPPORTED_OP, "swiglu pass: I %% 8 != 0");
-  swiglu_pass_kernel<<<grid_for(M * I / 8, c), 256, 0, (cudaStream_t)c.stream>>>(
-      (const __nv_bfloat16*)gu, M, I, (__nv_bfloat16*)h);
+  if (!vec_ok(vec)) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "swiglu pass: vector of %d bytes", vec);
+  const int g = grid_for(M * I / (vec / 2), c);
+  auto gp = (const __nv_bfloat16*)gu;
+  auto hp = (__nv_bfloat16*)h;
+  cudaStream_t st = (cudaStream_t)c.stream;
+  if (vec == 16) swiglu_pass_kernel<16><<<g, 256, 0, st>>>(gp, M, I, hp);
+  else if (vec == 8) swiglu_pass_kernel<8><<<g, 256, 0, st>>>(gp, M, I, hp);
+  else swiglu_pass_kernel<4><<<g, 256, 0, st>>>(gp, M, I, hp);
   return launched("swiglu pass");
 }
 
 rc_status rc_launch_bias_silu_pass(const void* y, const void* bias, int64_t rows, int64_t C, bool silu, void* out,
                                    int vec, const LaunchCtx& c) {
-  (void)vec;
   if (C % 8) return rc_fail(RC_ERR_UNSUPPORTED_OP, "bias/SiLU pass: C %% 8 != 0");
-  bias_silu_pass_kernel<<<grid_for(rows * C / 8, c), 256, 0, (cudaStream_t)c.stream>>>(
-      (const __nv_bfloat16*)y, (const __nv_bfloat16*)bias, rows, C, silu ? 1 : 0, (__nv_bfloat16*)out);
+  if (!vec_ok(vec)) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "bias/SiLU pass: vector of %d bytes", vec);
+  const int g = grid_for(rows * C / (vec / 2), c);
+  auto yp = (const __nv_bfloat16*)y;
+  auto bp = (const __nv_bfloat16*)bias;
+  auto op = (__nv_bfloat16*)out;
+  cudaStream_t st = (cudaStream_t)c.stream;
+  if (vec == 16) bias_silu_pass_kernel<16><<<g, 256, 0, st>>>(yp, bp, rows, C, silu ? 1 : 0, op);
+  else if (vec == 8) bias_silu_pass_kernel<8><<<g, 256, 0, st>>>(yp, bp, rows, C, silu ? 1 : 0, op);
+  else bias_silu_pass_kernel<4><<<g, 256, 0, st>>>(yp, bp, rows, C, silu ? 1 : 0, op);
   return launched("bias/SiLU pass");
 }
 
 rc_status rc_launch_splitk_reduce(const float* part, int splits, int64_t M, int64_t N, void* out, int vec,
                                   const LaunchCtx& c) {
-  (void)vec;
   if (N % 4) return rc_fail(RC_ERR_UNSUPPORTED_OP, "split-K reduce: N %% 4 != 0");
-  splitk_reduce_kernel<<<grid_for(M * N / 4, c), 256, 0, (cudaStream_t)c.stream>>>(part, splits, M * N,
-                                                                                   (__nv_bfloat16*)out);
+  if (!vec_ok(vec)) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "split-K reduce: vector of %d bytes", vec);
+  const int g = grid_for(M * N / (vec / 4), c);
+  auto op = (__nv_bfloat16*)out;
+  cudaStream_t st = (cudaStream_t)c.stream;
+  if (vec == 16) splitk_reduce_kernel<16><<<g, 256, 0, st>>>(part, splits, M * N, op);
+  else if (vec == 8) splitk_reduce_kernel<8><<<g, 256, 0, st>>>(part, splits, M * N, op);
+  else splitk_reduce_kernel<4><<<g, 256, 0, st>>>(part, splits, M * N, op);
   return launched("split-K reduce");
 }
 
-rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, const LaunchCtx& c) {
+rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, int vec, const LaunchCtx& c) {
   if (n % 4) return rc_fail(RC_ERR_UNSUPPORTED_OP, "f32->bf16: n %% 4 != 0");
-  f32_to_bf16_kernel<<<grid_for(n / 4, c), 256, 0, (cudaStream_t)c.stream>>>(in, n / 4, (__nv_bfloat16*)out);
+  if (!vec_ok(vec)) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "f32->bf16: vector of %d bytes", vec);
+  const int g = grid_for(n / (vec / 4), c);
+  auto op = (__nv_bfloat16*)out;
+  cudaStream_t st = (cudaStream_t)c.stream;
+  if (vec == 16) f32_to_bf16_kernel<16><<<g, 256, 0, st>>>(in, n, op);
+  else if (vec == 8) f32_to_bf16_kernel<8><<<g, 256, 0, st>>>(in, n, op);
+  else f32_to_bf16_kernel<4><<<g, 256, 0, st>>>(in, n, op);
   return launched("f32->bf16");
 }
 

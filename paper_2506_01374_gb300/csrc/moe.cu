@@ -18,9 +18,10 @@
 //      per-warp hit counts per chunk), so slot s = t*k + j lands at
 //      perm[offset[e] + rank] - the (expert, token, j) order - with no
 //      dependence on thread timing.
-// Gather: Xp[pos] = X[perm[pos] / k], 16-byte vectors, one warp per row.
+// Gather: Xp[pos] = X[perm[pos] / k], one warp per row, 4-, 8- or 16-byte
+//   vectors (the Vectorize knob).
 // Combine: out[t] = sum_{j<k} w[t,j] * Y[inv_perm[t*k+j]] in fp32, in j order,
-//   rounded once to bf16.
+//   rounded once to bf16, with the same choice of vector width.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -226,25 +227,46 @@ __global__ void __launch_bounds__(kPermThreads)
   }
 }
 
-__global__ void gather_rows_kernel(const uint4* __restrict__ X, const int* __restrict__ perm, int rows, int H16,
-                                   int K, uint4* __restrict__ Xp) {
+// VB-byte vectors of the Vectorize knob (4, 8 or 16 bytes per access).
+template <int VB>
+struct Vec;
+template <>
+struct Vec<16> {
+  using T = uint4;
+};
+template <>
+struct Vec<8> {
+  using T = uint2;
+};
+template <>
+struct Vec<4> {
+  using T = uint32_t;
+};
+
+template <int VB>
+__global__ void gather_rows_kernel(const typename Vec<VB>::T* __restrict__ X, const int* __restrict__ perm, int rows,
+                                   int HV, int K, typename Vec<VB>::T* __restrict__ Xp) {
   const int warps = blockDim.x / 32;
   const int lane = threadIdx.x % 32;
   for (int r = blockIdx.x * warps + threadIdx.x / 32; r < rows; r += gridDim.x * warps) {
     const int t = perm[r] / K;
-    const uint4* src = X + (size_t)t * H16;
-    uint4* dst = Xp + (size_t)r * H16;
-    for (int i = lane; i < H16; i += 32) dst[i] = src[i];
+    const typename Vec<VB>::T* src = X + (size_t)t * HV;
+    typename Vec<VB>::T* dst = Xp + (size_t)r * HV;
+    for (int i = lane; i < HV; i += 32) dst[i] = src[i];
   }
 }
 
-union V8 {
-  uint4 u;
-  __nv_bfloat162 h[4];
+template <int VB>
+union VecH {
+  typename Vec<VB>::T u;
+  __nv_bfloat162 h[VB / 4];
 };
 
-__global__ void combine_kernel(const uint4* __restrict__ Y, const float* __restrict__ w,
-                               const int* __restrict__ inv_perm, int T, int H8, int K, uint4* __restrict__ out) {
+template <int VB>
+__global__ void combine_kernel(const typename Vec<VB>::T* __restrict__ Y, const float* __restrict__ w,
+                               const int* __restrict__ inv_perm, int T, int HV, int K,
+                               typename Vec<VB>::T* __restrict__ out) {
+  constexpr int P = VB / 4;  // bf16 pairs per vector
   const int warps = blockDim.x / 32;
   const int lane = threadIdx.x % 32;
   for (int t = blockIdx.x * warps + threadIdx.x / 32; t < T; t += gridDim.x * warps) {
@@ -254,22 +276,24 @@ __global__ void combine_kernel(const uint4* __restrict__ Y, const float* __restr
       rows[j] = inv_perm[(size_t)t * K + j];
       ws[j] = w[(size_t)t * K + j];
     }
-    for (int i = lane; i < H8; i += 32) {
-      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      for (int j = 0; j < K; ++j) {
-        V8 y;
-        y.u = Y[(size_t)rows[j] * H8 + i];
+    for (int i = lane; i < HV; i += 32) {
+      float acc[2 * P];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
+      for (int q = 0; q < 2 * P; ++q) acc[q] = 0.f;
+      for (int j = 0; j < K; ++j) {
+        VecH<VB> y;
+        y.u = Y[(size_t)rows[j] * HV + i];
+#pragma unroll
+        for (int q = 0; q < P; ++q) {
           const float2 f = __bfloat1622float2(y.h[q]);
           acc[2 * q] = fmaf(ws[j], f.x, acc[2 * q]);
           acc[2 * q + 1] = fmaf(ws[j], f.y, acc[2 * q + 1]);
         }
       }
-      V8 o;
+      VecH<VB> o;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) o.h[q] = __floats2bfloat162_rn(acc[2 * q], acc[2 * q + 1]);
-      out[(size_t)t * H8 + i] = o.u;
+      for (int q = 0; q < P; ++q) o.h[q] = __floats2bfloat162_rn(acc[2 * q], acc[2 * q + 1]);
+      out[(size_t)t * HV + i] = o.u;
     }
   }
 }
@@ -307,24 +331,42 @@ rc_status rc_launch_moe_route(const rc_knobs& k, const rc_op_desc& d, const void
 
 rc_status rc_launch_moe_gather(const void* X, const int* perm, int64_t rows, int64_t H, int topk, void* Xp, int vec,
                                const LaunchCtx& c) {
-  (void)vec;
   if (H % 8) return rc_fail(RC_ERR_UNSUPPORTED_OP, "gather: H %% 8 != 0");
+  if (vec != 4 && vec != 8 && vec != 16) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "gather: vector of %d bytes", vec);
   const int warps = 8;
   int64_t blocks = (rows + warps - 1) / warps;
   if (blocks > (int64_t)c.num_sms * 16) blocks = (int64_t)c.num_sms * 16;
-  gather_rows_kernel<<<(unsigned)blocks, 32 * warps, 0, (cudaStream_t)c.stream>>>(
-      (const uint4*)X, perm, (int)rows, (int)(H / 8), topk, (uint4*)Xp);
+  const int hv = (int)(H * 2 / vec);  // vectors per row
+  cudaStream_t st = (cudaStream_t)c.stream;
+  if (vec == 16)
+    gather_rows_kernel<16><<<(unsigned)blocks, 32 * warps, 0, st>>>((const uint4*)X, perm, (int)rows, hv, topk,
+                                                                     (uint4*)Xp);
+  else if (vec == 8)
+    gather_rows_kernel<8><<<(unsigned)blocks, 32 * warps, 0, st>>>((const uint2*)X, perm, (int)rows, hv, topk,
+                                                                    (uint2*)Xp);
+  else
+    gather_rows_kernel<4><<<(unsigned)blocks, 32 * warps, 0, st>>>((const uint32_t*)X, perm, (int)rows, hv, topk,
+                                                                    (uint32_t*)Xp);
   return launched("gather");
 }
 
 rc_status rc_launch_moe_combine(const void* Y, const float* w, const int* inv_perm, int64_t T, int64_t H, int topk,
                                 void* out, int vec, const LaunchCtx& c) {
-  (void)vec;
   if (H % 8 || topk > kMaxK) return rc_fail(RC_ERR_UNSUPPORTED_OP, "combine: H %% 8 != 0 or k > 16");
+  if (vec != 4 && vec != 8 && vec != 16) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "combine: vector of %d bytes", vec);
   const int warps = 8;
   int64_t blocks = (T + warps - 1) / warps;
   if (blocks > (int64_t)c.num_sms * 16) blocks = (int64_t)c.num_sms * 16;
-  combine_kernel<<<(unsigned)blocks, 32 * warps, 0, (cudaStream_t)c.stream>>>(
-      (const uint4*)Y, w, inv_perm, (int)T, (int)(H / 8), topk, (uint4*)out);
+  const int hv = (int)(H * 2 / vec);
+  cudaStream_t st = (cudaStream_t)c.stream;
+  if (vec == 16)
+    combine_kernel<16><<<(unsigned)blocks, 32 * warps, 0, st>>>((const uint4*)Y, w, inv_perm, (int)T, hv, topk,
+                                                                 (uint4*)out);
+  else if (vec == 8)
+    combine_kernel<8><<<(unsigned)blocks, 32 * warps, 0, st>>>((const uint2*)Y, w, inv_perm, (int)T, hv, topk,
+                                                                (uint2*)out);
+  else
+    combine_kernel<4><<<(unsigned)blocks, 32 * warps, 0, st>>>((const uint32_t*)Y, w, inv_perm, (int)T, hv, topk,
+                                                                (uint32_t*)out);
   return launched("combine");
 }

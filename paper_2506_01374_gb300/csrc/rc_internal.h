@@ -176,7 +176,7 @@ rc_status rc_launch_moe_gather(const void* X, const int* perm, int64_t rows, int
                                void* Xp, int vec, const LaunchCtx& c);
 rc_status rc_launch_moe_combine(const void* Y, const float* w, const int* inv_perm, int64_t T,
                                 int64_t H, int topk, void* out, int vec, const LaunchCtx& c);
-rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, const LaunchCtx& c);
+rc_status rc_launch_f32_to_bf16(const float* in, int64_t n, void* out, int vec, const LaunchCtx& c);
 // Explicitly zero-padded copy of an NHWC tensor ([N][H+2p][W+2p][C]).
 rc_status rc_launch_pad_nhwc(const void* x, int64_t N, int64_t H, int64_t W, int64_t C, int64_t pad, void* xp,
                              const LaunchCtx& c);

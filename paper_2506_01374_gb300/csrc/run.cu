@@ -256,7 +256,8 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
       // gate/up compute location 1: the GEMM's producer gathers X's rows itself (no gathered copy)
       const bool gather_in_gemm = s->k[1].location == 1;
       RC_TRY(rc_launch_moe_route(s->k[0], d, p[0], ids, w, offsets, perm, inv, counts, c));
-      if (!gather_in_gemm) RC_TRY(rc_launch_moe_gather(p[1], perm, slots, d.hidden, (int)d.top_k, Xp, 16, c));
+      if (!gather_in_gemm)
+        RC_TRY(rc_launch_moe_gather(p[1], perm, slots, d.hidden, (int)d.top_k, Xp, s->k[0].vec, c));
       RC_TRY(rc_mark_stage(c));
       const int64_t max_tiles = slots / 128 + d.experts;
       TcGemmArgs g1 =
@@ -288,11 +289,11 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
         g2.row_div = (int)d.top_k;
         g2.ldd = d.hidden;
         RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
-        RC_TRY(rc_launch_f32_to_bf16(acc, d.tokens * d.hidden, p[4], c));
+        RC_TRY(rc_launch_f32_to_bf16(acc, d.tokens * d.hidden, p[4], s->k[2].vec, c));
         return rc_mark_stage(c);
       }
       RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
-      RC_TRY(rc_launch_moe_combine(Yb, w, inv, d.tokens, d.hidden, (int)d.top_k, p[4], 16, c));
+      RC_TRY(rc_launch_moe_combine(Yb, w, inv, d.tokens, d.hidden, (int)d.top_k, p[4], s->k[2].vec, c));
       return rc_mark_stage(c);
     }
   }

@@ -177,3 +177,28 @@ def test_binding_constants_match_the_header():
     opts = re.search(r"typedef struct \{([^{}]*)\} rc_search_opts;", src).group(1)
     names = re.findall(r"(\w+);", opts)
     assert names == [f for f, _ in rc.SearchOpts._fields_]
+
+
+def test_vectorize_offered_and_normalised_where_no_pass_runs():
+    # Vectorize sets the access width of a stage's memory-bound pass; a stage that runs none keeps the default
+    op = rc.Op(rc.OP_MLP, m=64, n=128, k=64)
+    kinds = {(t.kind, t.stage) for t in op.transform_space()}
+    assert (rc.T_VECTORIZE, 0) in kinds and (rc.T_VECTORIZE, 1) in kinds
+    fused = op.schedule(rc.T(rc.T_FUSE, 1, stage=0), rc.T(rc.T_VECTORIZE, 4, stage=0))
+    assert fused.knobs(0)["vec"] == 16 and str(fused) == str(op.schedule(rc.T(rc.T_FUSE, 1, stage=0)))
+    unfused = op.schedule(rc.T(rc.T_VECTORIZE, 8, stage=0))
+    assert unfused.knobs(0)["vec"] == 8 and str(unfused) != str(op.schedule())
+    no_split = op.schedule(rc.T(rc.T_VECTORIZE, 4, stage=1))
+    assert no_split.knobs(1)["vec"] == 16
+    split = op.schedule(rc.T(rc.T_SPLIT_K, 2, stage=1), rc.T(rc.T_VECTORIZE, 4, stage=1))
+    assert split.knobs(1)["vec"] == 4
+    with pytest.raises(rc.RcError) as e:
+        op.schedule(rc.T(rc.T_VECTORIZE, 2, stage=0))
+    assert e.value.status == rc.ERR_ILLEGAL_SCHEDULE
+    moe = rc.Op(rc.OP_MOE, tokens=64, hidden=128, experts=4, inter=64, top_k=2)
+    g = moe.schedule(rc.T(rc.T_VECTORIZE, 4, stage=0))
+    assert g.knobs(0)["vec"] == 4
+    # rows gathered inside the gate/up GEMM: stage 0 runs no gather pass
+    assert moe.schedule(rc.T(rc.T_COMPUTE_LOCATION, 1, stage=1), rc.T(rc.T_VECTORIZE, 4, stage=0)).knobs(0)["vec"] == 16
+    att = rc.Op(rc.OP_ATTENTION, batch=1, seq=128, heads_q=2, heads_kv=1, head_dim=128, causal=1)
+    assert all(t.kind != rc.T_VECTORIZE for t in att.transform_space())

@@ -1,6 +1,7 @@
 """Host logic of bench.py that needs no GPU: schedule text round trips, the
 stage-by-stage search driver on a synthetic separable landscape, and the
 launch counts the bench reports."""
+import json
 import math
 import os
 import random
@@ -133,3 +134,61 @@ def test_cpu_baseline_reports_all_threads_and_one_thread():
     assert one["value"] > 0 and f"{max(1, 32 // before)} of 64 token rows" in one["sample"]
     ref = bench.Workload("attention", {"seq": 64, "heads_q": 2, "heads_kv": 1}).cpu_sample(8, single_thread=False)
     assert "single_thread" not in ref and "8 of 64 query positions" in ref["sample"]
+
+
+def test_reference_arm_does_not_load_the_library():
+    # the oracle arm (--impl reference) times the CPU oracle alone: the product library stays unloaded
+    import subprocess
+    import sys
+    script = (
+        "import sys, json; sys.argv = ['bench.py', '--impl', 'reference', '--workload', 'gemm_f32', '--steps', '1', "
+        "'--warmup', '0', '--cpu-sample', '1']\n"
+        "import bench\n"
+        "bench.main()\n"
+        "maps = open('/proc/self/maps').read()\n"
+        "from paper_2506_01374_gb300 import rc\n"
+        "print('LIBRC', rc._lib is not None or 'librc.so' in maps)\n")
+    r = subprocess.run([sys.executable, "-c", script], capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = [x for x in r.stdout.splitlines() if x.startswith("{")][0]
+    rec = json.loads(line)
+    assert rec["impl"] == "reference" and rec["cpu_baseline"]["kind"] == "oracle"
+    assert rec["cpu_baseline"]["cpu_model"] and rec["cpu_baseline"]["nproc"] >= 1
+    assert "LIBRC False" in r.stdout
+
+
+def _table1():
+    import csv
+    path = os.path.join(ROOT, "tests", "golden", "table1_sample_efficiency.csv")
+    rows = list(csv.DictReader(line for line in open(path) if not line.startswith("#")))
+    return rows[:-1], rows[-1]
+
+
+def test_sample_efficiency_reproduces_table1():
+    # the paper's Table 1: efficiency = speedup / samples; the gain divides the two methods' efficiencies.
+    # Recomputed from the printed samples and (1-decimal) speedups, every printed gain and reduction is
+    # matched within the printed rounding, and so are the printed geomeans.
+    rows, geo = _table1()
+    assert len(rows) == 25
+    gains, reds = [], []
+    for r in rows:
+        tn, ts, mn, ms = float(r["tvm_samples"]), float(r["tvm_speedup"]), float(r["mcts_samples"]), \
+            float(r["mcts_speedup"])
+        g = bench.efficiency_gain(ts, tn, ms, mn)
+        red = bench.sample_reduction(tn, mn)
+        assert abs(g - float(r["gain"])) <= 0.025 * float(r["gain"]), r
+        assert abs(red - float(r["reduction"])) <= 0.05 + 1e-9, r
+        gains.append(g)
+        reds.append(red)
+    assert round(bench.geomean(float(r["tvm_speedup"]) for r in rows), 1) == float(geo["tvm_speedup"])
+    assert round(bench.geomean(float(r["mcts_speedup"]) for r in rows), 1) == float(geo["mcts_speedup"])
+    assert round(bench.geomean(reds), 1) == float(geo["reduction"])
+    assert round(bench.geomean(gains), 1) == float(geo["gain"])
+    # the gain is the speedup ratio times the sample reduction
+    assert math.isclose(bench.efficiency_gain(3.9, 510, 5.1, 60), (5.1 / 3.9) * (510 / 60), rel_tol=1e-12)
+
+
+def test_reach_of_a_best_so_far_curve():
+    curve = [(1, 10.0), (2, 8.0), (3, 8.0), (4, 5.0), (5, 5.0), (6, 5.0)]
+    assert bench.reach(curve, 10.0) == (4, 2.0)
+    assert bench.reach([(1, 3.0)], 3.0) == (1, 1.0)

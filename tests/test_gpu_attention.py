@@ -58,12 +58,13 @@ def test_attention_schedule_sweep(B, S, Hq, Hkv, causal):
         assert rel_err(L, L_ref) <= TOL_LSE, (bn, st, ra, lay, loc, un, par)
         n += 1
     assert n >= 40
-    with pytest.raises(rc.RcError):  # split UMMA issue keeps P in tensor memory
-        sched(op, 64, 2, 0, 0, 0, 1, 1)
     with pytest.raises(rc.RcError):  # row sums on the tensor core read V as given
         sched(op, 64, 2, 0, 1, 2, 1, 1)
-    with pytest.raises(rc.RcError):  # one issuing warp: one S buffer
-        sched(op, 64, 2, 0, 0, 0, 2, 0)
+    # each kernel family's canonical form: one issuing warp keeps P in shared memory and one S buffer,
+    # split issue keeps P in tensor memory, so one Parallel transformation moves between them
+    assert str(sched(op, 64, 2, 0, 0, 0, 2, 0)) == str(sched(op, 64, 2, 0, 0, 0, 1, 0))
+    assert str(sched(op, 64, 2, 0, 0, 0, 1, 1)) == str(sched(op, 64, 2, 0, 0, 1, 1, 1))
+    assert op.schedule(rc.T(rc.T_PARALLEL, 1)).knobs(0)["location"] == 1
 
 
 def test_attention_single_token_and_no_lse():
