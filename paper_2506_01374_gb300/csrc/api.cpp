@@ -32,8 +32,13 @@ bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, 
     if (why) *why = "UMMA N must be a multiple of 16 in [16, 256]";
     return false;
   }
-  if (tile_m != 128 && tile_m != 256) {
-    if (why) *why = "M tile must be 128 (one CTA) or 256 (a CTA pair)";
+  if (tile_m != 128 && tile_m != 256 && tile_m != 512) {
+    if (why) *why = "M tile must be 128 (one CTA), 256 (a CTA pair) or 512 (four CTAs sharing B)";
+    return false;
+  }
+  if (tile_m == 512 && (bn_mma % 32 != 0 || persistent)) {
+    // each of the four CTAs loads BN / 4 rows of B: whole 8-row swizzle atoms
+    if (why) *why = "a B-multicast cluster needs an N tile divisible by 32 and one tile per cluster";
     return false;
   }
   if (tile_m == 256 && bn_mma < 32) {
@@ -125,7 +130,8 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       break;
     case RC_OP_LINEAR:
       gemm_common({64, 128, 224, 256});
-      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});  // one CTA, or a CTA pair sharing each UMMA
+      // one CTA, a CTA pair sharing each UMMA, or four CTAs sharing the B tile by TMA multicast
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256, 512}, {}});
       v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       vectorize();
       break;
@@ -143,12 +149,14 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_SPLIT_K, 0, {1, 2, 4}, {}});
       }
-      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+      // the down projection may also share its B tile across four CTAs
+      v.push_back({RC_T_TILE_SIZE, 0, stage == 0 ? std::vector<int32_t>{128, 256} : std::vector<int32_t>{128, 256, 512},
+                   {}});
       vectorize();
       break;
     case RC_OP_CONV2D:
       gemm_common({64, 80, 160});
-      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256, 512}, {}});
       v.push_back({RC_T_SPLIT_K, 0, {1, 3, 5}, {}});
       v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
       vectorize();
@@ -163,7 +171,8 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       if (stage != 2) {
         // 0: QKV projection, 3: O projection, 4: gate/up + SwiGLU, 5: down projection
         gemm_common(stage == 4 ? std::vector<int32_t>{32, 64, 128} : std::vector<int32_t>{64, 128, 224, 256});
-        v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+        v.push_back({RC_T_TILE_SIZE, 0, stage == 4 ? std::vector<int32_t>{128, 256} : std::vector<int32_t>{128, 256, 512},
+                     {}});
         if (stage == 4) {
           v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
           vectorize();  // the SwiGLU pass of the unfused gate/up GEMM
@@ -309,8 +318,12 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
         if (why) *why = "conv N tile must divide Cout";
         return false;
       }
-      if (k.tile_m == 256 && k.layout == 2) {
-        if (why) *why = "a CTA pair loads A as one 4-D box (layouts 0 and 1)";
+      if (k.tile_m >= 256 && k.layout == 2) {
+        if (why) *why = "a CTA pair or a B-multicast cluster loads A as one 4-D box (layouts 0 and 1)";
+        return false;
+      }
+      if (k.tile_m == 512 && (o.img_n * o.img_h * o.img_w) % 512 != 0) {
+        if (why) *why = "a B-multicast cluster needs whole 512-row tiles of output pixels";
         return false;
       }
       return tc_gemm_ok(k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);

@@ -13,6 +13,7 @@ rc_status tc_dispatch_conv_pair(const rc_knobs& k, const TcGemmArgs& a, const La
 rc_status tc_dispatch_grouped_pair(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_conv(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_grouped(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
+rc_status tc_dispatch_mc(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 
 namespace tcg {
 namespace {
@@ -80,7 +81,9 @@ rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const Launch
   if (a.M > 0x7fffffff || a.N > 0x7fffffff || a.K > 0x7fffffff)
     return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: dimension exceeds 2^31");
   if (k.stages < 1) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: stages < 1");
-  if (k.tile_m != 128 && k.tile_m != 256) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: M tile %d", k.tile_m);
+  if (k.tile_m != 128 && k.tile_m != 256 && k.tile_m != 512)
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: M tile %d", k.tile_m);
+  if (k.tile_m == 512) return tc_dispatch_mc(k, a, c);  // four CTAs sharing the B tile by multicast
   const bool pair = k.tile_m == 256;  // a CTA pair per 256-row tile
   if (a.a_mode == TC_A_CONV || a.a_mode == TC_A_CONV_ROWS)
     return pair ? tc_dispatch_conv_pair(k, a, c) : tc_dispatch_conv(k, a, c);

@@ -297,14 +297,29 @@ __device__ __forceinline__ Item resolve_item(const Params& p, long long w, const
 // UMMAs and multicasts its commits to both CTAs' "empty" and "accumulator
 // full" barriers; each CTA's epilogue drains its own TMEM rows and arrives
 // on the leader's "accumulator empty" barrier (one arrival per warp).
-template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
+//
+// MC > 1 (TileSize M = 128 MC): a cluster of MC CTAs along M computes MC
+// consecutive 128 x BN tiles of one N tile with cta_group::1 UMMAs. They
+// need the same B tile, so each CTA loads 1 / MC of its rows and multicasts
+// them into every CTA of the cluster: B is read from L2 once per cluster
+// instead of once per CTA. A stage of a CTA is overwritten by its peers'
+// copies, so every CTA's MMA thread releases a stage into all the cluster's
+// "empty" barriers (a multicast commit; each counts MC arrivals) and a
+// producer refills a stage only once every CTA has released it.
+template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false, int MC = 1>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const Params p,
                 const int stages) {
   constexpr int A_BYTES = BM * BK * 2;                    // one 64-wide K sub-block of A
   constexpr int B_BYTES = (PAIR ? BN / 2 : BN) * BK * 2;  // and this CTA's rows of B
   constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  constexpr bool CLUSTER = PAIR || MC > 1;
   static_assert(B_BYTES % 1024 == 0, "B tile must keep stage buffers 1024-byte aligned");
+  static_assert(MC == 1 || MC == 2 || MC == 4 || MC == 8, "cluster size");
+  static_assert(MC == 1 || (!PAIR && !GROUPED && EPI != TC_EPI_SWIGLU && AMODE != TC_A_GATHER &&
+                            (BN / MC) % 8 == 0),
+                "B multicast: one-CTA tiles of a dense or convolution GEMM, 8-row swizzle atoms per slice");
+  constexpr uint16_t MC_MASK = (uint16_t)((1u << MC) - 1u);
   // stage layout: A sub-blocks [0, ksub), then B sub-blocks [0, ksub)
   const int ksub = p.ksub;
   const uint32_t STAGE_BYTES = (uint32_t)ksub * (A_BYTES + B_BYTES);
@@ -332,12 +347,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_acc = p.persistent ? 2 : 1;  // accumulator buffers in TMEM
   const uint32_t tmem_cols = ACC_COLS * (uint32_t)n_acc;
   const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;  // tiles of 128 (PAIR: 256) rows
-  const uint32_t rank = PAIR ? tc::cluster_ctarank() : 0u;              // 0 = leader of the pair
-  const long long w_first = PAIR ? blockIdx.x / 2 : blockIdx.x;
-  const long long w_step = PAIR ? gridDim.x / 2 : gridDim.x;
+  const uint32_t rank = CLUSTER ? tc::cluster_ctarank() : 0u;  // PAIR: 0 = leader of the pair
+  constexpr int PER_ITEM = PAIR ? 2 : MC;                        // CTAs per work item
+  const long long w_first = blockIdx.x / PER_ITEM;
+  const long long w_step = gridDim.x / PER_ITEM;
   auto item = [&](long long w) -> Item {
-    Item it = resolve_item<GROUPED, PAIR ? 2 * BM : BM>(p, w, s_goff, s_gtile);
-    if constexpr (PAIR) it.row0 += (int)rank * BM;  // this CTA's half of the 256-row tile
+    Item it = resolve_item<GROUPED, PER_ITEM * BM>(p, w, s_goff, s_gtile);
+    it.row0 += (int)rank * BM;  // this CTA's 128 rows of the PER_ITEM x 128-row tile
     return it;
   };
 
@@ -350,7 +366,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int s = 0; s < stages; ++s) {
       // gathered A: lane 0's arrival with the B bytes and one arrival per lane for its A copies
       tc::mbar_init(&full[s], AMODE == TC_A_GATHER ? 33 : 1);
-      tc::mbar_init(&empty[s], 1);
+      tc::mbar_init(&empty[s], MC);  // MC > 1: released by every CTA of the cluster
     }
     for (int b = 0; b < 2; ++b) {
       tc::mbar_init(&acc_full[b], 1);
@@ -370,8 +386,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 2) build_group_table<PAIR ? 2 * BM : BM>(p, lane, s_goff, s_gtile);
   }
   tc::tc_fence_before();
-  if constexpr (PAIR)
-    tc::cluster_sync();  // both CTAs' barriers exist before any copy or commit reaches them
+  if constexpr (CLUSTER)
+    tc::cluster_sync();  // every CTA's barriers exist before any copy or commit reaches them
   else
     __syncthreads();
   tc::tc_fence_after();
@@ -481,7 +497,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* stage = smem + (size_t)s * STAGE_BYTES;
           // PAIR: the leader's barrier counts both CTAs' bytes
           const uint32_t cbar = PAIR ? tc::mapa_shared(tc::smem_u32(&full[s]), 0) : 0u;
-          if (rank == 0) tc::mbar_expect_tx(&full[s], (uint32_t)nsub * (PAIR ? 2 : 1) * (A_BYTES + B_BYTES));
+          // MC > 1: every CTA's barrier counts its own A and the whole B tile (all the slices)
+          if (rank == 0 || !PAIR)
+            tc::mbar_expect_tx(&full[s], (uint32_t)nsub * (PAIR ? 2 : 1) * (A_BYTES + B_BYTES));
           auto ld2 = [&](void* dst, const CUtensorMap* m, int x, int y) {
             if constexpr (PAIR)
               tc::tma_load_2d_pair(dst, m, cbar, x, y);
@@ -521,6 +539,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ld2(sb, &tmB, kb * BK, it.brow0 + nh);
                 ld2(sb + (BN / 2) * 128, &tmB, kb * BK, it.brow0 + p.swiglu_I + nh);
               }
+            } else if constexpr (MC > 1) {
+              // this CTA's 1 / MC of the B tile's rows, into every CTA of the cluster
+              tc::tma_load_2d_mc(sb + rank * (BN / MC) * 128, &tmB, &full[s], kb * BK,
+                                 it.brow0 + it.nt * BN + (int)rank * (BN / MC), MC_MASK);
             } else {
               ld2(sb, &tmB, kb * BK, it.brow0 + it.nt * BN + (int)rank * (BN / 2));
             }
@@ -536,7 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // instead, bounded, for the leader's release of those slots)
       const uint32_t first = g > (uint32_t)stages ? g - (uint32_t)stages : 0u;
       for (uint32_t j = first; j < g; ++j) {
-        if (rank == 0) {
+        if (rank == 0 || !PAIR) {
           if (!tc::mbar_wait_drain(&full[j % (uint32_t)stages], (j / (uint32_t)stages) & 1u))
             fail(RC_DEV_TIMEOUT_DRAIN);
         } else {
@@ -546,7 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
-    if (lane == 0 && rank == 0) {
+    if (lane == 0 && (rank == 0 || !PAIR)) {
       constexpr uint32_t idesc = tc::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN);
       uint32_t li = 0;
       int s = 0;        // ring slot, advanced in step with the producer
@@ -591,6 +613,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if constexpr (PAIR)
             tc::umma_commit_pair(&empty[s], 3);  // the slot is free in both CTAs
+          else if constexpr (MC > 1)
+            tc::umma_commit_mc(&empty[s], MC_MASK);  // this CTA has read the slot: every producer may refill it
           else
             tc::umma_commit(&empty[s]);
           if (++s == stages) {
@@ -650,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   tc::tc_fence_before();
-  if constexpr (PAIR)
+  if constexpr (CLUSTER)
     tc::cluster_sync();  // no copy, commit or arrival may reach a CTA that has exited
   else
     __syncthreads();
@@ -671,10 +695,10 @@ rc_status encode_conv(CUtensorMap* m, const void* x, uint64_t c, uint64_t w, uin
 
 template <typename Kern>
 rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tmB, const Params& p, int stages,
-                        int acc_cols, size_t smem, bool pair, const LaunchCtx& c) {
+                        int acc_cols, size_t smem, int per_item, const LaunchCtx& c) {
   const long long items = (long long)p.tiles_m * p.tiles_n * p.splits;
   if (items <= 0 || items > 0x3fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: %lld work items", items);
-  const int per_item = pair ? 2 : 1;  // CTAs per work item
+  // per_item: CTAs per work item (the cluster: 2 for a CTA pair, MC for B multicast)
   long long ctas = items * per_item;
   if (p.persistent) {
     // as many CTAs as fit on the SMs at once (shared memory and 512 TMEM columns)
@@ -698,7 +722,7 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pair ? 1 : 0;
+  cfg.numAttrs = per_item > 1 ? 1 : 0;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmA, tmB, p, stages);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return rc_fail(RC_ERR_CUDA, "tc_gemm launch: %s", cudaGetErrorString(e));
@@ -715,9 +739,9 @@ inline size_t smem_bytes(int bn, int stages, int ksub, bool pair = false) {
          kGroupTableBytes;
 }
 
-template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false>
+template <int BN, int EPI, int AMODE, bool GROUPED, bool PAIR = false, int MC = 1>
 rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
-  auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED, PAIR>;
+  auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED, PAIR, MC>;
   if (k.tile_k != 64 && k.tile_k != 128) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: K tile %d", k.tile_k);
   constexpr int acc_cols_tile = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   if (PAIR && (k.persistent ? 2 : 1) * acc_cols_tile > 256)
@@ -748,7 +772,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   if (GROUPED && (a.groups < 1 || a.groups > kSmemGroups))
     return rc_fail(RC_ERR_UNSUPPORTED_OP, "tc_gemm: grouped GEMM with %d segments (1 .. %d)", a.groups, kSmemGroups);
   const int64_t b_rows = GROUPED ? (int64_t)a.groups * a.b_group_rows : a.N;
-  RC_TRY(encode_2d(&tmB, a.B, a.K, b_rows, (PAIR || EPI == TC_EPI_SWIGLU) ? BN / 2 : BN));
+  RC_TRY(encode_2d(&tmB, a.B, a.K, b_rows, (PAIR || EPI == TC_EPI_SWIGLU) ? BN / 2 : BN / MC));
   Params p;
   memset(&p, 0, sizeof p);
   p.M = (int)a.M;
@@ -757,7 +781,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   const int out_w = EPI == TC_EPI_SWIGLU ? (int)(a.N / 2) : (int)a.N;
   const int tile_out = EPI == TC_EPI_SWIGLU ? BN / 2 : BN;
   p.tiles_n = (out_w + tile_out - 1) / tile_out;
-  const int64_t tile_rows = PAIR ? 2 * BM : BM;
+  const int64_t tile_rows = (PAIR ? 2 : MC) * BM;
   // grouped: an upper bound of the tiles the segments need (spare tiles are skipped)
   p.tiles_m = GROUPED ? (int)(PAIR ? a.M / tile_rows + a.groups : a.max_tiles_m)
                       : (int)((a.M + tile_rows - 1) / tile_rows);
@@ -795,7 +819,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.a_src = (const __nv_bfloat16*)a.A;
   p.status = c.status;
   constexpr int acc_cols = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
-  return launch_kernel(kern, tmA, tmB, p, k.stages, acc_cols, smem, PAIR, c);
+  return launch_kernel(kern, tmA, tmB, p, k.stages, acc_cols, smem, PAIR ? 2 : MC, c);
 }
 
 }  // namespace tcg

@@ -101,3 +101,26 @@ def test_conv_full_size_sampled_pixels():
         op.check()
         got = from_dev_bf16(dy).reshape(-1, C)[pix]
         assert rel_err(got, ref) <= TOL, str(s)
+
+
+def test_conv_b_multicast_clusters():
+    # TileSize M = 512: four CTAs along M share each B (weight) tile through TMA multicast
+    N, H, W, Cin, Cout = 2, 16, 32, 128, 320
+    x, w, b = inputs.conv2d(N, H, W, Cin, Cout, seed=32)
+    ref = oracle.conv2d_nhwc_bf16(x, w, b)
+    op = conv_op(N, H, W, Cin, Cout)
+    n = 0
+    for tn, st, tk, split, fuse, lay in itertools.product((64, 160), (1, 3, 4), (64, 128), (1, 3), (0, 1), (0, 1)):
+        try:
+            s = sched(op, tn, st, split, fuse, 0, lay, tk, 512)
+        except rc.RcError:
+            continue  # shared memory
+        dy = empty_bf16(N, H, W, Cout).fill_(0x7FC0)
+        op.run(s, [to_dev(x), to_dev(w), to_dev(b), dy])
+        op.check()
+        assert rel_err(from_dev_bf16(dy).reshape(-1, Cout), ref) <= TOL, str(s)
+        n += 1
+    assert n >= 30
+    with pytest.raises(rc.RcError):  # B slices of 80 / 4 rows are not whole swizzle atoms
+        sched(op, 80, 2, 1, 1, 0, 0, 64, 512)
+

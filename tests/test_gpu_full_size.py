@@ -80,6 +80,8 @@ def test_conv2d_full_size_reported_schedules():
     ref = oracle.conv2d_nhwc_bf16(x, w, b, pix=pix)
     dx, dw, db = to_dev(x), to_dev(w), to_dev(b)
     for c in [dict(s0=dict(tile_n=160, tile_k=128, stages=3, fuse=1, persistent=1)),
+              dict(s0=dict(tile_m=512, tile_n=160, tile_k=64, stages=4, fuse=1)),
+              dict(s0=dict(tile_m=512, tile_n=160, tile_k=128, stages=3, fuse=1)),
               dict(s0=dict(tile_n=160, tile_k=128, stages=3, fuse=1, persistent=0)),
               dict(s0=dict(tile_n=160, tile_k=64, stages=6, fuse=1, persistent=1))]:
         s = schedule(op, **c)

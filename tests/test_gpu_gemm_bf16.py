@@ -148,3 +148,26 @@ def test_mlp_host_path_matches_device_path():
     op.check()
     np.testing.assert_array_equal(Yh, dY.cpu().numpy().view(np.uint16))
     assert rel_err(inputs.bf16_bits_to_f64(Yh), oracle.mlp_bf16(X, W1, W2)) <= TOL
+
+
+@pytest.mark.parametrize("M,N,K", [(1000, 512, 520), (2048, 256, 1024), (130, 128, 64)])
+def test_linear_b_multicast_clusters(M, N, K):
+    # TileSize M = 512: four CTAs along M share each B tile through TMA multicast; a ragged last
+    # cluster reads zero rows past M and stores nothing there
+    X, W = inputs.linear_bf16(M, N, K, seed=26)
+    ref = oracle.linear_bf16(X, W)
+    op = rc.Op(rc.OP_LINEAR, m=M, n=N, k=K)
+    dX, dW = to_dev(X), to_dev(W)
+    n = 0
+    for tn, st, tk, split in itertools.product((64, 128, 256), (1, 2, 4), (64, 128), (1, 2)):
+        try:
+            s = sched(op, tile_m=512, tile_n=tn, stages=st, tile_k=tk, split_k=split)
+        except rc.RcError:
+            continue
+        dY = empty_bf16(M, N).fill_(0x7FC0)
+        op.run(s, [dX, dW, dY])
+        op.check()
+        assert rel_err(from_dev_bf16(dY), ref) <= TOL, str(s)
+        n += 1
+    assert n >= 20
+
