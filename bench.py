@@ -85,7 +85,9 @@ def parse():
                     help="instead of the benchmark line: 'search' prints best-so-far curves (JSON lines) of the "
                          "search variants on --workload: MCTS with measured rollouts at B = 2 and 4, MCTS with the "
                          "learned surrogate and 4x screening, random search, and (composite ops) stage-by-stage "
-                         "tuning then a joint search, over seeds --seed .. --seed+1")
+                         "tuning then a joint search, over seeds --seed .. --seed+1; 'library' times the vendor "
+                         "libraries (cuDNN attention and convolution, cuBLAS GEMMs through torch) on --workload's "
+                         "inputs under the bench's timing protocol")
     ap.add_argument("--study-variants", default="",
                     help="with --study search: comma-separated variant names to run (default: all)")
     ap.add_argument("--shape", default="",
@@ -896,6 +898,93 @@ def search_study(wl, io, samples, seed, only=""):
                                                              for v, r in rows)}), flush=True)
 
 
+def library_study(wl, sched_text="", reps=20):
+    """Vendor-library baselines on the workload's inputs (cuDNN attention and convolution, cuBLAS GEMMs,
+    called through torch), timed like the search's candidates: inputs resident in HBM, the L2 flushed
+    before every repeat, CUDA events around the call, the median reported. Printed as JSON lines, with the
+    op's own flop count so the rates compare with the bench line's. With a schedule, this library's
+    program is timed in the same process first (same clocks, same inputs). Context for the kernels'
+    figures."""
+    import statistics
+
+    import numpy as np
+    import torch
+    import torch.nn.functional as F
+
+    peak = peaks()["bf16_tflops"]
+    flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
+
+    def bf16(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.bfloat16)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        ts = []
+        for _ in range(reps):
+            flush.fill_(1.0)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts)
+
+    flops = wl.op.info["flops"]
+    if sched_text:
+        from paper_2506_01374_gb300 import rc
+        m = wl.op.measure([parse_schedule(wl.op, sched_text, rc)], wl.device_io(), warmup=3, repeats=reps)[0]
+        print(json.dumps({"study": "library", "workload": wl.label, "library": "this repository", "schedule": sched_text,
+                          "value": round(m.tflops, 1), "unit": "TFLOP/s", "us": round(m.ms_median * 1e3, 2),
+                          "frac": round(m.tflops / peak, 3), "status": m.status}), flush=True)
+
+    def line(lib, fn, note=""):
+        try:
+            ms = timed(fn)
+        except Exception as e:  # a backend this torch build or GPU does not offer
+            rec = {"study": "library", "workload": wl.label, "library": lib, "unavailable": str(e).splitlines()[0][:160]}
+        else:
+            tf = flops / (ms * 1e-3) / 1e12
+            rec = {"study": "library", "workload": wl.label, "library": lib, "value": round(tf, 1), "unit": "TFLOP/s",
+                   "us": round(ms * 1e3, 2), "frac": round(tf / peak, 3)}
+        if note:
+            rec["note"] = note
+        print(json.dumps(rec), flush=True)
+
+    if wl.name in ("attention", "attention_flux"):
+        from torch.nn.attention import SDPBackend, sdpa_kernel
+        causal = bool(wl.config["causal"])
+        Q, K, V = [bf16(a).transpose(1, 2).contiguous() for a in wl.host[:3]]  # [B][H][S][D]
+        gqa = Q.shape[1] != K.shape[1]
+        for name, bk in (("cudnn sdpa", SDPBackend.CUDNN_ATTENTION), ("flash sdpa", SDPBackend.FLASH_ATTENTION)):
+            def call(bk=bk):
+                with sdpa_kernel([bk]):
+                    return F.scaled_dot_product_attention(Q, K, V, is_causal=causal, enable_gqa=gqa)
+            line(name, call)
+    elif wl.name == "conv2d":
+        x, w, b = wl.host[:3]
+        xt = bf16(x).permute(0, 3, 1, 2)  # NHWC storage seen as NCHW: channels_last
+        wt = bf16(w).permute(0, 3, 1, 2)
+        bt = bf16(b)
+        torch.backends.cudnn.benchmark = True
+        line("cudnn conv2d + bias", lambda: F.conv2d(xt, wt, bt, padding=1), "SiLU not included")
+        line("cudnn conv2d + bias, then torch SiLU", lambda: F.silu(F.conv2d(xt, wt, bt, padding=1)))
+    elif wl.name == "linear":
+        X, Wt = bf16(wl.host[0]), bf16(wl.host[1])
+        line("cublas matmul", lambda: X @ Wt.t())
+    elif wl.name == "mlp":
+        X, W1, W2 = [bf16(a) for a in wl.host[:3]]
+        I = W2.shape[1]
+
+        def block():
+            h = X @ W1.t()
+            return (F.silu(h[:, :I]) * h[:, I:]) @ W2.t()
+        line("cublas gate/up matmul + torch SiLU/mul + cublas down matmul", block)
+    else:
+        print(json.dumps({"study": "library", "workload": wl.label, "unavailable": "no library equivalent compared"}))
+
+
 def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None,
               layer_samples=None, hbm_gbs=None):
     """Search each other workload briefly and report its best schedule."""
@@ -1017,6 +1106,9 @@ def run_ours(args):
     wl = Workload(args.workload, parse_shape(args.shape))
     if args.study == "search":
         search_study(wl, wl.device_io(), args.samples, args.seed, args.study_variants)
+        return
+    if args.study == "library":
+        library_study(wl, args.schedule)
         return
     if args.study:
         raise SystemExit(f"unknown --study {args.study}")

@@ -182,6 +182,9 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
       [[fallthrough]];  // 2: the attention core
     case RC_OP_ATTENTION:
       v.push_back({RC_T_TILE_SIZE, 1, {64, 128}, {}});  // key block BN
+      // query rows per CTA: one 128-row tile, or two tiles sharing each K and V block (128-key
+      // blocks, one CTA per SM, the tensor core working on one tile while the other's softmax runs)
+      v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
       v.push_back({RC_T_PIPELINE_STAGES, 0, {1, 2, 3, 4, 5}, {}});
       v.push_back({RC_T_LOOP_ORDER, 0, {0, 1}, {1}});  // 0 = head-major tiles, 1 = longest causal rows first
       v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});        // V as [keys][d] or transposed to [d][keys]
@@ -353,6 +356,16 @@ static bool attention_knobs_ok(const rc_knobs& k, int64_t seq, std::string* why)
     return false;
   };
   // (rc_schedule_apply canonicalises location and unroll per kernel family before this check)
+  if (k.tile_m == 256) {
+    if (k.tile_n != 128 || k.persistent != 1 || k.location != 1 || k.unroll != 1)
+      return no("two query tiles per CTA take 128-key blocks, P in tensor memory and one S buffer per tile");
+    if (k.layout == 1 && seq % 8) return no("transposed V needs seq % 8 == 0 (16-byte TMA rows)");
+    // two query tiles, the K ring, a two-slot V ring, barriers, TMEM address and abort flag, slack
+    const int64_t smem2 = 2 * 128 * 128 * 2 + (k.stages + 2) * 128 * 128 * 2 + (14 + k.stages) * 8 + 8 + 1024;
+    if (smem2 > kSmemLimit) return no("attention ring exceeds 227 KB of shared memory");
+    return true;
+  }
+  if (k.tile_m != 128) return no("query tiles of 128 or 256 rows");
   if (k.persistent == 0) {
     if (k.location != 0 || k.unroll != 1) return no("one UMMA-issuing warp keeps P in shared memory and one S buffer");
   } else if (k.location == 0) {
@@ -734,13 +747,19 @@ extern "C" rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base,
   // leaves the program unchanged, so the canonical form keeps the default
   for (int i = 0; i < s.n_stages; ++i)
     if (!vectorize_used(op, s, i)) s.k[i].vec = rc_default_knobs(op, i).vec;
-  // attention: the one-issuing-warp kernel keeps P in shared memory and one S buffer, and the
-  // split-issue kernels keep P in tensor memory, so each family's canonical form fixes the knobs it
-  // does not offer (a single Parallel transformation then moves between the families)
+  // attention: the one-issuing-warp kernel keeps P in shared memory and one S buffer, the
+  // split-issue kernels keep P in tensor memory, and the two-query-tile kernel has one form for each
+  // key block, so each family's canonical form fixes the knobs it does not offer (a single Parallel
+  // or TileSize transformation then moves between the families)
   for (int i = 0; i < s.n_stages; ++i) {
     if (!(op->d.kind == RC_OP_ATTENTION || (op->d.kind == RC_OP_DECODER_LAYER && i == 2))) continue;
     rc_knobs& k = s.k[i];
-    if (k.persistent == 0) {
+    if (k.tile_m == 256) {  // two query tiles per CTA: one kernel, whatever the other families' knobs
+      k.tile_n = 128;
+      k.persistent = 1;
+      k.location = 1;
+      k.unroll = 1;
+    } else if (k.persistent == 0) {
       k.location = 0;
       k.unroll = 1;
     } else if (k.location == 0) {

@@ -9,13 +9,17 @@
 // than 2^8, and write P_j as bf16; the tensor core then adds P_j V_j to O.
 // The epilogue divides O by l and stores bf16 O and LSE = ln 2 * (m + log2 l).
 //
-// Two kernel families, chosen by the schedule's Parallel knob:
-//   0: attn_kernel - one warp issues every UMMA, P goes through shared
-//      memory (the unoptimised program P0);
-//   1, 2: attn4_kernel - S and P V issued by warps of their own, P in TMEM,
-//      one or two S buffers (Unroll), one or two softmax threads per row
-//      (Parallel 2), and optionally the row sums formed by the tensor core
-//      (ComputeLocation 2).
+// Three kernel families, chosen by the schedule's Parallel and TileSize M
+// knobs:
+//   Parallel 0: attn_kernel - one warp issues every UMMA, P goes through
+//      shared memory (the unoptimised program P0);
+//   Parallel 1, 2: attn4_kernel - S and P V issued by warps of their own, P
+//      in TMEM, one or two S buffers (Unroll), one or two softmax threads per
+//      row (Parallel 2), and optionally the row sums formed by the tensor
+//      core (ComputeLocation 2);
+//   TileSize M 256: attn2q_kernel - two 128-row query tiles per CTA sharing
+//      each 128-key K and V block, one CTA per SM, the tensor core working on
+//      one tile while the other's softmax runs.
 // Other knobs: BN (TileSize N), ring depth (PipelineStages), query-block
 // order (natural or longest causal rows first), and the layout of V: as given
 // ([keys][d], an MN-major UMMA B operand) or pre-transposed by a pass into
@@ -999,6 +1003,396 @@ __global__ void __launch_bounds__(attn4_threads<SPLIT>(), (Attn4Cols<BN, NSB, SU
   }
 }
 
+// Two query tiles per CTA (TileSize M = 256) with 128-key blocks. The CTA
+// holds the whole SM: TMEM columns [0, 128) and [128, 256) are S_0 and S_1
+// (fp32), [256, 384) and [384, 512) are O_0 and O_1; P_t (bf16 pairs) is
+// written over the first 64 columns of S_t. One thread issues every UMMA in
+// the order P_0 V_{j-1}, S_0(j), P_1 V_{j-1}, S_1(j): while tile t's softmax
+// works on S_t(j), the tensor core runs the other tile's P V and S products,
+// and K_j and V_j are loaded once for both tiles.
+//   warps 0..7 : softmax, one thread per query row; warp w serves tile w / 4,
+//                TMEM lane quadrant w % 4
+//   warp 8     : TMA producer of Q and of the K ring; owns TMEM
+//   warp 9     : TMA producer of the V ring
+//   warp 10    : the UMMA issue loop, run by all 32 lanes on warp-uniform
+//                descriptors, one elected lane issuing (a lane-0 branch
+//                spends far longer per UMMA forming its operands)
+// S_t(j) overwrites the columns P_t(j-1) V_{j-1} read as its A operand; both
+// are issued by the same thread, and tcgen05.mma operations of one thread
+// execute in issue order. The commit that signals S_t(j) also covers
+// P_t(j-1) V_{j-1}, so the softmax may rescale O_t as soon as S_t(j) is
+// ready. One commit per iteration (it_done) releases both rings: K_j's slot
+// after S_1(j), V_{j-1}'s after P_1 V_{j-1}. A tile's key blocks: every
+// block up to its diagonal when causal (the second tile has one more than
+// the first), all blocks otherwise; a tile with no query row inside the
+// sequence takes none.
+constexpr int kBN2q = 128;
+constexpr int kVStages2q = 2;
+constexpr int kItRing2q = 4;  // it_done barriers: more than the K (<= 3) and V (2) ring depths
+constexpr int kThreads2q = 32 * 11;
+
+// Bytes of dynamic shared memory: two query tiles, the K ring (the schedule's
+// stages), a two-slot V ring, barriers (q_full, k_full[stages], v_full[2],
+// it_done[4], s_full[2], p_full[2], o_full[2], drain), the TMEM address and
+// abort flag, and 1 KB of alignment slack.
+__host__ __device__ constexpr size_t attn2q_smem(int stages) {
+  return (size_t)2 * BM * D * 2 + (size_t)(stages + kVStages2q) * kBN2q * D * 2 + (size_t)(14 + stages) * 8 + 8 + 1024;
+}
+
+// Adds the two bf16 halves of v to a and b in fp32 (mixed-precision adds of sm_100+).
+__device__ __forceinline__ void acc_bf16x2(float& a, float& b, uint32_t v) {
+  asm("{\n\t.reg .b16 lo, hi;\n\t"
+      "mov.b32 {lo, hi}, %2;\n\t"
+      "add.rn.f32.bf16 %0, lo, %0;\n\t"
+      "add.rn.f32.bf16 %1, hi, %1;\n\t}"
+      : "+f"(a), "+f"(b)
+      : "r"(v));
+}
+
+// exp_pack_bf16 in place: the bf16 pair of scores i, i + 1 goes to r[i / 2],
+// which has been read by then, so P needs no registers of its own. Four
+// pairs per volatile block: the compiler keeps the blocks in order, so at
+// most four pairs' exponents are live at once (hoisting every packed FMA
+// ahead of the exponentials would need 64 more registers).
+template <int N>
+__device__ __forceinline__ void exp_pack_bf16_inplace(uint32_t* r, uint64_t sc2, uint64_t nm2) {
+  static_assert(N % 8 == 0, "four pairs per block");
+#pragma unroll
+  for (int i = 0; i < N; i += 8) {
+    uint32_t e0, e1, e2, e3;
+    asm volatile(
+        "{\n\t.reg .b64 x0, x1, x2, x3;\n\t.reg .f32 a0, b0, a1, b1, a2, b2, a3, b3;\n\t"
+        ".reg .b32 c0, c1, c2, c3;\n\t"
+        "mov.b64 x0, {%4, %5};\n\tmov.b64 x1, {%6, %7};\n\tmov.b64 x2, {%8, %9};\n\tmov.b64 x3, {%10, %11};\n\t"
+        "fma.rn.f32x2 x0, x0, %12, %13;\n\tfma.rn.f32x2 x1, x1, %12, %13;\n\t"
+        "fma.rn.f32x2 x2, x2, %12, %13;\n\tfma.rn.f32x2 x3, x3, %12, %13;\n\t"
+        "mov.b64 {a0, b0}, x0;\n\tmov.b64 {a1, b1}, x1;\n\tmov.b64 {a2, b2}, x2;\n\tmov.b64 {a3, b3}, x3;\n\t"
+        "cvt.rn.bf16x2.f32 c0, b0, a0;\n\tcvt.rn.bf16x2.f32 c1, b1, a1;\n\t"
+        "cvt.rn.bf16x2.f32 c2, b2, a2;\n\tcvt.rn.bf16x2.f32 c3, b3, a3;\n\t"
+        "ex2.approx.ftz.bf16x2 %0, c0;\n\tex2.approx.ftz.bf16x2 %1, c1;\n\t"
+        "ex2.approx.ftz.bf16x2 %2, c2;\n\tex2.approx.ftz.bf16x2 %3, c3;\n\t}"
+        : "=r"(e0), "=r"(e1), "=r"(e2), "=r"(e3)
+        : "r"(r[i]), "r"(r[i + 1]), "r"(r[i + 2]), "r"(r[i + 3]), "r"(r[i + 4]), "r"(r[i + 5]), "r"(r[i + 6]),
+          "r"(r[i + 7]), "l"(sc2), "l"(nm2));
+    r[i / 2] = e0;
+    r[i / 2 + 1] = e1;
+    r[i / 2 + 2] = e2;
+    r[i / 2 + 3] = e3;
+  }
+}
+
+// Softmax of query tile t (of the two) for TMEM lane quadrant qd, one
+// thread per query row: the block's 128 scores in registers, the row
+// maximum, the exponentials packed to bf16 pairs in place and written over
+// S_t as P_t, the row sum of those bf16 values in fp32, and O_t rescaled when
+// the maximum has grown by more than 2^8.
+__device__ __forceinline__ void softmax_2q(const Params& p, int t, int qd, int lane, int q0, int nk, int b, int h,
+                                           uint32_t tmem, uint64_t* s_full, uint64_t* p_full, uint64_t* o_full,
+                                           volatile int* abort_flag, volatile int* status) {
+  constexpr int BN = kBN2q;
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+  const int row = 32 * qd + lane;
+  const int qi = q0 + t * BM + row;
+  const uint32_t lane_base = (uint32_t)(32 * qd) << 16;
+  const uint32_t tS = tmem + lane_base + (uint32_t)(t * 128);
+  const uint32_t tO = tmem + lane_base + 256u + (uint32_t)(t * 128);
+  float m_ref = -INFINITY, l = 0.f;
+  for (int j = 0; j < nk; ++j) {
+    if (!tc::mbar_wait(&s_full[t], (uint32_t)j & 1u, abort_flag, status)) {
+      if (!*abort_flag) fail(RC_DEV_TIMEOUT_ACCUM);
+      return;
+    }
+    tc::tc_fence_after();
+    uint32_t r[BN];
+#pragma unroll
+    for (int c = 0; c < BN; c += 32) tc::tmem_ld32(tS + (uint32_t)c, *reinterpret_cast<uint32_t(*)[32]>(&r[c]));
+    tc::tmem_ld_wait();
+    const int k0 = j * BN;
+    int nvis = min(BN, p.S - k0);
+    if (p.causal) nvis = min(nvis, max(0, qi - k0 + 1));
+    if (nvis < BN) {
+#pragma unroll
+      for (int i = 0; i < BN; ++i)
+        if (i >= nvis) r[i] = __float_as_uint(-INFINITY);
+    }
+    const float mxs = row_max<BN>(r) * p.scale_log2;
+    float factor = 1.f;
+    if (m_ref == -INFINITY) {
+      m_ref = mxs;  // first visible scores: O and l are still zero
+    } else if (mxs > m_ref + kRescaleLog2) {
+      factor = exp2f(m_ref - mxs);
+      m_ref = mxs;
+    }
+    const float mref = m_ref == -INFINITY ? 0.f : m_ref;
+    const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-mref, -mref);
+    float ls0 = 0.f, ls1 = 0.f, ls2 = 0.f, ls3 = 0.f;
+#pragma unroll
+    for (int hf = 0; hf < BN / 64; ++hf) {
+      uint32_t* pk = r + hf * 64;  // the 32 bf16 pairs of scores [hf * 64, + 64), packed in place
+      exp_pack_bf16_inplace<64>(pk, sc2, nm2);
+#pragma unroll
+      for (int i = 0; i < 32; i += 2) {
+        acc_bf16x2(ls0, ls1, pk[i]);
+        acc_bf16x2(ls2, ls3, pk[i + 1]);
+      }
+      // P_t(j) over S_t(j), whose scores are in registers
+      tc::tmem_st32(tS + (uint32_t)(hf * 32), *reinterpret_cast<uint32_t(*)[32]>(pk));
+    }
+    l = l * factor + ((ls0 + ls1) + (ls2 + ls3));
+    if (__any_sync(0xffffffffu, factor != 1.f)) {
+      // O_t holds P_t V up to block j - 1 (complete: its UMMAs precede S_t(j)); rescaled here,
+      // with the scores no longer live, before P_t V_j is released
+#pragma unroll 1
+      for (int c = 0; c < D; c += 32) {
+        uint32_t o[32];
+        tc::tmem_ld32(tO + (uint32_t)c, o);
+        tc::tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * factor);
+        tc::tmem_st32(tO + (uint32_t)c, o);
+      }
+    }
+    tc::tmem_st_wait();
+    tc::tc_fence_before();
+    tc::mbar_arrive(&p_full[t]);
+  }
+  if (nk == 0) return;
+  if (tc::mbar_wait(&o_full[t], 0, abort_flag, status)) {
+    tc::tc_fence_after();
+    const float inv_l = l > 0.f ? 1.f / l : 0.f;
+    const bool row_ok = qi < p.S;
+    __nv_bfloat16* orow = p.O + ((size_t)(b * p.S + (row_ok ? qi : 0)) * p.Hq + h) * D;
+    store_o_row(tO, inv_l, orow, row_ok);
+    if (p.lse && row_ok) p.lse[((size_t)b * p.Hq + h) * p.S + qi] = 0.6931471805599453f * (m_ref + log2f(l));
+  } else if (!*abort_flag) {
+    fail(RC_DEV_TIMEOUT_ACCUM);
+  }
+}
+
+template <bool VT>
+__global__ void __launch_bounds__(kThreads2q, 1)
+    attn2q_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                  const __grid_constant__ CUtensorMap tmV, const Params p, const int stages) {
+  constexpr int BN = kBN2q;
+  constexpr int VS = kVStages2q;
+  constexpr int QT = BM * D * 2;  // one query tile: two [128][64] swizzled halves
+  constexpr int KV = BN * D * 2;  // one K or V tile
+  constexpr int W_K = 8, W_V = 9, W_MMA = 10;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;
+  uint8_t* kring = sQ + 2 * QT;
+  uint8_t* vring = kring + (size_t)stages * KV;
+  uint64_t* q_full = (uint64_t*)(vring + (size_t)VS * KV);
+  uint64_t* k_full = q_full + 1;       // [stages]
+  uint64_t* v_full = k_full + stages;  // [VS]
+  uint64_t* it_done = v_full + VS;     // [kItRing2q]
+  uint64_t* s_full = it_done + kItRing2q;  // [2] per tile
+  uint64_t* p_full = s_full + 2;           // [2]
+  uint64_t* o_full = p_full + 2;           // [2]
+  uint64_t* drain = o_full + 2;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  volatile int* status = p.status;
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int BH = p.B * p.Hq;
+  int qb, bh;
+  if (p.raster == 0) {
+    qb = blockIdx.x % p.q_blocks;
+    bh = blockIdx.x / p.q_blocks;
+  } else {  // longest causal rows first
+    qb = p.q_blocks - 1 - (int)(blockIdx.x / BH);
+    bh = blockIdx.x % BH;
+  }
+  const int b = bh / p.Hq, h = bh - b * p.Hq, g = h / p.group;
+  const int q0 = qb * 2 * BM;
+  auto blocks_of = [&](int t) {
+    const int r0 = q0 + t * BM;
+    const int kv_end = p.causal ? min(r0 + BM, p.S) : p.S;
+    return r0 < p.S ? (kv_end + BN - 1) / BN : 0;
+  };
+  const int nkb0 = blocks_of(0), nkb1 = blocks_of(1);
+  const int NK = max(nkb0, nkb1);
+
+  auto fail = [&](int code) {
+    *abort_flag = 1;
+    tc::record_failure(status, code);
+  };
+
+  if (threadIdx.x == 0) {
+    tc::mbar_init(q_full, 1);
+    for (int s = 0; s < stages; ++s) tc::mbar_init(&k_full[s], 1);
+    for (int s = 0; s < VS; ++s) tc::mbar_init(&v_full[s], 1);
+    for (int i = 0; i < kItRing2q; ++i) tc::mbar_init(&it_done[i], 1);
+    for (int t = 0; t < 2; ++t) {
+      tc::mbar_init(&s_full[t], 1);
+      tc::mbar_init(&p_full[t], 128);
+      tc::mbar_init(&o_full[t], 1);
+    }
+    tc::mbar_init(drain, 1);
+    *abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  if (warp == W_K) tc::tmem_alloc(tmem_slot, 512);
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  // Block j goes into slot j % depth once iteration j - depth + lag has completed (that
+  // iteration issued the last UMMA reading the slot's previous block: K lag 0, V lag 1).
+  // A producer is never a full it_done ring behind: the UMMA issuer cannot finish
+  // iteration i + kItRing2q before this producer has loaded a block that iteration reads.
+  auto produce = [&](uint64_t* full, int depth, int lag, auto load) {
+    int j = 0;
+    for (; j < NK; ++j) {
+      if (j >= depth) {
+        const int it = j - depth + lag;
+        if (!tc::mbar_wait(&it_done[it % kItRing2q], (uint32_t)(it / kItRing2q) & 1u, abort_flag, status)) {
+          fail(RC_DEV_TIMEOUT_EMPTY);
+          break;
+        }
+      }
+      const int s = j % depth;
+      tc::mbar_expect_tx(&full[s], KV);
+      load(s, j, &full[s]);
+    }
+    for (int i = max(0, j - depth); i < j; ++i)
+      if (!tc::mbar_wait_drain(&full[i % depth], (uint32_t)(i / depth) & 1u)) fail(RC_DEV_TIMEOUT_DRAIN);
+  };
+
+  if (warp == W_K) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmQ);
+      tc::prefetch_tmap(&tmK);
+      tc::mbar_expect_tx(q_full, (uint32_t)(((nkb0 > 0) + (nkb1 > 0)) * QT));
+      for (int t = 0; t < 2; ++t) {
+        if ((t == 0 ? nkb0 : nkb1) == 0) continue;
+        const int qrow = b * p.S + q0 + t * BM;
+        tc::tma_load_2d(sQ + t * QT, &tmQ, q_full, h * D, qrow);
+        tc::tma_load_2d(sQ + t * QT + QT / 2, &tmQ, q_full, h * D + 64, qrow);
+      }
+      produce(k_full, stages, 0, [&](int s, int j, uint64_t* bar) {
+        uint8_t* sk = kring + (size_t)s * KV;
+        const int krow = b * p.S + j * BN;
+        tc::tma_load_2d(sk, &tmK, bar, g * D, krow);
+        tc::tma_load_2d(sk + BN * 128, &tmK, bar, g * D + 64, krow);
+      });
+      if (!tc::mbar_wait_drain(q_full, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+    }
+    __syncwarp();  // reconverge before the final block barrier
+  } else if (warp == W_V) {
+    if (lane == 0) {
+      tc::prefetch_tmap(&tmV);
+      produce(v_full, VS, 1, [&](int s, int j, uint64_t* bar) {
+        uint8_t* sv = vring + (size_t)s * KV;
+        if constexpr (VT) {
+#pragma unroll
+          for (int a = 0; a < BN / 64; ++a)
+            tc::tma_load_2d(sv + a * (BM * 128), &tmV, bar, j * BN + a * 64, (b * p.Hkv + g) * D);
+        } else {
+          const int krow = b * p.S + j * BN;
+          tc::tma_load_2d(sv, &tmV, bar, g * D, krow);
+          tc::tma_load_2d(sv + BN * 128, &tmV, bar, g * D + 64, krow);
+        }
+      });
+    }
+    __syncwarp();
+  } else if (warp == W_MMA) {
+    const bool leader = tc::elect_one();
+    constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
+    constexpr uint32_t idO = tc::idesc_bf16_f32(BM, D, !VT);
+    // Descriptors of Q_0, the first K slot and the first V slot. Q_1, a ring slot and each
+    // 16-wide K step add a constant to the 14-bit start-address field (addresses below
+    // 256 KB: no carry out of it).
+    const uint64_t q_desc = tc::sw128_desc(tc::smem_u32(sQ));
+    const uint64_t k_desc = tc::sw128_desc(tc::smem_u32(kring));
+    const uint64_t v_desc =
+        VT ? tc::sw128_desc(tc::smem_u32(vring)) : tc::sw128_desc_mn(tc::smem_u32(vring), BN * 128, 1024);
+    auto all = [](bool x) { return __all_sync(0xffffffffu, x); };
+    bool ok = all(tc::mbar_wait(q_full, 0, abort_flag, status));
+    // iteration j: P_t V_{j-1} then S_t(j) for t = 0, 1 (each where the tile has that block)
+    for (int j = 0; ok && j <= NK; ++j) {
+      const int jj = j - 1;
+      bool v_ready = false, k_ready = false;
+#pragma unroll
+      for (int t = 0; t < 2; ++t) {
+        const int nk = t == 0 ? nkb0 : nkb1;
+        if (ok && jj >= 0 && jj < nk) {
+          if (!v_ready) {
+            ok = all(tc::mbar_wait(&v_full[jj % VS], (uint32_t)(jj / VS) & 1u, abort_flag, status));
+            v_ready = true;
+          }
+          ok = ok && all(tc::mbar_wait(&p_full[t], (uint32_t)jj & 1u, abort_flag, status));
+          if (ok) {
+            tc::tc_fence_after();
+            if (leader) {
+              const uint64_t vd = v_desc + (uint64_t)((jj % VS) * (KV >> 4));
+              const uint32_t tP = tmem + (uint32_t)(t * 128), tO = tmem + 256u + (uint32_t)(t * 128);
+#pragma unroll
+              for (int ks = 0; ks < BN / 16; ++ks) {
+                const uint64_t db = VT ? vd + (uint64_t)((ks / 4) * ((BM * 128) >> 4) + (ks % 4) * 2)
+                                       : vd + (uint64_t)(ks * ((16 * 128) >> 4));
+                tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (jj > 0 || ks > 0) ? 1u : 0u);
+              }
+              if (jj == nk - 1) tc::umma_commit(&o_full[t]);
+            }
+            __syncwarp();
+          }
+        }
+        if (ok && j < nk) {
+          if (!k_ready) {
+            ok = all(tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status));
+            k_ready = true;
+            if (ok) tc::tc_fence_after();
+          }
+          if (ok) {
+            if (leader) {
+              const uint64_t kd = k_desc + (uint64_t)((j % stages) * (KV >> 4));
+              const uint64_t qd = q_desc + (uint64_t)(t * (QT >> 4));
+              const uint32_t tS = tmem + (uint32_t)(t * 128);
+#pragma unroll
+              for (int ks = 0; ks < D / 16; ++ks) {
+                const uint64_t off = (uint64_t)((ks / 4) * ((BM * 128) >> 4) + (ks % 4) * 2);
+                tc::umma_bf16(tS, qd + off, kd + off, idS, ks > 0 ? 1u : 0u);
+              }
+              tc::umma_commit(&s_full[t]);
+            }
+            __syncwarp();
+          }
+        }
+      }
+      if (ok) {
+        if (leader) tc::umma_commit(&it_done[j % kItRing2q]);
+        __syncwarp();
+      }
+    }
+    if (!ok) {
+      if (leader) {
+        fail(RC_DEV_TIMEOUT_FULL);
+        tc::umma_commit(drain);
+        if (!tc::mbar_wait_drain(drain, 0)) fail(RC_DEV_TIMEOUT_DRAIN);
+      }
+      __syncwarp();
+    }
+  } else {
+    const int t = warp / 4;
+    softmax_2q(p, t, warp & 3, lane, q0, t == 0 ? nkb0 : nkb1, b, h, tmem, s_full, p_full, o_full, abort_flag, status);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == W_K) {
+    __syncwarp();
+    tc::tc_fence_after();
+    tc::tmem_dealloc(tmem, 512);
+  }
+}
+
 // Vt[(b*Hkv + g)*D + d][s] = V[b][s][g][d] (64 x 64 tiles through shared memory).
 __global__ void transpose_v_kernel(const __nv_bfloat16* __restrict__ V, int S, int Hkv, __nv_bfloat16* __restrict__ Vt) {
   __shared__ __nv_bfloat16 tile[64][66];
@@ -1110,6 +1504,22 @@ rc_status launch_split(const rc_knobs& k, const rc_op_desc& d, const void* Q, co
   return launched(kern, threads, smem);
 }
 
+// The two-query-tile kernel (TileSize M = 256): 128-key blocks, one CTA per SM.
+template <bool VT>
+rc_status launch_2q(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
+                    float* lse, const LaunchCtx& c) {
+  auto kern = attn2q_kernel<VT>;
+  static bool attr = false;
+  RC_TRY(smem_attributes(kern, attr));
+  CUtensorMap tq, tk, tv;
+  Params p;
+  RC_TRY((prepare<kBN2q, VT>(k, d, Q, K, V, O, lse, c, &tq, &tk, &tv, &p)));
+  p.q_blocks = (int)((d.seq + 2 * BM - 1) / (2 * BM));
+  const size_t smem = attn2q_smem(k.stages);
+  kern<<<(unsigned)(p.B * p.Hq * p.q_blocks), kThreads2q, smem, (cudaStream_t)c.stream>>>(tq, tk, tv, p, k.stages);
+  return launched(kern, kThreads2q, smem);
+}
+
 template <int BN, bool VT>
 rc_status dispatch(const rc_knobs& k, const rc_op_desc& d, const void* Q, const void* K, const void* V, void* O,
                    float* lse, const LaunchCtx& c) {
@@ -1137,8 +1547,13 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
   if (d.head_dim != attn::D) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: head_dim must be 128");
   if (d.batch * d.seq > 0x7fffffffLL) return rc_fail(RC_ERR_UNSUPPORTED_OP, "attention: B*S too large");
   // the same rules as the schedule legality check, so a launch never gets a kernel it cannot run
-  if (k.tile_m != attn::BM || k.raster > 1 || (k.tile_n != 64 && k.tile_n != 128))
-    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: 128-row query tiles, 64- or 128-key blocks, loop order 0 or 1");
+  if ((k.tile_m != attn::BM && k.tile_m != 2 * attn::BM) || k.raster > 1 || (k.tile_n != 64 && k.tile_n != 128))
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: 128- or 256-row query tiles, 64- or 128-key blocks, loop order 0 or 1");
+  if (k.tile_m == 2 * attn::BM && (k.tile_n != attn::kBN2q || k.persistent != 1 || k.location != 1 || k.unroll != 1 ||
+                                   k.stages < 1 || k.stages > 3))
+    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE,
+                   "attention: two query tiles per CTA take 128-key blocks, P in tensor memory, one S buffer per tile, "
+                   "one softmax thread per row and 1 to 3 K stages");
   if (k.persistent == 0 && (k.location != 0 || k.unroll != 1))
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "attention: one issuing warp keeps P in shared memory, one S buffer");
   if (k.persistent > 0 && k.location == 0)
@@ -1156,6 +1571,8 @@ rc_status rc_launch_attention(const rc_knobs& k, const rc_op_desc& d, const void
     Vuse = workspace;
   }
   const bool vt = k.layout == 1;
+  if (k.tile_m == 2 * attn::BM)
+    return vt ? attn::launch_2q<true>(k, d, Q, K, Vuse, O, lse, c) : attn::launch_2q<false>(k, d, Q, K, Vuse, O, lse, c);
   if (k.tile_n == 64)
     return vt ? attn::dispatch<64, true>(k, d, Q, K, Vuse, O, lse, c) : attn::dispatch<64, false>(k, d, Q, K, Vuse, O, lse, c);
   return vt ? attn::dispatch<128, true>(k, d, Q, K, Vuse, O, lse, c) : attn::dispatch<128, false>(k, d, Q, K, Vuse, O, lse, c);
