@@ -911,26 +911,34 @@ __global__ void __launch_bounds__(attn4_threads<SPLIT>(), (Attn4Cols<BN, NSB, SU
     }
     __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
-    if (lane == 0 && nkb > 0) {
+    // S issuer. The whole warp runs the loop on warp-uniform values and one lane (elect.sync)
+    // issues: a lane-0 branch spends far longer per UMMA forming its operands.
+    if (nkb > 0) {
+      const bool leader = tc::elect_one();
+      auto all = [](bool x) { return __all_sync(0xffffffffu, x); };
       constexpr uint32_t idS = tc::idesc_bf16_f32(BM, BN);
-      const uint32_t sq = tc::smem_u32(sQ);
+      const uint64_t q_desc = tc::sw128_desc(tc::smem_u32(sQ));
+      const uint64_t k_desc = tc::sw128_desc(tc::smem_u32(kring));
       auto issue_s = [&](int j) {
         const int s = j % stages;
-        const uint32_t sk = tc::smem_u32(kring + (size_t)s * KV_TILE);
-        const uint32_t tS = tmem + (uint32_t)((j % NSB) * BN);
+        if (leader) {
+          const uint64_t kd = k_desc + (uint64_t)(s * (KV_TILE >> 4));
+          const uint32_t tS = tmem + (uint32_t)((j % NSB) * BN);
 #pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          tc::umma_bf16(tS, tc::sw128_desc(sq + (ks / 4) * (BM * 128) + off),
-                        tc::sw128_desc(sk + (ks / 4) * (BN * 128) + off), idS, ks > 0 ? 1u : 0u);
+          for (int ks = 0; ks < D / 16; ++ks) {
+            // 16-wide K steps: 32 B within a 64-wide swizzled half, halves [BM or BN][64] apart
+            tc::umma_bf16(tS, q_desc + (uint64_t)((ks / 4) * ((BM * 128) >> 4) + (ks % 4) * 2),
+                          kd + (uint64_t)((ks / 4) * ((BN * 128) >> 4) + (ks % 4) * 2), idS, ks > 0 ? 1u : 0u);
+          }
+          tc::umma_commit(&s_full[j % NSB]);
+          tc::umma_commit(&k_empty[s]);
         }
-        tc::umma_commit(&s_full[j % NSB]);
-        tc::umma_commit(&k_empty[s]);
+        __syncwarp();
       };
       auto await_k = [&](int j) -> bool {
-        return tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status);
+        return all(tc::mbar_wait(&k_full[j % stages], (uint32_t)(j / stages) & 1u, abort_flag, status));
       };
-      bool ok = tc::mbar_wait(q_full, 0, abort_flag, status);
+      bool ok = all(tc::mbar_wait(q_full, 0, abort_flag, status));
       for (int j = 0; ok && j < NSB && j < nkb; ++j) {
         if ((ok = await_k(j))) {
           tc::tc_fence_after();
@@ -941,15 +949,15 @@ __global__ void __launch_bounds__(attn4_threads<SPLIT>(), (Attn4Cols<BN, NSB, SU
         // one S buffer: free once the softmax holds S_j in registers; two: S buffer j % 2
         // holds P_j, free once P_j V_j has completed
         if constexpr (NSB == 1)
-          ok = tc::mbar_wait(&s_free[0], (uint32_t)j & 1u, abort_flag, status);
+          ok = all(tc::mbar_wait(&s_free[0], (uint32_t)j & 1u, abort_flag, status));
         else
-          ok = tc::mbar_wait(&pv_full[j % 2], (uint32_t)(j / 2) & 1u, abort_flag, status);
+          ok = all(tc::mbar_wait(&pv_full[j % 2], (uint32_t)(j / 2) & 1u, abort_flag, status));
         ok = ok && await_k(j + NSB);
         if (!ok) break;
         tc::tc_fence_after();
         issue_s(j + NSB);
       }
-      if (!ok) {
+      if (!ok && leader) {
         fail(RC_DEV_TIMEOUT_FULL);
         tc::umma_commit(&drain[0]);
         if (!tc::mbar_wait_drain(&drain[0], 0)) fail(RC_DEV_TIMEOUT_DRAIN);
@@ -957,33 +965,37 @@ __global__ void __launch_bounds__(attn4_threads<SPLIT>(), (Attn4Cols<BN, NSB, SU
     }
     __syncwarp();
   } else if (warp == 2) {
-    if (lane == 0 && nkb > 0) {
+    // P V issuer, warp-uniform like the S issuer
+    if (nkb > 0) {
+      const bool leader = tc::elect_one();
+      auto all = [](bool x) { return __all_sync(0xffffffffu, x); };
       constexpr uint32_t idO = tc::idesc_bf16_f32(BM, (int)Cols::OW, !VT);
       const uint32_t tO = tmem + O_COL;
+      const uint64_t v_desc = VT ? tc::sw128_desc(tc::smem_u32(vring))
+                                 : tc::sw128_desc_mn(tc::smem_u32(vring), BN * 128, 1024);
       bool ok = true;
       for (int j = 0; ok && j < nkb; ++j) {
         const int s = j % vstages;
         const int pb = NSB == 2 ? j % 2 : 0;  // P over S buffer j % 2, or the P columns
         const uint32_t tP = tmem + (NSB == 2 ? (uint32_t)(pb * BN) : P_COL);
-        ok = tc::mbar_wait(&v_full[s], (uint32_t)(j / vstages) & 1u, abort_flag, status) &&
-             tc::mbar_wait(&p_full[pb], (uint32_t)(j / (NSB == 2 ? 2 : 1)) & 1u, abort_flag, status);
+        ok = all(tc::mbar_wait(&v_full[s], (uint32_t)(j / vstages) & 1u, abort_flag, status) &&
+                 tc::mbar_wait(&p_full[pb], (uint32_t)(j / (NSB == 2 ? 2 : 1)) & 1u, abort_flag, status));
         if (!ok) break;
         tc::tc_fence_after();
-        const uint32_t sv = tc::smem_u32(vring + (size_t)s * VSLOT);
+        if (leader) {
+          const uint64_t vd = v_desc + (uint64_t)(s * (VSLOT >> 4));
 #pragma unroll
-        for (int ks = 0; ks < BN / 16; ++ks) {
-          const uint32_t off = (uint32_t)(ks % 4) * 32;
-          uint64_t db;
-          if constexpr (VT)
-            db = tc::sw128_desc(sv + (ks / 4) * (BM * 128) + off);
-          else
-            db = tc::sw128_desc_mn(sv + (uint32_t)ks * 16 * 128, BN * 128, 1024);
-          tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+          for (int ks = 0; ks < BN / 16; ++ks) {
+            const uint64_t db = VT ? vd + (uint64_t)((ks / 4) * ((BM * 128) >> 4) + (ks % 4) * 2)
+                                   : vd + (uint64_t)(ks * ((16 * 128) >> 4));
+            tc::umma_bf16_ts(tO, tP + (uint32_t)ks * 8, db, idO, (j > 0 || ks > 0) ? 1u : 0u);
+          }
+          tc::umma_commit(&pv_full[pb]);
+          tc::umma_commit(&v_empty[s]);
         }
-        tc::umma_commit(&pv_full[pb]);
-        tc::umma_commit(&v_empty[s]);
+        __syncwarp();
       }
-      if (!ok) {
+      if (!ok && leader) {
         fail(RC_DEV_TIMEOUT_FULL);
         tc::umma_commit(&drain[1]);
         if (!tc::mbar_wait_drain(&drain[1], 0)) fail(RC_DEV_TIMEOUT_DRAIN);

@@ -7,7 +7,8 @@
 //                shared-memory buffers, one or two such 64-wide K sub-blocks
 //                per stage (TileSize K = 64 or 128), signalling a "full"
 //                mbarrier per stage.
-//   warp 1     : allocates TMEM, and one elected thread issues 4 UMMAs
+//   warp 1     : allocates TMEM; the whole warp runs the issue loop on
+//                warp-uniform values and one lane (elect.sync) issues 4 UMMAs
 //                (K = 16 each) per sub-block, releasing the stage through
 //                tcgen05.commit onto its "empty" mbarrier; a final commit
 //                signals the accumulator.
@@ -568,8 +569,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();  // reconverge before the final block barrier
   } else if (warp == 1) {
-    if (lane == 0 && (rank == 0 || !PAIR)) {
+    // the whole warp runs the issue loop on warp-uniform values and one elected lane issues (a lane-0
+    // branch spends far longer per UMMA forming its operands); in a pair only the leader CTA issues
+    if (rank == 0 || !PAIR) {
+      const bool leader = tc::elect_one();
+      auto all = [](bool x) { return __all_sync(0xffffffffu, x); };
       constexpr uint32_t idesc = tc::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN);
+      const uint32_t sbase = tc::smem_u32(smem);
       uint32_t li = 0;
       int s = 0;        // ring slot, advanced in step with the producer
       uint32_t ph = 0;  // its phase parity
@@ -579,8 +585,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!it.valid) continue;
         const uint32_t buf = li % (uint32_t)n_acc;
         const uint32_t aph = (li / (uint32_t)n_acc) & 1u;
-        if (!tc::mbar_wait(&acc_empty[buf], aph ^ 1u, abort_flag, status)) {
-          fail(RC_DEV_TIMEOUT_ACCUM);
+        if (!all(tc::mbar_wait(&acc_empty[buf], aph ^ 1u, abort_flag, status))) {
+          if (leader) fail(RC_DEV_TIMEOUT_ACCUM);
           ok = false;
           break;
         }
@@ -588,48 +594,54 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t dacc = tmem + buf * ACC_COLS;
         for (int i = 0; i < it.nkb; i += ksub) {
           const int nsub = min(ksub, it.nkb - i);
-          if (!tc::mbar_wait(&full[s], ph, abort_flag, status)) {
-            fail(RC_DEV_TIMEOUT_FULL);
+          if (!all(tc::mbar_wait(&full[s], ph, abort_flag, status))) {
+            if (leader) fail(RC_DEV_TIMEOUT_FULL);
             ok = false;
             break;
           }
           // gathered A: cp.async wrote the rows through the generic proxy; order them before the UMMA reads
           if constexpr (AMODE == TC_A_GATHER) tc::fence_proxy_async_smem();
           tc::tc_fence_after();
-          const uint32_t sa = tc::smem_u32(smem + (size_t)s * STAGE_BYTES);
+          if (leader) {
+            const uint32_t sa = sbase + (uint32_t)s * (uint32_t)STAGE_BYTES;
 #pragma unroll
-          for (int q = 0; q < 2; ++q) {
-            if (q >= nsub) break;
-            const uint64_t da = tc::sw128_desc(sa + q * A_BYTES);
-            const uint64_t db = tc::sw128_desc(sa + ksub * A_BYTES + q * B_BYTES);
+            for (int q = 0; q < 2; ++q) {
+              if (q >= nsub) break;
+              const uint64_t da = tc::sw128_desc(sa + q * A_BYTES);
+              const uint64_t db = tc::sw128_desc(sa + ksub * A_BYTES + q * B_BYTES);
 #pragma unroll
-            for (int k = 0; k < BK / 16; ++k) {
-              const uint32_t acc = (i > 0 || q > 0 || k > 0) ? 1u : 0u;
-              if constexpr (PAIR)
-                tc::umma_bf16_pair(dacc, da + 2 * k, db + 2 * k, idesc, acc);
-              else
-                tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, acc);
+              for (int k = 0; k < BK / 16; ++k) {
+                const uint32_t acc = (i > 0 || q > 0 || k > 0) ? 1u : 0u;
+                if constexpr (PAIR)
+                  tc::umma_bf16_pair(dacc, da + 2 * k, db + 2 * k, idesc, acc);
+                else
+                  tc::umma_bf16(dacc, da + 2 * k, db + 2 * k, idesc, acc);
+              }
             }
+            if constexpr (PAIR)
+              tc::umma_commit_pair(&empty[s], 3);  // the slot is free in both CTAs
+            else if constexpr (MC > 1)
+              tc::umma_commit_mc(&empty[s], MC_MASK);  // this CTA has read the slot: every producer may refill it
+            else
+              tc::umma_commit(&empty[s]);
           }
-          if constexpr (PAIR)
-            tc::umma_commit_pair(&empty[s], 3);  // the slot is free in both CTAs
-          else if constexpr (MC > 1)
-            tc::umma_commit_mc(&empty[s], MC_MASK);  // this CTA has read the slot: every producer may refill it
-          else
-            tc::umma_commit(&empty[s]);
+          __syncwarp();
           if (++s == stages) {
             s = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        if constexpr (PAIR)
-          tc::umma_commit_pair(&acc_full[buf], 3);
-        else
-          tc::umma_commit(&acc_full[buf]);  // accumulator ready (also when nkb == 0)
+        if (leader) {
+          if constexpr (PAIR)
+            tc::umma_commit_pair(&acc_full[buf], 3);
+          else
+            tc::umma_commit(&acc_full[buf]);  // accumulator ready (also when nkb == 0)
+        }
+        __syncwarp();
         ++li;
       }
-      if (!ok) {
+      if (!ok && leader) {
         if constexpr (PAIR)
           tc::umma_commit_pair(drain, 1);
         else
