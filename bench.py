@@ -923,6 +923,9 @@ def library_study(wl, sched_text="", reps=20):
         ts = []
         for _ in range(reps):
             flush.fill_(1.0)
+            # hold the stream about 100 us after the flush, so that the library's host-side dispatch
+            # (Python, plan lookup) is done before its kernels' turn: device time only, as for ours
+            torch.cuda._sleep(200000)
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
             fn()
