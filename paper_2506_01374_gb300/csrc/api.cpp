@@ -11,21 +11,21 @@
 
 #include "rc_internal.h"
 
-namespace {
-thread_local std::string g_err;
-
-constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
-
 // Tensor-core GEMM shared-memory footprint per CTA: a ring of `stages`
 // stages of tile_k / 64 sub-blocks, each an A (128 x 64) and a B (bn x 64,
 // or bn/2 x 64 in each CTA of a pair) bf16 tile, plus 1 KB alignment slack,
 // barriers, four fp32 copies of a bias tile, a 128-entry row table and the
-// grouped segment tables (2 x 257 entries + 8 B).
+// grouped segment tables (3 x 257 entries + 8 B).
 int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k, int tile_m) {
   const int64_t b_rows = tile_m == 256 ? bn_mma / 2 : bn_mma;
   return (int64_t)stages * (tile_k / 64) * (128 * 64 * 2 + b_rows * 64 * 2) + 1024 + 256 + 4 * (int64_t)bn_mma * 4 +
-         128 * 4 + 2 * 257 * 4 + 8;
+         128 * 4 + 3 * 257 * 4 + 8;
 }
+
+namespace {
+thread_local std::string g_err;
+
+constexpr int64_t kSmemLimit = 232448;  // 227 KB opt-in shared memory per CTA
 
 bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, std::string* why) {
   if (bn_mma % 16 != 0 || bn_mma < 16 || bn_mma > 256) {
@@ -45,11 +45,8 @@ bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, 
     if (why) *why = "a CTA pair splits the N tile: at least 32 columns";
     return false;
   }
-  if (tile_m == 256 && persistent && bn_mma > 128) {
-    // a pair holds at most 256 TMEM columns (two accumulators of <= 128)
-    if (why) *why = "persistent CTA pairs need N tiles of at most 128";
-    return false;
-  }
+  // (persistent CTA pairs with N tiles above 128 take all 512 TMEM columns of their SMs; the
+  // launcher then asks for enough shared memory that no other CTA shares those SMs)
   if (tile_k != 64 && tile_k != 128) {
     if (why) *why = "K per stage must be 64 or 128";
     return false;
@@ -209,10 +206,14 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         // where the token rows are gathered: 0 = a separate pass writes the grouped copy (stage 0),
         // 1 = the grouped GEMM's producer gathers them from X (M tile 128)
         v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});
+        // how a CTA-pair launch tiles a ragged expert segment: 0 = whole pair tiles, 1 = pair tiles and a
+        // last 128-row single-CTA tile where the remainder fits it (a second, one-CTA launch)
+        v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});
       } else {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
         v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
+        v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // as in stage 1
         vectorize();  // the combine (or the fp32 -> bf16 pass of the atomic combine)
       }
       break;
@@ -751,6 +752,10 @@ extern "C" rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base,
   // split-issue kernels keep P in tensor memory, and the two-query-tile kernel has one form for each
   // key block, so each family's canonical form fixes the knobs it does not offer (a single Parallel
   // or TileSize transformation then moves between the families)
+  // MoE grouped GEMMs: splitting ragged segments (layout 1) applies to CTA-pair launches only
+  if (op->d.kind == RC_OP_MOE)
+    for (int i = 1; i < s.n_stages; ++i)
+      if (s.k[i].tile_m != 256) s.k[i].layout = 0;
   for (int i = 0; i < s.n_stages; ++i) {
     if (!(op->d.kind == RC_OP_ATTENTION || (op->d.kind == RC_OP_DECODER_LAYER && i == 2))) continue;
     rc_knobs& k = s.k[i];

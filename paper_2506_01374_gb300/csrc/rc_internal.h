@@ -118,6 +118,12 @@ enum TcEpilogue {
   TC_EPI_BIAS_SILU = 3,    // D + bias[n] -> silu -> bf16
   TC_EPI_SCALE_ATOMIC = 4  // row_scale[row] * D atomically added to fp32 out[row_map[row]]
 };
+// Which rows of each grouped segment a launch covers (see seg_rows in tc_gemm.cuh).
+enum TcSegMode {
+  TC_SEG_ALL = 0,    // every row, in tiles of the launch's M tile
+  TC_SEG_PAIRS = 1,  // a CTA-pair launch: the segment minus a last remainder of 1 .. 128 rows
+  TC_SEG_REST = 2    // a one-CTA launch: that remainder alone (one 128-row tile per segment at most)
+};
 enum TcAMode {
   TC_A_2D = 0,         // A is a row-major [M][K] matrix
   TC_A_CONV = 1,       // A rows are output pixels of an NHWC 'same' conv; K = (r, s, c); one 4-D box
@@ -145,6 +151,7 @@ struct TcGemmArgs {
   const int* offsets;
   int64_t b_group_rows;
   int64_t max_tiles_m;     // upper bound on m-tiles over all groups
+  int seg_mode;            // TcSegMode
   const float* row_scale;  // TC_EPI_SCALE_ATOMIC
   const int* row_map;      // TC_EPI_SCALE_ATOMIC: A row -> slot; output row = slot / row_div
   int row_div;             // (TC_A_GATHER: A row i is source row row_map[i] / row_div)
@@ -152,6 +159,8 @@ struct TcGemmArgs {
   const void* resid;       // TC_EPI_STORE_BF16: bf16 [M][ldd] added to D before the one rounding (NULL = none)
 };
 rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
+// Shared memory of one CTA of the tensor-core GEMM (the schedule legality check's figure).
+int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k, int tile_m);
 // Split-K reduction: out_bf16[M][N] = sum_z part[z][M][N].
 rc_status rc_launch_splitk_reduce(const float* part, int splits, int64_t M, int64_t N, void* out,
                                   int vec, const LaunchCtx& c);

@@ -108,6 +108,27 @@ TcGemmArgs gemm_args(int64_t M, int64_t N, int64_t K, const void* A, const void*
   return a;
 }
 
+// A grouped (MoE) GEMM. Layout 1 with CTA pairs splits every expert segment
+// whose last pair tile would hold at most 128 rows: one launch of CTA pairs
+// over the rest of the segments, then one launch of single CTAs over those
+// remainders (one 128-row tile each), so a ragged segment pads at most 127
+// rows instead of 255. The remainder launch keeps the knobs but the M tile,
+// with as many of the ring stages as fit one CTA's shared memory.
+rc_status launch_grouped(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
+  if (k.layout != 1 || k.tile_m != 256) return rc_launch_tc_gemm(k, a, c);
+  TcGemmArgs head = a;
+  head.seg_mode = TC_SEG_PAIRS;
+  RC_TRY(rc_launch_tc_gemm(k, head, c));
+  rc_knobs kr = k;
+  kr.tile_m = 128;
+  kr.layout = 0;
+  const int bn_mma = a.epilogue == TC_EPI_SWIGLU ? 2 * k.tile_n : k.tile_n;
+  while (kr.stages > 1 && tc_smem_bytes(bn_mma, kr.stages, kr.tile_k, 128) > 232448) --kr.stages;
+  TcGemmArgs rest = a;
+  rest.seg_mode = TC_SEG_REST;
+  return rc_launch_tc_gemm(kr, rest, c);
+}
+
 // Y[M,N] = X W^T with optional split-K through an fp32 partial buffer.
 rc_status run_linear(const rc_knobs& k, int64_t M, int64_t N, int64_t K, const void* X, const void* W, void* Y,
                      void* part, const LaunchCtx& c) {
@@ -272,7 +293,7 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
         g1.row_div = (int)d.top_k;
         g1.a_rows = d.tokens;
       }
-      RC_TRY(rc_launch_tc_gemm(s->k[1], g1, c));
+      RC_TRY(launch_grouped(s->k[1], g1, c));
       RC_TRY(rc_mark_stage(c));
       TcGemmArgs g2 = gemm_args(slots, d.hidden, d.inter, Hb, p[3], Yb, d.hidden, TC_EPI_STORE_BF16);
       g2.groups = (int)d.experts;
@@ -288,11 +309,11 @@ rc_status run_impl(const rc_op_s* op, const rc_schedule_s* s, const rc_tensors* 
         g2.row_map = perm;
         g2.row_div = (int)d.top_k;
         g2.ldd = d.hidden;
-        RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
+        RC_TRY(launch_grouped(s->k[2], g2, c));
         RC_TRY(rc_launch_f32_to_bf16(acc, d.tokens * d.hidden, p[4], s->k[2].vec, c));
         return rc_mark_stage(c);
       }
-      RC_TRY(rc_launch_tc_gemm(s->k[2], g2, c));
+      RC_TRY(launch_grouped(s->k[2], g2, c));
       RC_TRY(rc_launch_moe_combine(Yb, w, inv, d.tokens, d.hidden, (int)d.top_k, p[4], s->k[2].vec, c));
       return rc_mark_stage(c);
     }

@@ -66,6 +66,7 @@ struct Params {
   const int* offsets;
   int groups;
   int b_group_rows;
+  int seg_mode;  // which rows of each segment: TcSegMode (all, the pair part, the short remainder)
   const float* row_scale;
   const int* row_map;
   int row_div;
@@ -216,24 +217,40 @@ struct Item {
   int row0, row_end, brow0, nt, split, kb0, nkb;
 };
 
-// Grouped mode keeps, per CTA, the segment offsets and the exclusive prefix of
-// the segments' tile counts in shared memory (at most kSmemGroups segments,
-// checked on the host), built once by one warp at CTA start, so that
-// resolving an m tile is a binary search in shared memory instead of a scan
-// over every segment in global memory (2.6 us per CTA for 64 segments).
+// Grouped mode keeps, per CTA, the segment row ranges and the exclusive
+// prefix of the segments' tile counts in shared memory (at most kSmemGroups
+// segments, checked on the host), built once by one warp at CTA start, so
+// that resolving an m tile is a binary search in shared memory instead of a
+// scan over every segment in global memory (2.6 us per CTA for 64 segments).
 constexpr int kSmemGroups = 256;
-constexpr int kGroupTableBytes = 2 * (kSmemGroups + 1) * 4 + 8;
+constexpr int kGroupTableBytes = 3 * (kSmemGroups + 1) * 4 + 8;
+
+// Rows [lo, hi) of a segment of rows [s_lo, s_hi) that a grouped launch covers.
+// TC_SEG_ALL: all of them. With kSegSplit-row CTA-pair tiles a segment whose
+// last tile would hold 1 .. kSegSplit / 2 rows is split: TC_SEG_PAIRS takes
+// everything before that remainder (whole pair tiles, or a last pair tile
+// more than half full), TC_SEG_REST takes the remainder alone (one 128-row
+// tile), so the padding of a ragged segment is at most 127 rows, not 255.
+constexpr int kSegSplit = 256;
+__device__ __forceinline__ void seg_rows(int mode, int s_lo, int s_hi, int& lo, int& hi) {
+  const int rem = (s_hi - s_lo) % kSegSplit;
+  const int rest = rem > 0 && rem <= kSegSplit / 2 ? rem : 0;
+  lo = mode == TC_SEG_REST ? s_hi - rest : s_lo;
+  hi = mode == TC_SEG_PAIRS ? s_hi - rest : s_hi;
+}
 
 // TR: rows of a tile (128, or 256 for a CTA pair). One warp, all lanes.
 template <int TR>
-__device__ __forceinline__ void build_group_table(const Params& p, int lane, int* s_goff, int* s_gtile) {
+__device__ __forceinline__ void build_group_table(const Params& p, int lane, int* s_goff, int* s_gend, int* s_gtile) {
   const int G = p.groups;
   const int per = (G + 31) / 32;  // segments per lane, lane-major
   const int g0 = min(G, lane * per), g1 = min(G, g0 + per);
   int sum = 0;
   for (int g = g0; g < g1; ++g) {
-    const int lo = p.offsets[g], hi = p.offsets[g + 1];
+    int lo, hi;
+    seg_rows(p.seg_mode, p.offsets[g], p.offsets[g + 1], lo, hi);
     s_goff[g] = lo;
+    s_gend[g] = hi;
     sum += (hi - lo + TR - 1) / TR;
   }
   int incl = sum;  // inclusive scan of the lanes' tile counts
@@ -245,16 +262,14 @@ __device__ __forceinline__ void build_group_table(const Params& p, int lane, int
   int acc = incl - sum;
   for (int g = g0; g < g1; ++g) {
     s_gtile[g] = acc;
-    acc += (p.offsets[g + 1] - p.offsets[g] + TR - 1) / TR;
+    acc += (s_gend[g] - s_goff[g] + TR - 1) / TR;
   }
-  if (lane == 31) {
-    s_gtile[G] = incl;
-    s_goff[G] = p.offsets[G];
-  }
+  if (lane == 31) s_gtile[G] = incl;
 }
 
 template <bool GROUPED, int TR>
-__device__ __forceinline__ Item resolve_item(const Params& p, long long w, const int* s_goff, const int* s_gtile) {
+__device__ __forceinline__ Item resolve_item(const Params& p, long long w, const int* s_goff, const int* s_gend,
+                                             const int* s_gtile) {
   Item it;
   const long long tiles = (long long)p.tiles_m * p.tiles_n;
   it.split = (int)(w / tiles);
@@ -277,7 +292,7 @@ __device__ __forceinline__ Item resolve_item(const Params& p, long long w, const
       }
       g = lo;
       it.row0 = s_goff[g] + (mt - s_gtile[g]) * TR;
-      it.row_end = s_goff[g + 1];
+      it.row_end = s_gend[g];
       it.valid = true;
     }
     it.brow0 = g * p.b_group_rows;
@@ -339,9 +354,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* sbias_all = (float*)(((uintptr_t)(abort_flag + 1) + 15) & ~(uintptr_t)15);
   // gathered A: source row of each of the tile's 128 rows (-1 = past the segment)
   int* s_src = (int*)(sbias_all + 4 * BN);
-  // grouped: segment offsets and tile prefix (kSmemGroups + 1 entries each)
+  // grouped: segment row ranges and tile prefix (kSmemGroups + 1 entries each)
   int* s_goff = s_src + BM;
-  int* s_gtile = s_goff + kSmemGroups + 1;
+  int* s_gend = s_goff + kSmemGroups + 1;
+  int* s_gtile = s_gend + kSmemGroups + 1;
 
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -353,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const long long w_first = blockIdx.x / PER_ITEM;
   const long long w_step = gridDim.x / PER_ITEM;
   auto item = [&](long long w) -> Item {
-    Item it = resolve_item<GROUPED, PER_ITEM * BM>(p, w, s_goff, s_gtile);
+    Item it = resolve_item<GROUPED, PER_ITEM * BM>(p, w, s_goff, s_gend, s_gtile);
     it.row0 += (int)rank * BM;  // this CTA's 128 rows of the PER_ITEM x 128-row tile
     return it;
   };
@@ -384,7 +400,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::tmem_alloc(tmem_slot, tmem_cols);
   }
   if constexpr (GROUPED) {
-    if (warp == 2) build_group_table<PAIR ? 2 * BM : BM>(p, lane, s_goff, s_gtile);
+    if (warp == 2) build_group_table<PAIR ? 2 * BM : BM>(p, lane, s_goff, s_gend, s_gtile);
   }
   tc::tc_fence_before();
   if constexpr (CLUSTER)
@@ -745,6 +761,9 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
 // per sub-block + 1 KB alignment slack + barriers and flags (256 B) + four
 // fp32 bias copies of the bn-column tile + the gathered-A row table (512 B)
 // + the grouped segment tables
+// Dynamic shared memory above which two CTAs cannot share an SM (228 KB per SM, 1 KB reserved per CTA).
+constexpr size_t kSmemHalfPlus = 233472 / 2 - 1024 + 16;
+
 inline size_t smem_bytes(int bn, int stages, int ksub, bool pair = false) {
   const size_t b_rows = pair ? (size_t)bn / 2 : (size_t)bn;
   return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4 + BM * 4 +
@@ -756,10 +775,13 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   auto kern = gemm_kernel<BN, EPI, AMODE, GROUPED, PAIR, MC>;
   if (k.tile_k != 64 && k.tile_k != 128) return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: K tile %d", k.tile_k);
   constexpr int acc_cols_tile = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
-  if (PAIR && (k.persistent ? 2 : 1) * acc_cols_tile > 256)
-    return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: a CTA pair holds at most 256 TMEM columns");
+  const int tmem_cols = (k.persistent ? 2 : 1) * acc_cols_tile;
   const int ksub = k.tile_k / 64;
-  const size_t smem = smem_bytes(BN, k.stages, ksub, PAIR);
+  size_t smem = smem_bytes(BN, k.stages, ksub, PAIR);
+  // A CTA pair taking all 512 TMEM columns of each of its SMs must not share an SM with a CTA of
+  // another pair: their allocations could then wait on each other across SMs. Asking for more than
+  // half of an SM's shared memory keeps one such CTA per SM, so its allocation never waits.
+  if (PAIR && tmem_cols > 256 && smem < kSmemHalfPlus) smem = kSmemHalfPlus;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
@@ -795,7 +817,8 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   p.tiles_n = (out_w + tile_out - 1) / tile_out;
   const int64_t tile_rows = (PAIR ? 2 : MC) * BM;
   // grouped: an upper bound of the tiles the segments need (spare tiles are skipped)
-  p.tiles_m = GROUPED ? (int)(PAIR ? a.M / tile_rows + a.groups : a.max_tiles_m)
+  // (the remainder launch needs at most one tile per segment)
+  p.tiles_m = GROUPED ? (int)(a.seg_mode == TC_SEG_REST ? a.groups : PAIR ? a.M / tile_rows + a.groups : a.max_tiles_m)
                       : (int)((a.M + tile_rows - 1) / tile_rows);
   p.kb_total = (int)((a.K + BK - 1) / BK);
   const int splits = EPI == TC_EPI_PARTIAL_F32 ? k.split_k : 1;
@@ -824,6 +847,7 @@ rc_status launch(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c) {
   }
   p.offsets = a.offsets;
   p.groups = a.groups;
+  p.seg_mode = a.seg_mode;
   p.b_group_rows = (int)a.b_group_rows;
   p.row_scale = a.row_scale;
   p.row_map = a.row_map;

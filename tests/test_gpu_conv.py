@@ -61,7 +61,7 @@ def test_conv_split_k_and_unfused_epilogue():
         try:
             s = sched(op, tn, 3 if tk == 64 else 2, sk, fuse, pe, tile_k=tk, tile_m=tm)
         except rc.RcError:
-            continue  # persistent CTA pairs hold N tiles of at most 128
+            continue  # illegal here (shared memory of the ring)
         dy = empty_bf16(N, H, W, Cout).fill_(0x7FC0)
         op.run(s, [dx, dw, db, dy])
         op.check()

@@ -84,9 +84,11 @@ def moe_op(T, H, E, I, K):
     return rc.Op(rc.OP_MOE, tokens=T, hidden=H, experts=E, inter=I, top_k=K)
 
 
-def moe_sched(op, tm, tn1, st1, tn2, st2, fuse, persistent=0, tile_k=64, tile_m=128, gather=0):
-    # gather = 1: the grouped gate/up GEMM's producer gathers the token rows itself (compute location 1)
+def moe_sched(op, tm, tn1, st1, tn2, st2, fuse, persistent=0, tile_k=64, tile_m=128, gather=0, split=0):
+    # gather = 1: the grouped gate/up GEMM's producer gathers the token rows itself (compute location 1);
+    # split = 1 (layout 1, CTA pairs): a segment's last remainder of at most 128 rows goes to a one-CTA launch
     return op.schedule(rc.T(rc.T_COMPUTE_LOCATION, gather, stage=1),
+                       rc.T(rc.T_LAYOUT, split, stage=1), rc.T(rc.T_LAYOUT, split, stage=2),
                        rc.T(rc.T_TILE_SIZE, tm, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
                        rc.T(rc.T_PIPELINE_STAGES, st1, stage=1), rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2),
                        rc.T(rc.T_PIPELINE_STAGES, st2, stage=2), rc.T(rc.T_FUSE, fuse, stage=2),
@@ -107,7 +109,7 @@ def test_moe_layer_schedule_sweep():
         try:  # CTA pairs (tm = 256) take 256 rows of one expert's segment
             s = moe_sched(op, 8, tn1, st, tn2, st, fuse, pe, tk, tm, ga)
         except rc.RcError:
-            continue  # shared memory (K = 128, 3 stages, widest N); TMEM of persistent pairs; gather on pairs
+            continue  # shared memory (K = 128, 3 stages, widest N); gather on pairs
         out = empty_bf16(T, H).fill_(0x7FC0)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         gp = torch.empty(T * K, dtype=torch.int32, device="cuda")
@@ -117,6 +119,46 @@ def test_moe_layer_schedule_sweep():
         np.testing.assert_array_equal(gp.cpu().numpy(), perm)
         err = rel_err(from_dev_bf16(out), ref)
         assert err <= TOL, (tn1, tn2, fuse, st, pe, tk, tm, ga, err)
+
+
+@pytest.mark.parametrize("T,E,K,kinds", [(200, 8, 2, {"rest"}), (700, 16, 4, {"pairs"}),
+                                         (1000, 5, 3, {"pairs", "rest"}), (2000, 12, 3, {"pairs", "rest"})])
+def test_moe_split_segments(T, E, K, kinds):
+    # CTA pairs with each segment's short remainder (1 .. 128 rows past its last whole or more than
+    # half-full 256-row tile) in a second, one-CTA launch: both grouped GEMMs, fused and unfused combine,
+    # persistent or not, ring depths that the one-CTA launch has to trim
+    H, I = 128, 64
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=45 + T)
+    ids, w, off, perm = oracle.moe_route(logits, K)
+    rows = np.diff(off)
+    ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
+    op = moe_op(T, H, E, I, K)
+    dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
+    n = 0
+    for tn1, tn2, fuse, st, pe, tk in itertools.product((64, 128), (128, 256), (0, 1), (3, 6), (0, 1), (64, 128)):
+        try:
+            s = moe_sched(op, 8, tn1, st, tn2, st, fuse, pe, tk, 256, 0, 1)
+        except rc.RcError:
+            continue  # shared memory of the pair ring
+        assert s.knobs(1)["layout"] == 1 and s.knobs(2)["layout"] == 1
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(s, [dl, dX, d1, d2, out])
+        op.check()
+        err = rel_err(from_dev_bf16(out), ref)
+        assert err <= TOL, (tn1, tn2, fuse, st, pe, tk, err)
+        n += 1
+    assert n >= 16
+    # which launches this case exercises: a remainder of 1 .. 128 rows goes to the one-CTA launch, whole
+    # pair tiles or a remainder of 129 .. 255 rows to the pair launch
+    rem = rows % 256
+    seen = set()
+    if ((rem > 0) & (rem <= 128)).any():
+        seen.add("rest")
+    if ((rows >= 256) | (rem > 128)).any():
+        seen.add("pairs")
+    assert seen == kinds, (seen, rows.tolist())
+    # single-CTA M tiles have nothing to split: the canonical form drops the layout
+    assert moe_sched(op, 8, 64, 3, 128, 3, 0, tile_m=128, split=1).knobs(1)["layout"] == 0
 
 
 def test_moe_layer_imbalanced_and_empty_experts():
@@ -129,14 +171,14 @@ def test_moe_layer_imbalanced_and_empty_experts():
     assert (np.diff(off)[4:] == 0).all() and (np.diff(off)[:4] == T).all()
     ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
     op = moe_op(T, H, E, I, K)
-    for fuse, pe, tm, ga in itertools.product((0, 1), (0, 1), (128, 256), (0, 1)):
-        if ga and tm == 256:
+    for fuse, pe, tm, ga, sp in itertools.product((0, 1), (0, 1), (128, 256), (0, 1), (0, 1)):
+        if ga and tm == 256 or sp and tm == 128:
             continue
         out = empty_bf16(T, H).fill_(0x7FC0)
-        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse, pe, tile_m=tm, gather=ga),
+        op.run(moe_sched(op, 4, 64, 2, 128, 2, fuse, pe, tile_m=tm, gather=ga, split=sp),
                [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
-        assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm, ga)
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm, ga, sp)
 
 
 def test_moe_full_size_sampled_tokens():
@@ -151,7 +193,10 @@ def test_moe_full_size_sampled_tokens():
     del W1, W2
     for s in [op.schedule(), moe_sched(op, 8, 128, 2, 256, 2, 0), moe_sched(op, 16, 64, 4, 128, 3, 1),
               moe_sched(op, 8, 128, 4, 256, 3, 0, 1), moe_sched(op, 8, 64, 3, 224, 2, 0, gather=1),
-              moe_sched(op, 8, 128, 2, 224, 2, 1, 1, tile_k=128, gather=1)]:
+              moe_sched(op, 8, 128, 2, 224, 2, 1, 1, tile_k=128, gather=1),
+              # CTA pairs with short remainders split off to one-CTA launches
+              moe_sched(op, 8, 128, 3, 256, 4, 0, 1, tile_m=256, split=1),
+              moe_sched(op, 8, 128, 3, 256, 3, 1, 0, tile_m=256, split=1)]:
         out = empty_bf16(T, H)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         go = torch.empty(E + 1, dtype=torch.int32, device="cuda")
