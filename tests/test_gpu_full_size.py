@@ -58,6 +58,12 @@ def test_mlp_block_full_size_reported_schedules():
              s1=dict(tile_m=256, tile_n=224, stages=3, raster=(0, 1))),
         dict(s0=dict(tile_m=128, tile_n=128, stages=2, fuse=1),
              s1=dict(tile_m=256, tile_n=224, stages=3)),
+        # gate/up on persistent CTA pairs (two 256-column accumulators: all 512 TMEM columns), K 128 per stage
+        dict(s0=dict(tile_m=256, tile_n=128, tile_k=128, stages=3, fuse=1, persistent=1, raster=(0, 1)),
+             s1=dict(tile_m=256, tile_n=224, stages=3, raster=(0, 1))),
+        # and both GEMMs persistent
+        dict(s0=dict(tile_m=256, tile_n=128, tile_k=64, stages=6, fuse=1, persistent=1, raster=(0, 8)),
+             s1=dict(tile_m=256, tile_n=256, tile_k=128, stages=3, persistent=1, raster=(1, 8))),
     ]
     for c in cases:
         s = schedule(op, **c)
