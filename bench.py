@@ -988,6 +988,18 @@ def library_study(wl, sched_text="", reps=20):
         print(json.dumps({"study": "library", "workload": wl.label, "unavailable": "no library equivalent compared"}))
 
 
+def rest_gpu(seconds=2.0):
+    """Idle the GPU briefly before a final timing. A search keeps it launching back to back for minutes,
+    which holds it at its power limit with the SM clock lowered; the measured peaks a fraction divides by
+    are those of a kernel timed alone (the burst figures), so the kernel is timed from a rested GPU too.
+    The timed work itself is unchanged."""
+    import time
+
+    import torch
+    torch.cuda.synchronize()
+    time.sleep(seconds)
+
+
 def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False, screen=1, moe_samples=None,
               layer_samples=None, hbm_gbs=None):
     """Search each other workload briefly and report its best schedule."""
@@ -1003,6 +1015,7 @@ def extra_ops(names, samples, peak_tf, branching=4, restarts=1, surrogate=False,
         find = search_tasks if wl.tasks else search_best
         _, best, _, n, cps = find(wl.op, io, n_s, branching=branching, restarts=restarts, surrogate=surrogate,
                                   screen=screen, horizon=wl.horizon)[:5]
+        rest_gpu()
         m = wl.op.measure([best], io, warmup=3, repeats=20)[0]
         if m.status != rc.OK:
             out[name] = {"workload": wl.label, "error": rc.STATUS_NAMES.get(m.status, m.status)}
@@ -1137,8 +1150,9 @@ def run_ours(args):
                                                         branching=args.branching, restarts=args.restarts,
                                                         surrogate=bool(args.surrogate), screen=args.screen)
 
-    # 2) timed steps of the best schedule
+    # 2) timed steps of the best schedule, from a rested GPU (rest_gpu)
     flush = torch.empty(int(2.5 * 129e6) // 4, dtype=torch.float32, device="cuda")
+    rest_gpu()
     for _ in range(args.warmup):
         op.run(best, io)
     torch.cuda.synchronize()
