@@ -748,14 +748,14 @@ extern "C" rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base,
   // leaves the program unchanged, so the canonical form keeps the default
   for (int i = 0; i < s.n_stages; ++i)
     if (!vectorize_used(op, s, i)) s.k[i].vec = rc_default_knobs(op, i).vec;
-  // attention: the one-issuing-warp kernel keeps P in shared memory and one S buffer, the
-  // split-issue kernels keep P in tensor memory, and the two-query-tile kernel has one form for each
-  // key block, so each family's canonical form fixes the knobs it does not offer (a single Parallel
-  // or TileSize transformation then moves between the families)
   // MoE grouped GEMMs: splitting ragged segments (layout 1) applies to CTA-pair launches only
   if (op->d.kind == RC_OP_MOE)
     for (int i = 1; i < s.n_stages; ++i)
       if (s.k[i].tile_m != 256) s.k[i].layout = 0;
+  // attention: the one-issuing-warp kernel keeps P in shared memory and one S buffer, the
+  // split-issue kernels keep P in tensor memory, and the two-query-tile kernel has a single form,
+  // so each family's canonical form fixes the knobs it does not offer (a single Parallel or
+  // TileSize transformation then moves between the families)
   for (int i = 0; i < s.n_stages; ++i) {
     if (!(op->d.kind == RC_OP_ATTENTION || (op->d.kind == RC_OP_DECODER_LAYER && i == 2))) continue;
     rc_knobs& k = s.k[i];

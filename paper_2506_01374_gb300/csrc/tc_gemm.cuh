@@ -757,13 +757,13 @@ rc_status launch_kernel(Kern kern, const CUtensorMap& tmA, const CUtensorMap& tm
   return RC_OK;
 }
 
+// Dynamic shared memory above which two CTAs cannot share an SM (228 KB per SM, 1 KB reserved per CTA).
+constexpr size_t kSmemHalfPlus = 233472 / 2 - 1024 + 16;
+
 // ring of A (128 rows) and this CTA's B rows (bn, or bn / 2 for a CTA pair)
 // per sub-block + 1 KB alignment slack + barriers and flags (256 B) + four
 // fp32 bias copies of the bn-column tile + the gathered-A row table (512 B)
 // + the grouped segment tables
-// Dynamic shared memory above which two CTAs cannot share an SM (228 KB per SM, 1 KB reserved per CTA).
-constexpr size_t kSmemHalfPlus = 233472 / 2 - 1024 + 16;
-
 inline size_t smem_bytes(int bn, int stages, int ksub, bool pair = false) {
   const size_t b_rows = pair ? (size_t)bn / 2 : (size_t)bn;
   return (size_t)stages * ksub * (BM * BK * 2 + b_rows * BK * 2) + 1024 + 256 + 4 * (size_t)bn * 4 + BM * 4 +
