@@ -202,3 +202,51 @@ def test_vectorize_offered_and_normalised_where_no_pass_runs():
     assert moe.schedule(rc.T(rc.T_COMPUTE_LOCATION, 1, stage=1), rc.T(rc.T_VECTORIZE, 4, stage=0)).knobs(0)["vec"] == 16
     att = rc.Op(rc.OP_ATTENTION, batch=1, seq=128, heads_q=2, heads_kv=1, head_dim=128, causal=1)
     assert all(t.kind != rc.T_VECTORIZE for t in att.transform_space())
+
+
+def test_two_query_tile_attention_canonical_form_and_legality():
+    op = rc.Op(rc.OP_ATTENTION, batch=1, seq=2048, heads_q=32, heads_kv=8, head_dim=128, causal=1)
+    # TileSize M = 256 selects the two-query-tile kernel whatever the other families' knobs say
+    s = op.schedule(rc.T(rc.T_TILE_SIZE, 64, axis=1), rc.T(rc.T_PARALLEL, 2), rc.T(rc.T_UNROLL, 2),
+                    rc.T(rc.T_COMPUTE_LOCATION, 0), rc.T(rc.T_TILE_SIZE, 256, axis=0))
+    k = s.knobs(0)
+    assert (k["tile_m"], k["tile_n"], k["persistent"], k["location"], k["unroll"]) == (256, 128, 1, 1, 1)
+    assert str(s) == str(op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0), rc.T(rc.T_PARALLEL, 1)))
+    # two 32 KB query tiles, a 128-key K ring and a two-slot V ring: at most three K stages fit 227 KB
+    for st in (1, 2, 3):
+        op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0), rc.T(rc.T_PIPELINE_STAGES, st))
+    with pytest.raises(rc.RcError):
+        op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0), rc.T(rc.T_PIPELINE_STAGES, 4))
+    # the transposed V needs 16-byte rows: seq % 8 == 0
+    odd = rc.Op(rc.OP_ATTENTION, batch=1, seq=300, heads_q=4, heads_kv=2, head_dim=128, causal=1)
+    with pytest.raises(rc.RcError):
+        odd.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0), rc.T(rc.T_LAYOUT, 1))
+    assert any(t.kind == rc.T_TILE_SIZE and t.axis == 0 and t.value[0] == 256 for t in op.transform_space())
+
+
+def test_persistent_pairs_take_256_column_tiles():
+    # two 256-column accumulators fill a pair's 512 TMEM columns: legal (the launcher keeps one CTA per SM)
+    op = rc.Op(rc.OP_LINEAR, m=2048, n=4096, k=14336)
+    for tn in (224, 256):
+        s = op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0), rc.T(rc.T_TILE_SIZE, tn, axis=1), rc.T(rc.T_PARALLEL, 1))
+        assert s.knobs(0)["persistent"] == 1 and s.knobs(0)["tile_n"] == tn
+    mlp = rc.Op(rc.OP_MLP, m=2048, n=14336, k=4096)
+    s = mlp.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, 128, axis=1, stage=0),
+                     rc.T(rc.T_TILE_SIZE, 128, axis=2, stage=0), rc.T(rc.T_PIPELINE_STAGES, 3, stage=0),
+                     rc.T(rc.T_PARALLEL, 1, stage=0), rc.T(rc.T_FUSE, 1, stage=0))
+    assert s.knobs(0)["persistent"] == 1 and s.knobs(0)["tile_k"] == 128
+
+
+def test_moe_split_segments_canonical_form():
+    op = rc.Op(rc.OP_MOE, tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
+    both = op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0, stage=1), rc.T(rc.T_LAYOUT, 1, stage=1),
+                       rc.T(rc.T_TILE_SIZE, 256, axis=0, stage=2), rc.T(rc.T_LAYOUT, 1, stage=2))
+    assert both.knobs(1)["layout"] == 1 and both.knobs(2)["layout"] == 1
+    # single-CTA M tiles have no remainder to split off: the canonical form drops the layout
+    single = op.schedule(rc.T(rc.T_LAYOUT, 1, stage=1), rc.T(rc.T_TILE_SIZE, 128, axis=0, stage=1))
+    assert single.knobs(1)["layout"] == 0
+    assert str(single) == str(op.schedule(rc.T(rc.T_TILE_SIZE, 128, axis=0, stage=1)))
+    # the in-GEMM row gather needs one CTA per tile, so it leaves nothing to split either
+    g = op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0, stage=1), rc.T(rc.T_LAYOUT, 1, stage=1),
+                    rc.T(rc.T_TILE_SIZE, 128, axis=0, stage=1), rc.T(rc.T_COMPUTE_LOCATION, 1, stage=1))
+    assert g.knobs(1)["layout"] == 0 and g.knobs(1)["location"] == 1
