@@ -58,6 +58,26 @@ bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, 
   return true;
 }
 
+// MoE grouped GEMM with exchanged operand roles (Layout 2): one CTA computes 256 weight rows
+// (two UMMAs of M = 128) x a token tile of tn rows into two TMEM accumulators of tn columns.
+bool moe_t_ok(const rc_op_desc& o, int stage, const rc_knobs& k, std::string* why) {
+  auto no = [&](const char* m) {
+    if (why) *why = m;
+    return false;
+  };
+  const int tn = stage == 1 ? 2 * k.tile_n : k.tile_n;
+  if (k.tile_m != 128) return no("exchanged operand roles: one CTA per tile (M tile 128)");
+  if (tn != 64 && tn != 128 && tn != 256) return no("exchanged operand roles: token tile of 64, 128 or 256 rows");
+  if (stage == 1 && k.location != 0) return no("exchanged operand roles: token rows from the gathered copy");
+  if (stage == 2 && k.fuse) return no("exchanged operand roles: the bf16 store epilogue (combine as a pass)");
+  // (persistent CTAs with 256-row token tiles keep one accumulator of all 512 TMEM columns: the
+  // producer runs ahead into the next tile while the epilogue drains, the tensor core waits)
+  if (k.tile_k != 64 && k.tile_k != 128) return no("K per stage must be 64 or 128");
+  if (o.hidden % 8 || o.inter % 8) return no("exchanged operand roles: 16-byte runs of output features");
+  if (tc_t_smem_bytes(tn, k.stages, k.tile_k) > kSmemLimit) return no("operand ring exceeds 227 KB of shared memory");
+  return true;
+}
+
 const char* kind_name(int k) {
   switch (k) {
     case RC_OP_GEMM_F32: return "gemm_f32";
@@ -206,14 +226,16 @@ std::vector<KnobSpec> rc_knob_space(const rc_op_s* op, int stage) {
         // where the token rows are gathered: 0 = a separate pass writes the grouped copy (stage 0),
         // 1 = the grouped GEMM's producer gathers them from X (M tile 128)
         v.push_back({RC_T_COMPUTE_LOCATION, 0, {0, 1}, {}});
-        // how a CTA-pair launch tiles a ragged expert segment: 0 = whole pair tiles, 1 = pair tiles and a
-        // last 128-row single-CTA tile where the remainder fits it (a second, one-CTA launch)
-        v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});
+        // how the grouped GEMM lays out a ragged expert segment: 0 = whole M tiles of tokens, 1 = CTA-pair
+        // tiles and a last 128-row single-CTA tile where the remainder fits it (a second, one-CTA launch),
+        // 2 = the operand roles exchanged: weight rows on UMMA M, the segment's tokens on N in tiles of
+        // whole 16-row units (the tile transposed in TMEM; the N tile knob sets the token tile)
+        v.push_back({RC_T_LAYOUT, 0, {0, 1, 2}, {}});
       } else {
         gemm_common({64, 128, 224, 256});
         v.push_back({RC_T_FUSE, 0, {0, 1}, {}});
         v.push_back({RC_T_TILE_SIZE, 0, {128, 256}, {}});
-        v.push_back({RC_T_LAYOUT, 0, {0, 1}, {}});  // as in stage 1
+        v.push_back({RC_T_LAYOUT, 0, {0, 1, 2}, {}});  // as in stage 1
         vectorize();  // the combine (or the fp32 -> bf16 pass of the atomic combine)
       }
       break;
@@ -337,6 +359,7 @@ bool rc_knobs_legal(const rc_op_s* op, int stage, const rc_knobs& k, std::string
         if (why) *why = "rows gathered in the GEMM producer need one CTA per tile (M tile 128)";
         return false;
       }
+      if (k.layout == 2) return moe_t_ok(o, stage, k, why);
       return tc_gemm_ok(stage == 1 ? 2 * k.tile_n : k.tile_n, k.stages, k.tile_k, k.tile_m, k.persistent, why);
     case RC_OP_DECODER_LAYER:
       if (stage == 1) return true;
@@ -751,7 +774,7 @@ extern "C" rc_status rc_schedule_apply(const rc_op* op, const rc_schedule* base,
   // MoE grouped GEMMs: splitting ragged segments (layout 1) applies to CTA-pair launches only
   if (op->d.kind == RC_OP_MOE)
     for (int i = 1; i < s.n_stages; ++i)
-      if (s.k[i].tile_m != 256) s.k[i].layout = 0;
+      if (s.k[i].layout == 1 && s.k[i].tile_m != 256) s.k[i].layout = 0;
   // attention: the one-issuing-warp kernel keeps P in shared memory and one S buffer, the
   // split-issue kernels keep P in tensor memory, and the two-query-tile kernel has a single form,
   // so each family's canonical form fixes the knobs it does not offer (a single Parallel or

@@ -14,6 +14,7 @@ rc_status tc_dispatch_grouped_pair(const rc_knobs& k, const TcGemmArgs& a, const
 rc_status tc_dispatch_conv(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_grouped(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 rc_status tc_dispatch_mc(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
+rc_status tc_dispatch_grouped_t(const rc_knobs& k, const TcGemmArgs& a, const LaunchCtx& c);
 
 namespace tcg {
 namespace {
@@ -89,6 +90,10 @@ rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const Launch
     return pair ? tc_dispatch_conv_pair(k, a, c) : tc_dispatch_conv(k, a, c);
   if (a.a_mode == TC_A_GATHER && (pair || a.groups <= 0))
     return rc_fail(RC_ERR_ILLEGAL_SCHEDULE, "tc_gemm: gathered A rows need a grouped GEMM on one CTA (M tile 128)");
-  if (a.groups > 0) return pair ? tc_dispatch_grouped_pair(k, a, c) : tc_dispatch_grouped(k, a, c);
+  if (a.groups > 0) {
+    // Layout 2: weights on UMMA M, each segment's tokens on N (the tile transposed in TMEM)
+    if (k.layout == 2) return tc_dispatch_grouped_t(k, a, c);
+    return pair ? tc_dispatch_grouped_pair(k, a, c) : tc_dispatch_grouped(k, a, c);
+  }
   return pair ? tc_dispatch_dense_pair(k, a, c) : tc_dispatch_dense(k, a, c);
 }

@@ -79,7 +79,8 @@ struct Params {
 };
 
 // Linear CTA index -> (m tile, n tile) under the raster order knob.
-__device__ __forceinline__ void map_tile(const Params& p, int t, int& mt, int& nt) {
+template <class P>
+__device__ __forceinline__ void map_tile(const P& p, int t, int& mt, int& nt) {
   const int G = p.group;
   if (p.raster == 0) {  // M fastest within bands of G n-tiles
     const int band = t / (p.tiles_m * G), in = t - band * p.tiles_m * G;
@@ -115,17 +116,25 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
     constexpr int HALF = BN / 2;
     __nv_bfloat16* out = (__nv_bfloat16*)p.D + (long long)r * p.ldd;
     const int n0 = nt * HALF;
-#pragma unroll 1
+    // 16 columns per step, software-pipelined: the next step's TMEM loads are issued before this
+    // step's math and stores, and waited for at the top of the next step
+    uint32_t g[2][16], u[2][16];
+    tc::tmem_ld16(taddr, g[0]);
+    tc::tmem_ld16(taddr + HALF, u[0]);
+#pragma unroll
     for (int c = 0; c < HALF; c += 16) {
-      uint32_t g[16], u[16];
-      tc::tmem_ld16(taddr + c, g);
-      tc::tmem_ld16(taddr + HALF + c, u);
-      tc::tmem_ld_wait();
+      const int b = (c / 16) & 1;
+      tc::tmem_ld_wait(g[b]);
+      tc::tmem_ld_wait(u[b]);
+      if (c + 16 < HALF) {
+        tc::tmem_ld16(taddr + c + 16, g[b ^ 1]);
+        tc::tmem_ld16(taddr + HALF + c + 16, u[b ^ 1]);
+      }
       float v[16];
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
-        const float gv = have_acc ? __uint_as_float(g[j]) : 0.f;
-        const float uv = have_acc ? __uint_as_float(u[j]) : 0.f;
+        const float gv = have_acc ? __uint_as_float(g[b][j]) : 0.f;
+        const float uv = have_acc ? __uint_as_float(u[b][j]) : 0.f;
         v[j] = tc::silu(gv) * uv;
       }
       const int col = n0 + c;
@@ -146,15 +155,18 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
         orow = slot / p.row_div;
       }
     }
-#pragma unroll 1
+    // 16 columns per step, software-pipelined as in the SwiGLU epilogue
+    uint32_t a[2][16];
+    tc::tmem_ld16(taddr, a[0]);
+#pragma unroll
     for (int c = 0; c < BN; c += 16) {
+      const int b = (c / 16) & 1;
       const int col = n0 + c;
-      uint32_t a[16];
-      tc::tmem_ld16(taddr + c, a);
-      tc::tmem_ld_wait();
+      tc::tmem_ld_wait(a[b]);
+      if (c + 16 < BN) tc::tmem_ld16(taddr + c + 16, a[b ^ 1]);
       float v[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = have_acc ? __uint_as_float(a[j]) : 0.f;
+      for (int j = 0; j < 16; ++j) v[j] = have_acc ? __uint_as_float(a[b][j]) : 0.f;
       if (!row_ok) continue;
       if constexpr (EPI == TC_EPI_STORE_BF16 || EPI == TC_EPI_BIAS_SILU) {
         if constexpr (EPI == TC_EPI_BIAS_SILU) {

@@ -161,6 +161,64 @@ def test_moe_split_segments(T, E, K, kinds):
     assert moe_sched(op, 8, 64, 3, 128, 3, 0, tile_m=128, split=1).knobs(1)["layout"] == 0
 
 
+def moe_sched_t(op, tn1, tn2, st, pe, tk, l1=2, l2=2, raster=(0, 1), fuse=0, tm2=128):
+    # layout 2: each grouped GEMM computes W X^T (weights on UMMA M, a segment's token tile on N)
+    return op.schedule(rc.T(rc.T_LAYOUT, l1, stage=1), rc.T(rc.T_LAYOUT, l2, stage=2),
+                       rc.T(rc.T_TILE_SIZE, 8, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
+                       rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2), rc.T(rc.T_TILE_SIZE, tm2, axis=0, stage=2),
+                       rc.T(rc.T_PIPELINE_STAGES, st, stage=1), rc.T(rc.T_PIPELINE_STAGES, st, stage=2),
+                       rc.T(rc.T_PARALLEL, pe, stage=1), rc.T(rc.T_PARALLEL, pe, stage=2),
+                       rc.T(rc.T_TILE_SIZE, tk, axis=2, stage=1), rc.T(rc.T_TILE_SIZE, tk, axis=2, stage=2),
+                       rc.T(rc.T_LOOP_ORDER, raster[0], group=raster[1], stage=1),
+                       rc.T(rc.T_LOOP_ORDER, raster[0], group=raster[1], stage=2), rc.T(rc.T_FUSE, fuse, stage=2))
+
+
+@pytest.mark.parametrize("T,E,K,H,I", [(200, 8, 2, 128, 64), (1000, 5, 3, 256, 192), (2000, 12, 3, 384, 256),
+                                       (37, 4, 4, 192, 64)])
+def test_moe_exchanged_operands(T, E, K, H, I):
+    # Layout 2 on both grouped GEMMs: token tiles of 64, 128 or 256 rows cut into whole 16-row units
+    # (segments of 9 .. 700 rows), weight tiles past I or H (masked columns), K of one or several
+    # ring laps, persistent or not, both raster orders
+    logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=47 + T)
+    ids, w, off, perm = oracle.moe_route(logits, K)
+    ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
+    op = moe_op(T, H, E, I, K)
+    dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
+    n = 0
+    for tn1, tn2, st, pe, tk, ra in itertools.product((32, 64, 128), (64, 128, 256), (2, 4), (0, 1), (64, 128),
+                                                      ((0, 1), (1, 8))):
+        try:
+            s = moe_sched_t(op, tn1, tn2, st, pe, tk, raster=ra)
+        except rc.RcError:
+            continue  # shared memory
+        assert s.knobs(1)["layout"] == 2 and s.knobs(2)["layout"] == 2
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(s, [dl, dX, d1, d2, out])
+        op.check()
+        err = rel_err(from_dev_bf16(out), ref)
+        assert err <= TOL, (tn1, tn2, st, pe, tk, ra, err)
+        n += 1
+    assert n >= 50
+    # one stage exchanged, the other on M tiles of tokens (one CTA or a CTA pair)
+    for l1, l2, tm2 in ((2, 0, 128), (0, 2, 128), (2, 0, 256), (2, 1, 256)):
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(moe_sched_t(op, 64, 128, 3, 1, 64, l1, l2, tm2=tm2), [dl, dX, d1, d2, out])
+        op.check()
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (l1, l2, tm2)
+
+
+def test_moe_exchanged_operands_legality():
+    op = moe_op(256, 128, 8, 64, 2)
+    # persistent CTAs with 256-row token tiles keep a single accumulator of 512 TMEM columns
+    assert moe_sched_t(op, 128, 256, 2, 1, 64).knobs(2)["persistent"] == 1
+    with pytest.raises(rc.RcError):
+        moe_sched_t(op, 64, 224, 2, 0, 64)  # token tiles of 64, 128 or 256 rows
+    with pytest.raises(rc.RcError):
+        moe_sched_t(op, 64, 128, 2, 0, 64, fuse=1)  # the atomic combine epilogue is not offered
+    with pytest.raises(rc.RcError):
+        moe_sched_t(op, 64, 128, 2, 0, 64, tm2=256)  # one CTA per tile
+
+
 def test_moe_layer_imbalanced_and_empty_experts():
     T, H, E, I, K = 300, 128, 16, 128, 4
     logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=43)
@@ -179,6 +237,11 @@ def test_moe_layer_imbalanced_and_empty_experts():
                [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
         assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm, ga, sp)
+    for tn1, tn2, pe in itertools.product((32, 128), (64, 256), (0, 1)):  # exchanged operand roles
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(moe_sched_t(op, tn1, tn2, 2, pe, 64), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.check()
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (tn1, tn2, pe)
 
 
 def test_moe_full_size_sampled_tokens():
@@ -196,7 +259,10 @@ def test_moe_full_size_sampled_tokens():
               moe_sched(op, 8, 128, 2, 224, 2, 1, 1, tile_k=128, gather=1),
               # CTA pairs with short remainders split off to one-CTA launches
               moe_sched(op, 8, 128, 3, 256, 4, 0, 1, tile_m=256, split=1),
-              moe_sched(op, 8, 128, 3, 256, 3, 1, 0, tile_m=256, split=1)]:
+              moe_sched(op, 8, 128, 3, 256, 3, 1, 0, tile_m=256, split=1),
+              # exchanged operand roles: 256-row token tiles, and 128-row tiles on persistent CTAs
+              moe_sched_t(op, 128, 256, 3, 0, 64), moe_sched_t(op, 64, 128, 4, 1, 64, raster=(1, 8)),
+              moe_sched_t(op, 128, 224, 3, 0, 64, l2=0)]:
         out = empty_bf16(T, H)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         go = torch.empty(E + 1, dtype=torch.int32, device="cuda")
@@ -222,6 +288,11 @@ def test_moe_layer_256_experts():
         op.run(moe_sched(op, 8, 64, 2, 128, 2, fuse, tile_m=tm), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
         assert rel_err(from_dev_bf16(out), ref) <= TOL, (tm, fuse)
+    for pe in (0, 1):  # exchanged operand roles
+        out = empty_bf16(T, H).fill_(0x7FC0)
+        op.run(moe_sched_t(op, 32, 64, 2, pe, 64), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.check()
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, pe
 
 
 def test_moe_host_path_matches_device_path():
