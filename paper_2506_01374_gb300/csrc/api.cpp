@@ -59,14 +59,15 @@ bool tc_gemm_ok(int bn_mma, int stages, int tile_k, int tile_m, int persistent, 
 }
 
 // MoE grouped GEMM with exchanged operand roles (Layout 2): one CTA computes 256 weight rows
-// (two UMMAs of M = 128) x a token tile of tn rows into two TMEM accumulators of tn columns.
+// (two UMMAs of M = 128) x a token tile of tn rows into two TMEM accumulators of tn columns; a CTA
+// pair (M tile 256) 512 weight rows with the token tile's rows split over its two CTAs.
 bool moe_t_ok(const rc_op_desc& o, int stage, const rc_knobs& k, std::string* why) {
   auto no = [&](const char* m) {
     if (why) *why = m;
     return false;
   };
   const int tn = stage == 1 ? 2 * k.tile_n : k.tile_n;
-  if (k.tile_m != 128) return no("exchanged operand roles: one CTA per tile (M tile 128)");
+  if (k.tile_m != 128 && k.tile_m != 256) return no("exchanged operand roles: M tile 128 or 256 (a CTA pair)");
   if (tn != 64 && tn != 128 && tn != 256) return no("exchanged operand roles: token tile of 64, 128 or 256 rows");
   if (stage == 1 && k.location != 0) return no("exchanged operand roles: token rows from the gathered copy");
   if (stage == 2 && k.fuse) return no("exchanged operand roles: the bf16 store epilogue (combine as a pass)");
@@ -74,7 +75,8 @@ bool moe_t_ok(const rc_op_desc& o, int stage, const rc_knobs& k, std::string* wh
   // producer runs ahead into the next tile while the epilogue drains, the tensor core waits)
   if (k.tile_k != 64 && k.tile_k != 128) return no("K per stage must be 64 or 128");
   if (o.hidden % 8 || o.inter % 8) return no("exchanged operand roles: 16-byte runs of output features");
-  if (tc_t_smem_bytes(tn, k.stages, k.tile_k) > kSmemLimit) return no("operand ring exceeds 227 KB of shared memory");
+  if (tc_t_smem_bytes(tn, k.stages, k.tile_k, k.tile_m == 256) > kSmemLimit)
+    return no("operand ring exceeds 227 KB of shared memory");
   return true;
 }
 

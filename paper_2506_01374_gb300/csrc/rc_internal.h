@@ -162,8 +162,8 @@ rc_status rc_launch_tc_gemm(const rc_knobs& k, const TcGemmArgs& a, const Launch
 // Shared memory of one CTA of the tensor-core GEMM (the schedule legality check's figure).
 int64_t tc_smem_bytes(int bn_mma, int stages, int tile_k, int tile_m);
 // The same for the grouped GEMM with exchanged operand roles (Layout 2: weights on UMMA M, a token
-// tile of tn rows on N).
-int64_t tc_t_smem_bytes(int tn, int stages, int tile_k);
+// tile of tn rows on N, split over the two CTAs of a pair).
+int64_t tc_t_smem_bytes(int tn, int stages, int tile_k, bool pair);
 // Split-K reduction: out_bf16[M][N] = sum_z part[z][M][N].
 rc_status rc_launch_splitk_reduce(const float* part, int splits, int64_t M, int64_t N, void* out,
                                   int vec, const LaunchCtx& c);

@@ -161,11 +161,13 @@ def test_moe_split_segments(T, E, K, kinds):
     assert moe_sched(op, 8, 64, 3, 128, 3, 0, tile_m=128, split=1).knobs(1)["layout"] == 0
 
 
-def moe_sched_t(op, tn1, tn2, st, pe, tk, l1=2, l2=2, raster=(0, 1), fuse=0, tm2=128):
-    # layout 2: each grouped GEMM computes W X^T (weights on UMMA M, a segment's token tile on N)
+def moe_sched_t(op, tn1, tn2, st, pe, tk, l1=2, l2=2, raster=(0, 1), fuse=0, tm1=128, tm2=128):
+    # layout 2: each grouped GEMM computes W X^T (weights on UMMA M, a segment's token tile on N);
+    # M tile 256: a CTA pair, 128 weight rows per CTA and the token tile's rows split between them
     return op.schedule(rc.T(rc.T_LAYOUT, l1, stage=1), rc.T(rc.T_LAYOUT, l2, stage=2),
                        rc.T(rc.T_TILE_SIZE, 8, axis=0, stage=0), rc.T(rc.T_TILE_SIZE, tn1, axis=1, stage=1),
-                       rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2), rc.T(rc.T_TILE_SIZE, tm2, axis=0, stage=2),
+                       rc.T(rc.T_TILE_SIZE, tn2, axis=1, stage=2), rc.T(rc.T_TILE_SIZE, tm1, axis=0, stage=1),
+                       rc.T(rc.T_TILE_SIZE, tm2, axis=0, stage=2),
                        rc.T(rc.T_PIPELINE_STAGES, st, stage=1), rc.T(rc.T_PIPELINE_STAGES, st, stage=2),
                        rc.T(rc.T_PARALLEL, pe, stage=1), rc.T(rc.T_PARALLEL, pe, stage=2),
                        rc.T(rc.T_TILE_SIZE, tk, axis=2, stage=1), rc.T(rc.T_TILE_SIZE, tk, axis=2, stage=2),
@@ -177,18 +179,18 @@ def moe_sched_t(op, tn1, tn2, st, pe, tk, l1=2, l2=2, raster=(0, 1), fuse=0, tm2
                                        (37, 4, 4, 192, 64)])
 def test_moe_exchanged_operands(T, E, K, H, I):
     # Layout 2 on both grouped GEMMs: token tiles of 64, 128 or 256 rows cut into whole 16-row units
-    # (segments of 9 .. 700 rows), weight tiles past I or H (masked columns), K of one or several
-    # ring laps, persistent or not, both raster orders
+    # (32-row units on CTA pairs; segments of 9 .. 700 rows), weight tiles past I or H (masked
+    # columns), K of one or several ring laps, persistent or not, both raster orders, one CTA or a pair
     logits, X, W1, W2 = inputs.moe(T, H, E, I, seed=47 + T)
     ids, w, off, perm = oracle.moe_route(logits, K)
     ref = oracle.moe_ffn_bf16(X, W1, W2, ids, w)
     op = moe_op(T, H, E, I, K)
     dl, dX, d1, d2 = to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2)
     n = 0
-    for tn1, tn2, st, pe, tk, ra in itertools.product((32, 64, 128), (64, 128, 256), (2, 4), (0, 1), (64, 128),
-                                                      ((0, 1), (1, 8))):
+    for tn1, tn2, st, pe, tk, ra, tm in itertools.product((32, 64, 128), (64, 128, 256), (2, 4), (0, 1), (64, 128),
+                                                          ((0, 1), (1, 8)), (128, 256)):
         try:
-            s = moe_sched_t(op, tn1, tn2, st, pe, tk, raster=ra)
+            s = moe_sched_t(op, tn1, tn2, st, pe, tk, raster=ra, tm1=tm, tm2=tm)
         except rc.RcError:
             continue  # shared memory
         assert s.knobs(1)["layout"] == 2 and s.knobs(2)["layout"] == 2
@@ -196,9 +198,9 @@ def test_moe_exchanged_operands(T, E, K, H, I):
         op.run(s, [dl, dX, d1, d2, out])
         op.check()
         err = rel_err(from_dev_bf16(out), ref)
-        assert err <= TOL, (tn1, tn2, st, pe, tk, ra, err)
+        assert err <= TOL, (tn1, tn2, st, pe, tk, ra, tm, err)
         n += 1
-    assert n >= 50
+    assert n >= 120
     # one stage exchanged, the other on M tiles of tokens (one CTA or a CTA pair)
     for l1, l2, tm2 in ((2, 0, 128), (0, 2, 128), (2, 0, 256), (2, 1, 256)):
         out = empty_bf16(T, H).fill_(0x7FC0)
@@ -216,7 +218,7 @@ def test_moe_exchanged_operands_legality():
     with pytest.raises(rc.RcError):
         moe_sched_t(op, 64, 128, 2, 0, 64, fuse=1)  # the atomic combine epilogue is not offered
     with pytest.raises(rc.RcError):
-        moe_sched_t(op, 64, 128, 2, 0, 64, tm2=256)  # one CTA per tile
+        moe_sched_t(op, 64, 128, 2, 0, 64, fuse=1, tm2=256)
 
 
 def test_moe_layer_imbalanced_and_empty_experts():
@@ -237,11 +239,11 @@ def test_moe_layer_imbalanced_and_empty_experts():
                [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
         assert rel_err(from_dev_bf16(out), ref) <= TOL, (fuse, pe, tm, ga, sp)
-    for tn1, tn2, pe in itertools.product((32, 128), (64, 256), (0, 1)):  # exchanged operand roles
+    for tn1, tn2, pe, tm in itertools.product((32, 128), (64, 256), (0, 1), (128, 256)):  # exchanged operand roles
         out = empty_bf16(T, H).fill_(0x7FC0)
-        op.run(moe_sched_t(op, tn1, tn2, 2, pe, 64), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.run(moe_sched_t(op, tn1, tn2, 2, pe, 64, tm1=tm, tm2=tm), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
-        assert rel_err(from_dev_bf16(out), ref) <= TOL, (tn1, tn2, pe)
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (tn1, tn2, pe, tm)
 
 
 def test_moe_full_size_sampled_tokens():
@@ -262,7 +264,8 @@ def test_moe_full_size_sampled_tokens():
               moe_sched(op, 8, 128, 3, 256, 3, 1, 0, tile_m=256, split=1),
               # exchanged operand roles: 256-row token tiles, and 128-row tiles on persistent CTAs
               moe_sched_t(op, 128, 256, 3, 0, 64), moe_sched_t(op, 64, 128, 4, 1, 64, raster=(1, 8)),
-              moe_sched_t(op, 128, 224, 3, 0, 64, l2=0)]:
+              moe_sched_t(op, 128, 224, 3, 0, 64, l2=0),
+              moe_sched_t(op, 128, 256, 4, 1, 64, tm1=256, tm2=256), moe_sched_t(op, 64, 128, 2, 0, 128, tm1=256, tm2=256)]:
         out = empty_bf16(T, H)
         gi = torch.empty(T, K, dtype=torch.int32, device="cuda")
         go = torch.empty(E + 1, dtype=torch.int32, device="cuda")
@@ -288,11 +291,11 @@ def test_moe_layer_256_experts():
         op.run(moe_sched(op, 8, 64, 2, 128, 2, fuse, tile_m=tm), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
         assert rel_err(from_dev_bf16(out), ref) <= TOL, (tm, fuse)
-    for pe in (0, 1):  # exchanged operand roles
+    for pe, tm in itertools.product((0, 1), (128, 256)):  # exchanged operand roles
         out = empty_bf16(T, H).fill_(0x7FC0)
-        op.run(moe_sched_t(op, 32, 64, 2, pe, 64), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
+        op.run(moe_sched_t(op, 32, 64, 2, pe, 64, tm1=tm, tm2=tm), [to_dev(logits), to_dev(X), to_dev(W1), to_dev(W2), out])
         op.check()
-        assert rel_err(from_dev_bf16(out), ref) <= TOL, pe
+        assert rel_err(from_dev_bf16(out), ref) <= TOL, (pe, tm)
 
 
 def test_moe_host_path_matches_device_path():
