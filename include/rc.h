@@ -180,7 +180,14 @@ typedef enum {
                               * runs two CTAs per SM */
   RC_T_LOOP_ORDER = 4,       /* value[0]: tile raster 0 = M fastest, 1 = N fastest; value[1] = group */
   RC_T_FUSE = 5,             /* value[0]: 1 = epilogue fused into the producing kernel, 0 = separate pass */
-  RC_T_LAYOUT = 6,           /* value[0]: op-specific data layout choice */
+  RC_T_LAYOUT = 6,           /* value[0]: op-specific data layout choice; CONV2D: 0 = implicit zero
+                              * padding, 1 and 2 = a padded copy read as one box or as row boxes;
+                              * ATTENTION: 1 = V transposed to [d][keys]; MOE stages 1 and 2 (the
+                              * grouped GEMMs): 0 = each expert's tokens in M tiles, 1 = CTA-pair
+                              * tiles with a segment's short remainder in a second one-CTA launch,
+                              * 2 = operand roles exchanged (expert weight rows on UMMA M, the
+                              * segment's tokens on N in tiles of whole 16-row units, 32 on a CTA
+                              * pair; the N tile knob sets the token tile) */
   RC_T_VECTORIZE = 7,        /* value[0]: bytes per global access in the vectorised passes */
   RC_T_PIPELINE_STAGES = 8,  /* value[0]: depth of the shared-memory operand ring */
   RC_T_SPLIT_K = 9,          /* value[0]: number of reduction splits */
