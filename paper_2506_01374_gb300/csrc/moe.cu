@@ -243,16 +243,27 @@ struct Vec<4> {
   using T = uint32_t;
 };
 
+// One warp per grouped row: four vector loads in flight per lane before their stores. The source
+// rows (each read by k slots) are left in L2; the grouped copy is written with the streaming hint.
 template <int VB>
 __global__ void gather_rows_kernel(const typename Vec<VB>::T* __restrict__ X, const int* __restrict__ perm, int rows,
                                    int HV, int K, typename Vec<VB>::T* __restrict__ Xp) {
+  using V = typename Vec<VB>::T;
   const int warps = blockDim.x / 32;
   const int lane = threadIdx.x % 32;
   for (int r = blockIdx.x * warps + threadIdx.x / 32; r < rows; r += gridDim.x * warps) {
     const int t = perm[r] / K;
-    const typename Vec<VB>::T* src = X + (size_t)t * HV;
-    typename Vec<VB>::T* dst = Xp + (size_t)r * HV;
-    for (int i = lane; i < HV; i += 32) dst[i] = src[i];
+    const V* src = X + (size_t)t * HV;
+    V* dst = Xp + (size_t)r * HV;
+    int i = lane;
+    for (; i + 96 < HV; i += 128) {
+      const V a = src[i], b = src[i + 32], c = src[i + 64], d = src[i + 96];
+      __stcs(dst + i, a);
+      __stcs(dst + i + 32, b);
+      __stcs(dst + i + 64, c);
+      __stcs(dst + i + 96, d);
+    }
+    for (; i < HV; i += 32) __stcs(dst + i, src[i]);
   }
 }
 
