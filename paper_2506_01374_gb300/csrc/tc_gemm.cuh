@@ -107,10 +107,20 @@ __device__ __forceinline__ uint4 pack8(const float* v) {
   return p.u;
 }
 
-// sbias: this warp's copy of the tile's bias (fp32, BN values; BIAS_SILU only)
+// Row pitch of an epilogue warp's staging area: BN bf16 plus 16 bytes, an odd number of 16-byte
+// chunks (BN % 16 == 0), so that eight consecutive rows' chunks c fall on distinct bank groups.
+template <int BN>
+constexpr int stage_pitch() {
+  return 2 * BN + 16;
+}
+
+// sbias: this warp's copy of the tile's bias (fp32, BN values; BIAS_SILU only). stage: NULL, or
+// this warp's 32 x stage_pitch<BN>() bytes of idle operand ring (the plain bf16 store): the rows
+// are converted into it, then stored as runs of whole rows, so that a warp store covers 512
+// contiguous bytes instead of 16 bytes in each of 32 rows.
 template <int BN, int EPI>
 __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r, int row_end, int nt, int split,
-                                         bool have_acc, const float* sbias) {
+                                         bool have_acc, const float* sbias, uint8_t* stage = nullptr) {
   const bool row_ok = r < row_end;
   if constexpr (EPI == TC_EPI_SWIGLU) {
     constexpr int HALF = BN / 2;
@@ -199,9 +209,15 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
             }
           }
         }
-        __nv_bfloat16* out = (__nv_bfloat16*)p.D + (long long)r * p.ldd;
-        if (col < p.out_cols) *reinterpret_cast<uint4*>(out + col) = pack8(v);
-        if (col + 8 < p.out_cols) *reinterpret_cast<uint4*>(out + col + 8) = pack8(v + 8);
+        if (stage) {
+          uint8_t* srow = stage + (threadIdx.x & 31) * stage_pitch<BN>() + c * 2;
+          *reinterpret_cast<uint4*>(srow) = pack8(v);
+          *reinterpret_cast<uint4*>(srow + 16) = pack8(v + 8);
+        } else {
+          __nv_bfloat16* out = (__nv_bfloat16*)p.D + (long long)r * p.ldd;
+          if (col < p.out_cols) *reinterpret_cast<uint4*>(out + col) = pack8(v);
+          if (col + 8 < p.out_cols) *reinterpret_cast<uint4*>(out + col + 8) = pack8(v + 8);
+        }
       } else if constexpr (EPI == TC_EPI_PARTIAL_F32) {
         float* out = (float*)p.D + (long long)split * p.M * p.ldd + (long long)r * p.ldd;
 #pragma unroll
@@ -216,6 +232,21 @@ __device__ __forceinline__ void epilogue(const Params& p, uint32_t taddr, int r,
           if (col + 4 * q < p.out_cols)
             atomicAdd(reinterpret_cast<float4*>(out + col + 4 * q),
                       make_float4(s * v[4 * q], s * v[4 * q + 1], s * v[4 * q + 2], s * v[4 * q + 3]));
+      }
+    }
+    if constexpr (EPI == TC_EPI_STORE_BF16) {
+      if (stage) {  // the warp's 32 rows, 16-byte chunks in row order: lane l takes chunks l, l + 32, ...
+        __syncwarp();
+        constexpr int NCH = BN / 8;
+        const int ln = threadIdx.x & 31, row0 = r - ln;
+#pragma unroll 4
+        for (int qc = ln; qc < 32 * NCH; qc += 32) {
+          const int rr = qc / NCH, ch = qc - rr * NCH;
+          const int row = row0 + rr, col = n0 + ch * 8;
+          if (row < row_end && col < p.out_cols)
+            *reinterpret_cast<uint4*>((__nv_bfloat16*)p.D + (long long)row * p.ldd + col) =
+                *reinterpret_cast<const uint4*>(stage + rr * stage_pitch<BN>() + ch * 16);
+        }
       }
     }
   }
@@ -701,8 +732,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc::tc_fence_after();
+      // one tile per CTA: every ring stage has been read by the tensor core and none is refilled,
+      // so the ring can stage the rows of the plain bf16 store, whose time is all in its stores (not
+      // with B multicast, whose peers write into the ring; the bias/SiLU epilogue's arithmetic
+      // already overlaps its stores, and staging only added to it: conv pair tiles 641 -> 614
+      // TFLOP/s, where the plain store gained 1-3% on the down-projection GEMM)
+      uint8_t* stg = nullptr;
+      if constexpr (MC == 1 && EPI == TC_EPI_STORE_BF16) {
+        if (!p.persistent && (size_t)stages * STAGE_BYTES >= (size_t)4 * 32 * stage_pitch<BN>())
+          stg = smem + (size_t)(warp - 2) * 32 * stage_pitch<BN>();
+      }
       epilogue<BN, EPI>(p, tmem + buf * ACC_COLS + ((uint32_t)(32 * q) << 16), it.row0 + 32 * q + lane,
-                        it.row_end, it.nt, it.split, it.nkb > 0, sbias);
+                        it.row_end, it.nt, it.split, it.nkb > 0, sbias, stg);
       tc::tc_fence_before();
       if constexpr (PAIR) {
         __syncwarp();
