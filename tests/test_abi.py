@@ -250,3 +250,34 @@ def test_moe_split_segments_canonical_form():
     g = op.schedule(rc.T(rc.T_TILE_SIZE, 256, axis=0, stage=1), rc.T(rc.T_LAYOUT, 1, stage=1),
                     rc.T(rc.T_TILE_SIZE, 128, axis=0, stage=1), rc.T(rc.T_COMPUTE_LOCATION, 1, stage=1))
     assert g.knobs(1)["layout"] == 0 and g.knobs(1)["location"] == 1
+
+
+def test_moe_exchanged_operands_canonical_form_and_legality():
+    # Layout 2 of the grouped GEMMs: weights on UMMA M, each expert's tokens on N (token tiles of 64,
+    # 128 or 256 rows: 2x the SwiGLU output tile in stage 1, the N tile in stage 2), one CTA or a pair
+    op = rc.Op(rc.OP_MOE, tokens=4096, hidden=7168, experts=64, inter=2048, top_k=8)
+    T = rc.T
+    s = op.schedule(T(rc.T_LAYOUT, 2, stage=1), T(rc.T_TILE_SIZE, 128, axis=1, stage=1),
+                    T(rc.T_LAYOUT, 2, stage=2), T(rc.T_TILE_SIZE, 256, axis=1, stage=2), T(rc.T_PARALLEL, 1, stage=2))
+    assert s.knobs(1)["layout"] == 2 and s.knobs(2)["layout"] == 2 and s.knobs(2)["persistent"] == 1
+    # unlike layout 1, layout 2 stays on single-CTA tiles, and on CTA pairs
+    assert op.schedule(T(rc.T_LAYOUT, 2, stage=1)).knobs(1)["layout"] == 2
+    pair = op.schedule(T(rc.T_LAYOUT, 2, stage=2), T(rc.T_TILE_SIZE, 256, axis=0, stage=2),
+                       T(rc.T_TILE_SIZE, 256, axis=1, stage=2), T(rc.T_PIPELINE_STAGES, 4, stage=2))
+    assert pair.knobs(2)["layout"] == 2 and pair.knobs(2)["tile_m"] == 256
+    assert str(pair) != str(op.schedule(T(rc.T_TILE_SIZE, 256, axis=0, stage=2), T(rc.T_TILE_SIZE, 256, axis=1, stage=2),
+                                        T(rc.T_PIPELINE_STAGES, 4, stage=2)))
+    illegal = [
+        [T(rc.T_LAYOUT, 2, stage=2), T(rc.T_TILE_SIZE, 224, axis=1, stage=2)],  # token tile of 224 rows
+        [T(rc.T_LAYOUT, 2, stage=2), T(rc.T_FUSE, 1, stage=2)],  # the atomic combine epilogue
+        [T(rc.T_LAYOUT, 2, stage=1), T(rc.T_COMPUTE_LOCATION, 1, stage=1)],  # rows gathered in the GEMM
+        # a single-CTA ring of 4 stages of 256 token rows and two 128-row weight boxes, K 128: 512 KB
+        [T(rc.T_LAYOUT, 2, stage=1), T(rc.T_TILE_SIZE, 128, axis=1, stage=1), T(rc.T_TILE_SIZE, 128, axis=2, stage=1),
+         T(rc.T_PIPELINE_STAGES, 4, stage=1)],
+    ]
+    for ts in illegal:
+        with pytest.raises(rc.RcError):
+            op.schedule(*ts)
+    # the search's space offers the layout on both grouped GEMMs
+    kinds = {(t.kind, t.stage, t.value[0]) for t in op.transform_space()}
+    assert (rc.T_LAYOUT, 1, 2) in kinds and (rc.T_LAYOUT, 2, 2) in kinds
